@@ -1,0 +1,250 @@
+/*
+ * memspec.h - C ABI of the GB300 (sm_103a) draft-then-verify step.
+ *
+ * The library implements the data-parallel hot path of speculative decoding
+ * as MemSpec runs it (arxiv 2608.10362, Section 3.5: "the standard
+ * draft-and-verify process"; throughput ~ E[A] / L_iter, Section 2.1 Eq. 1):
+ *
+ *   memspec_draft_step    the draft model's K autoregressive M=1 proposals
+ *   memspec_verify_step   one target pass over the K+1 positions
+ *                         [last committed token, x_1..x_K] against its KV cache
+ *   memspec_accept_commit speculative-sampling acceptance (accept x_i with
+ *                         probability min(1, p_i(x_i)/q_i(x_i)), else resample
+ *                         from norm(max(0, p - q)); bonus token when all K are
+ *                         accepted; Leviathan et al. ICML'23 Alg. 1, cited by
+ *                         the paper in Section 1) and KV commit / rollback
+ *   memspec_load_draft_async  side-stream load of a non-resident draft's
+ *                         weights into the device draft arena (Section 3.3,
+ *                         Algorithm 2: "asynchronously prefetch d"; Section 3.5:
+ *                         prefetching overlapped with decoding)
+ *
+ * The scheduling policy of MemSpec (Algorithms 1-3: prediction, cache update,
+ * best-resident selection) is host-side control logic that sits ABOVE this
+ * ABI and calls it.
+ *
+ * Conventions for every call:
+ *  - Device memory is owned by the caller (weights, KV caches, workspace, draft
+ *    arena).  The library borrows pointers and never frees them.
+ *  - Pointers named *_dev are device pointers; *_host are host pointers
+ *    (pinned where stated).  Streams are cudaStream_t passed as void*.
+ *  - Step calls only enqueue work on the main stream and return; results are
+ *    ready after memspec_sync() or a caller-side stream synchronisation.
+ *  - Every call returns a memspec_status; nothing throws across the ABI.
+ *    On error, memspec_last_error() describes the first failure of the call.
+ *    Arguments are validated before any work is enqueued: a call that returns
+ *    MEMSPEC_ERR_INVALID_ARG has enqueued nothing.
+ *  - Device-side errors (a bounded wait that ran out, an out-of-range token)
+ *    set a status word that memspec_sync() returns as
+ *    MEMSPEC_ERR_DEVICE_STATUS.  Kernels never trap.
+ *  - One context per host thread.
+ */
+#ifndef MEMSPEC_H_
+#define MEMSPEC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum memspec_status {
+  MEMSPEC_OK = 0,
+  MEMSPEC_ERR_INVALID_ARG = 1,
+  MEMSPEC_ERR_CUDA = 2,
+  MEMSPEC_ERR_BUDGET = 3,        /* draft does not fit the arena without evicting the active draft */
+  MEMSPEC_ERR_NOT_RESIDENT = 4,  /* draft named by a step is not loaded */
+  MEMSPEC_ERR_BUSY = 5,          /* draft is loading / in use */
+  MEMSPEC_ERR_TIMEOUT = 6,       /* host-side wait ran out */
+  MEMSPEC_ERR_DEVICE_STATUS = 7, /* a kernel reported an error in the device status word */
+  MEMSPEC_ERR_UNSUPPORTED = 8    /* shape outside what the kernels implement */
+} memspec_status;
+
+/* Device status word bits (memspec_sync / memspec_device_status). */
+#define MEMSPEC_DEV_TIMEOUT    0x1u  /* a bounded in-kernel wait gave up */
+#define MEMSPEC_DEV_BAD_TOKEN  0x2u  /* a token id outside [0, vocab) was fed */
+#define MEMSPEC_DEV_BAD_LENGTH 0x4u  /* sequence would exceed max_seq / draft not caught up */
+
+/* Llama-style decoder hyper-parameters (RMSNorm, RoPE on pairs (i, i+hd/2),
+ * grouped-query attention, SwiGLU).  Constraints checked by memspec_init /
+ * memspec_register_draft: head_dim in {64, 128}; n_heads % n_kv_heads == 0;
+ * n_heads*head_dim and n_kv_heads*head_dim multiples of 128; d_model a
+ * multiple of 128; d_ffn a multiple of 8; vocab >= 2. */
+typedef struct memspec_model_cfg {
+  int32_t n_layers;
+  int32_t d_model;
+  int32_t n_heads;
+  int32_t n_kv_heads;
+  int32_t head_dim;
+  int32_t d_ffn;
+  int32_t vocab;
+  int32_t tied_embeddings;  /* 1: LM head reuses the token embedding */
+  float rope_base;          /* theta_i = rope_base^(-2i/head_dim) */
+  float norm_eps;           /* RMSNorm epsilon */
+} memspec_model_cfg;
+
+/* ---- weight blob layout ------------------------------------------------
+ * A model's weights live in ONE contiguous blob (device memory for the
+ * target, pinned host memory for drafts that get loaded into the arena).
+ * Every tensor is bf16, row-major, 256-byte aligned inside the blob:
+ *   TOK_EMB [vocab][d]            LM_HEAD [vocab][d] (absent if tied)
+ *   per layer: ATTN_NORM [d], WQKV [(H + 2 Hkv) hd][d] (q rows, then k, then v),
+ *   WO [d][H hd], FFN_NORM [d], WGATE [F][d], WUP [F][d], WDOWN [d][F]
+ *   FINAL_NORM [d]
+ * Linear weights are [out][in], i.e. y = x W^T. */
+typedef enum memspec_tensor {
+  MEMSPEC_T_TOK_EMB = 0,
+  MEMSPEC_T_ATTN_NORM = 1,
+  MEMSPEC_T_WQKV = 2,
+  MEMSPEC_T_WO = 3,
+  MEMSPEC_T_FFN_NORM = 4,
+  MEMSPEC_T_WGATE = 5,
+  MEMSPEC_T_WUP = 6,
+  MEMSPEC_T_WDOWN = 7,
+  MEMSPEC_T_FINAL_NORM = 8,
+  MEMSPEC_T_LM_HEAD = 9
+} memspec_tensor;
+
+/* Total blob bytes for cfg.  Errors: INVALID_ARG (null / bad cfg). */
+memspec_status memspec_weights_bytes(const memspec_model_cfg* cfg, size_t* bytes);
+
+/* Byte offset and size of one tensor inside the blob.  layer is ignored for
+ * the non-layer tensors.  LM_HEAD of a tied model reports TOK_EMB's offset.
+ * Errors: INVALID_ARG (bad tensor id / layer). */
+memspec_status memspec_weights_offset(const memspec_model_cfg* cfg, int32_t tensor,
+                                      int32_t layer, size_t* offset, size_t* bytes);
+
+/* Bytes of one model's KV cache: n_layers * 2 * max_batch * n_kv_heads *
+ * max_seq * head_dim bf16, layout [layer][K|V][request][kv_head][pos][hd]. */
+memspec_status memspec_kv_bytes(const memspec_model_cfg* cfg, int32_t max_batch,
+                                int32_t max_seq, size_t* bytes);
+
+/* ---- context --------------------------------------------------------------*/
+typedef struct memspec_ctx memspec_ctx;
+
+typedef struct memspec_init_params {
+  memspec_model_cfg target;
+  const void* target_weights_dev;   /* blob, memspec_weights_bytes(target) bytes */
+  void* target_kv_dev;              /* memspec_kv_bytes(target, max_batch, max_seq) */
+  int32_t max_batch;                /* requests verified together (1..64) */
+  int32_t max_seq;                  /* prefix + generated tokens per request */
+  int32_t max_k;                    /* largest draft length K (1..15) */
+  int32_t max_drafts;               /* draft ids 0..max_drafts-1 (<= 16) */
+  memspec_model_cfg draft_shape_max;/* largest draft shape that will be registered
+                                       (sizes the activation workspace) */
+  void* draft_arena_dev;            /* device arena for resident draft weights */
+  size_t draft_budget_bytes;        /* arena size = the enforced draft budget */
+  void* stream_main;                /* cudaStream_t for all step calls */
+  void* stream_side;                /* cudaStream_t for draft loads (may equal main) */
+  int32_t use_graphs;               /* 1: capture each step once and replay it */
+} memspec_init_params;
+
+/* Device workspace bytes memspec_init needs for these params. */
+memspec_status memspec_workspace_bytes(const memspec_init_params* p, size_t* bytes);
+
+/* Create a context.  workspace_dev: device memory of memspec_workspace_bytes
+ * bytes, 256-byte aligned, caller-owned, untouched by the caller afterwards.
+ * Builds TMA descriptors for the target weights.  Errors: INVALID_ARG,
+ * UNSUPPORTED (shape), CUDA. */
+memspec_status memspec_init(const memspec_init_params* p, void* workspace_dev,
+                            memspec_ctx** out);
+
+/* Release host-side resources (graphs, events).  Does not free caller memory. */
+void memspec_destroy(memspec_ctx* ctx);
+
+/* Message describing the last error of this context (never NULL). */
+const char* memspec_last_error(const memspec_ctx* ctx);
+
+/* ---- drafts (Section 3.3: candidate set D, resident set G under a budget) --*/
+
+/* Register draft draft_id with its weights in pinned host memory (the backing
+ * tier) and its own device KV cache (memspec_kv_bytes(cfg, max_batch,
+ * max_seq)).  The host blob must stay valid while the draft is registered.
+ * Errors: INVALID_ARG, UNSUPPORTED, BUSY (id already registered). */
+memspec_status memspec_register_draft(memspec_ctx* ctx, int32_t draft_id,
+                                      const memspec_model_cfg* cfg,
+                                      const void* weights_host_pinned,
+                                      void* kv_dev);
+
+/* Start copying draft_id's weights into the arena on the side stream
+ * (non-blocking).  Places the draft first-fit in the arena.  If it does not
+ * fit, returns MEMSPEC_ERR_BUDGET and changes nothing: the caller chooses what
+ * to evict (the active draft is never evicted implicitly).  Already resident
+ * or loading: returns OK.  *slot_offset (optional) receives the arena offset. */
+memspec_status memspec_load_draft_async(memspec_ctx* ctx, int32_t draft_id,
+                                        size_t* slot_offset);
+
+/* *state: 0 = not resident, 1 = resident, 2 = loading (copy in flight). */
+memspec_status memspec_query_draft(memspec_ctx* ctx, int32_t draft_id, int32_t* state);
+
+/* Drop draft_id from the arena.  Refuses (BUSY) while its copy is in flight
+ * or while it is the active draft (the draft of the last draft step that has
+ * not been followed by memspec_set_active_draft to another draft). */
+memspec_status memspec_evict_draft(memspec_ctx* ctx, int32_t draft_id);
+
+/* Make draft_id the active draft.  It must be resident or loading (a loading
+ * draft makes the next draft step wait on the GPU, never on the host).  The
+ * new draft's KV cache is brought up to date with the committed tokens by a
+ * chunked prefill on the main stream (host-synchronising: it reads the
+ * committed lengths). */
+memspec_status memspec_set_active_draft(memspec_ctx* ctx, int32_t draft_id);
+
+/* ---- requests ----------------------------------------------------------- */
+
+/* Start request req with prompt tokens_host[0..n) (n >= 1) and Philox seed:
+ * copies the prompt, runs the target and the active draft over all prompt
+ * tokens but the last (chunks of up to 128 rows), and resets the request's
+ * iteration counter.  Host-synchronising.  Errors: INVALID_ARG, CUDA. */
+memspec_status memspec_prefill(memspec_ctx* ctx, int32_t req, const int32_t* tokens_host,
+                               int32_t n, uint64_t seed);
+
+/* Number of requests stepped together by the step calls (1..max_batch). All
+ * of them must have been prefilled. */
+memspec_status memspec_set_batch(memspec_ctx* ctx, int32_t batch);
+
+/* ---- the draft-then-verify step ----------------------------------------- */
+
+/* The active draft proposes x_1..x_K for every request: K forward passes of
+ * one position each (two for the first pass after a fully accepted step),
+ * each followed by sampling x_j ~ softmax(z/T) with Philox uniform slot j-1
+ * (T == 0: argmax).  Draft logits are kept for acceptance.  Enqueue only. */
+memspec_status memspec_draft_step(memspec_ctx* ctx, int32_t K, float temperature);
+
+/* One target pass over [t_{L-1}, x_1..x_K] at positions L-1..L-1+K per request,
+ * appending their K,V to the target cache and writing fp32 logits for
+ * positions L..L+K.  Enqueue only. */
+memspec_status memspec_verify_step(memspec_ctx* ctx, int32_t K);
+
+/* Acceptance, resampling and commit for every request (see the file header):
+ * n accepted tokens, the correction/bonus token y, L += n + 1, KV rollback by
+ * length (target KV valid below L-1; draft KV below L-1, or L-2 when n = K).
+ * If results_host_pinned is not NULL, an async copy of int32
+ * [batch][K+2] = {n, x_1..x_n, y, unused...} to it is enqueued.  Enqueue only. */
+memspec_status memspec_accept_commit(memspec_ctx* ctx, int32_t K, float temperature,
+                                     int32_t* results_host_pinned);
+
+/* Wait for the main stream (timeout_ms < 0: no limit) and return the device
+ * status word as MEMSPEC_ERR_DEVICE_STATUS if any bit is set (the word is then
+ * cleared; *bits, if given, receives it).  Errors: TIMEOUT, CUDA. */
+memspec_status memspec_sync(memspec_ctx* ctx, int32_t timeout_ms, uint32_t* bits);
+
+/* ---- inspection (tests, tooling) ----------------------------------------- */
+typedef enum memspec_buffer {
+  MEMSPEC_BUF_TARGET_LOGITS = 0, /* fp32 [batch][K+1][vocab] of the last verify */
+  MEMSPEC_BUF_DRAFT_LOGITS = 1,  /* fp32 [batch][K][vocab] of the last draft step */
+  MEMSPEC_BUF_DRAFT_TOKENS = 2,  /* int32 [batch][max_k] */
+  MEMSPEC_BUF_TOKENS = 3,        /* int32 [max_batch][max_seq] committed tokens */
+  MEMSPEC_BUF_SEQ_STATE = 4,     /* int32 [max_batch][4] = {L, Lt, step, active Ld} */
+  MEMSPEC_BUF_ACCEPT_DEBUG = 5,  /* fp32 [batch][2K+2] = {p_i(x_i), q_i(x_i), residual mass, u'} */
+  MEMSPEC_BUF_RESIDUAL = 6       /* fp32 residual stream [rows][d] of the last forward */
+} memspec_buffer;
+
+/* Synchronously copy `bytes` of an internal buffer to host memory (waits for
+ * the main stream first).  Errors: INVALID_ARG (bytes too large), CUDA. */
+memspec_status memspec_read_buffer(memspec_ctx* ctx, int32_t buffer, void* dst_host,
+                                   size_t bytes);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MEMSPEC_H_ */

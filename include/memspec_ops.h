@@ -1,0 +1,60 @@
+/*
+ * memspec_ops.h - op-level entry points of the same library (libmemspec.so).
+ *
+ * These expose single kernels of the draft-then-verify step so that each can
+ * be checked and timed on its own.  Same conventions as memspec.h: device
+ * pointers are caller-owned, work is enqueued on the given stream, arguments
+ * are validated before anything is enqueued.
+ */
+#ifndef MEMSPEC_OPS_H_
+#define MEMSPEC_OPS_H_
+
+#include "memspec.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Scratch bytes that memspec_op_linear needs for (rows, n_out, k): split-K
+ * partial sums and per-row-tile arrival counters. */
+memspec_status memspec_op_linear_scratch_bytes(int32_t rows, int32_t n_out, int32_t k,
+                                               size_t* bytes);
+
+/* y[rows][n_out] (fp32) = x[rows][k] (bf16, row-major) . w[n_out][k]^T (bf16).
+ * This is the weight-streaming GEMM every projection of the verify and draft
+ * passes runs (Q/K/V, O, gate/up, down, LM head): TMA-staged weight tiles,
+ * tcgen05 MMA into TMEM, stream-K over all SMs, deterministic split-K
+ * reduction.  rows in 1..256, k a multiple of 8, n_out >= 1.
+ * scratch_dev: memspec_op_linear_scratch_bytes bytes, 256-byte aligned; its
+ * counters must be zero on entry and are left zero on exit (zero it once).
+ * status_dev: uint32 device word, bits set on in-kernel errors (may be NULL).
+ * x, w: 16-byte aligned.  Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
+memspec_status memspec_op_linear(const void* x_dev, const void* w_dev, float* y_dev,
+                                 int32_t rows, int32_t n_out, int32_t k,
+                                 void* scratch_dev, size_t scratch_bytes,
+                                 uint32_t* status_dev, void* stream);
+
+/* Categorical sampling of each row of logits[rows][vocab] (fp32): with T > 0,
+ * out[r] = smallest j with sum_{i<=j} exp(z_i/T - m) > u[r] * sum_i exp(z_i/T - m);
+ * with T == 0, out[r] = argmax (lowest id on ties).  u_dev: fp32 [rows] in
+ * (0,1) (ignored for T == 0).  This is the draft-token sampler of
+ * memspec_draft_step. */
+memspec_status memspec_op_sample(const float* logits_dev, int32_t rows, int32_t vocab,
+                                 float temperature, const float* u_dev, int32_t* out_dev,
+                                 void* stream);
+
+/* Message describing the last failed op-level call (or memspec_init) on this
+ * host thread; never NULL. */
+const char* memspec_op_last_error(void);
+
+/* Overwrite an internal buffer of ctx (same ids as memspec_read_buffer) from
+ * host memory; synchronous.  Lets tests feed the acceptance step synthetic
+ * logits and set sequence state.  Writable: TARGET_LOGITS, DRAFT_LOGITS,
+ * DRAFT_TOKENS, TOKENS, SEQ_STATE. */
+memspec_status memspec_write_buffer(memspec_ctx* ctx, int32_t buffer, const void* src_host,
+                                    size_t bytes);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MEMSPEC_OPS_H_ */

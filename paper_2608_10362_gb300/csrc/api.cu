@@ -1,0 +1,1395 @@
+// api.cu - host runtime behind the C ABI of include/memspec.h and memspec_ops.h.
+//
+// Responsibilities: validate arguments, carve the caller's workspace, encode TMA
+// descriptors for every weight matrix, enqueue the forward passes of the
+// draft-then-verify step (optionally captured once as CUDA graphs and
+// replayed), manage the draft arena (first-fit placement under the byte budget,
+// side-stream copies fenced by events), and report errors as status codes.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <ctime>
+#include <map>
+#include <mutex>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "../../include/memspec.h"
+#include "../../include/memspec_ops.h"
+#include "internal.h"
+
+using namespace memspec;
+
+namespace {
+
+thread_local std::string g_op_error;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// 2D bf16 tensor map over a row-major [rows][cols] matrix, box {64 cols, box_rows},
+// 128-byte swizzle, zero fill out of bounds.
+bool encode_map(CUtensorMap* map, const void* base, int rows, int cols, int box_rows) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (fn == nullptr) return false;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) != 0 || (cols * 2) % 16 != 0) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
+  cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+int round_up(int x, int m) { return (x + m - 1) / m * m; }
+int ceil_div(int a, int b) { return (a + b - 1) / b; }
+
+int sm_count() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+bool ensure_func_attrs() {
+  static bool done = false;
+  if (done) return true;
+  if (gemm_set_max_smem() != cudaSuccess) return false;
+  if (attention_set_max_smem() != cudaSuccess) return false;
+  done = true;
+  return true;
+}
+
+// ---------------------------------------------------------------- blob layout
+struct Layout {
+  size_t emb, final_norm, lm_head, total;
+  std::vector<size_t> attn_norm, wqkv, wo, ffn_norm, wgate, wup, wdown;
+};
+
+bool cfg_valid(const memspec_model_cfg* c, std::string* why) {
+  if (c == nullptr) {
+    *why = "null model cfg";
+    return false;
+  }
+  if (c->n_layers < 1 || c->d_model < 128 || c->n_heads < 1 || c->n_kv_heads < 1 ||
+      c->head_dim < 1 || c->d_ffn < 8 || c->vocab < 2) {
+    *why = "model cfg: a dimension is out of range";
+    return false;
+  }
+  if (c->n_heads % c->n_kv_heads != 0) {
+    *why = "model cfg: n_heads must be a multiple of n_kv_heads";
+    return false;
+  }
+  if (!(c->rope_base > 0.f) || !(c->norm_eps >= 0.f)) {
+    *why = "model cfg: rope_base must be > 0 and norm_eps >= 0";
+    return false;
+  }
+  return true;
+}
+
+memspec_status cfg_supported(const memspec_model_cfg* c, std::string* why) {
+  if (c->head_dim != 64 && c->head_dim != 128) {
+    *why = "head_dim must be 64 or 128";
+    return MEMSPEC_ERR_UNSUPPORTED;
+  }
+  if (c->d_model % 128 || (c->n_heads * c->head_dim) % 128 || (c->n_kv_heads * c->head_dim) % 128) {
+    *why = "d_model, n_heads*head_dim and n_kv_heads*head_dim must be multiples of 128";
+    return MEMSPEC_ERR_UNSUPPORTED;
+  }
+  if (c->d_ffn % 8) {
+    *why = "d_ffn must be a multiple of 8";
+    return MEMSPEC_ERR_UNSUPPORTED;
+  }
+  if (c->vocab > 131072) {
+    *why = "vocab must be <= 131072";
+    return MEMSPEC_ERR_UNSUPPORTED;
+  }
+  return MEMSPEC_OK;
+}
+
+Layout make_layout(const memspec_model_cfg& c) {
+  Layout L;
+  const size_t d = c.d_model, q = static_cast<size_t>(c.n_heads) * c.head_dim,
+               kv = static_cast<size_t>(c.n_kv_heads) * c.head_dim, f = c.d_ffn, v = c.vocab;
+  size_t off = 0;
+  auto take = [&](size_t elems) {
+    const size_t o = off;
+    off = align256(off + elems * 2);
+    return o;
+  };
+  L.emb = take(v * d);
+  for (int l = 0; l < c.n_layers; ++l) {
+    L.attn_norm.push_back(take(d));
+    L.wqkv.push_back(take((q + 2 * kv) * d));
+    L.wo.push_back(take(d * q));
+    L.ffn_norm.push_back(take(d));
+    L.wgate.push_back(take(f * d));
+    L.wup.push_back(take(f * d));
+    L.wdown.push_back(take(d * f));
+  }
+  L.final_norm = take(d);
+  L.lm_head = c.tied_embeddings ? L.emb : take(v * d);
+  L.total = off;
+  return L;
+}
+
+size_t kv_bytes(const memspec_model_cfg& c, int max_batch, int max_seq) {
+  return static_cast<size_t>(c.n_layers) * 2 * max_batch * c.n_kv_heads * max_seq * c.head_dim * 2;
+}
+
+// ---------------------------------------------------------------- attention launch geometry
+struct AttnGeo {
+  int rows_per_block, row_blocks, n_splits, chunk, qmax;
+  size_t part_floats() const { return 0; }
+};
+
+AttnGeo attn_geometry(const memspec_model_cfg& c, int groups, int R, int max_seq) {
+  AttnGeo g;
+  const int gs = c.n_heads / c.n_kv_heads;
+  const int qlimit = c.head_dim == 128 ? 64 : 128;
+  int rpb = std::max(1, qlimit / gs);
+  rpb = std::min(rpb, R);
+  g.rows_per_block = rpb;
+  g.row_blocks = ceil_div(R, rpb);
+  g.qmax = gs * rpb;
+  const int units = groups * c.n_kv_heads * g.row_blocks;
+  const int max_splits = ceil_div(max_seq, 64);
+  int want = std::max(1, ceil_div(2 * sm_count(), units));
+  want = std::min(want, max_splits);
+  g.chunk = round_up(ceil_div(max_seq, want), 64);
+  g.n_splits = ceil_div(max_seq, g.chunk);
+  return g;
+}
+
+size_t attn_part_floats(const memspec_model_cfg& c, const AttnGeo& g, int groups) {
+  const size_t units = static_cast<size_t>(groups) * c.n_kv_heads * g.row_blocks;
+  return units * g.n_splits * g.qmax * c.head_dim;
+}
+size_t attn_units(const memspec_model_cfg& c, const AttnGeo& g, int groups) {
+  return static_cast<size_t>(groups) * c.n_kv_heads * g.row_blocks;
+}
+
+// ---------------------------------------------------------------- models
+struct ModelRT {
+  memspec_model_cfg cfg{};
+  Layout lay;
+  const uint8_t* w = nullptr;  // device blob
+  bf16* kv = nullptr;
+  std::vector<CUtensorMap> m_qkv, m_o, m_gate, m_up, m_down;
+  CUtensorMap m_lm{};
+  int l2_hint = L2_EVICT_FIRST;
+  bool ready = false;
+};
+
+bool build_maps(ModelRT& m, std::string* why) {
+  const memspec_model_cfg& c = m.cfg;
+  const int d = c.d_model, q = c.n_heads * c.head_dim, kv = c.n_kv_heads * c.head_dim,
+            f = c.d_ffn;
+  m.m_qkv.resize(c.n_layers);
+  m.m_o.resize(c.n_layers);
+  m.m_gate.resize(c.n_layers);
+  m.m_up.resize(c.n_layers);
+  m.m_down.resize(c.n_layers);
+  bool ok = true;
+  for (int l = 0; l < c.n_layers; ++l) {
+    ok &= encode_map(&m.m_qkv[l], m.w + m.lay.wqkv[l], q + 2 * kv, d, 128);
+    ok &= encode_map(&m.m_o[l], m.w + m.lay.wo[l], d, q, 128);
+    ok &= encode_map(&m.m_gate[l], m.w + m.lay.wgate[l], f, d, 64);
+    ok &= encode_map(&m.m_up[l], m.w + m.lay.wup[l], f, d, 64);
+    ok &= encode_map(&m.m_down[l], m.w + m.lay.wdown[l], d, f, 128);
+  }
+  ok &= encode_map(&m.m_lm, m.w + m.lay.lm_head, c.vocab, d, 128);
+  if (!ok) *why = "cuTensorMapEncodeTiled failed (driver entry point or alignment)";
+  m.ready = ok;
+  return ok;
+}
+
+struct DraftRec {
+  bool registered = false;
+  memspec_model_cfg cfg{};
+  const void* host_blob = nullptr;
+  size_t bytes = 0;
+  int state = 0;  // 0 not resident, 1 resident, 2 loading
+  size_t arena_off = 0;
+  cudaEvent_t ev = nullptr;
+  ModelRT rt;
+  int* d_len = nullptr;  // device [max_batch]
+};
+
+struct GraphKey {
+  int kind, draft, K;
+  uint32_t tbits;
+  int batch;
+  bool operator<(const GraphKey& o) const {
+    return std::tie(kind, draft, K, tbits, batch) < std::tie(o.kind, o.draft, o.K, o.tbits, o.batch);
+  }
+};
+
+}  // namespace
+
+struct memspec_ctx {
+  memspec_init_params p{};
+  cudaStream_t main = nullptr, side = nullptr;
+  std::string err;
+  // workspace
+  float* h = nullptr;
+  float* ss = nullptr;
+  int ss_stride = kMaxRows;
+  float* q = nullptr;
+  bf16* o = nullptr;
+  bf16* act = nullptr;
+  float* gemm_part = nullptr;
+  int* gemm_cnt = nullptr;
+  float* att_po = nullptr;
+  float* att_pml = nullptr;
+  int* att_cnt = nullptr;
+  size_t att_po_cap = 0, att_cnt_cap = 0;
+  float* zt = nullptr;
+  float* zd = nullptr;
+  int* tokens = nullptr;
+  int* state = nullptr;
+  int* draft_tokens = nullptr;
+  int* d_len_all = nullptr;
+  unsigned long long* seeds = nullptr;
+  RowPlan* plan = nullptr;
+  uint32_t* status = nullptr;
+  int* results = nullptr;
+  float* acc_part = nullptr;
+  float* acc_dbg = nullptr;
+  int* acc_cnt = nullptr;
+  int* smp_cnt = nullptr;
+  float* rope_cos[2] = {nullptr, nullptr};  // hd 64, hd 128
+  float* rope_sin[2] = {nullptr, nullptr};
+  size_t ws_bytes = 0;
+  int max_rows = 0;
+  int vocab = 0;
+  // models
+  ModelRT target;
+  DraftRec drafts[kMaxDrafts];
+  int active = -1;
+  int batch = 1;
+  int last_K = 0;
+  std::map<GraphKey, cudaGraphExec_t> graphs;
+};
+
+namespace {
+
+memspec_status fail(memspec_ctx* c, memspec_status s, const std::string& why) {
+  if (c) c->err = why;
+  return s;
+}
+memspec_status cuda_fail(memspec_ctx* c, cudaError_t e, const char* where) {
+  std::string m = std::string(where) + ": " + cudaGetErrorString(e);
+  if (c) c->err = m;
+  return MEMSPEC_ERR_CUDA;
+}
+
+struct WsPlan {
+  size_t off = 0;
+  size_t take(size_t bytes) {
+    const size_t o = off;
+    off = align256(off + bytes);
+    return o;
+  }
+};
+
+int model_q(const memspec_model_cfg& c) { return c.n_heads * c.head_dim; }
+int model_kv(const memspec_model_cfg& c) { return c.n_kv_heads * c.head_dim; }
+
+// Computes (and optionally binds) the workspace layout.
+size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* base) {
+  const memspec_model_cfg& t = p->target;
+  const memspec_model_cfg& dm = p->draft_shape_max;
+  const bool has_draft = p->max_drafts > 0;
+  auto mx = [&](int a, int b) { return has_draft ? std::max(a, b) : a; };
+  const int dmax = mx(t.d_model, dm.d_model);
+  const int qmax_dim = mx(model_q(t), model_q(dm));
+  const int fmax = mx(t.d_ffn, dm.d_ffn);
+  const int B = p->max_batch, K = p->max_k;
+  const int rows = std::max({B * (K + 1), kPrefillChunk, 2 * B});
+  const int V = t.vocab;
+  const int nsm = sm_count();
+  // attention partial sizing: max over the passes this context runs
+  size_t po = 0, cnt = 0;
+  auto acc_att = [&](const memspec_model_cfg& m, int groups, int R) {
+    AttnGeo g = attn_geometry(m, groups, R, p->max_seq);
+    po = std::max(po, attn_part_floats(m, g, groups));
+    cnt = std::max(cnt, attn_units(m, g, groups));
+  };
+  acc_att(t, B, K + 1);
+  acc_att(t, 1, kPrefillChunk);
+  if (has_draft) {
+    acc_att(dm, B, 2);
+    acc_att(dm, B, 1);
+    acc_att(dm, 1, kPrefillChunk);
+  }
+  const int max_rt = std::max({ceil_div(V, 128), ceil_div(fmax, 64),
+                               ceil_div(model_q(t) + 2 * model_kv(t), 128),
+                               has_draft ? ceil_div(model_q(dm) + 2 * model_kv(dm), 128) : 1,
+                               ceil_div(dmax, 128)});
+  WsPlan w;
+  const size_t o_h = w.take(static_cast<size_t>(kMaxRows) * dmax * 4);
+  const size_t o_ss = w.take(static_cast<size_t>(ceil_div(dmax, 128)) * kMaxRows * 4);
+  const size_t o_q = w.take(static_cast<size_t>(kMaxRows) * qmax_dim * 4);
+  const size_t o_o = w.take(static_cast<size_t>(kMaxRows) * qmax_dim * 2);
+  const size_t o_act = w.take(static_cast<size_t>(kMaxRows) * fmax * 2);
+  const size_t o_gp = w.take(static_cast<size_t>(2) * nsm * kMaxRows * 128 * 4);
+  const size_t o_gc = w.take(static_cast<size_t>(max_rt) * 4);
+  const size_t o_apo = w.take(po * 4);
+  const size_t o_apml = w.take(po / 64 * 2 * 4 + 1024);
+  const size_t o_acnt = w.take(cnt * 4);
+  const size_t o_zt = w.take(static_cast<size_t>(B) * (K + 1) * V * 4);
+  const size_t o_zd = w.take(static_cast<size_t>(B) * K * V * 4);
+  const size_t o_tok = w.take(static_cast<size_t>(B) * p->max_seq * 4);
+  const size_t o_st = w.take(static_cast<size_t>(B) * kStateInts * 4);
+  const size_t o_dt = w.take(static_cast<size_t>(B) * K * 4);
+  const size_t o_dl = w.take(static_cast<size_t>(std::max(1, p->max_drafts)) * B * 4);
+  const size_t o_seed = w.take(static_cast<size_t>(B) * 8);
+  const size_t o_plan = w.take(sizeof(RowPlan));
+  const size_t o_status = w.take(4);
+  const size_t o_res = w.take(static_cast<size_t>(B) * (K + 2) * 4);
+  const size_t o_ap = w.take(static_cast<size_t>(B) * (2 * K + 1) * 4 * 4);
+  const size_t o_ad = w.take(static_cast<size_t>(B) * (2 * K + 2) * 4);
+  const size_t o_ac = w.take(static_cast<size_t>(B) * 4);
+  const size_t o_sc = w.take(static_cast<size_t>(B) * 4);
+  const size_t o_rc64 = w.take(static_cast<size_t>(p->max_seq) * 32 * 4);
+  const size_t o_rs64 = w.take(static_cast<size_t>(p->max_seq) * 32 * 4);
+  const size_t o_rc128 = w.take(static_cast<size_t>(p->max_seq) * 64 * 4);
+  const size_t o_rs128 = w.take(static_cast<size_t>(p->max_seq) * 64 * 4);
+  if (c != nullptr) {
+    c->h = reinterpret_cast<float*>(base + o_h);
+    c->ss = reinterpret_cast<float*>(base + o_ss);
+    c->q = reinterpret_cast<float*>(base + o_q);
+    c->o = reinterpret_cast<bf16*>(base + o_o);
+    c->act = reinterpret_cast<bf16*>(base + o_act);
+    c->gemm_part = reinterpret_cast<float*>(base + o_gp);
+    c->gemm_cnt = reinterpret_cast<int*>(base + o_gc);
+    c->att_po = reinterpret_cast<float*>(base + o_apo);
+    c->att_pml = reinterpret_cast<float*>(base + o_apml);
+    c->att_cnt = reinterpret_cast<int*>(base + o_acnt);
+    c->att_po_cap = po;
+    c->att_cnt_cap = cnt;
+    c->zt = reinterpret_cast<float*>(base + o_zt);
+    c->zd = reinterpret_cast<float*>(base + o_zd);
+    c->tokens = reinterpret_cast<int*>(base + o_tok);
+    c->state = reinterpret_cast<int*>(base + o_st);
+    c->draft_tokens = reinterpret_cast<int*>(base + o_dt);
+    c->d_len_all = reinterpret_cast<int*>(base + o_dl);
+    c->seeds = reinterpret_cast<unsigned long long*>(base + o_seed);
+    c->plan = reinterpret_cast<RowPlan*>(base + o_plan);
+    c->status = reinterpret_cast<uint32_t*>(base + o_status);
+    c->results = reinterpret_cast<int*>(base + o_res);
+    c->acc_part = reinterpret_cast<float*>(base + o_ap);
+    c->acc_dbg = reinterpret_cast<float*>(base + o_ad);
+    c->acc_cnt = reinterpret_cast<int*>(base + o_ac);
+    c->smp_cnt = reinterpret_cast<int*>(base + o_sc);
+    c->rope_cos[0] = reinterpret_cast<float*>(base + o_rc64);
+    c->rope_sin[0] = reinterpret_cast<float*>(base + o_rs64);
+    c->rope_cos[1] = reinterpret_cast<float*>(base + o_rc128);
+    c->rope_sin[1] = reinterpret_cast<float*>(base + o_rs128);
+    c->max_rows = rows;
+    c->vocab = V;
+  }
+  return w.off;
+}
+
+memspec_status validate_params(const memspec_init_params* p, std::string* why) {
+  if (p == nullptr) {
+    *why = "null params";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (!cfg_valid(&p->target, why)) return MEMSPEC_ERR_INVALID_ARG;
+  memspec_status s = cfg_supported(&p->target, why);
+  if (s != MEMSPEC_OK) return s;
+  if (p->max_batch < 1 || p->max_batch > kMaxGroups) {
+    *why = "max_batch must be in 1..64";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (p->max_k < 1 || p->max_k > kMaxK) {
+    *why = "max_k must be in 1..15";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (p->max_batch * (p->max_k + 1) > kMaxRows) {
+    *why = "max_batch * (max_k + 1) must be <= 256";
+    return MEMSPEC_ERR_UNSUPPORTED;
+  }
+  if (p->max_seq < 2 || p->max_seq > (1 << 20)) {
+    *why = "max_seq must be in 2..2^20";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (p->max_drafts < 0 || p->max_drafts > kMaxDrafts) {
+    *why = "max_drafts must be in 0..16";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (p->max_drafts > 0) {
+    if (!cfg_valid(&p->draft_shape_max, why)) return MEMSPEC_ERR_INVALID_ARG;
+    s = cfg_supported(&p->draft_shape_max, why);
+    if (s != MEMSPEC_OK) return s;
+  }
+  return MEMSPEC_OK;
+}
+
+// ---------------------------------------------------------------- forward pass
+struct FwdSpec {
+  int mode, n_groups, R, j;
+  int pre_req, pre_start, pre_count;
+  const int* d_len;  // draft pass 1: processed counts of the draft
+  float* logits;     // nullptr: no LM head
+  int last_only;
+  long long out_group_stride;
+};
+
+memspec_status run_gemm(memspec_ctx* c, GemmArgs& a, const char* what) {
+  const int T = a.row_tiles * a.k_tiles;
+  const int grid = std::min(T, sm_count());
+  a.stages = gemm_pick_stages(a.n_pad);
+  a.partials = c->gemm_part;
+  a.counters = c->gemm_cnt;
+  a.status = c->status;
+  cudaError_t e = launch_gemm(a, grid, gemm_smem_bytes(a.n_pad, a.stages), c->main, true);
+  if (e != cudaSuccess) return cuda_fail(c, e, what);
+  return MEMSPEC_OK;
+}
+
+memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
+  const memspec_model_cfg& cf = m.cfg;
+  const int d = cf.d_model, qd = model_q(cf), kvd = model_kv(cf), F = cf.d_ffn;
+  const int rows = f.n_groups * f.R;
+  const int n_pad = round_up(rows, 16);
+  const int hsel = cf.head_dim == 128 ? 1 : 0;
+  EmbedArgs ea{};
+  ea.mode = f.mode;
+  ea.n_groups = f.n_groups;
+  ea.R = f.R;
+  ea.j = f.j;
+  ea.prefill_req = f.pre_req;
+  ea.prefill_start = f.pre_start;
+  ea.prefill_count = f.pre_count;
+  ea.seq_state = c->state;
+  ea.draft_len = f.d_len;
+  ea.tokens = c->tokens;
+  ea.max_seq = c->p.max_seq;
+  ea.draft_tokens = c->draft_tokens;
+  ea.max_k = c->p.max_k;
+  ea.emb = reinterpret_cast<const bf16*>(m.w + m.lay.emb);
+  ea.d = d;
+  ea.vocab = cf.vocab;
+  ea.h = c->h;
+  ea.ss = c->ss;
+  ea.ss_stride = c->ss_stride;
+  ea.plan = c->plan;
+  ea.status = c->status;
+  cudaError_t e = launch_embed(ea, rows, c->main, true);
+  if (e != cudaSuccess) return cuda_fail(c, e, "embed launch");
+
+  const size_t layer_kv = static_cast<size_t>(c->p.max_batch) * cf.n_kv_heads * c->p.max_seq * cf.head_dim;
+  AttnGeo geo = attn_geometry(cf, f.n_groups, f.R, c->p.max_seq);
+  if (attn_part_floats(cf, geo, f.n_groups) > c->att_po_cap ||
+      attn_units(cf, geo, f.n_groups) > c->att_cnt_cap)
+    return fail(c, MEMSPEC_ERR_UNSUPPORTED, "attention partial buffer too small for this pass");
+  int ss_count = 1;
+  for (int l = 0; l < cf.n_layers; ++l) {
+    bf16* kl = m.kv + static_cast<size_t>(l) * 2 * layer_kv;
+    bf16* vl = kl + layer_kv;
+    {  // QKV + RoPE + KV append, RMSNorm fused into the activation producer
+      GemmArgs a{};
+      a.map_a = m.m_qkv[l];
+      a.n_out = qd + 2 * kvd;
+      a.k_in = d;
+      a.pair = 0;
+      a.rows_total = rows;
+      a.n_pad = n_pad;
+      a.row_tiles = ceil_div(a.n_out, 128);
+      a.k_tiles = ceil_div(d, 64);
+      a.l2_hint = m.l2_hint;
+      a.b_mode = B_F32_RMSNORM;
+      a.b_src = c->h;
+      a.b_ld = d;
+      a.gain = reinterpret_cast<const bf16*>(m.w + m.lay.attn_norm[l]);
+      a.ss = c->ss;
+      a.ss_count = ss_count;
+      a.ss_stride = c->ss_stride;
+      a.eps = cf.norm_eps;
+      a.epi = EPI_QKV;
+      a.q_out = c->q;
+      a.q_dim = qd;
+      a.kv_dim = kvd;
+      a.head_dim = cf.head_dim;
+      a.n_kv_heads = cf.n_kv_heads;
+      a.max_seq = c->p.max_seq;
+      a.kcache = kl;
+      a.vcache = vl;
+      a.rope_cos = c->rope_cos[hsel];
+      a.rope_sin = c->rope_sin[hsel];
+      a.plan = c->plan;
+      memspec_status s = run_gemm(c, a, "qkv gemm launch");
+      if (s != MEMSPEC_OK) return s;
+    }
+    {  // attention
+      AttnArgs at{};
+      at.q = c->q;
+      at.kcache = kl;
+      at.vcache = vl;
+      at.H = cf.n_heads;
+      at.Hkv = cf.n_kv_heads;
+      at.hd = cf.head_dim;
+      at.max_seq = c->p.max_seq;
+      at.rows_per_block = geo.rows_per_block;
+      at.row_blocks = geo.row_blocks;
+      at.chunk = geo.chunk;
+      at.n_splits = geo.n_splits;
+      at.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(cf.head_dim));
+      at.part_o = c->att_po;
+      at.part_ml = c->att_pml;
+      at.qmax = geo.qmax;
+      at.counters = c->att_cnt;
+      at.out = c->o;
+      at.plan = c->plan;
+      at.status = c->status;
+      e = launch_attention(at, f.n_groups, c->main, true);
+      if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
+    }
+    {  // O projection + residual
+      GemmArgs a{};
+      a.map_a = m.m_o[l];
+      a.n_out = d;
+      a.k_in = qd;
+      a.rows_total = rows;
+      a.n_pad = n_pad;
+      a.row_tiles = ceil_div(d, 128);
+      a.k_tiles = ceil_div(qd, 64);
+      a.l2_hint = m.l2_hint;
+      a.b_mode = B_BF16;
+      a.b_src = c->o;
+      a.b_ld = qd;
+      a.epi = EPI_RESIDUAL;
+      a.h = c->h;
+      a.h_ld = d;
+      a.ss_out = c->ss;
+      a.ss_stride = c->ss_stride;
+      a.plan = c->plan;
+      memspec_status s = run_gemm(c, a, "o gemm launch");
+      if (s != MEMSPEC_OK) return s;
+      ss_count = ceil_div(d, 128);
+    }
+    {  // gate/up + SwiGLU
+      GemmArgs a{};
+      a.map_a = m.m_gate[l];
+      a.map_a2 = m.m_up[l];
+      a.pair = 1;
+      a.n_out = F;
+      a.k_in = d;
+      a.rows_total = rows;
+      a.n_pad = n_pad;
+      a.row_tiles = ceil_div(F, 64);
+      a.k_tiles = ceil_div(d, 64);
+      a.l2_hint = m.l2_hint;
+      a.b_mode = B_F32_RMSNORM;
+      a.b_src = c->h;
+      a.b_ld = d;
+      a.gain = reinterpret_cast<const bf16*>(m.w + m.lay.ffn_norm[l]);
+      a.ss = c->ss;
+      a.ss_count = ss_count;
+      a.ss_stride = c->ss_stride;
+      a.eps = cf.norm_eps;
+      a.epi = EPI_SWIGLU;
+      a.act = c->act;
+      a.act_ld = F;
+      a.plan = c->plan;
+      memspec_status s = run_gemm(c, a, "gate/up gemm launch");
+      if (s != MEMSPEC_OK) return s;
+    }
+    {  // down projection + residual
+      GemmArgs a{};
+      a.map_a = m.m_down[l];
+      a.n_out = d;
+      a.k_in = F;
+      a.rows_total = rows;
+      a.n_pad = n_pad;
+      a.row_tiles = ceil_div(d, 128);
+      a.k_tiles = ceil_div(F, 64);
+      a.l2_hint = m.l2_hint;
+      a.b_mode = B_BF16;
+      a.b_src = c->act;
+      a.b_ld = F;
+      a.epi = EPI_RESIDUAL;
+      a.h = c->h;
+      a.h_ld = d;
+      a.ss_out = c->ss;
+      a.ss_stride = c->ss_stride;
+      a.plan = c->plan;
+      memspec_status s = run_gemm(c, a, "down gemm launch");
+      if (s != MEMSPEC_OK) return s;
+    }
+  }
+  if (f.logits != nullptr) {  // final RMSNorm + LM head -> fp32 logits
+    GemmArgs a{};
+    a.map_a = m.m_lm;
+    a.n_out = cf.vocab;
+    a.k_in = d;
+    a.rows_total = rows;
+    a.n_pad = n_pad;
+    a.row_tiles = ceil_div(cf.vocab, 128);
+    a.k_tiles = ceil_div(d, 64);
+    a.l2_hint = m.l2_hint;
+    a.b_mode = B_F32_RMSNORM;
+    a.b_src = c->h;
+    a.b_ld = d;
+    a.gain = reinterpret_cast<const bf16*>(m.w + m.lay.final_norm);
+    a.ss = c->ss;
+    a.ss_count = ss_count;
+    a.ss_stride = c->ss_stride;
+    a.eps = cf.norm_eps;
+    a.epi = EPI_F32;
+    a.out = f.logits;
+    a.out_ld = cf.vocab;
+    a.last_only = f.last_only;
+    a.out_group_stride = f.out_group_stride;
+    a.plan = c->plan;
+    memspec_status s = run_gemm(c, a, "lm head gemm launch");
+    if (s != MEMSPEC_OK) return s;
+  }
+  return MEMSPEC_OK;
+}
+
+// ---------------------------------------------------------------- graphs
+template <class F>
+memspec_status run_maybe_graphed(memspec_ctx* c, const GraphKey& key, F&& enqueue) {
+  if (!c->p.use_graphs) return enqueue();
+  auto it = c->graphs.find(key);
+  if (it == c->graphs.end()) {
+    cudaError_t e = cudaStreamBeginCapture(c->main, cudaStreamCaptureModeThreadLocal);
+    if (e != cudaSuccess) return cuda_fail(c, e, "begin capture");
+    memspec_status s = enqueue();
+    cudaGraph_t g = nullptr;
+    e = cudaStreamEndCapture(c->main, &g);
+    if (s != MEMSPEC_OK) {
+      if (g) cudaGraphDestroy(g);
+      return s;
+    }
+    if (e != cudaSuccess) return cuda_fail(c, e, "end capture");
+    cudaGraphExec_t ex = nullptr;
+    e = cudaGraphInstantiate(&ex, g, 0);
+    cudaGraphDestroy(g);
+    if (e != cudaSuccess) return cuda_fail(c, e, "graph instantiate");
+    it = c->graphs.emplace(key, ex).first;
+  }
+  cudaError_t e = cudaGraphLaunch(it->second, c->main);
+  if (e != cudaSuccess) return cuda_fail(c, e, "graph launch");
+  return MEMSPEC_OK;
+}
+
+void drop_graphs_of_draft(memspec_ctx* c, int draft) {
+  for (auto it = c->graphs.begin(); it != c->graphs.end();) {
+    if (it->first.draft == draft) {
+      cudaGraphExecDestroy(it->second);
+      it = c->graphs.erase(it);
+    } else {
+      ++it;
+    }
+  }
+}
+
+uint32_t fbits(float x) {
+  uint32_t u;
+  std::memcpy(&u, &x, 4);
+  return u;
+}
+
+memspec_status draft_wait_ready(memspec_ctx* c, DraftRec& dr) {
+  if (dr.state == 2) {
+    cudaError_t e = cudaStreamWaitEvent(c->main, dr.ev, 0);
+    if (e != cudaSuccess) return cuda_fail(c, e, "wait for draft load");
+  }
+  return MEMSPEC_OK;
+}
+
+// Bring draft `id`'s KV cache up to the committed tokens of requests [0, batch).
+memspec_status draft_catch_up(memspec_ctx* c, int id) {
+  DraftRec& dr = c->drafts[id];
+  const int B = c->p.max_batch;
+  std::vector<int> st(static_cast<size_t>(B) * kStateInts), dl(B);
+  cudaError_t e = cudaStreamSynchronize(c->main);
+  if (e != cudaSuccess) return cuda_fail(c, e, "sync");
+  e = cudaMemcpy(st.data(), c->state, st.size() * 4, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemcpy(dl.data(), dr.d_len, dl.size() * 4, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(c, e, "read lengths");
+  for (int b = 0; b < c->batch; ++b) {
+    const int L = st[b * kStateInts];
+    for (int start = dl[b]; start < L - 1; start += kPrefillChunk) {
+      FwdSpec f{};
+      f.mode = PLAN_PREFILL;
+      f.n_groups = 1;
+      f.R = kPrefillChunk;
+      f.pre_req = b;
+      f.pre_start = start;
+      f.pre_count = std::min(kPrefillChunk, L - 1 - start);
+      memspec_status s = enqueue_forward(c, dr.rt, f);
+      if (s != MEMSPEC_OK) return s;
+    }
+    if (L - 1 > dl[b]) {
+      const int v = L - 1;
+      e = cudaMemcpyAsync(dr.d_len + b, &v, 4, cudaMemcpyHostToDevice, c->main);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(c->main);
+      if (e != cudaSuccess) return cuda_fail(c, e, "set draft length");
+    }
+  }
+  return MEMSPEC_OK;
+}
+
+}  // namespace
+
+// =================================================================== C ABI
+extern "C" {
+
+memspec_status memspec_weights_bytes(const memspec_model_cfg* cfg, size_t* bytes) {
+  std::string why;
+  if (!cfg_valid(cfg, &why) || bytes == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  *bytes = make_layout(*cfg).total;
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_weights_offset(const memspec_model_cfg* cfg, int32_t tensor, int32_t layer,
+                                      size_t* offset, size_t* bytes) {
+  std::string why;
+  if (!cfg_valid(cfg, &why) || offset == nullptr || bytes == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  const Layout L = make_layout(*cfg);
+  const size_t d = cfg->d_model, q = static_cast<size_t>(model_q(*cfg)),
+               kv = static_cast<size_t>(model_kv(*cfg)), f = cfg->d_ffn, v = cfg->vocab;
+  const bool per_layer = tensor >= MEMSPEC_T_ATTN_NORM && tensor <= MEMSPEC_T_WDOWN;
+  if (per_layer && (layer < 0 || layer >= cfg->n_layers)) return MEMSPEC_ERR_INVALID_ARG;
+  switch (tensor) {
+    case MEMSPEC_T_TOK_EMB: *offset = L.emb; *bytes = v * d * 2; break;
+    case MEMSPEC_T_ATTN_NORM: *offset = L.attn_norm[layer]; *bytes = d * 2; break;
+    case MEMSPEC_T_WQKV: *offset = L.wqkv[layer]; *bytes = (q + 2 * kv) * d * 2; break;
+    case MEMSPEC_T_WO: *offset = L.wo[layer]; *bytes = d * q * 2; break;
+    case MEMSPEC_T_FFN_NORM: *offset = L.ffn_norm[layer]; *bytes = d * 2; break;
+    case MEMSPEC_T_WGATE: *offset = L.wgate[layer]; *bytes = f * d * 2; break;
+    case MEMSPEC_T_WUP: *offset = L.wup[layer]; *bytes = f * d * 2; break;
+    case MEMSPEC_T_WDOWN: *offset = L.wdown[layer]; *bytes = d * f * 2; break;
+    case MEMSPEC_T_FINAL_NORM: *offset = L.final_norm; *bytes = d * 2; break;
+    case MEMSPEC_T_LM_HEAD: *offset = L.lm_head; *bytes = v * d * 2; break;
+    default: return MEMSPEC_ERR_INVALID_ARG;
+  }
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_kv_bytes(const memspec_model_cfg* cfg, int32_t max_batch, int32_t max_seq,
+                                size_t* bytes) {
+  std::string why;
+  if (!cfg_valid(cfg, &why) || bytes == nullptr || max_batch < 1 || max_seq < 1)
+    return MEMSPEC_ERR_INVALID_ARG;
+  *bytes = kv_bytes(*cfg, max_batch, max_seq);
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_workspace_bytes(const memspec_init_params* p, size_t* bytes) {
+  std::string why;
+  memspec_status s = validate_params(p, &why);
+  if (s != MEMSPEC_OK) return s;
+  if (bytes == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  *bytes = layout_workspace(p, nullptr, nullptr);
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_init(const memspec_init_params* p, void* workspace_dev, memspec_ctx** out) {
+  std::string why;
+  if (out == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  *out = nullptr;
+  memspec_status s = validate_params(p, &why);
+  if (s != MEMSPEC_OK) {
+    g_op_error = why;
+    return s;
+  }
+  if (workspace_dev == nullptr || (reinterpret_cast<uintptr_t>(workspace_dev) & 255) != 0 ||
+      p->target_weights_dev == nullptr || p->target_kv_dev == nullptr ||
+      (p->max_drafts > 0 && p->draft_arena_dev == nullptr && p->draft_budget_bytes > 0)) {
+    g_op_error = "null or misaligned device pointer";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  memspec_ctx* c = new memspec_ctx();
+  c->p = *p;
+  c->main = static_cast<cudaStream_t>(p->stream_main);
+  c->side = p->stream_side ? static_cast<cudaStream_t>(p->stream_side) : c->main;
+  c->ws_bytes = layout_workspace(p, c, static_cast<uint8_t*>(workspace_dev));
+  if (!ensure_func_attrs()) {
+    g_op_error = "cudaFuncSetAttribute failed";
+    delete c;
+    return MEMSPEC_ERR_CUDA;
+  }
+  c->target.cfg = p->target;
+  c->target.lay = make_layout(p->target);
+  c->target.w = static_cast<const uint8_t*>(p->target_weights_dev);
+  c->target.kv = static_cast<bf16*>(p->target_kv_dev);
+  c->target.l2_hint = L2_EVICT_FIRST;
+  if (!build_maps(c->target, &why)) {
+    g_op_error = why;
+    delete c;
+    return MEMSPEC_ERR_CUDA;
+  }
+  cudaError_t e = cudaMemsetAsync(workspace_dev, 0, c->ws_bytes, c->main);
+  if (e == cudaSuccess)
+    e = launch_rope_table(c->rope_cos[0], c->rope_sin[0], p->max_seq, 32, p->target.rope_base, c->main);
+  if (e == cudaSuccess)
+    e = launch_rope_table(c->rope_cos[1], c->rope_sin[1], p->max_seq, 64, p->target.rope_base, c->main);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->main);
+  if (e != cudaSuccess) {
+    g_op_error = std::string("init: ") + cudaGetErrorString(e);
+    delete c;
+    return MEMSPEC_ERR_CUDA;
+  }
+  for (int i = 0; i < kMaxDrafts; ++i) c->drafts[i].d_len = c->d_len_all + i * p->max_batch;
+  *out = c;
+  return MEMSPEC_OK;
+}
+
+void memspec_destroy(memspec_ctx* c) {
+  if (c == nullptr) return;
+  for (auto& kv : c->graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& d : c->drafts)
+    if (d.ev) cudaEventDestroy(d.ev);
+  delete c;
+}
+
+const char* memspec_last_error(const memspec_ctx* c) {
+  if (c == nullptr) return g_op_error.c_str();
+  return c->err.c_str();
+}
+
+memspec_status memspec_register_draft(memspec_ctx* c, int32_t id, const memspec_model_cfg* cfg,
+                                      const void* host_blob, void* kv_dev) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  std::string why;
+  if (id < 0 || id >= c->p.max_drafts) return fail(c, MEMSPEC_ERR_INVALID_ARG, "draft id out of range");
+  if (!cfg_valid(cfg, &why)) return fail(c, MEMSPEC_ERR_INVALID_ARG, why);
+  memspec_status s = cfg_supported(cfg, &why);
+  if (s != MEMSPEC_OK) return fail(c, s, why);
+  if (cfg->vocab != c->p.target.vocab)
+    return fail(c, MEMSPEC_ERR_INVALID_ARG, "draft and target must share the vocabulary");
+  if (cfg->rope_base != c->p.target.rope_base)
+    return fail(c, MEMSPEC_ERR_UNSUPPORTED, "draft rope_base must equal the target's");
+  const memspec_model_cfg& dm = c->p.draft_shape_max;
+  if (cfg->d_model > dm.d_model || model_q(*cfg) > model_q(dm) || cfg->d_ffn > dm.d_ffn)
+    return fail(c, MEMSPEC_ERR_INVALID_ARG, "draft larger than draft_shape_max");
+  if (host_blob == nullptr || kv_dev == nullptr)
+    return fail(c, MEMSPEC_ERR_INVALID_ARG, "null draft weights or KV pointer");
+  DraftRec& d = c->drafts[id];
+  if (d.registered) return fail(c, MEMSPEC_ERR_BUSY, "draft id already registered");
+  // the draft's attention passes must fit the partial buffers
+  for (int R : {1, 2}) {
+    AttnGeo g = attn_geometry(*cfg, c->p.max_batch, R, c->p.max_seq);
+    if (attn_part_floats(*cfg, g, c->p.max_batch) > c->att_po_cap ||
+        attn_units(*cfg, g, c->p.max_batch) > c->att_cnt_cap)
+      return fail(c, MEMSPEC_ERR_UNSUPPORTED, "draft attention does not fit the workspace");
+  }
+  d.registered = true;
+  d.cfg = *cfg;
+  d.host_blob = host_blob;
+  d.bytes = make_layout(*cfg).total;
+  d.state = 0;
+  d.rt = ModelRT();
+  d.rt.cfg = *cfg;
+  d.rt.lay = make_layout(*cfg);
+  d.rt.kv = static_cast<bf16*>(kv_dev);
+  d.rt.l2_hint = L2_EVICT_NORMAL;
+  if (d.ev == nullptr) {
+    cudaError_t e = cudaEventCreateWithFlags(&d.ev, cudaEventDisableTiming);
+    if (e != cudaSuccess) return cuda_fail(c, e, "event create");
+  }
+  cudaError_t e = cudaMemsetAsync(d.d_len, 0, c->p.max_batch * 4, c->main);
+  if (e != cudaSuccess) return cuda_fail(c, e, "reset draft lengths");
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_load_draft_async(memspec_ctx* c, int32_t id, size_t* slot_offset) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (id < 0 || id >= c->p.max_drafts || !c->drafts[id].registered)
+    return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown draft id");
+  DraftRec& d = c->drafts[id];
+  if (d.state != 0) {
+    if (slot_offset) *slot_offset = d.arena_off;
+    return MEMSPEC_OK;
+  }
+  // first fit over the resident / loading drafts, sorted by offset
+  std::vector<std::pair<size_t, size_t>> used;
+  for (int i = 0; i < kMaxDrafts; ++i)
+    if (c->drafts[i].registered && c->drafts[i].state != 0)
+      used.push_back({c->drafts[i].arena_off, align256(c->drafts[i].bytes)});
+  std::sort(used.begin(), used.end());
+  size_t pos = 0;
+  const size_t need = align256(d.bytes);
+  bool found = false;
+  for (auto& u : used) {
+    if (u.first >= pos + need) {
+      found = true;
+      break;
+    }
+    pos = std::max(pos, u.first + u.second);
+  }
+  if (!found && pos + need <= c->p.draft_budget_bytes) found = true;
+  if (!found || pos + need > c->p.draft_budget_bytes)
+    return fail(c, MEMSPEC_ERR_BUDGET, "draft does not fit the draft budget; evict first");
+  uint8_t* dst = static_cast<uint8_t*>(c->p.draft_arena_dev) + pos;
+  cudaError_t e = cudaMemcpyAsync(dst, d.host_blob, d.bytes, cudaMemcpyHostToDevice, c->side);
+  if (e == cudaSuccess) e = cudaEventRecord(d.ev, c->side);
+  if (e != cudaSuccess) return cuda_fail(c, e, "draft copy");
+  d.arena_off = pos;
+  d.state = 2;
+  d.rt.w = dst;
+  std::string why;
+  if (!build_maps(d.rt, &why)) return fail(c, MEMSPEC_ERR_CUDA, why);
+  drop_graphs_of_draft(c, id);
+  if (slot_offset) *slot_offset = pos;
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_query_draft(memspec_ctx* c, int32_t id, int32_t* state) {
+  if (c == nullptr || state == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (id < 0 || id >= c->p.max_drafts || !c->drafts[id].registered)
+    return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown draft id");
+  DraftRec& d = c->drafts[id];
+  if (d.state == 2) {
+    cudaError_t e = cudaEventQuery(d.ev);
+    if (e == cudaSuccess) d.state = 1;
+    else if (e != cudaErrorNotReady) return cuda_fail(c, e, "event query");
+  }
+  *state = d.state;
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_evict_draft(memspec_ctx* c, int32_t id) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (id < 0 || id >= c->p.max_drafts || !c->drafts[id].registered)
+    return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown draft id");
+  DraftRec& d = c->drafts[id];
+  if (id == c->active) return fail(c, MEMSPEC_ERR_BUSY, "the active draft is never evicted");
+  if (d.state == 2) {
+    cudaError_t e = cudaEventQuery(d.ev);
+    if (e == cudaErrorNotReady) return fail(c, MEMSPEC_ERR_BUSY, "draft copy in flight");
+    if (e != cudaSuccess) return cuda_fail(c, e, "event query");
+  }
+  // work already enqueued on the main stream may still read the weights
+  cudaError_t e = cudaStreamSynchronize(c->main);
+  if (e != cudaSuccess) return cuda_fail(c, e, "sync");
+  d.state = 0;
+  d.rt.w = nullptr;
+  d.rt.ready = false;
+  drop_graphs_of_draft(c, id);
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_set_active_draft(memspec_ctx* c, int32_t id) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (id < 0 || id >= c->p.max_drafts || !c->drafts[id].registered)
+    return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown draft id");
+  DraftRec& d = c->drafts[id];
+  if (d.state == 0) return fail(c, MEMSPEC_ERR_NOT_RESIDENT, "draft is not resident");
+  memspec_status s = draft_wait_ready(c, d);
+  if (s != MEMSPEC_OK) return s;
+  c->active = id;
+  return draft_catch_up(c, id);
+}
+
+memspec_status memspec_prefill(memspec_ctx* c, int32_t req, const int32_t* tokens, int32_t n,
+                               uint64_t seed) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (req < 0 || req >= c->p.max_batch) return fail(c, MEMSPEC_ERR_INVALID_ARG, "request out of range");
+  if (tokens == nullptr || n < 1 || n >= c->p.max_seq)
+    return fail(c, MEMSPEC_ERR_INVALID_ARG, "prompt length must be in 1..max_seq-1");
+  for (int i = 0; i < n; ++i)
+    if (tokens[i] < 0 || tokens[i] >= c->vocab)
+      return fail(c, MEMSPEC_ERR_INVALID_ARG, "prompt token outside the vocabulary");
+  cudaError_t e = cudaStreamSynchronize(c->main);
+  if (e != cudaSuccess) return cuda_fail(c, e, "sync");
+  int st[kStateInts] = {n, n - 1, 0, 0};
+  const unsigned long long sd = seed;
+  e = cudaMemcpy(c->tokens + static_cast<size_t>(req) * c->p.max_seq, tokens,
+                 static_cast<size_t>(n) * 4, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(c->state + req * kStateInts, st, sizeof(st), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(c->seeds + req, &sd, 8, cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(c, e, "prefill copies");
+  for (int start = 0; start < n - 1; start += kPrefillChunk) {
+    FwdSpec f{};
+    f.mode = PLAN_PREFILL;
+    f.n_groups = 1;
+    f.R = kPrefillChunk;
+    f.pre_req = req;
+    f.pre_start = start;
+    f.pre_count = std::min(kPrefillChunk, n - 1 - start);
+    memspec_status s = enqueue_forward(c, c->target, f);
+    if (s != MEMSPEC_OK) return s;
+  }
+  // every registered draft restarts from zero for this request; the active one
+  // is brought up to date now, the others when they become active
+  for (int i = 0; i < c->p.max_drafts; ++i) {
+    if (!c->drafts[i].registered) continue;
+    const int zero = 0;
+    e = cudaMemcpy(c->drafts[i].d_len + req, &zero, 4, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(c, e, "reset draft length");
+  }
+  if (c->active >= 0) {
+    DraftRec& d = c->drafts[c->active];
+    memspec_status s = draft_wait_ready(c, d);
+    if (s != MEMSPEC_OK) return s;
+    for (int start = 0; start < n - 1; start += kPrefillChunk) {
+      FwdSpec f{};
+      f.mode = PLAN_PREFILL;
+      f.n_groups = 1;
+      f.R = kPrefillChunk;
+      f.pre_req = req;
+      f.pre_start = start;
+      f.pre_count = std::min(kPrefillChunk, n - 1 - start);
+      s = enqueue_forward(c, d.rt, f);
+      if (s != MEMSPEC_OK) return s;
+    }
+    const int v = n - 1;
+    e = cudaMemcpyAsync(d.d_len + req, &v, 4, cudaMemcpyHostToDevice, c->main);
+    if (e != cudaSuccess) return cuda_fail(c, e, "set draft length");
+  }
+  e = cudaStreamSynchronize(c->main);
+  if (e != cudaSuccess) return cuda_fail(c, e, "prefill sync");
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_set_batch(memspec_ctx* c, int32_t batch) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (batch < 1 || batch > c->p.max_batch) return fail(c, MEMSPEC_ERR_INVALID_ARG, "batch out of range");
+  c->batch = batch;
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_draft_step(memspec_ctx* c, int32_t K, float T) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (K < 1 || K > c->p.max_k) return fail(c, MEMSPEC_ERR_INVALID_ARG, "K out of range");
+  if (!(T >= 0.f)) return fail(c, MEMSPEC_ERR_INVALID_ARG, "temperature must be >= 0");
+  if (c->active < 0) return fail(c, MEMSPEC_ERR_NOT_RESIDENT, "no active draft");
+  DraftRec& d = c->drafts[c->active];
+  if (d.state == 0) return fail(c, MEMSPEC_ERR_NOT_RESIDENT, "active draft not resident");
+  memspec_status s = draft_wait_ready(c, d);
+  if (s != MEMSPEC_OK) return s;
+  const int B = c->batch;
+  const int id = c->active;
+  GraphKey key{0, id, K, fbits(T), B};
+  return run_maybe_graphed(c, key, [&]() -> memspec_status {
+    for (int j = 1; j <= K; ++j) {
+      FwdSpec f{};
+      f.mode = j == 1 ? PLAN_DRAFT_FIRST : PLAN_DRAFT_NEXT;
+      f.n_groups = B;
+      f.R = j == 1 ? 2 : 1;
+      f.j = j;
+      f.d_len = d.d_len;
+      f.logits = c->zd + static_cast<size_t>(j - 1) * c->vocab;
+      f.last_only = 1;
+      f.out_group_stride = static_cast<long long>(K) * c->vocab;
+      memspec_status st = enqueue_forward(c, d.rt, f);
+      if (st != MEMSPEC_OK) return st;
+      SampleArgs sa{};
+      sa.logits = f.logits;
+      sa.row_stride = f.out_group_stride;
+      sa.vocab = c->vocab;
+      sa.n_groups = B;
+      sa.greedy = T == 0.f;
+      sa.inv_temp = T == 0.f ? 0.f : 1.f / T;
+      sa.slot = j - 1;
+      sa.seq_state = c->state;
+      sa.seeds = c->seeds;
+      sa.out_tok = c->draft_tokens + (j - 1);
+      sa.out_stride = c->p.max_k;
+      sa.counters = c->smp_cnt;
+      sa.status = c->status;
+      cudaError_t e = launch_sample(sa, c->main, true);
+      if (e != cudaSuccess) return cuda_fail(c, e, "sample launch");
+    }
+    return MEMSPEC_OK;
+  });
+}
+
+memspec_status memspec_verify_step(memspec_ctx* c, int32_t K) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (K < 1 || K > c->p.max_k) return fail(c, MEMSPEC_ERR_INVALID_ARG, "K out of range");
+  const int B = c->batch;
+  GraphKey key{1, -1, K, 0, B};
+  return run_maybe_graphed(c, key, [&]() -> memspec_status {
+    FwdSpec f{};
+    f.mode = PLAN_VERIFY;
+    f.n_groups = B;
+    f.R = K + 1;
+    f.logits = c->zt;
+    f.last_only = 0;
+    return enqueue_forward(c, c->target, f);
+  });
+}
+
+memspec_status memspec_accept_commit(memspec_ctx* c, int32_t K, float T, int32_t* results_host) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (K < 1 || K > c->p.max_k) return fail(c, MEMSPEC_ERR_INVALID_ARG, "K out of range");
+  if (!(T >= 0.f)) return fail(c, MEMSPEC_ERR_INVALID_ARG, "temperature must be >= 0");
+  const int B = c->batch;
+  const int id = c->active;
+  if (id < 0) return fail(c, MEMSPEC_ERR_NOT_RESIDENT, "no active draft");
+  GraphKey key{2, id, K, fbits(T), B};
+  memspec_status s = run_maybe_graphed(c, key, [&]() -> memspec_status {
+    AcceptArgs a{};
+    a.zt = c->zt;
+    a.zd = c->zd;
+    a.draft_tokens = c->draft_tokens;
+    a.max_k = c->p.max_k;
+    a.K = K;
+    a.vocab = c->vocab;
+    a.n_groups = B;
+    a.greedy = T == 0.f;
+    a.inv_temp = T == 0.f ? 0.f : 1.f / T;
+    a.part = c->acc_part;
+    a.counters = c->acc_cnt;
+    a.seq_state = c->state;
+    a.seeds = c->seeds;
+    a.draft_len = c->drafts[id].d_len;
+    a.tokens = c->tokens;
+    a.max_seq = c->p.max_seq;
+    a.results = c->results;
+    a.debug = c->acc_dbg;
+    a.status = c->status;
+    cudaError_t e = launch_accept(a, c->main, false);
+    if (e != cudaSuccess) return cuda_fail(c, e, "accept launch");
+    return MEMSPEC_OK;
+  });
+  if (s != MEMSPEC_OK) return s;
+  c->last_K = K;
+  if (results_host != nullptr) {
+    cudaError_t e = cudaMemcpyAsync(results_host, c->results, static_cast<size_t>(B) * (K + 2) * 4,
+                                    cudaMemcpyDeviceToHost, c->main);
+    if (e != cudaSuccess) return cuda_fail(c, e, "results copy");
+  }
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_sync(memspec_ctx* c, int32_t timeout_ms, uint32_t* bits) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  cudaError_t e;
+  if (timeout_ms < 0) {
+    e = cudaStreamSynchronize(c->main);
+  } else {
+    cudaEvent_t ev;
+    e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+    if (e != cudaSuccess) return cuda_fail(c, e, "event create");
+    e = cudaEventRecord(ev, c->main);
+    int waited = 0;
+    while (e == cudaSuccess) {
+      e = cudaEventQuery(ev);
+      if (e != cudaErrorNotReady) break;
+      if (waited >= timeout_ms) {
+        cudaEventDestroy(ev);
+        return fail(c, MEMSPEC_ERR_TIMEOUT, "sync timed out");
+      }
+      struct timespec ts = {0, 1000000};
+      nanosleep(&ts, nullptr);
+      ++waited;
+    }
+    cudaEventDestroy(ev);
+  }
+  if (e != cudaSuccess) return cuda_fail(c, e, "sync");
+  uint32_t st = 0;
+  e = cudaMemcpy(&st, c->status, 4, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(c, e, "status read");
+  if (bits) *bits = st;
+  if (st != 0) {
+    // a kernel gave up part-way: clear the status and the arrival counters so the
+    // context can be used again
+    cudaMemset(c->status, 0, 4);
+    cudaMemset(c->gemm_cnt, 0, 4);
+    return fail(c, MEMSPEC_ERR_DEVICE_STATUS, "device status word set");
+  }
+  return MEMSPEC_OK;
+}
+
+static memspec_status buffer_span(memspec_ctx* c, int32_t buf, void** ptr, size_t* cap) {
+  const int B = c->p.max_batch, K = c->p.max_k, V = c->vocab;
+  switch (buf) {
+    case MEMSPEC_BUF_TARGET_LOGITS: *ptr = c->zt; *cap = static_cast<size_t>(B) * (K + 1) * V * 4; break;
+    case MEMSPEC_BUF_DRAFT_LOGITS: *ptr = c->zd; *cap = static_cast<size_t>(B) * K * V * 4; break;
+    case MEMSPEC_BUF_DRAFT_TOKENS: *ptr = c->draft_tokens; *cap = static_cast<size_t>(B) * K * 4; break;
+    case MEMSPEC_BUF_TOKENS: *ptr = c->tokens; *cap = static_cast<size_t>(B) * c->p.max_seq * 4; break;
+    case MEMSPEC_BUF_SEQ_STATE: *ptr = c->state; *cap = static_cast<size_t>(B) * kStateInts * 4; break;
+    case MEMSPEC_BUF_ACCEPT_DEBUG: *ptr = c->acc_dbg; *cap = static_cast<size_t>(B) * (2 * K + 2) * 4; break;
+    case MEMSPEC_BUF_RESIDUAL: *ptr = c->h; *cap = static_cast<size_t>(kMaxRows) * c->p.target.d_model * 4; break;
+    default: return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown buffer id");
+  }
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_read_buffer(memspec_ctx* c, int32_t buf, void* dst, size_t bytes) {
+  if (c == nullptr || dst == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  void* p;
+  size_t cap;
+  memspec_status s = buffer_span(c, buf, &p, &cap);
+  if (s != MEMSPEC_OK) return s;
+  if (bytes > cap) return fail(c, MEMSPEC_ERR_INVALID_ARG, "read larger than the buffer");
+  cudaError_t e = cudaStreamSynchronize(c->main);
+  if (e == cudaSuccess) e = cudaMemcpy(dst, p, bytes, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(c, e, "read buffer");
+  if (buf == MEMSPEC_BUF_SEQ_STATE && c->active >= 0) {
+    // slot 3 of each request reports the active draft's processed count
+    std::vector<int> dl(c->p.max_batch);
+    e = cudaMemcpy(dl.data(), c->drafts[c->active].d_len, dl.size() * 4, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(c, e, "read draft lengths");
+    int* out = static_cast<int*>(dst);
+    for (size_t b = 0; b < dl.size() && (b * kStateInts + 3) * 4 < bytes; ++b) out[b * kStateInts + 3] = dl[b];
+  }
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_write_buffer(memspec_ctx* c, int32_t buf, const void* src, size_t bytes) {
+  if (c == nullptr || src == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (buf != MEMSPEC_BUF_TARGET_LOGITS && buf != MEMSPEC_BUF_DRAFT_LOGITS &&
+      buf != MEMSPEC_BUF_DRAFT_TOKENS && buf != MEMSPEC_BUF_TOKENS && buf != MEMSPEC_BUF_SEQ_STATE)
+    return fail(c, MEMSPEC_ERR_INVALID_ARG, "buffer is not writable");
+  void* p;
+  size_t cap;
+  memspec_status s = buffer_span(c, buf, &p, &cap);
+  if (s != MEMSPEC_OK) return s;
+  if (bytes > cap) return fail(c, MEMSPEC_ERR_INVALID_ARG, "write larger than the buffer");
+  cudaError_t e = cudaStreamSynchronize(c->main);
+  if (e == cudaSuccess) e = cudaMemcpy(p, src, bytes, cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(c, e, "write buffer");
+  if (buf == MEMSPEC_BUF_SEQ_STATE && c->active >= 0) {
+    // slot 3 sets the active draft's processed count
+    const int* in = static_cast<const int*>(src);
+    for (size_t b = 0; (b * kStateInts + 3) * 4 < bytes && b < static_cast<size_t>(c->p.max_batch); ++b) {
+      e = cudaMemcpy(c->drafts[c->active].d_len + b, in + b * kStateInts + 3, 4, cudaMemcpyHostToDevice);
+      if (e != cudaSuccess) return cuda_fail(c, e, "write draft length");
+    }
+  }
+  return MEMSPEC_OK;
+}
+
+// ---------------------------------------------------------------- op-level entry points
+const char* memspec_op_last_error(void) { return g_op_error.c_str(); }
+
+static size_t op_linear_scratch(int rows, int n_out, int k) {
+  const int n_pad = round_up(rows, 16);
+  const int rt = ceil_div(n_out, 128);
+  (void)k;
+  return align256(static_cast<size_t>(2) * sm_count() * n_pad * 128 * 4) + align256(static_cast<size_t>(rt) * 4) + 256;
+}
+
+memspec_status memspec_op_linear_scratch_bytes(int32_t rows, int32_t n_out, int32_t k, size_t* bytes) {
+  if (bytes == nullptr || rows < 1 || rows > kMaxRows || n_out < 1 || k < 8) return MEMSPEC_ERR_INVALID_ARG;
+  *bytes = op_linear_scratch(rows, n_out, k);
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_op_linear(const void* x, const void* w, float* y, int32_t rows, int32_t n_out,
+                                 int32_t k, void* scratch, size_t scratch_bytes, uint32_t* status,
+                                 void* stream) {
+  if (x == nullptr || w == nullptr || y == nullptr || scratch == nullptr) {
+    g_op_error = "null pointer";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (rows < 1 || rows > kMaxRows || n_out < 1 || k < 8 || k % 8 != 0) {
+    g_op_error = "rows must be in 1..256, n_out >= 1, k a positive multiple of 8";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(w) & 15) ||
+      (reinterpret_cast<uintptr_t>(scratch) & 255)) {
+    g_op_error = "x and w must be 16-byte aligned, scratch 256-byte aligned";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (scratch_bytes < op_linear_scratch(rows, n_out, k)) {
+    g_op_error = "scratch too small";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (!ensure_func_attrs()) {
+    g_op_error = "cudaFuncSetAttribute failed";
+    return MEMSPEC_ERR_CUDA;
+  }
+  GemmArgs a{};
+  if (!encode_map(&a.map_a, w, n_out, k, 128)) {
+    g_op_error = "cuTensorMapEncodeTiled failed";
+    return MEMSPEC_ERR_CUDA;
+  }
+  const int n_pad = round_up(rows, 16);
+  a.n_out = n_out;
+  a.k_in = k;
+  a.rows_total = rows;
+  a.n_pad = n_pad;
+  a.row_tiles = ceil_div(n_out, 128);
+  a.k_tiles = ceil_div(k, 64);
+  a.stages = gemm_pick_stages(n_pad);
+  a.l2_hint = L2_EVICT_FIRST;
+  a.b_mode = B_BF16;
+  a.b_src = x;
+  a.b_ld = k;
+  a.epi = EPI_F32;
+  a.out = y;
+  a.out_ld = n_out;
+  uint8_t* sb = static_cast<uint8_t*>(scratch);
+  a.partials = reinterpret_cast<float*>(sb);
+  const size_t part_bytes = align256(static_cast<size_t>(2) * sm_count() * n_pad * 128 * 4);
+  a.counters = reinterpret_cast<int*>(sb + part_bytes);
+  a.status = status != nullptr ? status
+                               : reinterpret_cast<uint32_t*>(sb + part_bytes +
+                                                             align256(static_cast<size_t>(a.row_tiles) * 4));
+  a.plan = nullptr;
+  const int T = a.row_tiles * a.k_tiles;
+  const int grid = std::min(T, sm_count());
+  cudaError_t e = launch_gemm(a, grid, gemm_smem_bytes(n_pad, a.stages),
+                              static_cast<cudaStream_t>(stream), false);
+  if (e != cudaSuccess) {
+    g_op_error = std::string("gemm launch: ") + cudaGetErrorString(e);
+    return MEMSPEC_ERR_CUDA;
+  }
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_op_sample(const float* logits, int32_t rows, int32_t vocab, float T,
+                                 const float* u, int32_t* out, void* stream) {
+  if (logits == nullptr || out == nullptr || rows < 1 || rows > 65535 || vocab < 1 ||
+      vocab > 131072 || !(T >= 0.f) || (T > 0.f && u == nullptr)) {
+    g_op_error = "invalid sampling arguments";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  SampleArgs sa{};
+  sa.logits = logits;
+  sa.row_stride = vocab;
+  sa.vocab = vocab;
+  sa.n_groups = rows;
+  sa.greedy = T == 0.f;
+  sa.inv_temp = T == 0.f ? 0.f : 1.f / T;
+  sa.u_explicit = u;
+  sa.out_tok = out;
+  sa.out_stride = 1;
+  cudaError_t e = launch_sample(sa, static_cast<cudaStream_t>(stream), false);
+  if (e != cudaSuccess) {
+    g_op_error = std::string("sample launch: ") + cudaGetErrorString(e);
+    return MEMSPEC_ERR_CUDA;
+  }
+  return MEMSPEC_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,494 @@
+// gemm.cu - weight-streaming projection GEMM for the verify and draft passes.
+//
+// Y[rows][n_out] = X[rows][k] . W[n_out][k]^T with rows <= 256 (K+1 verify rows,
+// 1-2 draft rows, up to 128 prefill rows).  At these row counts every projection
+// of the decoder (QKV, O, gate/up, down, LM head) reads each weight exactly once
+// and is bound by HBM bandwidth, so the kernel is organised around streaming
+// weights:
+//
+//  * swap-AB: the weight tile is the MMA's M=128 operand, the activation rows
+//    are its N (16..256) operand; tcgen05.mma.kind::f16 (bf16 in, fp32 out)
+//    accumulates in TMEM;
+//  * weight tiles [128 rows x 64 k] arrive by TMA (128-byte swizzle) into a
+//    multi-stage mbarrier ring; they are independent of earlier kernels, so the
+//    producer starts streaming before griddepcontrol.wait (programmatic
+//    dependent launch hides the previous kernel's tail);
+//  * activation tiles are written into shared memory by two producer warps,
+//    which fuse the RMSNorm of the fp32 residual stream (rms from per-row-tile
+//    partial sums of squares written by the previous epilogue);
+//  * stream-K: the (row-tile, k-tile) space is cut into one contiguous range
+//    per CTA, one CTA per SM; a row tile split over several CTAs is reduced by
+//    the last-arriving CTA in ascending CTA order (deterministic, no float
+//    atomics) from an fp32 partial buffer;
+//  * fused epilogues: fp32 logits; residual add (+ the row sums of squares
+//    the next RMSNorm needs); SwiGLU of interleaved gate/up tiles; RoPE on q/k
+//    with K/V appended to the KV cache at each row's position.
+#include <cuda_bf16.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace memspec {
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kTileM = 128;
+constexpr int kTileK = 64;
+constexpr int kABytes = kTileM * kTileK * 2;  // 16 KB
+constexpr int kMaxStages = 8;
+constexpr int kStagePitch = 17;                // epilogue staging row pitch (floats)
+constexpr int kNumBThreads = 64;               // warps 2-3
+
+struct SmemCtl {
+  uint64_t full_a[kMaxStages];
+  uint64_t full_b[kMaxStages];
+  uint64_t empty[kMaxStages];
+  uint64_t acc_full[2];
+  uint64_t acc_empty[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort_flag;
+  int reduce_flag;
+  float red[4][16];
+};
+
+__device__ __forceinline__ uint32_t tmem_cols_for(int n_pad) {
+  uint32_t need = 2u * static_cast<uint32_t>(n_pad);
+  uint32_t c = 32;
+  while (c < need) c <<= 1;
+  return c;
+}
+
+__device__ __forceinline__ bool row_valid(const GemmArgs& a, int r) {
+  if (r >= a.rows_total) return false;
+  return a.plan == nullptr ? true : plan_row_valid(a.plan, r);
+}
+
+// Pack 8 floats into 8 bf16 (round to nearest even) as a uint4.
+__device__ __forceinline__ uint4 pack8_bf16(const float* f) {
+  uint4 u;
+  __nv_bfloat162 t;
+  t = __floats2bfloat162_rn(f[0], f[1]);
+  u.x = *reinterpret_cast<uint32_t*>(&t);
+  t = __floats2bfloat162_rn(f[2], f[3]);
+  u.y = *reinterpret_cast<uint32_t*>(&t);
+  t = __floats2bfloat162_rn(f[4], f[5]);
+  u.z = *reinterpret_cast<uint32_t*>(&t);
+  t = __floats2bfloat162_rn(f[6], f[7]);
+  u.w = *reinterpret_cast<uint32_t*>(&t);
+  return u;
+}
+
+// Epilogue for one 16-row chunk of a finished 128-feature row tile.  Called by
+// the 128 epilogue threads together; et = feature within the tile (= TMEM lane).
+__device__ void apply_epilogue(const GemmArgs& a, SmemCtl& ctl, float* stage, int rt, int chunk,
+                               int et, const float* v) {
+  const int ew = et >> 5, lane = et & 31;
+  if (a.epi == EPI_F32) {
+    const int f = rt * kTileM + et;
+    if (f < a.n_out) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int r = chunk * 16 + j;
+        if (!row_valid(a, r)) continue;
+        if (a.last_only) {
+          const int g = r / a.plan->rows_per_group;
+          const int i = r - g * a.plan->rows_per_group;
+          if (i != a.plan->valid[g] - 1) continue;
+          a.out[g * a.out_group_stride + f] = v[j];
+        } else {
+          a.out[static_cast<size_t>(r) * a.out_ld + f] = v[j];
+        }
+      }
+    }
+    return;
+  }
+  if (a.epi == EPI_RESIDUAL) {
+    const int f = rt * kTileM + et;  // n_out is a multiple of 128 (d_model)
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const int r = chunk * 16 + j;
+      float sq = 0.f;
+      if (r < a.rows_total) {
+        float* hp = a.h + static_cast<size_t>(r) * a.h_ld + f;
+        const float hn = *hp + v[j];
+        *hp = hn;
+        sq = hn * hn;
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+      if (lane == 0) ctl.red[ew][j] = sq;
+    }
+    named_bar_sync(1, 128);
+    if (et < 16) {
+      const int r = chunk * 16 + et;
+      if (r < a.rows_total) {
+        const float s = ((ctl.red[0][et] + ctl.red[1][et]) + ctl.red[2][et]) + ctl.red[3][et];
+        a.ss_out[static_cast<size_t>(rt) * a.ss_stride + r] = s;
+      }
+    }
+    named_bar_sync(1, 128);
+    return;
+  }
+  // staged epilogues: make the whole 128 x 16 chunk visible to all 128 threads
+#pragma unroll
+  for (int j = 0; j < 16; ++j) stage[et * kStagePitch + j] = v[j];
+  named_bar_sync(1, 128);
+  if (a.epi == EPI_SWIGLU) {
+    if (et < 64) {
+      const int f = rt * 64 + et;
+      if (f < a.n_out) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int r = chunk * 16 + j;
+          if (r >= a.rows_total) continue;
+          const float g = stage[et * kStagePitch + j];
+          const float u = stage[(et + 64) * kStagePitch + j];
+          const float sg = g / (1.0f + expf(-g));
+          a.act[static_cast<size_t>(r) * a.act_ld + f] = __float2bfloat16_rn(sg * u);
+        }
+      }
+    }
+  } else {  // EPI_QKV: RoPE on q and k, K/V appended to the cache
+    const int f = rt * kTileM + et;
+    const int hd = a.head_dim, half = hd >> 1;
+    int seg, fs;
+    if (f < a.q_dim) {
+      seg = 0;
+      fs = f;
+    } else if (f < a.q_dim + a.kv_dim) {
+      seg = 1;
+      fs = f - a.q_dim;
+    } else {
+      seg = 2;
+      fs = f - a.q_dim - a.kv_dim;
+    }
+    const int head = fs / hd, d = fs - head * hd;
+    const int ip = d < half ? d : d - half;   // rotation pair index
+    const int e1 = et - d + ip;               // staging index of element ip of this head
+#pragma unroll 1
+    for (int j = 0; j < 16; ++j) {
+      const int r = chunk * 16 + j;
+      if (!row_valid(a, r)) continue;
+      const int g = r / a.plan->rows_per_group;
+      const int i = r - g * a.plan->rows_per_group;
+      const int pos = a.plan->pos0[g] + i;
+      if (pos < 0 || pos >= a.max_seq) continue;   // flagged by the embedding kernel
+      float val = stage[et * kStagePitch + j];
+      if (seg < 2) {
+        const float x1 = stage[e1 * kStagePitch + j];
+        const float x2 = stage[(e1 + half) * kStagePitch + j];
+        const float c = a.rope_cos[static_cast<size_t>(pos) * half + ip];
+        const float s = a.rope_sin[static_cast<size_t>(pos) * half + ip];
+        val = d < half ? (x1 * c - x2 * s) : (x1 * s + x2 * c);
+      }
+      if (seg == 0) {
+        a.q_out[static_cast<size_t>(r) * a.q_dim + f] = val;
+      } else {
+        const int req = a.plan->req[g];
+        const size_t off =
+            ((static_cast<size_t>(req) * a.n_kv_heads + head) * a.max_seq + pos) * hd + d;
+        (seg == 1 ? a.kcache : a.vcache)[off] = __float2bfloat16_rn(val);
+      }
+    }
+  }
+  named_bar_sync(1, 128);  // staging buffer is reused by the next chunk
+}
+
+__global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_constant__ GemmArgs a) {
+  __shared__ SmemCtl ctl;
+  extern __shared__ uint8_t dsmem_raw[];
+  uint8_t* dsmem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const int S = a.stages;
+  const int b_bytes = a.n_pad * 128;
+  uint8_t* smem_a = dsmem;
+  uint8_t* smem_b = dsmem + static_cast<size_t>(S) * kABytes;
+  float* stage = reinterpret_cast<float*>(smem_b + static_cast<size_t>(S) * b_bytes);
+  float* rms = stage + kTileM * kStagePitch;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int T = a.row_tiles * a.k_tiles;
+  const int G = gridDim.x, c = blockIdx.x;
+  const int t_begin = sk_begin(c, T, G), t_end = sk_begin(c + 1, T, G);
+  const int KT = a.k_tiles;
+  const uint32_t tmem_cols = tmem_cols_for(a.n_pad);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&ctl.full_a[s], 1);
+      mbar_init(&ctl.full_b[s], kNumBThreads);
+      mbar_init(&ctl.empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&ctl.acc_full[b], 1);
+      mbar_init(&ctl.acc_empty[b], 4);
+    }
+    mbar_init(&ctl.drain, 1);
+    ctl.abort_flag = 0;
+    ctl.reduce_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    __syncwarp();
+    tmem_alloc(&ctl.tmem_base, tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  pdl_launch_dependents();
+  const uint32_t tmem_base = ctl.tmem_base;
+  volatile int* abort_flag = &ctl.abort_flag;
+
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer (weights)
+    if (lane == 0) {
+      tma_prefetch_desc(&a.map_a);
+      if (a.pair) tma_prefetch_desc(&a.map_a2);
+      const uint64_t pol = a.l2_hint == L2_EVICT_FIRST  ? l2_policy_evict_first()
+                           : a.l2_hint == L2_EVICT_LAST ? l2_policy_evict_last()
+                                                        : l2_policy_evict_normal();
+      uint32_t issued_mask = 0, last_par = 0;
+      int it = 0;
+      bool ok = true;
+      for (int t = t_begin; t < t_end && ok; ++t, ++it) {
+        const int rt = t / KT, kt = t - rt * KT;
+        const int s = it % S;
+        const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
+        if (!mbar_wait_bounded(&ctl.empty[s], ph ^ 1u, abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        uint8_t* dst = smem_a + static_cast<size_t>(s) * kABytes;
+        mbar_arrive_expect_tx(&ctl.full_a[s], kABytes);
+        if (a.pair) {
+          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * 64, &ctl.full_a[s], pol);
+          tma_load_2d(dst + kABytes / 2, &a.map_a2, kt * kTileK, rt * 64, &ctl.full_a[s], pol);
+        } else {
+          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * kTileM, &ctl.full_a[s], pol);
+        }
+        issued_mask |= 1u << s;
+        last_par = (last_par & ~(1u << s)) | (ph << s);
+      }
+      if (!ok) {  // tear-down: let every copy still in flight land before exit
+        for (int s = 0; s < S; ++s)
+          if (issued_mask & (1u << s)) mbar_wait_drain(&ctl.full_a[s], (last_par >> s) & 1u);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
+    pdl_wait();
+    if (lane == 0) {
+      const uint32_t idesc = make_idesc_bf16_f32(kTileM, a.n_pad);
+      int it = 0, seg = 0;
+      bool ok = true;
+      for (int t = t_begin; t < t_end && ok; ++seg) {
+        const int rt = t / KT;
+        const int seg_end = min(t_end, (rt + 1) * KT);
+        const int buf = seg & 1;
+        if (seg >= 2 &&
+            !mbar_wait_bounded(&ctl.acc_empty[buf], static_cast<uint32_t>((seg >> 1) - 1) & 1u,
+                               abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * a.n_pad);
+        for (int tt = t; tt < seg_end; ++tt, ++it) {
+          const int s = it % S;
+          const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
+          if (!mbar_wait_bounded(&ctl.full_a[s], ph, abort_flag, a.status) ||
+              !mbar_wait_bounded(&ctl.full_b[s], ph, abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_addr = smem_addr(smem_a + static_cast<size_t>(s) * kABytes);
+          const uint32_t b_addr = smem_addr(smem_b + static_cast<size_t>(s) * b_bytes);
+#pragma unroll
+          for (int kk = 0; kk < kTileK / 16; ++kk) {
+            tc_mma_bf16(d_tmem, make_smem_desc_sw128(a_addr + kk * 32),
+                        make_smem_desc_sw128(b_addr + kk * 32), idesc,
+                        (tt > t || kk > 0) ? 1u : 0u);
+          }
+          tc_commit(&ctl.empty[s]);
+        }
+        if (!ok) break;
+        tc_commit(&ctl.acc_full[buf]);
+        t = seg_end;
+      }
+      if (!ok) {  // tear-down: wait for every MMA already issued
+        tc_commit(&ctl.drain);
+        mbar_wait_drain(&ctl.drain, 0);
+      }
+    }
+  } else if (warp < 4) {
+    // ------------------------------------------------ activation producers
+    const int tb = threadIdx.x - 64;
+    pdl_wait();
+    if (a.b_mode == B_F32_RMSNORM) {
+      for (int r = tb; r < a.n_pad; r += kNumBThreads) {
+        float val = 0.f;
+        if (r < a.rows_total) {
+          float s = 0.f;
+          for (int i = 0; i < a.ss_count; ++i) s += a.ss[static_cast<size_t>(i) * a.ss_stride + r];
+          val = rsqrtf(s / static_cast<float>(a.k_in) + a.eps);
+        }
+        rms[r] = val;
+      }
+      named_bar_sync(2, kNumBThreads);
+    }
+    int it = 0;
+    for (int t = t_begin; t < t_end; ++t, ++it) {
+      const int rt = t / KT, kt = t - rt * KT;
+      (void)rt;
+      const int s = it % S;
+      const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
+      if (!mbar_wait_bounded(&ctl.empty[s], ph ^ 1u, abort_flag, a.status)) break;
+      uint8_t* bs = smem_b + static_cast<size_t>(s) * b_bytes;
+      for (int ch = tb; ch < a.n_pad * 8; ch += kNumBThreads) {
+        const int row = ch >> 3, kc = ch & 7;
+        const int k = kt * kTileK + kc * 8;
+        uint4 val = make_uint4(0u, 0u, 0u, 0u);
+        if (row < a.rows_total && k < a.k_in) {
+          if (a.b_mode == B_BF16) {
+            val = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(a.b_src) +
+                                                   static_cast<size_t>(row) * a.b_ld + k);
+          } else {
+            const float* src = static_cast<const float*>(a.b_src) + static_cast<size_t>(row) * a.b_ld + k;
+            const float4 x0 = *reinterpret_cast<const float4*>(src);
+            const float4 x1 = *reinterpret_cast<const float4*>(src + 4);
+            const uint4 graw = *reinterpret_cast<const uint4*>(a.gain + k);
+            const __nv_bfloat16* g = reinterpret_cast<const __nv_bfloat16*>(&graw);
+            const float sc = rms[row];
+            float f[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+            for (int q = 0; q < 8; ++q) f[q] = f[q] * sc * __bfloat162float(g[q]);
+            val = pack8_bf16(f);
+          }
+        }
+        *reinterpret_cast<uint4*>(bs + row * 128 + ((kc ^ (row & 7)) << 4)) = val;
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(&ctl.full_b[s]);
+    }
+  } else {
+    // ------------------------------------------------ epilogue (warps 4-7)
+    const int et = threadIdx.x - 128;  // tile feature == TMEM lane
+    const int ew = warp & 3;
+    pdl_wait();
+    int seg = 0;
+    for (int t = t_begin; t < t_end; ++seg) {
+      const int rt = t / KT;
+      const int k0 = t - rt * KT;
+      const int seg_end = min(t_end, (rt + 1) * KT);
+      const int k1 = seg_end - rt * KT;
+      const int buf = seg & 1;
+      int ok = 1;
+      if (lane == 0)
+        ok = mbar_wait_bounded(&ctl.acc_full[buf], static_cast<uint32_t>(seg >> 1) & 1u, abort_flag,
+                               a.status)
+                 ? 1
+                 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);   // the warp proceeds (or stops) together
+      if (!ok) break;
+      tc_fence_after();
+      const bool full = (k0 == 0 && k1 == KT);
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(ew * 32) << 16) +
+                             static_cast<uint32_t>(buf * a.n_pad);
+      float v[16];
+      if (full) {
+        for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
+          tmem_ld_32x32b_x16(tbase + chunk * 16, v);
+          apply_epilogue(a, ctl, stage, rt, chunk, et, v);
+        }
+      } else {
+        const int slot = (seg == 0) ? 0 : 1;
+        float* pb = a.partials + static_cast<size_t>(2 * c + slot) * a.n_pad * kTileM;
+        for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
+          tmem_ld_32x32b_x16(tbase + chunk * 16, v);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) pb[(chunk * 16 + j) * kTileM + et] = v[j];
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.acc_empty[buf]);
+      if (!full) {
+        __threadfence();
+        named_bar_sync(1, 128);
+        const int c_first = sk_cta_of(rt * KT, T, G);
+        const int c_last = sk_cta_of((rt + 1) * KT - 1, T, G);
+        if (et == 0) {
+          const int old = atomicAdd(&a.counters[rt], 1);
+          ctl.reduce_flag = (old == c_last - c_first) ? 1 : 0;
+        }
+        named_bar_sync(1, 128);
+        if (ctl.reduce_flag) {
+          __threadfence();
+          for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) v[j] = 0.f;
+            for (int cc = c_first; cc <= c_last; ++cc) {
+              const int sl = (sk_begin(cc, T, G) >= rt * KT) ? 0 : 1;
+              const float* pp = a.partials + static_cast<size_t>(2 * cc + sl) * a.n_pad * kTileM;
+#pragma unroll
+              for (int j = 0; j < 16; ++j) v[j] += ld_cg_f(pp + (chunk * 16 + j) * kTileM + et);
+            }
+            apply_epilogue(a, ctl, stage, rt, chunk, et, v);
+          }
+          if (et == 0) a.counters[rt] = 0;
+        }
+      }
+      t = seg_end;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, tmem_cols);
+  }
+}
+
+}  // namespace
+
+int gemm_pick_stages(int n_pad) {
+  const int stage = kABytes + n_pad * 128;
+  const int budget = n_pad <= 32 ? 100 * 1024 : 190 * 1024;
+  const int fixed = kTileM * kStagePitch * 4 + kMaxRows * 4 + 1024;
+  int s = (budget - fixed) / stage;
+  if (s > kMaxStages) s = kMaxStages;
+  if (s < 2) s = 2;
+  return s;
+}
+
+size_t gemm_smem_bytes(int n_pad, int stages) {
+  return static_cast<size_t>(stages) * (kABytes + n_pad * 128) + kTileM * kStagePitch * 4 +
+         kMaxRows * 4 + 1024;
+}
+
+cudaError_t gemm_set_max_smem() {
+  return cudaFuncSetAttribute(gemm_stream_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              227 * 1024);
+}
+
+cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s, bool pdl) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, gemm_stream_kernel, a);
+}
+
+}  // namespace memspec

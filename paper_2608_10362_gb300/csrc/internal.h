@@ -1,0 +1,224 @@
+// internal.h - launch-parameter structs shared by the host runtime (api.cu) and
+// the kernels.  Not part of the public ABI.
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace memspec {
+
+typedef __nv_bfloat16 bf16;
+
+constexpr int kMaxGroups = 64;      // requests stepped together
+constexpr int kMaxRows = 256;       // rows of one forward pass (MMA N <= 256)
+constexpr int kPrefillChunk = 128;  // rows per prefill forward
+constexpr int kMaxK = 15;           // largest draft length
+constexpr int kMaxDrafts = 16;
+constexpr int kStateInts = 4;       // per request: L, Lt, step, unused
+
+// Which rows a forward pass processes.  Row r belongs to group g = r / R
+// (a request), index i = r % R; it is valid iff i < valid[g]; its position is
+// pos0[g] + i.  Written by the embedding kernel, read by every later kernel of
+// the same forward pass.
+struct RowPlan {
+  int n_groups;
+  int rows_per_group;  // R
+  int rows_total;      // n_groups * R
+  int max_pos;         // largest valid position of the pass
+  int req[kMaxGroups];
+  int valid[kMaxGroups];
+  int pos0[kMaxGroups];
+};
+
+__host__ __device__ inline bool plan_row_valid(const RowPlan* p, int r) {
+  if (r >= p->rows_total) return false;
+  const int g = r / p->rows_per_group;
+  return (r - g * p->rows_per_group) < p->valid[g];
+}
+
+enum PlanMode : int { PLAN_VERIFY = 0, PLAN_DRAFT_FIRST = 1, PLAN_DRAFT_NEXT = 2, PLAN_PREFILL = 3 };
+
+struct EmbedArgs {
+  int mode;
+  int n_groups;
+  int R;
+  int j;               // draft pass index (1-based) for PLAN_DRAFT_NEXT
+  int prefill_req, prefill_start, prefill_count;
+  const int* seq_state;     // [max_batch][kStateInts]
+  const int* draft_len;     // [max_batch] processed count of the model being run (drafts)
+  const int* tokens;        // [max_batch][max_seq]
+  int max_seq;
+  const int* draft_tokens;  // [max_batch][max_k]
+  int max_k;
+  const bf16* emb;          // [vocab][d]
+  int d, vocab;
+  float* h;                 // [rows][d] residual stream
+  float* ss;                // [ss_tiles][ss_stride]: row sums of squares (partial)
+  int ss_stride;
+  RowPlan* plan;
+  uint32_t* status;
+};
+
+enum GemmBMode : int { B_BF16 = 0, B_F32_RMSNORM = 1 };
+enum GemmEpi : int { EPI_F32 = 0, EPI_RESIDUAL = 1, EPI_SWIGLU = 2, EPI_QKV = 3 };
+enum L2Hint : int { L2_EVICT_FIRST = 0, L2_EVICT_NORMAL = 1, L2_EVICT_LAST = 2 };
+
+struct GemmArgs {
+  CUtensorMap map_a;        // weights [n_out][k] bf16, box {64, 128} (or {64, 64} for pairs)
+  CUtensorMap map_a2;       // second matrix of a SwiGLU pair (up), box {64, 64}
+  int n_out;                // output features (F for pairs)
+  int k_in;
+  int pair;                 // 1: tile = 64 rows of map_a + 64 rows of map_a2
+  int rows_total;           // rows of B (activations)
+  int n_pad;                // MMA N: rows_total rounded up to 16
+  int row_tiles, k_tiles, stages;
+  int l2_hint;
+  // B operand source
+  int b_mode;
+  const void* b_src;        // bf16 [rows][b_ld] or fp32 [rows][b_ld]
+  int b_ld;
+  const bf16* gain;         // RMSNorm gain [k_in] (B_F32_RMSNORM)
+  const float* ss;          // [ss_count][ss_stride]
+  int ss_count, ss_stride;
+  float eps;
+  // split-K scratch
+  float* partials;          // [2 * grid][n_pad * 128]
+  int* counters;            // [row_tiles], zero on entry, left zero
+  // epilogue
+  int epi;
+  float* out;               // EPI_F32
+  int out_ld;
+  int last_only;            // EPI_F32: only the last valid row of each group
+  long long out_group_stride;
+  float* h;                 // EPI_RESIDUAL: residual [rows][h_ld], updated in place
+  int h_ld;
+  float* ss_out;            // EPI_RESIDUAL: [row_tiles][ss_stride]
+  bf16* act;                // EPI_SWIGLU: [rows][act_ld]
+  int act_ld;
+  float* q_out;             // EPI_QKV: fp32 [rows][q_dim]
+  int q_dim, kv_dim, head_dim, n_kv_heads, max_seq;
+  bf16* kcache;             // [req][kv_head][max_seq][hd] for this layer
+  bf16* vcache;
+  const float* rope_cos;    // [max_seq][hd/2]
+  const float* rope_sin;
+  const RowPlan* plan;      // nullptr: rows < rows_total are valid, no positions
+  uint32_t* status;
+};
+
+struct AttnArgs {
+  const float* q;           // [rows][H][hd] fp32, rotated
+  const bf16* kcache;       // [req][Hkv][max_seq][hd]
+  const bf16* vcache;
+  int H, Hkv, hd, max_seq;
+  int rows_per_block;       // query rows (positions) per CTA
+  int row_blocks;           // blocks per group
+  int chunk;                // keys per split
+  int n_splits;             // gridDim.x
+  float scale_log2;         // log2(e) / sqrt(hd)
+  float* part_o;            // [groups][Hkv][row_blocks][n_splits][qmax][hd]
+  float* part_ml;           // [groups][Hkv][row_blocks][n_splits][qmax][2]
+  int qmax;                 // group_size * rows_per_block
+  int* counters;            // [groups][Hkv][row_blocks]
+  bf16* out;                // [rows][H][hd]
+  const RowPlan* plan;
+  uint32_t* status;
+};
+
+struct SampleArgs {         // draft sampling of pass j
+  const float* logits;      // [groups][row_stride] (row for this pass)
+  long long row_stride;
+  int vocab;
+  int n_groups;
+  float inv_temp;           // 0: greedy
+  int greedy;
+  int slot;                 // Philox slot (j-1)
+  const int* seq_state;     // for Philox step; nullptr for explicit uniforms
+  const unsigned long long* seeds;
+  const float* u_explicit;  // [groups] (op-level entry)
+  int* out_tok;             // [groups] at stride out_stride
+  int out_stride;
+  float* part;              // [groups][chunks][4] scratch
+  int* counters;            // [groups]
+  int chunks;               // CTAs per group (gridDim.x)
+  uint32_t* status;
+};
+
+struct AcceptArgs {
+  const float* zt;          // [groups][K+1][vocab]
+  const float* zd;          // [groups][K][vocab]
+  const int* draft_tokens;  // [groups][max_k]
+  int max_k;
+  int K, vocab, n_groups;
+  float inv_temp;
+  int greedy;
+  int chunks;               // CTAs per row
+  float* part;              // [groups][2K+1][chunks][4]
+  int* counters;            // [groups]
+  int* seq_state;           // [max_batch][kStateInts]
+  const unsigned long long* seeds;
+  int* draft_len;           // [max_batch] Ld of the active draft
+  int* tokens;              // [max_batch][max_seq]
+  int max_seq;
+  int* results;             // [groups][K+2]
+  float* debug;             // [groups][2K+2]
+  uint32_t* status;
+};
+
+// launchers (each returns the launch's cudaError_t)
+cudaError_t launch_embed(const EmbedArgs& a, int rows, cudaStream_t s, bool pdl);
+cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s, bool pdl);
+size_t gemm_smem_bytes(int n_pad, int stages);
+int gemm_pick_stages(int n_pad);
+cudaError_t gemm_set_max_smem();
+cudaError_t launch_attention(const AttnArgs& a, int n_groups, cudaStream_t s, bool pdl);
+size_t attention_smem_bytes(const AttnArgs& a);
+cudaError_t attention_set_max_smem();
+cudaError_t launch_sample(const SampleArgs& a, cudaStream_t s, bool pdl);
+cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t s, bool pdl);
+cudaError_t launch_rope_table(float* cos_t, float* sin_t, int max_seq, int half, float base,
+                              cudaStream_t s);
+
+// Philox4x32-10 (Salmon et al., SC'11), device side.
+__host__ __device__ inline uint32_t philox_u01_bits(uint32_t c0, uint32_t c1, uint32_t c2,
+                                                    uint32_t c3, uint32_t k0, uint32_t k1) {
+  const uint32_t M0 = 0xD2511F53u, M1 = 0xCD9E8D57u, W0 = 0x9E3779B9u, W1 = 0xBB67AE85u;
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r > 0) {
+      k0 += W0;
+      k1 += W1;
+    }
+    const uint64_t p0 = static_cast<uint64_t>(M0) * c0;
+    const uint64_t p1 = static_cast<uint64_t>(M1) * c2;
+    const uint32_t hi0 = static_cast<uint32_t>(p0 >> 32), lo0 = static_cast<uint32_t>(p0);
+    const uint32_t hi1 = static_cast<uint32_t>(p1 >> 32), lo1 = static_cast<uint32_t>(p1);
+    const uint32_t n0 = hi1 ^ c1 ^ k0, n2 = hi0 ^ c3 ^ k1;
+    c0 = n0;
+    c1 = lo1;
+    c2 = n2;
+    c3 = lo0;
+  }
+  return c0;
+}
+
+// Uniform for (seed, request, step, slot): odd multiple of 2^-24 in (0, 1).
+__host__ __device__ inline float philox_uniform(unsigned long long seed, int req, int step,
+                                                int slot) {
+  const uint32_t w = philox_u01_bits(static_cast<uint32_t>(req), static_cast<uint32_t>(step), 0u,
+                                     static_cast<uint32_t>(slot),
+                                     static_cast<uint32_t>(seed & 0xFFFFFFFFull),
+                                     static_cast<uint32_t>(seed >> 32));
+  return static_cast<float>(2u * (w >> 9) + 1u) * (1.0f / 16777216.0f);
+}
+
+// Stream-K schedule: CTA c of G processes global tiles [begin(c), begin(c+1)).
+__host__ __device__ inline int sk_begin(int c, int T, int G) {
+  return static_cast<int>((static_cast<long long>(c) * T) / G);
+}
+// The CTA whose range contains tile t.
+__host__ __device__ inline int sk_cta_of(int t, int T, int G) {
+  return static_cast<int>(((static_cast<long long>(t) + 1) * G + T - 1) / T) - 1;
+}
+
+}  // namespace memspec

@@ -1,0 +1,77 @@
+"""End-to-end parity of the draft-then-verify step on the GPU against the oracle,
+in lock step (tests/lockstep.py), on the tiny pair and on the edge-class pair."""
+import numpy as np
+import pytest
+
+from lockstep import LockstepReport, check_step
+from oracle.llama import LlamaOracle
+from oracle.speculative import SpecDecoder
+from seeded_inputs import SHAPES, gen_prompt, gen_weights
+
+pytestmark = pytest.mark.gpu
+
+
+def _run_lockstep(eng, target_o, draft_o, prompt, K, T, seed, steps, use_graphs_note=""):
+    eng.prefill(0, prompt, seed=seed)
+    sd = SpecDecoder(target_o, draft_o, prompt, len(prompt) + steps * (K + 1) + 4)
+    rep = LockstepReport()
+    for step in range(steps):
+        eng.step(K, T, eng.results_host)
+        check_step(eng, sd, K, T, seed, step, rep)
+    return rep, sd
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    from paper_2608_10362_gb300 import Engine
+    t, d = SHAPES["tiny_target"], SHAPES["tiny_draft"]
+    wt, wd = gen_weights(t, 0), gen_weights(d, 1)
+    engines = {}
+    for graphs in (False, True):
+        eng = Engine(t, wt, max_batch=1, max_seq=512, max_k=8, max_drafts=1, draft_shape_max=d,
+                     draft_budget_bytes=32 << 20, use_graphs=graphs)
+        eng.register_draft(0, d, wd)
+        eng.load_draft_async(0)
+        eng.set_active_draft(0)
+        engines[graphs] = eng
+    yield engines, LlamaOracle(t, wt), LlamaOracle(d, wd)
+    for e in engines.values():
+        e.close()
+
+
+@pytest.mark.parametrize("graphs", [False, True])
+@pytest.mark.parametrize("T", [0.0, 1.0])
+def test_tiny_pair_lockstep(tiny, T, graphs):
+    engines, to, do = tiny
+    eng = engines[graphs]
+    prompt = gen_prompt(7, 128, 2048)
+    rep, sd = _run_lockstep(eng, to, do, prompt, 4, T, seed=3, steps=16)
+    print(f"tiny T={T} graphs={graphs}: steps {rep.steps} tokens {rep.tokens_committed} "
+          f"flags {rep.flags}/{rep.decisions} max logit err {rep.max_logit_err_frac:.2e}")
+    assert rep.flags <= max(1, rep.decisions // 20)
+    assert list(eng.committed_tokens(0)) == sd.tokens
+
+
+def test_tiny_greedy_stream_equals_oracle_target_greedy(tiny):
+    """Greedy speculative output == greedy target-only output (token-identical)."""
+    from oracle.speculative import greedy_generate
+    engines, to, do = tiny
+    eng = engines[True]
+    prompt = gen_prompt(8, 128, 2048)
+    eng.prefill(0, prompt, seed=0)
+    while int(eng.seq_state()[0, 0]) < len(prompt) + 40:
+        eng.step(4, 0.0, eng.results_host)
+        assert eng.sync() == 0
+    got = list(eng.committed_tokens(0)[len(prompt):len(prompt) + 40])
+    assert got == greedy_generate(to, prompt, 40)
+
+
+def test_tiny_prompt_edge_cases(tiny):
+    """Prompt of one token (nothing to prefill) and a prompt crossing the
+    128-row prefill chunk boundary by one."""
+    engines, to, do = tiny
+    eng = engines[False]
+    for n in (1, 129):
+        prompt = gen_prompt(9 + n, n, 2048)
+        rep, sd = _run_lockstep(eng, to, do, prompt, 3, 1.0, seed=5, steps=4)
+        assert rep.steps == 4
