@@ -77,11 +77,21 @@ int sm_count() {
   return n;
 }
 
+std::string g_attr_error;
+
 bool ensure_func_attrs() {
   static bool done = false;
   if (done) return true;
-  if (gemm_set_max_smem() != cudaSuccess) return false;
-  if (attention_set_max_smem() != cudaSuccess) return false;
+  cudaError_t e = gemm_set_max_smem();
+  if (e != cudaSuccess) {
+    g_attr_error = std::string("gemm smem attribute: ") + cudaGetErrorString(e);
+    return false;
+  }
+  e = attention_set_max_smem();
+  if (e != cudaSuccess) {
+    g_attr_error = std::string("attention smem attribute: ") + cudaGetErrorString(e);
+    return false;
+  }
   done = true;
   return true;
 }
@@ -166,13 +176,12 @@ size_t kv_bytes(const memspec_model_cfg& c, int max_batch, int max_seq) {
 // ---------------------------------------------------------------- attention launch geometry
 struct AttnGeo {
   int rows_per_block, row_blocks, n_splits, chunk, qmax;
-  size_t part_floats() const { return 0; }
 };
 
 AttnGeo attn_geometry(const memspec_model_cfg& c, int groups, int R, int max_seq) {
   AttnGeo g;
   const int gs = c.n_heads / c.n_kv_heads;
-  const int qlimit = c.head_dim == 128 ? 64 : 128;
+  const int qlimit = 64;   // query vectors per CTA (4 m-tiles of 16)
   int rpb = std::max(1, qlimit / gs);
   rpb = std::min(rpb, R);
   g.rows_per_block = rpb;
@@ -259,6 +268,7 @@ struct memspec_ctx {
   std::string err;
   // workspace
   float* h = nullptr;
+  bf16* xg = nullptr;
   float* ss = nullptr;
   int ss_stride = kMaxRows;
   float* q = nullptr;
@@ -296,6 +306,7 @@ struct memspec_ctx {
   int batch = 1;
   int last_K = 0;
   std::map<GraphKey, cudaGraphExec_t> graphs;
+  std::map<std::tuple<const void*, int, int, int>, CUtensorMap> bmaps;
 };
 
 namespace {
@@ -355,6 +366,7 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
                                ceil_div(dmax, 128)});
   WsPlan w;
   const size_t o_h = w.take(static_cast<size_t>(kMaxRows) * dmax * 4);
+  const size_t o_xg = w.take(static_cast<size_t>(kMaxRows) * dmax * 2);
   const size_t o_ss = w.take(static_cast<size_t>(ceil_div(dmax, 128)) * kMaxRows * 4);
   const size_t o_q = w.take(static_cast<size_t>(kMaxRows) * qmax_dim * 4);
   const size_t o_o = w.take(static_cast<size_t>(kMaxRows) * qmax_dim * 2);
@@ -384,6 +396,7 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   const size_t o_rs128 = w.take(static_cast<size_t>(p->max_seq) * 64 * 4);
   if (c != nullptr) {
     c->h = reinterpret_cast<float*>(base + o_h);
+    c->xg = reinterpret_cast<bf16*>(base + o_xg);
     c->ss = reinterpret_cast<float*>(base + o_ss);
     c->q = reinterpret_cast<float*>(base + o_q);
     c->o = reinterpret_cast<bf16*>(base + o_o);
@@ -455,6 +468,20 @@ memspec_status validate_params(const memspec_init_params* p, std::string* why) {
   return MEMSPEC_OK;
 }
 
+// Tensor map over a bf16 activation buffer [rows][cols] with box {64, n_pad}:
+// rows >= `rows` read as zero.  Cached per (buffer, rows, cols, n_pad).
+bool act_map(memspec_ctx* c, const void* ptr, int rows, int cols, int n_pad, CUtensorMap* out) {
+  auto key = std::make_tuple(ptr, rows, cols, n_pad);
+  auto it = c->bmaps.find(key);
+  if (it == c->bmaps.end()) {
+    CUtensorMap m;
+    if (!encode_map(&m, ptr, rows, cols, n_pad)) return false;
+    it = c->bmaps.emplace(key, m).first;
+  }
+  *out = it->second;
+  return true;
+}
+
 // ---------------------------------------------------------------- forward pass
 struct FwdSpec {
   int mode, n_groups, R, j;
@@ -501,6 +528,8 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
   ea.d = d;
   ea.vocab = cf.vocab;
   ea.h = c->h;
+  ea.xg = c->xg;
+  ea.gain = reinterpret_cast<const bf16*>(m.w + m.lay.attn_norm[0]);
   ea.ss = c->ss;
   ea.ss_stride = c->ss_stride;
   ea.plan = c->plan;
@@ -528,10 +557,9 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.row_tiles = ceil_div(a.n_out, 128);
       a.k_tiles = ceil_div(d, 64);
       a.l2_hint = m.l2_hint;
-      a.b_mode = B_F32_RMSNORM;
-      a.b_src = c->h;
-      a.b_ld = d;
-      a.gain = reinterpret_cast<const bf16*>(m.w + m.lay.attn_norm[l]);
+      if (!act_map(c, c->xg, rows, d, n_pad, &a.map_b))
+        return fail(c, MEMSPEC_ERR_CUDA, "activation tensor map");
+      a.rms = 1;
       a.ss = c->ss;
       a.ss_count = ss_count;
       a.ss_stride = c->ss_stride;
@@ -585,13 +613,14 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.row_tiles = ceil_div(d, 128);
       a.k_tiles = ceil_div(qd, 64);
       a.l2_hint = m.l2_hint;
-      a.b_mode = B_BF16;
-      a.b_src = c->o;
-      a.b_ld = qd;
+      if (!act_map(c, c->o, rows, qd, n_pad, &a.map_b))
+        return fail(c, MEMSPEC_ERR_CUDA, "activation tensor map");
       a.epi = EPI_RESIDUAL;
       a.h = c->h;
       a.h_ld = d;
       a.ss_out = c->ss;
+      a.gain_next = reinterpret_cast<const bf16*>(m.w + m.lay.ffn_norm[l]);
+      a.xg_out = c->xg;
       a.ss_stride = c->ss_stride;
       a.plan = c->plan;
       memspec_status s = run_gemm(c, a, "o gemm launch");
@@ -610,10 +639,9 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.row_tiles = ceil_div(F, 64);
       a.k_tiles = ceil_div(d, 64);
       a.l2_hint = m.l2_hint;
-      a.b_mode = B_F32_RMSNORM;
-      a.b_src = c->h;
-      a.b_ld = d;
-      a.gain = reinterpret_cast<const bf16*>(m.w + m.lay.ffn_norm[l]);
+      if (!act_map(c, c->xg, rows, d, n_pad, &a.map_b))
+        return fail(c, MEMSPEC_ERR_CUDA, "activation tensor map");
+      a.rms = 1;
       a.ss = c->ss;
       a.ss_count = ss_count;
       a.ss_stride = c->ss_stride;
@@ -635,13 +663,15 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.row_tiles = ceil_div(d, 128);
       a.k_tiles = ceil_div(F, 64);
       a.l2_hint = m.l2_hint;
-      a.b_mode = B_BF16;
-      a.b_src = c->act;
-      a.b_ld = F;
+      if (!act_map(c, c->act, rows, F, n_pad, &a.map_b))
+        return fail(c, MEMSPEC_ERR_CUDA, "activation tensor map");
       a.epi = EPI_RESIDUAL;
       a.h = c->h;
       a.h_ld = d;
       a.ss_out = c->ss;
+      a.gain_next = reinterpret_cast<const bf16*>(
+          m.w + (l + 1 < cf.n_layers ? m.lay.attn_norm[l + 1] : m.lay.final_norm));
+      a.xg_out = c->xg;
       a.ss_stride = c->ss_stride;
       a.plan = c->plan;
       memspec_status s = run_gemm(c, a, "down gemm launch");
@@ -658,10 +688,9 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
     a.row_tiles = ceil_div(cf.vocab, 128);
     a.k_tiles = ceil_div(d, 64);
     a.l2_hint = m.l2_hint;
-    a.b_mode = B_F32_RMSNORM;
-    a.b_src = c->h;
-    a.b_ld = d;
-    a.gain = reinterpret_cast<const bf16*>(m.w + m.lay.final_norm);
+    if (!act_map(c, c->xg, rows, d, n_pad, &a.map_b))
+      return fail(c, MEMSPEC_ERR_CUDA, "activation tensor map");
+    a.rms = 1;
     a.ss = c->ss;
     a.ss_count = ss_count;
     a.ss_stride = c->ss_stride;
@@ -839,7 +868,7 @@ memspec_status memspec_init(const memspec_init_params* p, void* workspace_dev, m
   c->side = p->stream_side ? static_cast<cudaStream_t>(p->stream_side) : c->main;
   c->ws_bytes = layout_workspace(p, c, static_cast<uint8_t*>(workspace_dev));
   if (!ensure_func_attrs()) {
-    g_op_error = "cudaFuncSetAttribute failed";
+    g_op_error = g_attr_error;
     delete c;
     return MEMSPEC_ERR_CUDA;
   }
@@ -1325,7 +1354,7 @@ memspec_status memspec_op_linear(const void* x, const void* w, float* y, int32_t
     return MEMSPEC_ERR_INVALID_ARG;
   }
   if (!ensure_func_attrs()) {
-    g_op_error = "cudaFuncSetAttribute failed";
+    g_op_error = g_attr_error;
     return MEMSPEC_ERR_CUDA;
   }
   GemmArgs a{};
@@ -1342,9 +1371,10 @@ memspec_status memspec_op_linear(const void* x, const void* w, float* y, int32_t
   a.k_tiles = ceil_div(k, 64);
   a.stages = gemm_pick_stages(n_pad);
   a.l2_hint = L2_EVICT_FIRST;
-  a.b_mode = B_BF16;
-  a.b_src = x;
-  a.b_ld = k;
+  if (!encode_map(&a.map_b, x, rows, k, n_pad)) {
+    g_op_error = "cuTensorMapEncodeTiled failed for x";
+    return MEMSPEC_ERR_CUDA;
+  }
   a.epi = EPI_F32;
   a.out = y;
   a.out_ld = n_out;

@@ -3,13 +3,18 @@
 // against that request's KV cache.
 //
 // Grid: (key split, kv_head x row_block, request group).  A CTA takes the query
-// vectors of one KV head's group of query heads for a block of rows, streams its
-// chunk of keys/values once, keeps an online softmax (running max m, sum l,
-// unnormalised o) and writes (m, l, o) to a partial buffer.  The last-arriving
-// split CTA of each (group, kv head, row block) combines the partials in split
-// order (deterministic, no float atomics): o = sum_s e^(m_s - M) o_s /
-// sum_s e^(m_s - M) l_s with M = max_s m_s.  Query row i of a group sits at
-// position pos0 + i and sees keys 0..pos0+i.
+// vectors of one KV head's group of query heads for a block of rows (at most 64
+// vectors, 16 per m-tile), streams its chunk of keys/values once through a
+// 3-stage cp.async pipeline into XOR-swizzled shared memory, and computes on
+// tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate):
+//   S = Q K^T (Q pre-scaled by log2(e)/sqrt(hd)), online softmax in registers
+//   (running max m, sum l), O += P V with P re-packed from the S fragments.
+// With few query vectors the four warps split each 64-key tile between them
+// and are merged at the end.  Each split writes (m, l, o) to a partial buffer;
+// the last-arriving split CTA of each (group, kv head, row block) combines them
+// in split order (deterministic, no float atomics):
+//   o = sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s.
+// Query row i of a group sits at position pos0 + i and sees keys 0..pos0+i.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -17,35 +22,61 @@ namespace memspec {
 
 namespace {
 
-constexpr int kAttThreads = 256;
+constexpr int kAttThreads = 128;
 constexpr int kKeyTile = 64;
+constexpr int kStages = 3;
+constexpr int kMaxQ = 64;   // query vectors per CTA (4 m-tiles of 16)
 
-__device__ __forceinline__ float dot8(const float* q, const uint4& raw) {
-  const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&raw);
-  float s = 0.f;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float2 f = __bfloat1622float2(b[i]);
-    s = fmaf(q[2 * i], f.x, s);
-    s = fmaf(q[2 * i + 1], f.y, s);
-  }
-  return s;
-}
-
-__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(smem_dst)), "l"(gsrc)
+__device__ __forceinline__ void cp_async16_zfill(void* smem_dst, const void* gsrc, bool valid) {
+  const int n = valid ? 16 : 0;
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(smem_dst)),
+               "l"(gsrc), "r"(n)
                : "memory");
 }
-__device__ __forceinline__ void cp_async_wait_all() {
-  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 t = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&t);
+}
+
+// byte offset of 16-byte chunk `ch` of row `row` in a swizzled [rows][HD] bf16 tile
+template <int HD>
+__device__ __forceinline__ uint32_t swz(int row, int ch) {
+  return static_cast<uint32_t>(row * (HD * 2) + ((ch ^ (row & 7)) << 4));
 }
 
 template <int HD>
 __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant__ AttnArgs a) {
-  constexpr int kNvg = kAttThreads / HD;       // PV thread groups
-  constexpr int kAcc = 32;                     // max query vectors per PV thread
-  constexpr int kSv = 32;                      // max query vectors per score thread
-  extern __shared__ __align__(16) uint8_t smem_raw[];
+  constexpr int kChunks = HD / 8;                        // 16-byte chunks per row
+  constexpr int kTileBytes = kKeyTile * HD * 2;          // one K (or V) tile
+  constexpr int kNT = HD / 8;                            // n8 tiles of the output
+  extern __shared__ __align__(128) uint8_t smem_raw[];
   pdl_launch_dependents();
   pdl_wait();
 
@@ -63,7 +94,7 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
   const int gs = a.H / a.Hkv;
   const int nq = gs * nr;
   const int kmax = pos0 + r_hi - 1;
-  if (pos0 < 0 || kmax >= a.max_seq) {   // out-of-range positions are reported, never read
+  if (pos0 < 0 || kmax >= a.max_seq || nq > kMaxQ) {   // reported, never read
     if (threadIdx.x == 0 && split == 0) atomicOr(a.status, 0x4u);
     return;
   }
@@ -71,128 +102,209 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
   if (split >= n_active) return;
   const int k0 = split * a.chunk;
   const int k1 = min(k0 + a.chunk, kmax + 1);
+  const int n_tiles = (k1 - k0 + kKeyTile - 1) / kKeyTile;
 
-  float* qs = reinterpret_cast<float*>(smem_raw);                  // [qmax][HD]
-  float* sp = qs + a.qmax * HD;                                    // [qmax][kKeyTile]
-  float* m_s = sp + a.qmax * kKeyTile;                             // [qmax]
-  float* l_s = m_s + a.qmax;
-  float* al_s = l_s + a.qmax;
-  bf16* vs = reinterpret_cast<bf16*>(al_s + a.qmax + (4 - (3 * a.qmax) % 4) % 4);  // [kKeyTile][HD]
+  const int n_mt = (nq + 15) >> 4;
+  const int kg = n_mt == 1 ? 4 : (n_mt == 2 ? 2 : 1);    // warps per m-tile (key groups)
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int mt = warp / kg, kgi = warp - mt * kg;
+  const bool active = mt < n_mt;
 
-  const int tid = threadIdx.x;
-  for (int idx = tid; idx < nq * HD; idx += kAttThreads) {
-    const int v = idx / HD, d = idx - v * HD;
-    const int hl = v / nr, rr = v - hl * nr;
-    const int row = g * R + r_lo + rr;
-    const int h = kvh * gs + hl;
-    qs[idx] = a.q[(static_cast<size_t>(row) * a.H + h) * HD + d] * a.scale_log2;
-  }
-  for (int v = tid; v < nq; v += kAttThreads) {
-    m_s[v] = -INFINITY;
-    l_s[v] = 0.f;
-  }
+  uint8_t* qs = smem_raw;                                 // [64][HD] bf16, swizzled
+  uint8_t* kv = smem_raw + kMaxQ * HD * 2;                // kStages x (K tile, V tile)
   const size_t kv_base = (static_cast<size_t>(req) * a.Hkv + kvh) * a.max_seq;
   const bf16* kc = a.kcache + kv_base * HD;
   const bf16* vc = a.vcache + kv_base * HD;
 
-  const int pd = tid % HD, pvg = tid / HD;     // PV mapping
-  float acc[kAcc];
+  auto load_tile = [&](int t) {
+    uint8_t* ks = kv + (t % kStages) * 2 * kTileBytes;
+    uint8_t* vs = ks + kTileBytes;
+    const int kt0 = k0 + t * kKeyTile;
+    for (int c = tid; c < kKeyTile * kChunks; c += kAttThreads) {
+      const int row = c / kChunks, ch = c - row * kChunks;
+      const bool ok = kt0 + row < k1;
+      const size_t off = ok ? static_cast<size_t>(kt0 + row) * HD + ch * 8 : 0;
+      cp_async16_zfill(ks + swz<HD>(row, ch), kc + off, ok);
+      cp_async16_zfill(vs + swz<HD>(row, ch), vc + off, ok);
+    }
+  };
+
+  // prologue: start the first kStages-1 tiles, then stage Q (fp32 -> bf16, scaled)
+  for (int s = 0; s < kStages - 1; ++s) {
+    if (s < n_tiles) load_tile(s);
+    cp_async_commit();
+  }
+  for (int c = tid; c < kMaxQ * kChunks; c += kAttThreads) {
+    const int v = c / kChunks, ch = c - v * kChunks;
+    __nv_bfloat16 e[8];
+    if (v < nq) {
+      const int hl = v / nr, rr = v - hl * nr;
+      const int row = g * R + r_lo + rr;
+      const int h = kvh * gs + hl;
+      const float* src = a.q + (static_cast<size_t>(row) * a.H + h) * HD + ch * 8;
+      const float4 x0 = *reinterpret_cast<const float4*>(src);
+      const float4 x1 = *reinterpret_cast<const float4*>(src + 4);
+      const float f[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
 #pragma unroll
-  for (int i = 0; i < kAcc; ++i) acc[i] = 0.f;
-  const int sj = tid % kKeyTile, svv = tid / kKeyTile;   // score mapping (4 groups)
+      for (int i = 0; i < 8; ++i) e[i] = __float2bfloat16_rn(f[i] * a.scale_log2);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) e[i] = __float2bfloat16_rn(0.f);
+    }
+    *reinterpret_cast<uint4*>(qs + swz<HD>(v, ch)) = *reinterpret_cast<const uint4*>(e);
+  }
   __syncthreads();
 
-  for (int kt0 = k0; kt0 < k1; kt0 += kKeyTile) {
-    const int nk = min(kKeyTile, k1 - kt0);
-    // V tile -> shared memory (async, overlaps the score computation)
-    for (int c = tid; c < nk * (HD / 8); c += kAttThreads) {
-      const int j = c / (HD / 8), cc = c - j * (HD / 8);
-      cp_async16(vs + j * HD + cc * 8, vc + static_cast<size_t>(kt0 + j) * HD + cc * 8);
+  // Q fragments of this warp's m-tile stay in registers
+  uint32_t qa[HD / 16][4];
+  if (active) {
+#pragma unroll
+    for (int ks = 0; ks < HD / 16; ++ks) {
+      const int row = mt * 16 + (lane & 15);
+      const int ch = ks * 2 + (lane >> 4);
+      ldsm_x4(smem_addr(qs) + swz<HD>(row, ch), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
     }
-    // scores: thread (key sj, query vectors svv, svv+4, ...)
-    {
-      float s[kSv];
-#pragma unroll
-      for (int i = 0; i < kSv; ++i) s[i] = 0.f;
-      if (sj < nk) {
-        const bf16* krow = kc + static_cast<size_t>(kt0 + sj) * HD;
-#pragma unroll 4
-        for (int dc = 0; dc < HD / 8; ++dc) {
-          const uint4 raw = __ldg(reinterpret_cast<const uint4*>(krow) + dc);
-#pragma unroll
-          for (int i = 0; i < kSv; ++i) {
-            const int v = svv + 4 * i;
-            if (v < nq) s[i] += dot8(qs + v * HD + dc * 8, raw);
-          }
-        }
-      }
-#pragma unroll
-      for (int i = 0; i < kSv; ++i) {
-        const int v = svv + 4 * i;
-        if (v < nq) {
-          const int rr = v % nr;
-          const int pos = pos0 + r_lo + rr;
-          const int key = kt0 + sj;
-          sp[v * kKeyTile + sj] = (sj < nk && key <= pos) ? s[i] : -INFINITY;
-        }
-      }
-    }
-    __syncthreads();
-    // online softmax update, one warp per query vector
-    {
-      const int w = tid >> 5, lane = tid & 31;
-      for (int v = w; v < nq; v += kAttThreads / 32) {
-        const float x0 = sp[v * kKeyTile + lane], x1 = sp[v * kKeyTile + lane + 32];
-        float mx = fmaxf(x0, x1);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        const float m_old = m_s[v];
-        const float m_new = fmaxf(m_old, mx);
-        float p0 = 0.f, p1 = 0.f, alpha = 1.f;
-        if (m_new != -INFINITY) {
-          p0 = exp2f(x0 - m_new);
-          p1 = exp2f(x1 - m_new);
-          alpha = exp2f(m_old - m_new);
-        }
-        sp[v * kKeyTile + lane] = p0;
-        sp[v * kKeyTile + lane + 32] = p1;
-        float sum = p0 + p1;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-        if (lane == 0) {
-          l_s[v] = l_s[v] * alpha + sum;
-          m_s[v] = m_new;
-          al_s[v] = alpha;
-        }
-      }
-    }
-    cp_async_wait_all();
-    __syncthreads();
-    // o += p V
-#pragma unroll
-    for (int i = 0; i < kAcc; ++i) {
-      const int v = pvg + kNvg * i;
-      if (v < nq) {
-        float o = acc[i] * al_s[v];
-        const float* pr = sp + v * kKeyTile;
-        for (int j = 0; j < nk; ++j) o = fmaf(pr[j], __bfloat162float(vs[j * HD + pd]), o);
-        acc[i] = o;
-      }
-    }
-    __syncthreads();
   }
+  // positions of this thread's two rows (v = mt*16 + lane/4 and +8); -1: padding row
+  int prow[2];
+#pragma unroll
+  for (int h2 = 0; h2 < 2; ++h2) {
+    const int v = mt * 16 + (lane >> 2) + 8 * h2;
+    prow[h2] = (active && v < nq) ? pos0 + r_lo + (v % nr) : -1;
+  }
+  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  float o[kNT][4];
+#pragma unroll
+  for (int i = 0; i < kNT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
 
-  // partials -> global
+  const int sub_per_warp = (kKeyTile / 16) / kg;          // 16-key sub-blocks per warp per tile
+  for (int t = 0; t < n_tiles; ++t) {
+    cp_async_wait<kStages - 2>();
+    __syncthreads();
+    if (t + kStages - 1 < n_tiles) load_tile(t + kStages - 1);
+    cp_async_commit();
+    if (!active) continue;
+    const uint32_t ks_addr = smem_addr(kv + (t % kStages) * 2 * kTileBytes);
+    const uint32_t vs_addr = ks_addr + kTileBytes;
+    const int kt0 = k0 + t * kKeyTile;
+    for (int sb = 0; sb < sub_per_warp; ++sb) {
+      const int kb = (kgi * sub_per_warp + sb) * 16;      // key offset within the tile
+      float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int ks = 0; ks < HD / 16; ++ks) {
+        uint32_t b0, b1, b2, b3;
+        const int row = kb + (lane & 7) + ((lane >> 4) << 3);
+        const int ch = ks * 2 + ((lane >> 3) & 1);
+        ldsm_x4(ks_addr + swz<HD>(row, ch), b0, b1, b2, b3);
+        mma16816(s0, qa[ks], b0, b1);
+        mma16816(s1, qa[ks], b2, b3);
+      }
+      // causal / range mask, then online softmax (base 2)
+      const int key_c = kt0 + kb + ((lane & 3) << 1);
+      float mx[2];
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const int p = prow[h2];
+        const int lim = min(p, k1 - 1);
+        float* a0 = s0 + 2 * h2;
+        float* a1 = s1 + 2 * h2;
+        a0[0] = (key_c <= lim) ? a0[0] : -INFINITY;
+        a0[1] = (key_c + 1 <= lim) ? a0[1] : -INFINITY;
+        a1[0] = (key_c + 8 <= lim) ? a1[0] : -INFINITY;
+        a1[1] = (key_c + 9 <= lim) ? a1[1] : -INFINITY;
+        mx[h2] = fmaxf(fmaxf(a0[0], a0[1]), fmaxf(a1[0], a1[1]));
+        mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 1));
+        mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 2));
+      }
+      float scale[2];
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const float m_new = fmaxf(m_run[h2], mx[h2]);
+        float* a0 = s0 + 2 * h2;
+        float* a1 = s1 + 2 * h2;
+        if (m_new == -INFINITY) {
+          scale[h2] = 1.f;
+          a0[0] = a0[1] = a1[0] = a1[1] = 0.f;
+        } else {
+          scale[h2] = exp2f(m_run[h2] - m_new);
+          a0[0] = exp2f(a0[0] - m_new);
+          a0[1] = exp2f(a0[1] - m_new);
+          a1[0] = exp2f(a1[0] - m_new);
+          a1[1] = exp2f(a1[1] - m_new);
+        }
+        float rs = (a0[0] + a0[1]) + (a1[0] + a1[1]);
+        rs += __shfl_xor_sync(0xffffffffu, rs, 1);
+        rs += __shfl_xor_sync(0xffffffffu, rs, 2);
+        l_run[h2] = l_run[h2] * scale[h2] + rs;
+        m_run[h2] = m_new;
+      }
+#pragma unroll
+      for (int i = 0; i < kNT; ++i) {
+        o[i][0] *= scale[0];
+        o[i][1] *= scale[0];
+        o[i][2] *= scale[1];
+        o[i][3] *= scale[1];
+      }
+      uint32_t pa[4];
+      pa[0] = pack_bf16x2(s0[0], s0[1]);
+      pa[1] = pack_bf16x2(s0[2], s0[3]);
+      pa[2] = pack_bf16x2(s1[0], s1[1]);
+      pa[3] = pack_bf16x2(s1[2], s1[3]);
+#pragma unroll
+      for (int n2 = 0; n2 < HD / 16; ++n2) {
+        uint32_t b0, b1, b2, b3;
+        const int row = kb + (lane & 7) + (((lane >> 3) & 1) << 3);
+        const int ch = n2 * 2 + (lane >> 4);
+        ldsm_x4_t(vs_addr + swz<HD>(row, ch), b0, b1, b2, b3);
+        mma16816(o[2 * n2], pa, b0, b1);
+        mma16816(o[2 * n2 + 1], pa, b2, b3);
+      }
+    }
+  }
+  cp_async_wait<0>();
+  __syncthreads();
+
+  // merge the key groups of each m-tile (shared memory reuses the K/V stages)
+  float* mo = reinterpret_cast<float*>(kv);                 // [4 warps][16][HD]
+  float* ml = mo + 4 * 16 * HD;                             // [4 warps][16][2]
+  if (active) {
+    const int r0 = lane >> 2, cc = (lane & 3) << 1;
+#pragma unroll
+    for (int i = 0; i < kNT; ++i) {
+      float* dst = mo + (warp * 16) * HD + i * 8 + cc;
+      dst[r0 * HD] = o[i][0];
+      dst[r0 * HD + 1] = o[i][1];
+      dst[(r0 + 8) * HD] = o[i][2];
+      dst[(r0 + 8) * HD + 1] = o[i][3];
+    }
+    if ((lane & 3) == 0) {
+      ml[(warp * 16 + r0) * 2] = m_run[0];
+      ml[(warp * 16 + r0) * 2 + 1] = l_run[0];
+      ml[(warp * 16 + r0 + 8) * 2] = m_run[1];
+      ml[(warp * 16 + r0 + 8) * 2 + 1] = l_run[1];
+    }
+  }
+  __syncthreads();
   const int unit = (g * a.Hkv + kvh) * a.row_blocks + rb;
   const size_t pbase = (static_cast<size_t>(unit) * a.n_splits + split) * a.qmax;
-#pragma unroll
-  for (int i = 0; i < kAcc; ++i) {
-    const int v = pvg + kNvg * i;
-    if (v < nq) a.part_o[(pbase + v) * HD + pd] = acc[i];
-  }
-  for (int v = tid; v < nq; v += kAttThreads) {
-    a.part_ml[(pbase + v) * 2 + 0] = m_s[v];
-    a.part_ml[(pbase + v) * 2 + 1] = l_s[v];
+  for (int idx = tid; idx < nq * HD; idx += kAttThreads) {
+    const int v = idx / HD, d = idx - v * HD;
+    const int m_t = v >> 4, r = v & 15;
+    float M = -INFINITY;
+    for (int w = 0; w < kg; ++w) M = fmaxf(M, ml[((m_t * kg + w) * 16 + r) * 2]);
+    float L = 0.f, O = 0.f;
+    for (int w = 0; w < kg; ++w) {
+      const int ww = m_t * kg + w;
+      const float mw = ml[(ww * 16 + r) * 2];
+      const float f = mw == -INFINITY ? 0.f : exp2f(mw - M);
+      L += f * ml[(ww * 16 + r) * 2 + 1];
+      O += f * mo[(ww * 16 + r) * HD + d];
+    }
+    a.part_o[(pbase + v) * HD + d] = O;
+    if (d == 0) {
+      a.part_ml[(pbase + v) * 2 + 0] = M;
+      a.part_ml[(pbase + v) * 2 + 1] = L;
+    }
   }
   __threadfence();
   __syncthreads();
@@ -225,9 +337,10 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
 }  // namespace
 
 size_t attention_smem_bytes(const AttnArgs& a) {
-  const size_t f = static_cast<size_t>(a.qmax) * a.hd + static_cast<size_t>(a.qmax) * kKeyTile +
-                   3 * a.qmax + 4;
-  return f * 4 + static_cast<size_t>(kKeyTile) * a.hd * 2;
+  const size_t q = static_cast<size_t>(kMaxQ) * a.hd * 2;
+  const size_t stages = static_cast<size_t>(kStages) * 2 * kKeyTile * a.hd * 2;
+  const size_t merge = static_cast<size_t>(4) * 16 * a.hd * 4 + 4 * 16 * 2 * 4;
+  return q + (stages > merge ? stages : merge);
 }
 
 cudaError_t attention_set_max_smem() {

@@ -113,6 +113,15 @@ __global__ void __launch_bounds__(256) embed_kernel(const __grid_constant__ Embe
     for (int q = 0; q < 8; ++q) sq += f[q] * f[q];
     reinterpret_cast<float4*>(hr + c)[0] = make_float4(f[0], f[1], f[2], f[3]);
     reinterpret_cast<float4*>(hr + c)[1] = make_float4(f[4], f[5], f[6], f[7]);
+    // bf16(h * gain): the first projection's input, its RMSNorm scale applied
+    // per row in that projection's epilogue
+    const uint4 graw = *reinterpret_cast<const uint4*>(a.gain + c);
+    const __nv_bfloat16* gb = reinterpret_cast<const __nv_bfloat16*>(&graw);
+    __nv_bfloat16 o8[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) o8[q] = __float2bfloat16_rn(f[q] * __bfloat162float(gb[q]));
+    *reinterpret_cast<uint4*>(a.xg + static_cast<size_t>(r) * a.d + c) =
+        *reinterpret_cast<const uint4*>(o8);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);

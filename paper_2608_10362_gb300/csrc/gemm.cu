@@ -13,9 +13,11 @@
 //    multi-stage mbarrier ring; they are independent of earlier kernels, so the
 //    producer starts streaming before griddepcontrol.wait (programmatic
 //    dependent launch hides the previous kernel's tail);
-//  * activation tiles are written into shared memory by two producer warps,
-//    which fuse the RMSNorm of the fp32 residual stream (rms from per-row-tile
-//    partial sums of squares written by the previous epilogue);
+//  * activation tiles [n_pad rows x 64 k] arrive by TMA on the same barrier,
+//    issued only after griddepcontrol.wait (they are the previous kernel's
+//    output); RMSNorm is folded in: the previous epilogue wrote bf16(h * gain)
+//    and per-row-tile sums of squares, and this kernel's epilogue scales each
+//    output row by rsqrt(mean(h^2) + eps) (exact: the scale is per row);
 //  * stream-K: the (row-tile, k-tile) space is cut into one contiguous range
 //    per CTA, one CTA per SM; a row tile split over several CTAs is reduced by
 //    the last-arriving CTA in ascending CTA order (deterministic, no float
@@ -38,11 +40,9 @@ constexpr int kTileK = 64;
 constexpr int kABytes = kTileM * kTileK * 2;  // 16 KB
 constexpr int kMaxStages = 8;
 constexpr int kStagePitch = 17;                // epilogue staging row pitch (floats)
-constexpr int kNumBThreads = 64;               // warps 2-3
 
 struct SmemCtl {
-  uint64_t full_a[kMaxStages];
-  uint64_t full_b[kMaxStages];
+  uint64_t full[kMaxStages];
   uint64_t empty[kMaxStages];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
@@ -82,9 +82,12 @@ __device__ __forceinline__ uint4 pack8_bf16(const float* f) {
 
 // Epilogue for one 16-row chunk of a finished 128-feature row tile.  Called by
 // the 128 epilogue threads together; et = feature within the tile (= TMEM lane).
-__device__ void apply_epilogue(const GemmArgs& a, SmemCtl& ctl, float* stage, int rt, int chunk,
-                               int et, const float* v) {
+__device__ void apply_epilogue(const GemmArgs& a, SmemCtl& ctl, float* stage, const float* rms,
+                               int rt, int chunk, int et, const float* vin) {
   const int ew = et >> 5, lane = et & 31;
+  float v[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) v[j] = a.rms ? vin[j] * rms[chunk * 16 + j] : vin[j];
   if (a.epi == EPI_F32) {
     const int f = rt * kTileM + et;
     if (f < a.n_out) {
@@ -115,6 +118,9 @@ __device__ void apply_epilogue(const GemmArgs& a, SmemCtl& ctl, float* stage, in
         const float hn = *hp + v[j];
         *hp = hn;
         sq = hn * hn;
+        if (a.gain_next != nullptr)
+          a.xg_out[static_cast<size_t>(r) * a.h_ld + f] =
+              __float2bfloat16_rn(hn * __bfloat162float(a.gain_next[f]));
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
@@ -203,6 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
       (reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const int S = a.stages;
   const int b_bytes = a.n_pad * 128;
+  const uint32_t stage_tx = static_cast<uint32_t>(kABytes + b_bytes);
   uint8_t* smem_a = dsmem;
   uint8_t* smem_b = dsmem + static_cast<size_t>(S) * kABytes;
   float* stage = reinterpret_cast<float*>(smem_b + static_cast<size_t>(S) * b_bytes);
@@ -217,8 +224,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(&ctl.full_a[s], 1);
-      mbar_init(&ctl.full_b[s], kNumBThreads);
+      mbar_init(&ctl.full[s], 1);
       mbar_init(&ctl.empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -243,17 +249,44 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
   volatile int* abort_flag = &ctl.abort_flag;
 
   if (warp == 0) {
-    // ------------------------------------------------ TMA producer (weights)
+    // ------------------------------------------------ TMA producer
+    // Weight tiles do not depend on earlier kernels: the first S of them are
+    // requested before griddepcontrol.wait.  Activation tiles are requested after.
     if (lane == 0) {
       tma_prefetch_desc(&a.map_a);
       if (a.pair) tma_prefetch_desc(&a.map_a2);
+      tma_prefetch_desc(&a.map_b);
       const uint64_t pol = a.l2_hint == L2_EVICT_FIRST  ? l2_policy_evict_first()
                            : a.l2_hint == L2_EVICT_LAST ? l2_policy_evict_last()
                                                         : l2_policy_evict_normal();
+      const uint64_t pol_b = l2_policy_evict_last();   // activations are re-read by every CTA
       uint32_t issued_mask = 0, last_par = 0;
       int it = 0;
       bool ok = true;
-      for (int t = t_begin; t < t_end && ok; ++t, ++it) {
+      const int n_pre = min(S, t_end - t_begin);
+      // weights of the first n_pre tiles (the ring is empty: no wait needed)
+      for (int p = 0; p < n_pre; ++p) {
+        const int t = t_begin + p;
+        const int rt = t / KT, kt = t - rt * KT;
+        uint8_t* dst = smem_a + static_cast<size_t>(p) * kABytes;
+        mbar_arrive_expect_tx(&ctl.full[p], stage_tx);
+        if (a.pair) {
+          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * 64, &ctl.full[p], pol);
+          tma_load_2d(dst + kABytes / 2, &a.map_a2, kt * kTileK, rt * 64, &ctl.full[p], pol);
+        } else {
+          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * kTileM, &ctl.full[p], pol);
+        }
+        issued_mask |= 1u << p;
+      }
+      pdl_wait();
+      for (int p = 0; p < n_pre; ++p) {
+        const int t = t_begin + p;
+        const int kt = t - (t / KT) * KT;
+        tma_load_2d(smem_b + static_cast<size_t>(p) * b_bytes, &a.map_b, kt * kTileK, 0,
+                    &ctl.full[p], pol_b);
+      }
+      it = n_pre;
+      for (int t = t_begin + n_pre; t < t_end; ++t, ++it) {
         const int rt = t / KT, kt = t - rt * KT;
         const int s = it % S;
         const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
@@ -262,24 +295,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
           break;
         }
         uint8_t* dst = smem_a + static_cast<size_t>(s) * kABytes;
-        mbar_arrive_expect_tx(&ctl.full_a[s], kABytes);
+        mbar_arrive_expect_tx(&ctl.full[s], stage_tx);
         if (a.pair) {
-          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * 64, &ctl.full_a[s], pol);
-          tma_load_2d(dst + kABytes / 2, &a.map_a2, kt * kTileK, rt * 64, &ctl.full_a[s], pol);
+          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * 64, &ctl.full[s], pol);
+          tma_load_2d(dst + kABytes / 2, &a.map_a2, kt * kTileK, rt * 64, &ctl.full[s], pol);
         } else {
-          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * kTileM, &ctl.full_a[s], pol);
+          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * kTileM, &ctl.full[s], pol);
         }
+        tma_load_2d(smem_b + static_cast<size_t>(s) * b_bytes, &a.map_b, kt * kTileK, 0,
+                    &ctl.full[s], pol_b);
         issued_mask |= 1u << s;
         last_par = (last_par & ~(1u << s)) | (ph << s);
       }
       if (!ok) {  // tear-down: let every copy still in flight land before exit
         for (int s = 0; s < S; ++s)
-          if (issued_mask & (1u << s)) mbar_wait_drain(&ctl.full_a[s], (last_par >> s) & 1u);
+          if (issued_mask & (1u << s)) mbar_wait_drain(&ctl.full[s], (last_par >> s) & 1u);
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
-    pdl_wait();
     if (lane == 0) {
       const uint32_t idesc = make_idesc_bf16_f32(kTileM, a.n_pad);
       int it = 0, seg = 0;
@@ -299,8 +333,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
         for (int tt = t; tt < seg_end; ++tt, ++it) {
           const int s = it % S;
           const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
-          if (!mbar_wait_bounded(&ctl.full_a[s], ph, abort_flag, a.status) ||
-              !mbar_wait_bounded(&ctl.full_b[s], ph, abort_flag, a.status)) {
+          if (!mbar_wait_bounded(&ctl.full[s], ph, abort_flag, a.status)) {
             ok = false;
             break;
           }
@@ -324,61 +357,23 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
         mbar_wait_drain(&ctl.drain, 0);
       }
     }
-  } else if (warp < 4) {
-    // ------------------------------------------------ activation producers
-    const int tb = threadIdx.x - 64;
-    pdl_wait();
-    if (a.b_mode == B_F32_RMSNORM) {
-      for (int r = tb; r < a.n_pad; r += kNumBThreads) {
-        float val = 0.f;
-        if (r < a.rows_total) {
-          float s = 0.f;
-          for (int i = 0; i < a.ss_count; ++i) s += a.ss[static_cast<size_t>(i) * a.ss_stride + r];
-          val = rsqrtf(s / static_cast<float>(a.k_in) + a.eps);
-        }
-        rms[r] = val;
-      }
-      named_bar_sync(2, kNumBThreads);
-    }
-    int it = 0;
-    for (int t = t_begin; t < t_end; ++t, ++it) {
-      const int rt = t / KT, kt = t - rt * KT;
-      (void)rt;
-      const int s = it % S;
-      const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
-      if (!mbar_wait_bounded(&ctl.empty[s], ph ^ 1u, abort_flag, a.status)) break;
-      uint8_t* bs = smem_b + static_cast<size_t>(s) * b_bytes;
-      for (int ch = tb; ch < a.n_pad * 8; ch += kNumBThreads) {
-        const int row = ch >> 3, kc = ch & 7;
-        const int k = kt * kTileK + kc * 8;
-        uint4 val = make_uint4(0u, 0u, 0u, 0u);
-        if (row < a.rows_total && k < a.k_in) {
-          if (a.b_mode == B_BF16) {
-            val = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(a.b_src) +
-                                                   static_cast<size_t>(row) * a.b_ld + k);
-          } else {
-            const float* src = static_cast<const float*>(a.b_src) + static_cast<size_t>(row) * a.b_ld + k;
-            const float4 x0 = *reinterpret_cast<const float4*>(src);
-            const float4 x1 = *reinterpret_cast<const float4*>(src + 4);
-            const uint4 graw = *reinterpret_cast<const uint4*>(a.gain + k);
-            const __nv_bfloat16* g = reinterpret_cast<const __nv_bfloat16*>(&graw);
-            const float sc = rms[row];
-            float f[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-#pragma unroll
-            for (int q = 0; q < 8; ++q) f[q] = f[q] * sc * __bfloat162float(g[q]);
-            val = pack8_bf16(f);
-          }
-        }
-        *reinterpret_cast<uint4*>(bs + row * 128 + ((kc ^ (row & 7)) << 4)) = val;
-      }
-      fence_proxy_async_smem();
-      mbar_arrive(&ctl.full_b[s]);
-    }
-  } else {
+  } else if (warp >= 4) {
     // ------------------------------------------------ epilogue (warps 4-7)
     const int et = threadIdx.x - 128;  // tile feature == TMEM lane
     const int ew = warp & 3;
     pdl_wait();
+    if (a.rms) {   // per-row RMSNorm scale from the partial sums of squares
+      for (int r = et; r < a.n_pad; r += 128) {
+        float val = 0.f;
+        if (r < a.rows_total) {
+          float sum = 0.f;
+          for (int i = 0; i < a.ss_count; ++i) sum += a.ss[static_cast<size_t>(i) * a.ss_stride + r];
+          val = rsqrtf(sum / static_cast<float>(a.k_in) + a.eps);
+        }
+        rms[r] = val;
+      }
+      named_bar_sync(1, 128);
+    }
     int seg = 0;
     for (int t = t_begin; t < t_end; ++seg) {
       const int rt = t / KT;
@@ -402,7 +397,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
       if (full) {
         for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
           tmem_ld_32x32b_x16(tbase + chunk * 16, v);
-          apply_epilogue(a, ctl, stage, rt, chunk, et, v);
+          apply_epilogue(a, ctl, stage, rms, rt, chunk, et, v);
         }
       } else {
         const int slot = (seg == 0) ? 0 : 1;
@@ -437,7 +432,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
 #pragma unroll
               for (int j = 0; j < 16; ++j) v[j] += ld_cg_f(pp + (chunk * 16 + j) * kTileM + et);
             }
-            apply_epilogue(a, ctl, stage, rt, chunk, et, v);
+            apply_epilogue(a, ctl, stage, rms, rt, chunk, et, v);
           }
           if (et == 0) a.counters[rt] = 0;
         }
@@ -459,7 +454,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
 
 int gemm_pick_stages(int n_pad) {
   const int stage = kABytes + n_pad * 128;
-  const int budget = n_pad <= 32 ? 100 * 1024 : 190 * 1024;
+  const int budget = n_pad <= 32 ? 104 * 1024 : 200 * 1024;
   const int fixed = kTileM * kStagePitch * 4 + kMaxRows * 4 + 1024;
   int s = (budget - fixed) / stage;
   if (s > kMaxStages) s = kMaxStages;
@@ -473,8 +468,9 @@ size_t gemm_smem_bytes(int n_pad, int stages) {
 }
 
 cudaError_t gemm_set_max_smem() {
+  // 227 KB per block minus the kernel's static shared memory
   return cudaFuncSetAttribute(gemm_stream_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              227 * 1024);
+                              220 * 1024);
 }
 
 cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s, bool pdl) {

@@ -54,19 +54,21 @@ struct EmbedArgs {
   const bf16* emb;          // [vocab][d]
   int d, vocab;
   float* h;                 // [rows][d] residual stream
+  bf16* xg;                 // [rows][d] bf16(h * gain) for the first projection
+  const bf16* gain;         // first RMSNorm gain
   float* ss;                // [ss_tiles][ss_stride]: row sums of squares (partial)
   int ss_stride;
   RowPlan* plan;
   uint32_t* status;
 };
 
-enum GemmBMode : int { B_BF16 = 0, B_F32_RMSNORM = 1 };
 enum GemmEpi : int { EPI_F32 = 0, EPI_RESIDUAL = 1, EPI_SWIGLU = 2, EPI_QKV = 3 };
 enum L2Hint : int { L2_EVICT_FIRST = 0, L2_EVICT_NORMAL = 1, L2_EVICT_LAST = 2 };
 
 struct GemmArgs {
   CUtensorMap map_a;        // weights [n_out][k] bf16, box {64, 128} (or {64, 64} for pairs)
   CUtensorMap map_a2;       // second matrix of a SwiGLU pair (up), box {64, 64}
+  CUtensorMap map_b;        // activations [rows_total][k] bf16, box {64, n_pad}
   int n_out;                // output features (F for pairs)
   int k_in;
   int pair;                 // 1: tile = 64 rows of map_a + 64 rows of map_a2
@@ -74,11 +76,9 @@ struct GemmArgs {
   int n_pad;                // MMA N: rows_total rounded up to 16
   int row_tiles, k_tiles, stages;
   int l2_hint;
-  // B operand source
-  int b_mode;
-  const void* b_src;        // bf16 [rows][b_ld] or fp32 [rows][b_ld]
-  int b_ld;
-  const bf16* gain;         // RMSNorm gain [k_in] (B_F32_RMSNORM)
+  // RMSNorm folded into the epilogue: B = bf16(h * gain) was written by the
+  // previous epilogue; y[r] *= rsqrt(sum_i ss[i][r] / k_in + eps)
+  int rms;
   const float* ss;          // [ss_count][ss_stride]
   int ss_count, ss_stride;
   float eps;
@@ -94,6 +94,8 @@ struct GemmArgs {
   float* h;                 // EPI_RESIDUAL: residual [rows][h_ld], updated in place
   int h_ld;
   float* ss_out;            // EPI_RESIDUAL: [row_tiles][ss_stride]
+  const bf16* gain_next;    // EPI_RESIDUAL: gain of the next RMSNorm (nullptr: no xg)
+  bf16* xg_out;             // EPI_RESIDUAL: bf16(h_new * gain_next) [rows][h_ld]
   bf16* act;                // EPI_SWIGLU: [rows][act_ld]
   int act_ld;
   float* q_out;             // EPI_QKV: fp32 [rows][q_dim]
