@@ -271,6 +271,62 @@ def oracle_sample(tokens_per_iter: float, K: int, reps: int = 1):
     }
 
 
+def run_case(args):
+    """Diagnostic cases (not the headline metric)."""
+    import numpy as np
+    import torch
+
+    from seeded_inputs import SHAPES, bf16_round, gen_prompt, iter_weights
+    if args.case == "gemm":
+        from paper_2608_10362_gb300 import op_linear
+        rng = np.random.default_rng(0)
+        x = torch.from_numpy(bf16_round(rng.standard_normal((args.rows, args.kdim), dtype=np.float32)))
+        w = torch.randn(args.n, args.kdim, device="cuda", dtype=torch.bfloat16) * 0.02
+        xt = x.to(torch.bfloat16).cuda()
+        scratch = torch.zeros(64 << 20, dtype=torch.uint8, device="cuda")
+        for _ in range(args.warmup):
+            op_linear(xt, w, scratch)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(args.steps):
+            op_linear(xt, w, scratch)
+        b.record()
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / args.steps
+        nbytes = args.n * args.kdim * 2 + args.rows * (args.kdim * 2 + args.n * 4)
+        return {"case": "gemm", "n_out": args.n, "k": args.kdim, "rows": args.rows,
+                "us_per_launch": ms * 1e3, "GB/s": nbytes / ms / 1e6}
+    from paper_2608_10362_gb300 import Engine
+    t, d = SHAPES["draft_160m"], SHAPES["draft_68m"]
+    K = args.k
+    max_seq = 512 + (args.steps + args.warmup + 4) * (K + 1) + 16
+    eng = Engine(t, iter_weights(t, 0), max_batch=1, max_seq=max_seq, max_k=K, max_drafts=1,
+                 draft_shape_max=d, draft_budget_bytes=512 << 20, use_graphs=True)
+    eng.register_draft(0, d, iter_weights(d, 1))
+    eng.load_draft_async(0)
+    eng.set_active_draft(0)
+    eng.prefill(0, gen_prompt(3, 512, t.vocab), seed=1)
+    for _ in range(args.warmup):
+        eng.step(K, TEMP)
+    eng.sync()
+    L0 = int(eng.seq_state()[0, 0])
+    s = eng.stream
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(s)
+    for _ in range(args.steps):
+        eng.step(K, TEMP)
+    b.record(s)
+    torch.cuda.synchronize()
+    bits = eng.sync()
+    L1 = int(eng.seq_state()[0, 0])
+    ms = a.elapsed_time(b)
+    eng.close()
+    return {"case": "small", "target": "draft_160m", "draft": "draft_68m", "K": K,
+            "ms_per_step": ms / args.steps, "tokens_per_s": (L1 - L0) / ms * 1e3,
+            "device_status": bits}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -279,8 +335,17 @@ def main():
     ap.add_argument("--k", type=int, default=K_DRAFT)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--case", default="step", choices=["step", "gemm", "small"],
+                    help="step: the workload above; gemm / small: diagnostic cases sized for "
+                         "profiler captures (one projection GEMM; a 160M target with a 68M draft)")
+    ap.add_argument("--n", type=int, default=22016)
+    ap.add_argument("--kdim", type=int, default=4096)
+    ap.add_argument("--rows", type=int, default=5)
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.case != "step":
+        print(json.dumps(run_case(args)))
+        return
 
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))

@@ -10,6 +10,7 @@
 
 #include <algorithm>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <ctime>
 #include <map>
@@ -264,6 +265,7 @@ struct GraphKey {
 
 struct memspec_ctx {
   memspec_init_params p{};
+  bool pdl = true;   // programmatic dependent launch between the kernels of a pass
   cudaStream_t main = nullptr, side = nullptr;
   std::string err;
   // workspace
@@ -492,14 +494,23 @@ struct FwdSpec {
   long long out_group_stride;
 };
 
+// Stream-K grid: at most one CTA per SM, and at least ceil(k_tiles / 4) tiles per
+// CTA so that a row tile is shared by at most ~4 CTAs (the last of them sums the
+// partials; more contributors lengthen that serial tail more than they add
+// bandwidth on small matrices).
+int gemm_grid(int row_tiles, int k_tiles) {
+  const int T = row_tiles * k_tiles;
+  const int min_tiles = std::max(1, (k_tiles + 3) / 4);
+  return std::max(1, std::min({T, sm_count(), T / min_tiles}));
+}
+
 memspec_status run_gemm(memspec_ctx* c, GemmArgs& a, const char* what) {
-  const int T = a.row_tiles * a.k_tiles;
-  const int grid = std::min(T, sm_count());
+  const int grid = gemm_grid(a.row_tiles, a.k_tiles);
   a.stages = gemm_pick_stages(a.n_pad);
   a.partials = c->gemm_part;
   a.counters = c->gemm_cnt;
   a.status = c->status;
-  cudaError_t e = launch_gemm(a, grid, gemm_smem_bytes(a.n_pad, a.stages), c->main, true);
+  cudaError_t e = launch_gemm(a, grid, gemm_smem_bytes(a.n_pad, a.stages), c->main, c->pdl);
   if (e != cudaSuccess) return cuda_fail(c, e, what);
   return MEMSPEC_OK;
 }
@@ -534,7 +545,7 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
   ea.ss_stride = c->ss_stride;
   ea.plan = c->plan;
   ea.status = c->status;
-  cudaError_t e = launch_embed(ea, rows, c->main, true);
+  cudaError_t e = launch_embed(ea, rows, c->main, c->pdl);
   if (e != cudaSuccess) return cuda_fail(c, e, "embed launch");
 
   const size_t layer_kv = static_cast<size_t>(c->p.max_batch) * cf.n_kv_heads * c->p.max_seq * cf.head_dim;
@@ -600,7 +611,7 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       at.out = c->o;
       at.plan = c->plan;
       at.status = c->status;
-      e = launch_attention(at, f.n_groups, c->main, true);
+      e = launch_attention(at, f.n_groups, c->main, c->pdl);
       if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
     }
     {  // O projection + residual
@@ -865,6 +876,10 @@ memspec_status memspec_init(const memspec_init_params* p, void* workspace_dev, m
   memspec_ctx* c = new memspec_ctx();
   c->p = *p;
   c->main = static_cast<cudaStream_t>(p->stream_main);
+  // MEMSPEC_NO_PDL=1 launches every kernel without programmatic dependent launch
+  // (for measuring what the overlap buys)
+  const char* no_pdl = std::getenv("MEMSPEC_NO_PDL");
+  c->pdl = !(no_pdl != nullptr && no_pdl[0] == '1');
   c->side = p->stream_side ? static_cast<cudaStream_t>(p->stream_side) : c->main;
   c->ws_bytes = layout_workspace(p, c, static_cast<uint8_t*>(workspace_dev));
   if (!ensure_func_attrs()) {
@@ -1152,7 +1167,7 @@ memspec_status memspec_draft_step(memspec_ctx* c, int32_t K, float T) {
       sa.out_stride = c->p.max_k;
       sa.counters = c->smp_cnt;
       sa.status = c->status;
-      cudaError_t e = launch_sample(sa, c->main, true);
+      cudaError_t e = launch_sample(sa, c->main, c->pdl);
       if (e != cudaSuccess) return cuda_fail(c, e, "sample launch");
     }
     return MEMSPEC_OK;
@@ -1386,8 +1401,7 @@ memspec_status memspec_op_linear(const void* x, const void* w, float* y, int32_t
                                : reinterpret_cast<uint32_t*>(sb + part_bytes +
                                                              align256(static_cast<size_t>(a.row_tiles) * 4));
   a.plan = nullptr;
-  const int T = a.row_tiles * a.k_tiles;
-  const int grid = std::min(T, sm_count());
+  const int grid = gemm_grid(a.row_tiles, a.k_tiles);
   cudaError_t e = launch_gemm(a, grid, gemm_smem_bytes(n_pad, a.stages),
                               static_cast<cudaStream_t>(stream), false);
   if (e != cudaSuccess) {

@@ -314,22 +314,39 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
   if (!last) return;
   __threadfence();
   const size_t ubase = static_cast<size_t>(unit) * a.n_splits * a.qmax;
-  for (int idx = tid; idx < nq * HD; idx += kAttThreads) {
-    const int v = idx / HD, d = idx - v * HD;
+  // split weights 2^(m_s - M) and 1/L per query vector, computed once in shared memory
+  float* wsm = reinterpret_cast<float*>(kv);                // [n_active][nq]
+  float* linv = wsm + n_active * nq;                        // [nq]
+  for (int v = tid; v < nq; v += kAttThreads) {
     float M = -INFINITY;
     for (int s = 0; s < n_active; ++s) M = fmaxf(M, ld_cg_f(a.part_ml + (ubase + s * a.qmax + v) * 2));
-    float L = 0.f, O = 0.f;
+    float L = 0.f;
     for (int s = 0; s < n_active; ++s) {
       const size_t pv = ubase + s * a.qmax + v;
       const float ms = ld_cg_f(a.part_ml + pv * 2);
       const float w = ms == -INFINITY ? 0.f : exp2f(ms - M);
+      wsm[s * nq + v] = w;
       L += w * ld_cg_f(a.part_ml + pv * 2 + 1);
-      O += w * ld_cg_f(a.part_o + pv * HD + d);
+    }
+    linv[v] = 1.f / L;
+  }
+  __syncthreads();
+  for (int idx = tid; idx < nq * HD; idx += kAttThreads) {
+    const int v = idx / HD, d = idx - v * HD;
+    float O = 0.f;
+    for (int s0 = 0; s0 < n_active; s0 += 4) {   // four splits fetched at once, summed in order
+      float ov[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        ov[q] = (s0 + q < n_active) ? ld_cg_f(a.part_o + (ubase + (s0 + q) * a.qmax + v) * HD + d) : 0.f;
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if (s0 + q < n_active) O += wsm[(s0 + q) * nq + v] * ov[q];
     }
     const int hl = v / nr, rr = v - hl * nr;
     const int row = g * R + r_lo + rr;
     const int h = kvh * gs + hl;
-    a.out[(static_cast<size_t>(row) * a.H + h) * HD + d] = __float2bfloat16_rn(O / L);
+    a.out[(static_cast<size_t>(row) * a.H + h) * HD + d] = __float2bfloat16_rn(O * linv[v]);
   }
   if (tid == 0) a.counters[unit] = 0;
 }

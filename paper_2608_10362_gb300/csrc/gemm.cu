@@ -34,7 +34,7 @@ namespace memspec {
 
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 192;   // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr int kTileM = 128;
 constexpr int kTileK = 64;
 constexpr int kABytes = kTileM * kTileK * 2;  // 16 KB
@@ -63,21 +63,6 @@ __device__ __forceinline__ uint32_t tmem_cols_for(int n_pad) {
 __device__ __forceinline__ bool row_valid(const GemmArgs& a, int r) {
   if (r >= a.rows_total) return false;
   return a.plan == nullptr ? true : plan_row_valid(a.plan, r);
-}
-
-// Pack 8 floats into 8 bf16 (round to nearest even) as a uint4.
-__device__ __forceinline__ uint4 pack8_bf16(const float* f) {
-  uint4 u;
-  __nv_bfloat162 t;
-  t = __floats2bfloat162_rn(f[0], f[1]);
-  u.x = *reinterpret_cast<uint32_t*>(&t);
-  t = __floats2bfloat162_rn(f[2], f[3]);
-  u.y = *reinterpret_cast<uint32_t*>(&t);
-  t = __floats2bfloat162_rn(f[4], f[5]);
-  u.z = *reinterpret_cast<uint32_t*>(&t);
-  t = __floats2bfloat162_rn(f[6], f[7]);
-  u.w = *reinterpret_cast<uint32_t*>(&t);
-  return u;
 }
 
 // Epilogue for one 16-row chunk of a finished 128-feature row tile.  Called by
@@ -357,17 +342,26 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
         mbar_wait_drain(&ctl.drain, 0);
       }
     }
-  } else if (warp >= 4) {
-    // ------------------------------------------------ epilogue (warps 4-7)
-    const int et = threadIdx.x - 128;  // tile feature == TMEM lane
+  } else {
+    // ------------------------------------------------ epilogue (warps 2-5)
+    // a warp may only read TMEM lanes 32*(warp % 4) .. +31: that is its feature block
     const int ew = warp & 3;
+    const int et = ew * 32 + lane;  // tile feature == TMEM lane
     pdl_wait();
     if (a.rms) {   // per-row RMSNorm scale from the partial sums of squares
       for (int r = et; r < a.n_pad; r += 128) {
         float val = 0.f;
         if (r < a.rows_total) {
           float sum = 0.f;
-          for (int i = 0; i < a.ss_count; ++i) sum += a.ss[static_cast<size_t>(i) * a.ss_stride + r];
+          // partial sums added in index order; loads issued eight at a time
+          for (int i0 = 0; i0 < a.ss_count; i0 += 8) {
+            float t[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              t[q] = (i0 + q < a.ss_count) ? a.ss[static_cast<size_t>(i0 + q) * a.ss_stride + r] : 0.f;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) sum += t[q];
+          }
           val = rsqrtf(sum / static_cast<float>(a.k_in) + a.eps);
         }
         rms[r] = val;
@@ -400,12 +394,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
           apply_epilogue(a, ctl, stage, rms, rt, chunk, et, v);
         }
       } else {
+        // partial sums, feature-major: thread et owns n_pad consecutive floats
         const int slot = (seg == 0) ? 0 : 1;
-        float* pb = a.partials + static_cast<size_t>(2 * c + slot) * a.n_pad * kTileM;
+        float* pb = a.partials + static_cast<size_t>(2 * c + slot) * a.n_pad * kTileM +
+                    static_cast<size_t>(et) * a.n_pad;
         for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
           tmem_ld_32x32b_x16(tbase + chunk * 16, v);
+          float4* dst = reinterpret_cast<float4*>(pb + chunk * 16);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) pb[(chunk * 16 + j) * kTileM + et] = v[j];
+          for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
       }
       tc_fence_before();
@@ -426,11 +423,32 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
           for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
 #pragma unroll
             for (int j = 0; j < 16; ++j) v[j] = 0.f;
-            for (int cc = c_first; cc <= c_last; ++cc) {
-              const int sl = (sk_begin(cc, T, G) >= rt * KT) ? 0 : 1;
-              const float* pp = a.partials + static_cast<size_t>(2 * cc + sl) * a.n_pad * kTileM;
+            // contributors are summed in ascending CTA order; four are fetched at once
+            for (int cc0 = c_first; cc0 <= c_last; cc0 += 4) {
+              float4 tmp[4][4];
 #pragma unroll
-              for (int j = 0; j < 16; ++j) v[j] += ld_cg_f(pp + (chunk * 16 + j) * kTileM + et);
+              for (int q = 0; q < 4; ++q) {
+                const int cc = cc0 + q;
+                if (cc <= c_last) {
+                  const int sl = (sk_begin(cc, T, G) >= rt * KT) ? 0 : 1;
+                  const float* pp = a.partials + static_cast<size_t>(2 * cc + sl) * a.n_pad * kTileM +
+                                    static_cast<size_t>(et) * a.n_pad + chunk * 16;
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) tmp[q][e] = ld_cg_f4(pp + 4 * e);
+                }
+              }
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                if (cc0 + q <= c_last) {
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) {
+                    v[4 * e] += tmp[q][e].x;
+                    v[4 * e + 1] += tmp[q][e].y;
+                    v[4 * e + 2] += tmp[q][e].z;
+                    v[4 * e + 3] += tmp[q][e].w;
+                  }
+                }
+              }
             }
             apply_epilogue(a, ctl, stage, rms, rt, chunk, et, v);
           }

@@ -24,8 +24,7 @@ namespace {
 
 constexpr int kSThreads = 512;
 constexpr int kSWarps = kSThreads / 32;
-constexpr int kTileIds = kSThreads * 4;
-constexpr int kMaxTiles = 64;          // vocab <= 131072
+constexpr int kMaxTiles = 1024;        // 128-id tiles: vocab <= 131072
 
 struct RowStats {
   float m;     // max of z * inv_temp   (greedy: max of z)
@@ -46,19 +45,35 @@ __device__ float block_sum(float v, float* scratch) {
   return t;
 }
 
+__device__ __forceinline__ void stats_update(float raw, int x, bool greedy, float inv_temp,
+                                             float& m, float& s, int& arg) {
+  if (raw > m) {
+    if (!greedy) s = (m == -INFINITY) ? 0.f : s * __expf((m - raw) * inv_temp);
+    m = raw;
+    arg = x;
+  }
+  if (!greedy) s += __expf((raw - m) * inv_temp);
+}
+
 // max / first-argmax / rescaled exp-sum of one row, whole block.
 __device__ RowStats row_stats(const float* z, int V, float inv_temp, bool greedy, float* scr_f,
                               int* scr_i) {
   float m = -INFINITY, s = 0.f;
   int arg = 0x7fffffff;
-  for (int x = threadIdx.x; x < V; x += kSThreads) {
-    const float raw = z[x];
-    if (raw > m || (raw == m && x < arg)) {
-      if (!greedy) s = (m == -INFINITY) ? 0.f : s * __expf((m - raw) * inv_temp);
-      m = raw;
-      arg = x;
+  if ((V & 3) == 0 && (reinterpret_cast<uintptr_t>(z) & 15) == 0) {
+    const float4* z4 = reinterpret_cast<const float4*>(z);
+    const int V4 = V >> 2;
+#pragma unroll 4
+    for (int x4 = threadIdx.x; x4 < V4; x4 += kSThreads) {
+      const float4 r = __ldcg(z4 + x4);
+      stats_update(r.x, 4 * x4, greedy, inv_temp, m, s, arg);
+      stats_update(r.y, 4 * x4 + 1, greedy, inv_temp, m, s, arg);
+      stats_update(r.z, 4 * x4 + 2, greedy, inv_temp, m, s, arg);
+      stats_update(r.w, 4 * x4 + 3, greedy, inv_temp, m, s, arg);
     }
-    if (!greedy) s += __expf((raw - m) * inv_temp);
+  } else {
+#pragma unroll 4
+    for (int x = threadIdx.x; x < V; x += kSThreads) stats_update(__ldcg(z + x), x, greedy, inv_temp, m, s, arg);
   }
   // block combine: max first (with first index), then sums rescaled to it
   float bm = m;
@@ -99,107 +114,129 @@ __device__ RowStats row_stats(const float* z, int V, float inv_temp, bool greedy
 }
 
 // Smallest id j in [0, V) with sum_{i<=j} w(i) > u * sum w; whole block.
-// w(i) must be >= 0.  Returns -1 if the total weight is zero.
+// w(i) must be >= 0.  Returns -1 if the total weight is zero.  Weights are
+// summed in a fixed order: tiles of 128 consecutive ids (4 per lane, lanes
+// combined by a fixed shuffle tree), tiles combined in id order.
 template <class W>
 __device__ int block_sample(const W& wfun, int V, float u, float* tile_sums, float* scr,
                             float* total_out) {
-  const int ntiles = (V + kTileIds - 1) / kTileIds;
-  for (int tile = 0; tile < ntiles; ++tile) {
+  (void)scr;
+  constexpr int kTile = 128;
+  const int ntiles = (V + kTile - 1) / kTile;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll 2
+  for (int tile = w; tile < ntiles; tile += kSWarps) {
+    const int x0 = tile * kTile + lane * 4;
     float own = 0.f;
-    const int x0 = tile * kTileIds + threadIdx.x * 4;
 #pragma unroll
     for (int q = 0; q < 4; ++q)
       if (x0 + q < V) own += wfun(x0 + q);
-    const float ts = block_sum(own, scr);
-    if (threadIdx.x == 0) tile_sums[tile] = ts;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) own += __shfl_xor_sync(0xffffffffu, own, o);
+    if (lane == 0) tile_sums[tile] = own;
   }
   __syncthreads();
-  __shared__ float sh_target, sh_before;
-  __shared__ int sh_tile, sh_pick;
-  if (threadIdx.x == 0) {
-    float total = 0.f;
-    for (int t = 0; t < ntiles; ++t) total += tile_sums[t];
+  __shared__ int sh_pick;
+  if (w == 0) {
+    // each lane owns a contiguous range of tiles
+    const int tpl = (ntiles + 31) / 32;
+    const int t_lo = min(lane * tpl, ntiles), t_hi = min(t_lo + tpl, ntiles);
+    float ls = 0.f;
+    for (int t = t_lo; t < t_hi; ++t) ls += tile_sums[t];
+    float incl = ls;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
+    }
+    float excl = __shfl_up_sync(0xffffffffu, incl, 1);
+    if (lane == 0) excl = 0.f;
+    const float total = __shfl_sync(0xffffffffu, incl, 31);
     const float target = u * total;
-    float cum = 0.f;
-    int tsel = -1;
+    int sel = -1;
     float before = 0.f;
-    for (int t = 0; t < ntiles; ++t) {
-      if (tile_sums[t] > 0.f) {
-        if (cum + tile_sums[t] > target) {
-          tsel = t;
-          before = cum;
-          break;
+    if (ls > 0.f && excl <= target && target < incl) {
+      float c = excl;
+      for (int t = t_lo; t < t_hi; ++t) {
+        if (tile_sums[t] > 0.f) {
+          sel = t;
+          before = c;
+          if (c + tile_sums[t] > target) break;
         }
-        tsel = t;  // fallback: last tile with mass
-        before = cum;
+        c += tile_sums[t];
       }
-      cum += tile_sums[t];
     }
-    *total_out = total;
-    sh_target = target - before;
-    sh_tile = total > 0.f ? tsel : -1;
-    sh_pick = -1;
-  }
-  __syncthreads();
-  if (sh_tile < 0) return -1;
-  // inside the selected tile: exclusive scan of the per-thread sums
-  const int x0 = sh_tile * kTileIds + threadIdx.x * 4;
-  float wv[4];
-  float own = 0.f;
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    wv[q] = (x0 + q < V) ? wfun(x0 + q) : 0.f;
-    own += wv[q];
-  }
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  float incl = own;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const float n = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += n;
-  }
-  float excl = __shfl_up_sync(0xffffffffu, incl, 1);
-  if (lane == 0) excl = 0.f;
-  __syncthreads();
-  if (lane == 31) scr[w] = incl;
-  __syncthreads();
-  float woff = 0.f;
-  for (int i = 0; i < w; ++i) woff += scr[i];
-  // [lo, hi) of consecutive threads chain exactly: hi of lane l == lo of lane l+1,
-  // and hi of lane 31 == lo of the next warp's lane 0 (same additions).
-  const float lo = woff + excl, hi = woff + incl;
-  const float r = sh_target;
-  if (own > 0.f && lo <= r && r < hi) {
-    float c = lo;
+    // the claiming lane (at most one: ranges chain exactly); otherwise the last tile with mass
+    unsigned claim = __ballot_sync(0xffffffffu, sel >= 0);
+    int last_lane = 31 - __clz(__ballot_sync(0xffffffffu, ls > 0.f) | 1u);
+    int src = claim ? (__ffs(claim) - 1) : last_lane;
+    if (!claim && lane == src) {   // rounding put the target at/after the end: last tile with mass
+      float c = excl;
+      for (int t = t_lo; t < t_hi; ++t) {
+        if (tile_sums[t] > 0.f) {
+          sel = t;
+          before = c;
+        }
+        c += tile_sums[t];
+      }
+    }
+    sel = __shfl_sync(0xffffffffu, sel, src);
+    before = __shfl_sync(0xffffffffu, before, src);
     int pick = -1;
+    if (total > 0.f && sel >= 0) {
+      const float r = target - before;
+      const int x0 = sel * kTile + lane * 4;
+      float wv[4], own = 0.f;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      c += wv[q];
-      if (pick < 0 && wv[q] > 0.f && c > r) pick = x0 + q;
-    }
-    if (pick < 0) {  // rounding at the thread's upper edge: its last id with mass
-      for (int q = 3; q >= 0; --q)
-        if (wv[q] > 0.f) {
-          pick = x0 + q;
-          break;
+      for (int q = 0; q < 4; ++q) {
+        wv[q] = (x0 + q < V) ? wfun(x0 + q) : 0.f;
+        own += wv[q];
+      }
+      float in2 = own;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float n = __shfl_up_sync(0xffffffffu, in2, o);
+        if (lane >= o) in2 += n;
+      }
+      float ex2 = __shfl_up_sync(0xffffffffu, in2, 1);
+      if (lane == 0) ex2 = 0.f;
+      int mine = -1;
+      if (own > 0.f && ex2 <= r && r < in2) {
+        float c = ex2;
+        for (int q = 0; q < 4; ++q) {
+          c += wv[q];
+          if (wv[q] > 0.f && c > r) {
+            mine = x0 + q;
+            break;
+          }
         }
+        if (mine < 0)
+          for (int q = 3; q >= 0; --q)
+            if (wv[q] > 0.f) {
+              mine = x0 + q;
+              break;
+            }
+      }
+      unsigned cl = __ballot_sync(0xffffffffu, mine >= 0);
+      if (cl) {
+        pick = __shfl_sync(0xffffffffu, mine, __ffs(cl) - 1);
+      } else {   // r at/after the tile's scanned mass: its last id with mass
+        int lastq = -1;
+        for (int q = 3; q >= 0; --q)
+          if (wv[q] > 0.f) {
+            lastq = x0 + q;
+            break;
+          }
+        unsigned hm = __ballot_sync(0xffffffffu, lastq >= 0);
+        pick = hm ? __shfl_sync(0xffffffffu, lastq, 31 - __clz(hm)) : -1;
+      }
     }
-    atomicMax(&sh_pick, pick);
+    if (lane == 0) {
+      sh_pick = pick;
+      *total_out = total;
+    }
   }
   __syncthreads();
-  if (sh_pick < 0) {
-    // target at or beyond the tile's scanned mass (rounding): last id with mass
-    if (own > 0.f) {
-      int last_id = -1;
-      for (int q = 3; q >= 0; --q)
-        if (wv[q] > 0.f) {
-          last_id = x0 + q;
-          break;
-        }
-      atomicMax(&sh_pick, last_id);
-    }
-    __syncthreads();
-  }
   return sh_pick;
 }
 
