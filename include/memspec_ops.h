@@ -34,6 +34,26 @@ memspec_status memspec_op_linear(const void* x_dev, const void* w_dev, float* y_
                                  void* scratch_dev, size_t scratch_bytes,
                                  uint32_t* status_dev, void* stream);
 
+/* The same GEMM as memspec_op_linear (y = x . w^T, fp32 out), for callers
+ * that cannot allocate device memory: code running while a CUDA graph is
+ * being captured, plug-ins whose host application owns all device memory, and
+ * fixed-budget deployments that allocate only at start-up.  The paper has no
+ * counterpart; this is a property of the library's interface.
+ * Instead of a scratch argument it uses one file-scope device array of about
+ * 2.6 MB that every GPU loading the library keeps until the process exits.
+ * Limits: rows in 1..16, n_out in 1..131072, k a positive multiple of 8; x and w
+ * 16-byte aligned.  Larger sizes return MEMSPEC_ERR_INVALID_ARG (message in
+ * memspec_op_last_error) and enqueue nothing.  The call allocates nothing; it
+ * enqueues a clear of the array's counters and the kernel on `stream`.
+ * All calls share the array: calls that overlap on the GPU (other streams,
+ * other host threads) race - serialise them.  The first call on a device looks
+ * up the array's address on that device; make it before any stream capture.
+ * status_dev: optional uint32 device word for in-kernel error bits (NULL: an
+ * internal word is used). */
+memspec_status memspec_op_linear_noalloc(const void* x_dev, const void* w_dev, float* y_dev,
+                                         int32_t rows, int32_t n_out, int32_t k,
+                                         uint32_t* status_dev, void* stream);
+
 /* Categorical sampling of each row of logits[rows][vocab] (fp32): with T > 0,
  * out[r] = smallest j with sum_{i<=j} exp(z_i/T - m) > u[r] * sum_i exp(z_i/T - m);
  * with T == 0, out[r] = argmax (lowest id on ties).  u_dev: fp32 [rows] in

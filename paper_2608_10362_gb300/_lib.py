@@ -73,6 +73,8 @@ EXPORTS = {
                                                   C.POINTER(C.c_size_t)]),
     "memspec_op_linear": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32,
                                     C.c_int32, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
+    "memspec_op_linear_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
+                                            C.c_int32, C.c_int32, C.c_void_p, C.c_void_p]),
     "memspec_op_sample": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_float, C.c_void_p,
                                     C.c_void_p, C.c_void_p]),
     "memspec_op_last_error": (C.c_char_p, []),

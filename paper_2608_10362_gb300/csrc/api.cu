@@ -1334,6 +1334,11 @@ memspec_status memspec_write_buffer(memspec_ctx* c, int32_t buf, const void* src
 
 // ---------------------------------------------------------------- op-level entry points
 const char* memspec_op_last_error(void) { return g_op_error.c_str(); }
+}  // extern "C"
+
+void memspec::set_op_error(const char* msg) { g_op_error = msg; }
+
+extern "C" {
 
 static size_t op_linear_scratch(int rows, int n_out, int k) {
   const int n_pad = round_up(rows, 16);

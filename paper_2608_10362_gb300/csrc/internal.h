@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <string>
+
 namespace memspec {
 
 typedef __nv_bfloat16 bf16;
@@ -180,6 +182,10 @@ cudaError_t launch_sample(const SampleArgs& a, cudaStream_t s, bool pdl);
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t s, bool pdl);
 cudaError_t launch_rope_table(float* cos_t, float* sin_t, int max_seq, int half, float base,
                               cudaStream_t s);
+
+// Message returned by memspec_op_last_error() on this host thread.
+void set_op_error(const char* msg);
+inline void set_op_error(const std::string& msg) { set_op_error(msg.c_str()); }
 
 // Philox4x32-10 (Salmon et al., SC'11), device side.
 __host__ __device__ inline uint32_t philox_u01_bits(uint32_t c0, uint32_t c1, uint32_t c2,

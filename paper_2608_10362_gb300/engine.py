@@ -263,6 +263,20 @@ def op_linear(x: torch.Tensor, w: torch.Tensor, scratch: torch.Tensor | None = N
     return y
 
 
+def op_linear_noalloc(x: torch.Tensor, w: torch.Tensor,
+                      stream: torch.cuda.Stream | None = None) -> torch.Tensor:
+    """y = x . w^T through memspec_op_linear_noalloc (no scratch argument; the
+    library's fixed device array is used).  rows <= 16."""
+    lib = _lib.load()
+    rows, k = x.shape
+    n_out = w.shape[0]
+    y = torch.empty(rows, n_out, dtype=torch.float32, device=x.device)
+    s = stream or torch.cuda.current_stream(x.device)
+    _check(lib, lib.memspec_op_linear_noalloc(x.data_ptr(), w.data_ptr(), y.data_ptr(), rows,
+                                              n_out, k, None, s.cuda_stream))
+    return y
+
+
 def op_sample(logits: torch.Tensor, temperature: float, u: torch.Tensor | None = None):
     lib = _lib.load()
     rows, vocab = logits.shape
