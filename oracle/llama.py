@@ -99,19 +99,33 @@ class KVCache:
 class LlamaOracle:
     """One model (target or draft).  ``weights`` maps (name, layer) -> array."""
 
-    def __init__(self, shape, weights: dict):
+    def __init__(self, shape, weights: dict, keep_f64: bool = False):
+        """keep_f64: hold every matrix in float64 (memory for speed); otherwise
+        the matrices of the most recently used layer are kept converted."""
         self.shape = shape
         self.w = weights
         lm = ("tok_emb", -1) if shape.tied else ("lm_head", -1)
         self.lm_key = lm
+        self.keep_f64 = keep_f64
+        self._f64 = {}
+        self._f64_layer = None
 
     def new_cache(self, capacity: int) -> KVCache:
         s = self.shape
         return KVCache(s.n_layers, s.n_kv_heads, s.head_dim, capacity)
 
+    def _w64(self, name: str, layer: int) -> np.ndarray:
+        key = (name, layer)
+        if not self.keep_f64 and layer != self._f64_layer:
+            self._f64 = {}
+            self._f64_layer = layer
+        if key not in self._f64:
+            self._f64[key] = self.w[key].astype(np.float64)
+        return self._f64[key]
+
     def _lin(self, x: np.ndarray, name: str, layer: int) -> np.ndarray:
         # x [M, in] float64; W [out, in] float32 holding bf16 values -> x W^T in float64
-        return x @ self.w[(name, layer)].astype(np.float64).T
+        return x @ self._w64(name, layer).T
 
     def layer(self, li: int, h: np.ndarray, cache: KVCache, positions) -> np.ndarray:
         """One decoder layer over rows h [M, d]; appends their K, V to the cache."""
@@ -139,7 +153,7 @@ class LlamaOracle:
     def logits(self, h: np.ndarray) -> np.ndarray:
         s = self.shape
         hf = rmsnorm(h, self.w[("final_norm", -1)], s.norm_eps)
-        return hf @ self.w[self.lm_key].astype(np.float64).T
+        return hf @ self._w64(*self.lm_key).T
 
     def forward(self, cache: KVCache, tokens, want_logits: bool = True):
         """Feed ``tokens`` at positions cache.length .. cache.length+M-1.

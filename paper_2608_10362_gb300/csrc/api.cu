@@ -271,6 +271,9 @@ struct memspec_ctx {
   // workspace
   float* h = nullptr;
   bf16* xg = nullptr;
+  bf16* xg_lo = nullptr;   // low-order planes of the bf16 activations
+  bf16* o_lo = nullptr;
+  bf16* act_lo = nullptr;
   float* ss = nullptr;
   int ss_stride = kMaxRows;
   float* q = nullptr;
@@ -369,10 +372,13 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   WsPlan w;
   const size_t o_h = w.take(static_cast<size_t>(kMaxRows) * dmax * 4);
   const size_t o_xg = w.take(static_cast<size_t>(kMaxRows) * dmax * 2);
+  const size_t o_xgl = w.take(static_cast<size_t>(kMaxRows) * dmax * 2);
   const size_t o_ss = w.take(static_cast<size_t>(ceil_div(dmax, 128)) * kMaxRows * 4);
   const size_t o_q = w.take(static_cast<size_t>(kMaxRows) * qmax_dim * 4);
   const size_t o_o = w.take(static_cast<size_t>(kMaxRows) * qmax_dim * 2);
+  const size_t o_ol = w.take(static_cast<size_t>(kMaxRows) * qmax_dim * 2);
   const size_t o_act = w.take(static_cast<size_t>(kMaxRows) * fmax * 2);
+  const size_t o_actl = w.take(static_cast<size_t>(kMaxRows) * fmax * 2);
   const size_t o_gp = w.take(static_cast<size_t>(2) * nsm * kMaxRows * 128 * 4);
   const size_t o_gc = w.take(static_cast<size_t>(max_rt) * 4);
   const size_t o_apo = w.take(po * 4);
@@ -399,6 +405,9 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   if (c != nullptr) {
     c->h = reinterpret_cast<float*>(base + o_h);
     c->xg = reinterpret_cast<bf16*>(base + o_xg);
+    c->xg_lo = reinterpret_cast<bf16*>(base + o_xgl);
+    c->o_lo = reinterpret_cast<bf16*>(base + o_ol);
+    c->act_lo = reinterpret_cast<bf16*>(base + o_actl);
     c->ss = reinterpret_cast<float*>(base + o_ss);
     c->q = reinterpret_cast<float*>(base + o_q);
     c->o = reinterpret_cast<bf16*>(base + o_o);
@@ -506,11 +515,13 @@ int gemm_grid(int row_tiles, int k_tiles) {
 
 memspec_status run_gemm(memspec_ctx* c, GemmArgs& a, const char* what) {
   const int grid = gemm_grid(a.row_tiles, a.k_tiles);
-  a.stages = gemm_pick_stages(a.n_pad);
+  const int planes = a.split ? 2 : 1;
+  a.stages = gemm_pick_stages(a.n_pad, planes);
   a.partials = c->gemm_part;
   a.counters = c->gemm_cnt;
   a.status = c->status;
-  cudaError_t e = launch_gemm(a, grid, gemm_smem_bytes(a.n_pad, a.stages), c->main, c->pdl);
+  cudaError_t e =
+      launch_gemm(a, grid, gemm_smem_bytes(a.n_pad, a.stages, planes), c->main, c->pdl);
   if (e != cudaSuccess) return cuda_fail(c, e, what);
   return MEMSPEC_OK;
 }
@@ -540,6 +551,7 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
   ea.vocab = cf.vocab;
   ea.h = c->h;
   ea.xg = c->xg;
+  ea.xg_lo = c->xg_lo;
   ea.gain = reinterpret_cast<const bf16*>(m.w + m.lay.attn_norm[0]);
   ea.ss = c->ss;
   ea.ss_stride = c->ss_stride;
@@ -568,8 +580,10 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.row_tiles = ceil_div(a.n_out, 128);
       a.k_tiles = ceil_div(d, 64);
       a.l2_hint = m.l2_hint;
-      if (!act_map(c, c->xg, rows, d, n_pad, &a.map_b))
+      if (!act_map(c, c->xg, rows, d, n_pad, &a.map_b) ||
+          !act_map(c, c->xg_lo, rows, d, n_pad, &a.map_b2))
         return fail(c, MEMSPEC_ERR_CUDA, "activation tensor map");
+      a.split = 1;
       a.rms = 1;
       a.ss = c->ss;
       a.ss_count = ss_count;
@@ -609,6 +623,7 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       at.qmax = geo.qmax;
       at.counters = c->att_cnt;
       at.out = c->o;
+      at.out_lo = c->o_lo;
       at.plan = c->plan;
       at.status = c->status;
       e = launch_attention(at, f.n_groups, c->main, c->pdl);
@@ -624,14 +639,17 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.row_tiles = ceil_div(d, 128);
       a.k_tiles = ceil_div(qd, 64);
       a.l2_hint = m.l2_hint;
-      if (!act_map(c, c->o, rows, qd, n_pad, &a.map_b))
+      if (!act_map(c, c->o, rows, qd, n_pad, &a.map_b) ||
+          !act_map(c, c->o_lo, rows, qd, n_pad, &a.map_b2))
         return fail(c, MEMSPEC_ERR_CUDA, "activation tensor map");
+      a.split = 1;
       a.epi = EPI_RESIDUAL;
       a.h = c->h;
       a.h_ld = d;
       a.ss_out = c->ss;
       a.gain_next = reinterpret_cast<const bf16*>(m.w + m.lay.ffn_norm[l]);
       a.xg_out = c->xg;
+      a.xg_lo_out = c->xg_lo;
       a.ss_stride = c->ss_stride;
       a.plan = c->plan;
       memspec_status s = run_gemm(c, a, "o gemm launch");
@@ -650,8 +668,10 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.row_tiles = ceil_div(F, 64);
       a.k_tiles = ceil_div(d, 64);
       a.l2_hint = m.l2_hint;
-      if (!act_map(c, c->xg, rows, d, n_pad, &a.map_b))
+      if (!act_map(c, c->xg, rows, d, n_pad, &a.map_b) ||
+          !act_map(c, c->xg_lo, rows, d, n_pad, &a.map_b2))
         return fail(c, MEMSPEC_ERR_CUDA, "activation tensor map");
+      a.split = 1;
       a.rms = 1;
       a.ss = c->ss;
       a.ss_count = ss_count;
@@ -659,6 +679,7 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.eps = cf.norm_eps;
       a.epi = EPI_SWIGLU;
       a.act = c->act;
+      a.act_lo = c->act_lo;
       a.act_ld = F;
       a.plan = c->plan;
       memspec_status s = run_gemm(c, a, "gate/up gemm launch");
@@ -674,8 +695,10 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.row_tiles = ceil_div(d, 128);
       a.k_tiles = ceil_div(F, 64);
       a.l2_hint = m.l2_hint;
-      if (!act_map(c, c->act, rows, F, n_pad, &a.map_b))
+      if (!act_map(c, c->act, rows, F, n_pad, &a.map_b) ||
+          !act_map(c, c->act_lo, rows, F, n_pad, &a.map_b2))
         return fail(c, MEMSPEC_ERR_CUDA, "activation tensor map");
+      a.split = 1;
       a.epi = EPI_RESIDUAL;
       a.h = c->h;
       a.h_ld = d;
@@ -683,6 +706,7 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.gain_next = reinterpret_cast<const bf16*>(
           m.w + (l + 1 < cf.n_layers ? m.lay.attn_norm[l + 1] : m.lay.final_norm));
       a.xg_out = c->xg;
+      a.xg_lo_out = c->xg_lo;
       a.ss_stride = c->ss_stride;
       a.plan = c->plan;
       memspec_status s = run_gemm(c, a, "down gemm launch");
@@ -699,8 +723,10 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
     a.row_tiles = ceil_div(cf.vocab, 128);
     a.k_tiles = ceil_div(d, 64);
     a.l2_hint = m.l2_hint;
-    if (!act_map(c, c->xg, rows, d, n_pad, &a.map_b))
+    if (!act_map(c, c->xg, rows, d, n_pad, &a.map_b) ||
+        !act_map(c, c->xg_lo, rows, d, n_pad, &a.map_b2))
       return fail(c, MEMSPEC_ERR_CUDA, "activation tensor map");
+    a.split = 1;
     a.rms = 1;
     a.ss = c->ss;
     a.ss_count = ss_count;

@@ -9,6 +9,8 @@
 // tensor cores (mma.sync m16n8k16, bf16 in, fp32 accumulate):
 //   S = Q K^T (Q pre-scaled by log2(e)/sqrt(hd)), online softmax in registers
 //   (running max m, sum l), O += P V with P re-packed from the S fragments.
+// Q and P are carried as two bf16 planes (hi + lo, two MMAs each), so only the
+// bf16 K/V cache limits the precision; the output is written as hi + lo planes.
 // With few query vectors the four warps split each 64-key tile between them
 // and are merged at the end.  Each split writes (m, l, o) to a partial buffer;
 // the last-arriving split CTA of each (group, kv head, row block) combines them
@@ -110,8 +112,11 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
   const int mt = warp / kg, kgi = warp - mt * kg;
   const bool active = mt < n_mt;
 
-  uint8_t* qs = smem_raw;                                 // [64][HD] bf16, swizzled
-  uint8_t* kv = smem_raw + kMaxQ * HD * 2;                // kStages x (K tile, V tile)
+  uint8_t* kv = smem_raw;                                 // kStages x (K tile, V tile)
+  // Q (hi and lo planes, [64][HD] bf16 each, swizzled) is staged in the last
+  // pipeline stage, which the prologue leaves empty; the fragments move to
+  // registers before that stage is first filled.
+  uint8_t* qs = kv + (kStages - 1) * 2 * kTileBytes;
   const size_t kv_base = (static_cast<size_t>(req) * a.Hkv + kvh) * a.max_seq;
   const bf16* kc = a.kcache + kv_base * HD;
   const bf16* vc = a.vcache + kv_base * HD;
@@ -136,7 +141,7 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
   }
   for (int c = tid; c < kMaxQ * kChunks; c += kAttThreads) {
     const int v = c / kChunks, ch = c - v * kChunks;
-    __nv_bfloat16 e[8];
+    __nv_bfloat16 e[8], el[8];
     if (v < nq) {
       const int hl = v / nr, rr = v - hl * nr;
       const int row = g * R + r_lo + rr;
@@ -146,23 +151,26 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
       const float4 x1 = *reinterpret_cast<const float4*>(src + 4);
       const float f[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
 #pragma unroll
-      for (int i = 0; i < 8; ++i) e[i] = __float2bfloat16_rn(f[i] * a.scale_log2);
+      for (int i = 0; i < 8; ++i) split_bf16(f[i] * a.scale_log2, e[i], el[i]);
     } else {
 #pragma unroll
-      for (int i = 0; i < 8; ++i) e[i] = __float2bfloat16_rn(0.f);
+      for (int i = 0; i < 8; ++i) e[i] = el[i] = __float2bfloat16_rn(0.f);
     }
     *reinterpret_cast<uint4*>(qs + swz<HD>(v, ch)) = *reinterpret_cast<const uint4*>(e);
+    *reinterpret_cast<uint4*>(qs + kTileBytes + swz<HD>(v, ch)) = *reinterpret_cast<const uint4*>(el);
   }
   __syncthreads();
 
-  // Q fragments of this warp's m-tile stay in registers
-  uint32_t qa[HD / 16][4];
+  // Q fragments (hi and lo) of this warp's m-tile stay in registers
+  uint32_t qa[HD / 16][4], ql[HD / 16][4];
   if (active) {
 #pragma unroll
     for (int ks = 0; ks < HD / 16; ++ks) {
       const int row = mt * 16 + (lane & 15);
       const int ch = ks * 2 + (lane >> 4);
       ldsm_x4(smem_addr(qs) + swz<HD>(row, ch), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
+      ldsm_x4(smem_addr(qs + kTileBytes) + swz<HD>(row, ch), ql[ks][0], ql[ks][1], ql[ks][2],
+              ql[ks][3]);
     }
   }
   // positions of this thread's two rows (v = mt*16 + lane/4 and +8); -1: padding row
@@ -197,7 +205,9 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
         const int ch = ks * 2 + ((lane >> 3) & 1);
         ldsm_x4(ks_addr + swz<HD>(row, ch), b0, b1, b2, b3);
         mma16816(s0, qa[ks], b0, b1);
+        mma16816(s0, ql[ks], b0, b1);
         mma16816(s1, qa[ks], b2, b3);
+        mma16816(s1, ql[ks], b2, b3);
       }
       // causal / range mask, then online softmax (base 2)
       const int key_c = kt0 + kb + ((lane & 3) << 1);
@@ -245,11 +255,19 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
         o[i][2] *= scale[1];
         o[i][3] *= scale[1];
       }
-      uint32_t pa[4];
-      pa[0] = pack_bf16x2(s0[0], s0[1]);
-      pa[1] = pack_bf16x2(s0[2], s0[3]);
-      pa[2] = pack_bf16x2(s1[0], s1[1]);
-      pa[3] = pack_bf16x2(s1[2], s1[3]);
+      // P as hi + lo bf16 fragments
+      uint32_t pa[4], pl[4];
+      {
+        const float pv[8] = {s0[0], s0[1], s0[2], s0[3], s1[0], s1[1], s1[2], s1[3]};
+        float lo[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) lo[i] = pv[i] - __bfloat162float(__float2bfloat16_rn(pv[i]));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          pa[i] = pack_bf16x2(pv[2 * i], pv[2 * i + 1]);
+          pl[i] = pack_bf16x2(lo[2 * i], lo[2 * i + 1]);
+        }
+      }
 #pragma unroll
       for (int n2 = 0; n2 < HD / 16; ++n2) {
         uint32_t b0, b1, b2, b3;
@@ -257,7 +275,9 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
         const int ch = n2 * 2 + (lane >> 4);
         ldsm_x4_t(vs_addr + swz<HD>(row, ch), b0, b1, b2, b3);
         mma16816(o[2 * n2], pa, b0, b1);
+        mma16816(o[2 * n2], pl, b0, b1);
         mma16816(o[2 * n2 + 1], pa, b2, b3);
+        mma16816(o[2 * n2 + 1], pl, b2, b3);
       }
     }
   }
@@ -346,7 +366,12 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
     const int hl = v / nr, rr = v - hl * nr;
     const int row = g * R + r_lo + rr;
     const int h = kvh * gs + hl;
-    a.out[(static_cast<size_t>(row) * a.H + h) * HD + d] = __float2bfloat16_rn(O * linv[v]);
+    const size_t oi = (static_cast<size_t>(row) * a.H + h) * HD + d;
+    if (a.out_lo != nullptr) {
+      split_bf16(O * linv[v], a.out[oi], a.out_lo[oi]);
+    } else {
+      a.out[oi] = __float2bfloat16_rn(O * linv[v]);
+    }
   }
   if (tid == 0) a.counters[unit] = 0;
 }
@@ -354,10 +379,9 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
 }  // namespace
 
 size_t attention_smem_bytes(const AttnArgs& a) {
-  const size_t q = static_cast<size_t>(kMaxQ) * a.hd * 2;
   const size_t stages = static_cast<size_t>(kStages) * 2 * kKeyTile * a.hd * 2;
   const size_t merge = static_cast<size_t>(4) * 16 * a.hd * 4 + 4 * 16 * 2 * 4;
-  return q + (stages > merge ? stages : merge);
+  return stages > merge ? stages : merge;
 }
 
 cudaError_t attention_set_max_smem() {

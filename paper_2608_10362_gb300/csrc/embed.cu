@@ -122,6 +122,14 @@ __global__ void __launch_bounds__(256) embed_kernel(const __grid_constant__ Embe
     for (int q = 0; q < 8; ++q) o8[q] = __float2bfloat16_rn(f[q] * __bfloat162float(gb[q]));
     *reinterpret_cast<uint4*>(a.xg + static_cast<size_t>(r) * a.d + c) =
         *reinterpret_cast<const uint4*>(o8);
+    if (a.xg_lo != nullptr) {   // low-order plane: bf16(x - bf16(x))
+      __nv_bfloat16 l8[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        l8[q] = __float2bfloat16_rn(f[q] * __bfloat162float(gb[q]) - __bfloat162float(o8[q]));
+      *reinterpret_cast<uint4*>(a.xg_lo + static_cast<size_t>(r) * a.d + c) =
+          *reinterpret_cast<const uint4*>(l8);
+    }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);

@@ -27,6 +27,8 @@
 //    with K/V appended to the KV cache at each row's position.
 #include <cuda_bf16.h>
 
+#include <cstdlib>
+
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -38,7 +40,7 @@ constexpr int kThreads = 192;   // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
 constexpr int kTileM = 128;
 constexpr int kTileK = 64;
 constexpr int kABytes = kTileM * kTileK * 2;  // 16 KB
-constexpr int kMaxStages = 8;
+constexpr int kMaxStages = 12;
 constexpr int kStagePitch = 17;                // epilogue staging row pitch (floats)
 
 struct SmemCtl {
@@ -53,8 +55,19 @@ struct SmemCtl {
   float red[4][16];
 };
 
-__device__ __forceinline__ uint32_t tmem_cols_for(int n_pad) {
-  uint32_t need = 2u * static_cast<uint32_t>(n_pad);
+// MMA layouts of the activation operand:
+//   kPlain  one bf16 plane, N = n_pad
+//   kWide   hi and lo planes as one operand of N = 2 n_pad (one MMA per k-step);
+//           accumulator columns [0, n_pad) hold W.hi, [n_pad, 2 n_pad) W.lo
+//   kTwice  hi and lo planes as two MMAs into the same accumulator (2 n_pad > 256)
+enum BLayout : int { kPlain = 0, kWide = 1, kTwice = 2 };
+
+__device__ __forceinline__ int acc_cols(const GemmArgs& a, int layout) {
+  return layout == kWide ? 2 * a.n_pad : a.n_pad;
+}
+
+__device__ __forceinline__ uint32_t tmem_cols_for(int cols) {
+  uint32_t need = 2u * static_cast<uint32_t>(cols);
   uint32_t c = 32;
   while (c < need) c <<= 1;
   return c;
@@ -103,9 +116,15 @@ __device__ void apply_epilogue(const GemmArgs& a, SmemCtl& ctl, float* stage, co
         const float hn = *hp + v[j];
         *hp = hn;
         sq = hn * hn;
-        if (a.gain_next != nullptr)
-          a.xg_out[static_cast<size_t>(r) * a.h_ld + f] =
-              __float2bfloat16_rn(hn * __bfloat162float(a.gain_next[f]));
+        if (a.gain_next != nullptr) {
+          const float xv = hn * __bfloat162float(a.gain_next[f]);
+          const size_t o = static_cast<size_t>(r) * a.h_ld + f;
+          if (a.xg_lo_out != nullptr) {
+            split_bf16(xv, a.xg_out[o], a.xg_lo_out[o]);
+          } else {
+            a.xg_out[o] = __float2bfloat16_rn(xv);
+          }
+        }
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
@@ -137,7 +156,12 @@ __device__ void apply_epilogue(const GemmArgs& a, SmemCtl& ctl, float* stage, co
           const float g = stage[et * kStagePitch + j];
           const float u = stage[(et + 64) * kStagePitch + j];
           const float sg = g / (1.0f + expf(-g));
-          a.act[static_cast<size_t>(r) * a.act_ld + f] = __float2bfloat16_rn(sg * u);
+          const size_t o = static_cast<size_t>(r) * a.act_ld + f;
+          if (a.act_lo != nullptr) {
+            split_bf16(sg * u, a.act[o], a.act_lo[o]);
+          } else {
+            a.act[o] = __float2bfloat16_rn(sg * u);
+          }
         }
       }
     }
@@ -193,7 +217,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
   uint8_t* dsmem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const int S = a.stages;
-  const int b_bytes = a.n_pad * 128;
+  const int plane_bytes = a.n_pad * 128;              // one [n_pad][64] bf16 activation plane
+  const int b_bytes = plane_bytes * (a.split ? 2 : 1);
   const uint32_t stage_tx = static_cast<uint32_t>(kABytes + b_bytes);
   uint8_t* smem_a = dsmem;
   uint8_t* smem_b = dsmem + static_cast<size_t>(S) * kABytes;
@@ -205,7 +230,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
   const int G = gridDim.x, c = blockIdx.x;
   const int t_begin = sk_begin(c, T, G), t_end = sk_begin(c + 1, T, G);
   const int KT = a.k_tiles;
-  const uint32_t tmem_cols = tmem_cols_for(a.n_pad);
+  const int layout = !a.split ? kPlain : (2 * a.n_pad <= 256 ? kWide : kTwice);
+  const int acols = acc_cols(a, layout);                 // accumulator columns per buffer
+  const uint32_t tmem_cols = tmem_cols_for(acols);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -241,6 +268,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
       tma_prefetch_desc(&a.map_a);
       if (a.pair) tma_prefetch_desc(&a.map_a2);
       tma_prefetch_desc(&a.map_b);
+      if (a.split) tma_prefetch_desc(&a.map_b2);
       const uint64_t pol = a.l2_hint == L2_EVICT_FIRST  ? l2_policy_evict_first()
                            : a.l2_hint == L2_EVICT_LAST ? l2_policy_evict_last()
                                                         : l2_policy_evict_normal();
@@ -269,6 +297,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
         const int kt = t - (t / KT) * KT;
         tma_load_2d(smem_b + static_cast<size_t>(p) * b_bytes, &a.map_b, kt * kTileK, 0,
                     &ctl.full[p], pol_b);
+        if (a.split)
+          tma_load_2d(smem_b + static_cast<size_t>(p) * b_bytes + plane_bytes, &a.map_b2,
+                      kt * kTileK, 0, &ctl.full[p], pol_b);
       }
       it = n_pre;
       for (int t = t_begin + n_pre; t < t_end; ++t, ++it) {
@@ -289,6 +320,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
         }
         tma_load_2d(smem_b + static_cast<size_t>(s) * b_bytes, &a.map_b, kt * kTileK, 0,
                     &ctl.full[s], pol_b);
+        if (a.split)
+          tma_load_2d(smem_b + static_cast<size_t>(s) * b_bytes + plane_bytes, &a.map_b2,
+                      kt * kTileK, 0, &ctl.full[s], pol_b);
         issued_mask |= 1u << s;
         last_par = (last_par & ~(1u << s)) | (ph << s);
       }
@@ -300,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = make_idesc_bf16_f32(kTileM, a.n_pad);
+      const uint32_t idesc = make_idesc_bf16_f32(kTileM, layout == kWide ? 2 * a.n_pad : a.n_pad);
       int it = 0, seg = 0;
       bool ok = true;
       for (int t = t_begin; t < t_end && ok; ++seg) {
@@ -314,7 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
           break;
         }
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * a.n_pad);
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * acols);
         for (int tt = t; tt < seg_end; ++tt, ++it) {
           const int s = it % S;
           const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
@@ -325,11 +359,21 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
           tc_fence_after();
           const uint32_t a_addr = smem_addr(smem_a + static_cast<size_t>(s) * kABytes);
           const uint32_t b_addr = smem_addr(smem_b + static_cast<size_t>(s) * b_bytes);
+          if (layout != kTwice) {   // one MMA per k-step (N = n_pad or 2 n_pad)
 #pragma unroll
-          for (int kk = 0; kk < kTileK / 16; ++kk) {
-            tc_mma_bf16(d_tmem, make_smem_desc_sw128(a_addr + kk * 32),
-                        make_smem_desc_sw128(b_addr + kk * 32), idesc,
-                        (tt > t || kk > 0) ? 1u : 0u);
+            for (int kk = 0; kk < kTileK / 16; ++kk)
+              tc_mma_bf16(d_tmem, make_smem_desc_sw128(a_addr + kk * 32),
+                          make_smem_desc_sw128(b_addr + kk * 32), idesc,
+                          (tt > t || kk > 0) ? 1u : 0u);
+          } else {                  // hi then lo plane into the same accumulator
+#pragma unroll
+            for (int kk = 0; kk < kTileK / 16; ++kk) {
+              const uint64_t adesc = make_smem_desc_sw128(a_addr + kk * 32);
+              tc_mma_bf16(d_tmem, adesc, make_smem_desc_sw128(b_addr + kk * 32), idesc,
+                          (tt > t || kk > 0) ? 1u : 0u);
+              tc_mma_bf16(d_tmem, adesc, make_smem_desc_sw128(b_addr + plane_bytes + kk * 32),
+                          idesc, 1u);
+            }
           }
           tc_commit(&ctl.empty[s]);
         }
@@ -386,11 +430,21 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
       tc_fence_after();
       const bool full = (k0 == 0 && k1 == KT);
       const uint32_t tbase = tmem_base + (static_cast<uint32_t>(ew * 32) << 16) +
-                             static_cast<uint32_t>(buf * a.n_pad);
+                             static_cast<uint32_t>(buf * acols);
       float v[16];
+      // accumulator chunk (16 columns) -> v; the wide layout adds W.hi + W.lo
+      auto load_chunk = [&](int chunk) {
+        tmem_ld_32x32b_x16(tbase + chunk * 16, v);
+        if (layout == kWide) {
+          float lo[16];
+          tmem_ld_32x32b_x16(tbase + a.n_pad + chunk * 16, lo);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) v[j] += lo[j];
+        }
+      };
       if (full) {
         for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
-          tmem_ld_32x32b_x16(tbase + chunk * 16, v);
+          load_chunk(chunk);
           apply_epilogue(a, ctl, stage, rms, rt, chunk, et, v);
         }
       } else {
@@ -399,7 +453,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
         float* pb = a.partials + static_cast<size_t>(2 * c + slot) * a.n_pad * kTileM +
                     static_cast<size_t>(et) * a.n_pad;
         for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
-          tmem_ld_32x32b_x16(tbase + chunk * 16, v);
+          load_chunk(chunk);
           float4* dst = reinterpret_cast<float4*>(pb + chunk * 16);
 #pragma unroll
           for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
@@ -470,9 +524,23 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
 
 }  // namespace
 
-int gemm_pick_stages(int n_pad) {
-  const int stage = kABytes + n_pad * 128;
-  const int budget = n_pad <= 32 ? 104 * 1024 : 200 * 1024;
+// Shared-memory budget of the stage ring.  A deep ring keeps more weight bytes
+// in flight per SM; a budget under ~110 KB lets the next kernel's CTA start on
+// the same SM early (programmatic dependent launch).  MEMSPEC_GEMM_SMEM_KB
+// overrides the default (for measurement).
+static int gemm_budget_bytes(int n_pad) {
+  static int env_kb = -1;
+  if (env_kb < 0) {
+    const char* e = std::getenv("MEMSPEC_GEMM_SMEM_KB");
+    env_kb = e != nullptr ? std::atoi(e) : 0;
+  }
+  if (env_kb > 0) return env_kb * 1024;
+  return n_pad <= 32 ? 200 * 1024 : 200 * 1024;
+}
+
+int gemm_pick_stages(int n_pad, int planes) {
+  const int stage = kABytes + n_pad * 128 * planes;
+  const int budget = gemm_budget_bytes(n_pad);
   const int fixed = kTileM * kStagePitch * 4 + kMaxRows * 4 + 1024;
   int s = (budget - fixed) / stage;
   if (s > kMaxStages) s = kMaxStages;
@@ -480,8 +548,8 @@ int gemm_pick_stages(int n_pad) {
   return s;
 }
 
-size_t gemm_smem_bytes(int n_pad, int stages) {
-  return static_cast<size_t>(stages) * (kABytes + n_pad * 128) + kTileM * kStagePitch * 4 +
+size_t gemm_smem_bytes(int n_pad, int stages, int planes) {
+  return static_cast<size_t>(stages) * (kABytes + n_pad * 128 * planes) + kTileM * kStagePitch * 4 +
          kMaxRows * 4 + 1024;
 }
 

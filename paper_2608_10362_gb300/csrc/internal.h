@@ -57,6 +57,7 @@ struct EmbedArgs {
   int d, vocab;
   float* h;                 // [rows][d] residual stream
   bf16* xg;                 // [rows][d] bf16(h * gain) for the first projection
+  bf16* xg_lo;              // its low-order plane
   const bf16* gain;         // first RMSNorm gain
   float* ss;                // [ss_tiles][ss_stride]: row sums of squares (partial)
   int ss_stride;
@@ -71,6 +72,8 @@ struct GemmArgs {
   CUtensorMap map_a;        // weights [n_out][k] bf16, box {64, 128} (or {64, 64} for pairs)
   CUtensorMap map_a2;       // second matrix of a SwiGLU pair (up), box {64, 64}
   CUtensorMap map_b;        // activations [rows_total][k] bf16, box {64, n_pad}
+  CUtensorMap map_b2;       // low-order plane of the activations (split), same shape
+  int split;                // 1: activations = hi + lo bf16 planes, two MMAs per k-step
   int n_out;                // output features (F for pairs)
   int k_in;
   int pair;                 // 1: tile = 64 rows of map_a + 64 rows of map_a2
@@ -98,7 +101,9 @@ struct GemmArgs {
   float* ss_out;            // EPI_RESIDUAL: [row_tiles][ss_stride]
   const bf16* gain_next;    // EPI_RESIDUAL: gain of the next RMSNorm (nullptr: no xg)
   bf16* xg_out;             // EPI_RESIDUAL: bf16(h_new * gain_next) [rows][h_ld]
+  bf16* xg_lo_out;          // EPI_RESIDUAL: low-order plane (nullptr: none)
   bf16* act;                // EPI_SWIGLU: [rows][act_ld]
+  bf16* act_lo;             // EPI_SWIGLU: low-order plane (nullptr: none)
   int act_ld;
   float* q_out;             // EPI_QKV: fp32 [rows][q_dim]
   int q_dim, kv_dim, head_dim, n_kv_heads, max_seq;
@@ -125,6 +130,7 @@ struct AttnArgs {
   int qmax;                 // group_size * rows_per_block
   int* counters;            // [groups][Hkv][row_blocks]
   bf16* out;                // [rows][H][hd]
+  bf16* out_lo;             // low-order plane of out
   const RowPlan* plan;
   uint32_t* status;
 };
@@ -172,8 +178,8 @@ struct AcceptArgs {
 // launchers (each returns the launch's cudaError_t)
 cudaError_t launch_embed(const EmbedArgs& a, int rows, cudaStream_t s, bool pdl);
 cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s, bool pdl);
-size_t gemm_smem_bytes(int n_pad, int stages);
-int gemm_pick_stages(int n_pad);
+size_t gemm_smem_bytes(int n_pad, int stages, int planes = 1);
+int gemm_pick_stages(int n_pad, int planes = 1);
 cudaError_t gemm_set_max_smem();
 cudaError_t launch_attention(const AttnArgs& a, int n_groups, cudaStream_t s, bool pdl);
 size_t attention_smem_bytes(const AttnArgs& a);
@@ -182,6 +188,13 @@ cudaError_t launch_sample(const SampleArgs& a, cudaStream_t s, bool pdl);
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t s, bool pdl);
 cudaError_t launch_rope_table(float* cos_t, float* sin_t, int max_seq, int half, float base,
                               cudaStream_t s);
+
+// x ~= hi + lo with hi = bf16(x), lo = bf16(x - hi): two bf16 planes carry about
+// 16 significant bits, so bf16 tensor-core products see (almost) fp32 inputs.
+__device__ __forceinline__ void split_bf16(float x, bf16& hi, bf16& lo) {
+  hi = __float2bfloat16_rn(x);
+  lo = __float2bfloat16_rn(x - __bfloat162float(hi));
+}
 
 // Message returned by memspec_op_last_error() on this host thread.
 void set_op_error(const char* msg);
