@@ -194,6 +194,13 @@ AttnGeo attn_geometry(const memspec_model_cfg& c, int groups, int R, int max_seq
   want = std::min(want, max_splits);
   g.chunk = round_up(ceil_div(max_seq, want), 64);
   g.n_splits = ceil_div(max_seq, g.chunk);
+  // the combine keeps (n_splits + 1) x qmax floats of split weights in the CTA's
+  // shared memory (3 stages x 64 keys x hd x 2 x 2 bytes, last 16 bytes reserved)
+  const size_t smem = static_cast<size_t>(3) * 2 * 64 * c.head_dim * 2 - 16;
+  while (static_cast<size_t>(g.n_splits + 1) * g.qmax * 4 > smem) {
+    g.chunk *= 2;
+    g.n_splits = ceil_div(max_seq, g.chunk);
+  }
   return g;
 }
 

@@ -1,0 +1,371 @@
+// attn_body.cuh - split-KV attention CTA body, shared by the attention kernel and
+// the persistent pass kernel (see attention.cu for the algorithm).
+#pragma once
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace memspec {
+namespace attn {
+
+constexpr int kAttThreads = 128;
+constexpr int kKeyTile = 64;
+constexpr int kStages = 3;
+constexpr int kMaxQ = 64;   // query vectors per CTA (4 m-tiles of 16)
+
+__device__ __forceinline__ void cp_async16_zfill(void* smem_dst, const void* gsrc, bool valid) {
+  const int n = valid ? 16 : 0;
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(smem_dst)),
+               "l"(gsrc), "r"(n)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 t = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&t);
+}
+
+// byte offset of 16-byte chunk `ch` of row `row` in a swizzled [rows][HD] bf16 tile
+template <int HD>
+__device__ __forceinline__ uint32_t swz(int row, int ch) {
+  return static_cast<uint32_t>(row * (HD * 2) + ((ch ^ (row & 7)) << 4));
+}
+
+template <int HD>
+__host__ __device__ constexpr size_t attention_smem_bytes_hd() {
+  // kStages x (K tile + V tile); the merge buffers reuse it; the last 16 bytes hold a flag
+  return static_cast<size_t>(kStages) * 2 * kKeyTile * HD * 2 >
+                 static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + 16
+             ? static_cast<size_t>(kStages) * 2 * kKeyTile * HD * 2
+             : static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + 16;
+}
+
+// One CTA of split-KV attention for unit (g, kvh, rb, split), run by 128 threads
+// (tid 0..127); `sync` is a barrier over exactly those threads; smem_raw is the
+// CTA's attention shared memory (attention_smem_bytes).  Returns early, all
+// threads together, when the unit has no work.
+template <int HD, class Sync>
+__device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh, int rb, int split,
+                                              uint8_t* smem_raw, int tid, Sync sync) {
+  constexpr int kChunks = HD / 8;                        // 16-byte chunks per row
+  constexpr int kTileBytes = kKeyTile * HD * 2;          // one K (or V) tile
+  constexpr int kNT = HD / 8;                            // n8 tiles of the output
+  const RowPlan* plan = a.plan;
+  if (g >= plan->n_groups) return;
+  const int R = plan->rows_per_group;
+  const int req = plan->req[g], valid = plan->valid[g], pos0 = plan->pos0[g];
+  const int r_lo = rb * a.rows_per_block;
+  const int r_hi = min(r_lo + a.rows_per_block, valid);
+  if (r_lo >= r_hi) return;
+  const int nr = r_hi - r_lo;
+  const int gs = a.H / a.Hkv;
+  const int nq = gs * nr;
+  const int kmax = pos0 + r_hi - 1;
+  if (pos0 < 0 || kmax >= a.max_seq || nq > kMaxQ) {   // reported, never read
+    if (threadIdx.x == 0 && split == 0) atomicOr(a.status, 0x4u);
+    return;
+  }
+  const int n_active = (kmax + a.chunk) / a.chunk;   // ceil((kmax + 1) / chunk)
+  if (split >= n_active) return;
+  const int k0 = split * a.chunk;
+  const int k1 = min(k0 + a.chunk, kmax + 1);
+  const int n_tiles = (k1 - k0 + kKeyTile - 1) / kKeyTile;
+
+  const int n_mt = (nq + 15) >> 4;
+  const int kg = n_mt == 1 ? 4 : (n_mt == 2 ? 2 : 1);    // warps per m-tile (key groups)
+  const int warp = tid >> 5, lane = tid & 31;
+  const int mt = warp / kg, kgi = warp - mt * kg;
+  const bool active = mt < n_mt;
+
+  uint8_t* kv = smem_raw;                                 // kStages x (K tile, V tile)
+  // Q (hi and lo planes, [64][HD] bf16 each, swizzled) is staged in the last
+  // pipeline stage, which the prologue leaves empty; the fragments move to
+  // registers before that stage is first filled.
+  uint8_t* qs = kv + (kStages - 1) * 2 * kTileBytes;
+  const size_t kv_base = (static_cast<size_t>(req) * a.Hkv + kvh) * a.max_seq;
+  const bf16* kc = a.kcache + kv_base * HD;
+  const bf16* vc = a.vcache + kv_base * HD;
+
+  auto load_tile = [&](int t) {
+    uint8_t* ks = kv + (t % kStages) * 2 * kTileBytes;
+    uint8_t* vs = ks + kTileBytes;
+    const int kt0 = k0 + t * kKeyTile;
+    for (int c = tid; c < kKeyTile * kChunks; c += kAttThreads) {
+      const int row = c / kChunks, ch = c - row * kChunks;
+      const bool ok = kt0 + row < k1;
+      const size_t off = ok ? static_cast<size_t>(kt0 + row) * HD + ch * 8 : 0;
+      cp_async16_zfill(ks + swz<HD>(row, ch), kc + off, ok);
+      cp_async16_zfill(vs + swz<HD>(row, ch), vc + off, ok);
+    }
+  };
+
+  // prologue: start the first kStages-1 tiles, then stage Q (fp32 -> bf16, scaled)
+  for (int s = 0; s < kStages - 1; ++s) {
+    if (s < n_tiles) load_tile(s);
+    cp_async_commit();
+  }
+  for (int c = tid; c < kMaxQ * kChunks; c += kAttThreads) {
+    const int v = c / kChunks, ch = c - v * kChunks;
+    __nv_bfloat16 e[8], el[8];
+    if (v < nq) {
+      const int hl = v / nr, rr = v - hl * nr;
+      const int row = g * R + r_lo + rr;
+      const int h = kvh * gs + hl;
+      const float* src = a.q + (static_cast<size_t>(row) * a.H + h) * HD + ch * 8;
+      const float4 x0 = *reinterpret_cast<const float4*>(src);
+      const float4 x1 = *reinterpret_cast<const float4*>(src + 4);
+      const float f[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+      for (int i = 0; i < 8; ++i) split_bf16(f[i] * a.scale_log2, e[i], el[i]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) e[i] = el[i] = __float2bfloat16_rn(0.f);
+    }
+    *reinterpret_cast<uint4*>(qs + swz<HD>(v, ch)) = *reinterpret_cast<const uint4*>(e);
+    *reinterpret_cast<uint4*>(qs + kTileBytes + swz<HD>(v, ch)) = *reinterpret_cast<const uint4*>(el);
+  }
+  sync();
+
+  // Q fragments (hi and lo) of this warp's m-tile stay in registers
+  uint32_t qa[HD / 16][4], ql[HD / 16][4];
+  if (active) {
+#pragma unroll
+    for (int ks = 0; ks < HD / 16; ++ks) {
+      const int row = mt * 16 + (lane & 15);
+      const int ch = ks * 2 + (lane >> 4);
+      ldsm_x4(smem_addr(qs) + swz<HD>(row, ch), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
+      ldsm_x4(smem_addr(qs + kTileBytes) + swz<HD>(row, ch), ql[ks][0], ql[ks][1], ql[ks][2],
+              ql[ks][3]);
+    }
+  }
+  // positions of this thread's two rows (v = mt*16 + lane/4 and +8); -1: padding row
+  int prow[2];
+#pragma unroll
+  for (int h2 = 0; h2 < 2; ++h2) {
+    const int v = mt * 16 + (lane >> 2) + 8 * h2;
+    prow[h2] = (active && v < nq) ? pos0 + r_lo + (v % nr) : -1;
+  }
+  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  float o[kNT][4];
+#pragma unroll
+  for (int i = 0; i < kNT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+
+  const int sub_per_warp = (kKeyTile / 16) / kg;          // 16-key sub-blocks per warp per tile
+  for (int t = 0; t < n_tiles; ++t) {
+    cp_async_wait<kStages - 2>();
+    sync();
+    if (t + kStages - 1 < n_tiles) load_tile(t + kStages - 1);
+    cp_async_commit();
+    if (!active) continue;
+    const uint32_t ks_addr = smem_addr(kv + (t % kStages) * 2 * kTileBytes);
+    const uint32_t vs_addr = ks_addr + kTileBytes;
+    const int kt0 = k0 + t * kKeyTile;
+    for (int sb = 0; sb < sub_per_warp; ++sb) {
+      const int kb = (kgi * sub_per_warp + sb) * 16;      // key offset within the tile
+      float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int ks = 0; ks < HD / 16; ++ks) {
+        uint32_t b0, b1, b2, b3;
+        const int row = kb + (lane & 7) + ((lane >> 4) << 3);
+        const int ch = ks * 2 + ((lane >> 3) & 1);
+        ldsm_x4(ks_addr + swz<HD>(row, ch), b0, b1, b2, b3);
+        mma16816(s0, qa[ks], b0, b1);
+        mma16816(s0, ql[ks], b0, b1);
+        mma16816(s1, qa[ks], b2, b3);
+        mma16816(s1, ql[ks], b2, b3);
+      }
+      // causal / range mask, then online softmax (base 2)
+      const int key_c = kt0 + kb + ((lane & 3) << 1);
+      float mx[2];
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const int p = prow[h2];
+        const int lim = min(p, k1 - 1);
+        float* a0 = s0 + 2 * h2;
+        float* a1 = s1 + 2 * h2;
+        a0[0] = (key_c <= lim) ? a0[0] : -INFINITY;
+        a0[1] = (key_c + 1 <= lim) ? a0[1] : -INFINITY;
+        a1[0] = (key_c + 8 <= lim) ? a1[0] : -INFINITY;
+        a1[1] = (key_c + 9 <= lim) ? a1[1] : -INFINITY;
+        mx[h2] = fmaxf(fmaxf(a0[0], a0[1]), fmaxf(a1[0], a1[1]));
+        mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 1));
+        mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 2));
+      }
+      float scale[2];
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const float m_new = fmaxf(m_run[h2], mx[h2]);
+        float* a0 = s0 + 2 * h2;
+        float* a1 = s1 + 2 * h2;
+        if (m_new == -INFINITY) {
+          scale[h2] = 1.f;
+          a0[0] = a0[1] = a1[0] = a1[1] = 0.f;
+        } else {
+          scale[h2] = exp2f(m_run[h2] - m_new);
+          a0[0] = exp2f(a0[0] - m_new);
+          a0[1] = exp2f(a0[1] - m_new);
+          a1[0] = exp2f(a1[0] - m_new);
+          a1[1] = exp2f(a1[1] - m_new);
+        }
+        float rs = (a0[0] + a0[1]) + (a1[0] + a1[1]);
+        rs += __shfl_xor_sync(0xffffffffu, rs, 1);
+        rs += __shfl_xor_sync(0xffffffffu, rs, 2);
+        l_run[h2] = l_run[h2] * scale[h2] + rs;
+        m_run[h2] = m_new;
+      }
+#pragma unroll
+      for (int i = 0; i < kNT; ++i) {
+        o[i][0] *= scale[0];
+        o[i][1] *= scale[0];
+        o[i][2] *= scale[1];
+        o[i][3] *= scale[1];
+      }
+      // P as hi + lo bf16 fragments
+      uint32_t pa[4], pl[4];
+      {
+        const float pv[8] = {s0[0], s0[1], s0[2], s0[3], s1[0], s1[1], s1[2], s1[3]};
+        float lo[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) lo[i] = pv[i] - __bfloat162float(__float2bfloat16_rn(pv[i]));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          pa[i] = pack_bf16x2(pv[2 * i], pv[2 * i + 1]);
+          pl[i] = pack_bf16x2(lo[2 * i], lo[2 * i + 1]);
+        }
+      }
+#pragma unroll
+      for (int n2 = 0; n2 < HD / 16; ++n2) {
+        uint32_t b0, b1, b2, b3;
+        const int row = kb + (lane & 7) + (((lane >> 3) & 1) << 3);
+        const int ch = n2 * 2 + (lane >> 4);
+        ldsm_x4_t(vs_addr + swz<HD>(row, ch), b0, b1, b2, b3);
+        mma16816(o[2 * n2], pa, b0, b1);
+        mma16816(o[2 * n2], pl, b0, b1);
+        mma16816(o[2 * n2 + 1], pa, b2, b3);
+        mma16816(o[2 * n2 + 1], pl, b2, b3);
+      }
+    }
+  }
+  cp_async_wait<0>();
+  sync();
+
+  // merge the key groups of each m-tile (shared memory reuses the K/V stages)
+  float* mo = reinterpret_cast<float*>(kv);                 // [4 warps][16][HD]
+  float* ml = mo + 4 * 16 * HD;                             // [4 warps][16][2]
+  if (active) {
+    const int r0 = lane >> 2, cc = (lane & 3) << 1;
+#pragma unroll
+    for (int i = 0; i < kNT; ++i) {
+      float* dst = mo + (warp * 16) * HD + i * 8 + cc;
+      dst[r0 * HD] = o[i][0];
+      dst[r0 * HD + 1] = o[i][1];
+      dst[(r0 + 8) * HD] = o[i][2];
+      dst[(r0 + 8) * HD + 1] = o[i][3];
+    }
+    if ((lane & 3) == 0) {
+      ml[(warp * 16 + r0) * 2] = m_run[0];
+      ml[(warp * 16 + r0) * 2 + 1] = l_run[0];
+      ml[(warp * 16 + r0 + 8) * 2] = m_run[1];
+      ml[(warp * 16 + r0 + 8) * 2 + 1] = l_run[1];
+    }
+  }
+  sync();
+  const int unit = (g * a.Hkv + kvh) * a.row_blocks + rb;
+  const size_t pbase = (static_cast<size_t>(unit) * a.n_splits + split) * a.qmax;
+  for (int idx = tid; idx < nq * HD; idx += kAttThreads) {
+    const int v = idx / HD, d = idx - v * HD;
+    const int m_t = v >> 4, r = v & 15;
+    float M = -INFINITY;
+    for (int w = 0; w < kg; ++w) M = fmaxf(M, ml[((m_t * kg + w) * 16 + r) * 2]);
+    float L = 0.f, O = 0.f;
+    for (int w = 0; w < kg; ++w) {
+      const int ww = m_t * kg + w;
+      const float mw = ml[(ww * 16 + r) * 2];
+      const float f = mw == -INFINITY ? 0.f : exp2f(mw - M);
+      L += f * ml[(ww * 16 + r) * 2 + 1];
+      O += f * mo[(ww * 16 + r) * HD + d];
+    }
+    a.part_o[(pbase + v) * HD + d] = O;
+    if (d == 0) {
+      a.part_ml[(pbase + v) * 2 + 0] = M;
+      a.part_ml[(pbase + v) * 2 + 1] = L;
+    }
+  }
+  __threadfence();
+  sync();
+  int* last = reinterpret_cast<int*>(kv + attention_smem_bytes_hd<HD>() - 16);
+  if (tid == 0) *last = (atomicAdd(&a.counters[unit], 1) == n_active - 1) ? 1 : 0;
+  sync();
+  if (!*last) return;
+  __threadfence();
+  const size_t ubase = static_cast<size_t>(unit) * a.n_splits * a.qmax;
+  // split weights 2^(m_s - M) and 1/L per query vector, computed once in shared memory
+  float* wsm = reinterpret_cast<float*>(kv);                // [n_active][nq]
+  float* linv = wsm + n_active * nq;                        // [nq]
+  for (int v = tid; v < nq; v += kAttThreads) {
+    float M = -INFINITY;
+    for (int s = 0; s < n_active; ++s) M = fmaxf(M, ld_cg_f(a.part_ml + (ubase + s * a.qmax + v) * 2));
+    float L = 0.f;
+    for (int s = 0; s < n_active; ++s) {
+      const size_t pv = ubase + s * a.qmax + v;
+      const float ms = ld_cg_f(a.part_ml + pv * 2);
+      const float w = ms == -INFINITY ? 0.f : exp2f(ms - M);
+      wsm[s * nq + v] = w;
+      L += w * ld_cg_f(a.part_ml + pv * 2 + 1);
+    }
+    linv[v] = 1.f / L;
+  }
+  sync();
+  for (int idx = tid; idx < nq * HD; idx += kAttThreads) {
+    const int v = idx / HD, d = idx - v * HD;
+    float O = 0.f;
+    for (int s0 = 0; s0 < n_active; s0 += 4) {   // four splits fetched at once, summed in order
+      float ov[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        ov[q] = (s0 + q < n_active) ? ld_cg_f(a.part_o + (ubase + (s0 + q) * a.qmax + v) * HD + d) : 0.f;
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if (s0 + q < n_active) O += wsm[(s0 + q) * nq + v] * ov[q];
+    }
+    const int hl = v / nr, rr = v - hl * nr;
+    const int row = g * R + r_lo + rr;
+    const int h = kvh * gs + hl;
+    const size_t oi = (static_cast<size_t>(row) * a.H + h) * HD + d;
+    if (a.out_lo != nullptr) {
+      split_bf16(O * linv[v], a.out[oi], a.out_lo[oi]);
+    } else {
+      a.out[oi] = __float2bfloat16_rn(O * linv[v]);
+    }
+  }
+  if (tid == 0) a.counters[unit] = 0;
+}
+
+
+}  // namespace attn
+}  // namespace memspec

@@ -1,402 +1,31 @@
-// sampling.cu - vocab-wide softmax statistics, categorical sampling with Philox
-// uniforms, speculative-sampling acceptance, residual resampling, and the
-// commit / rollback of the sequence state.
-//
-// Acceptance (Leviathan et al. ICML'23 Alg. 1, which MemSpec cites and runs
-// unchanged, Section 3.5): with p_i = softmax(z_target,i / T) and
-// q_i = softmax(z_draft,i / T), draft token x_i is accepted iff
-// u_i * q_i(x_i) <= p_i(x_i); at the first rejection n, the extra token is drawn
-// from norm(max(0, p_{n+1} - q_{n+1})) (from p_{n+1} if that residual has no
-// mass); if all K are accepted it is drawn from p_{K+1}.  T == 0 is greedy:
-// accept while x_i == argmax p_i, extra token = argmax p_{n+1}.
-//
-// Categorical sampling of weights w with uniform u returns the smallest id j with
-// sum_{i<=j} w_i > u * sum_i w_i (weights summed in a fixed order: tiles of
-// blockDim*4 consecutive ids, tile sums added in id order).
-#include <float.h>
-
+// sampling.cu - the draft-token sampler and the acceptance / resample / commit
+// kernel (algorithms in sample_body.cuh).
 #include "internal.h"
 #include "ptx.cuh"
+#include "sample_body.cuh"
 
 namespace memspec {
 
 namespace {
 
+using namespace smp;
+
 constexpr int kSThreads = 512;
-constexpr int kSWarps = kSThreads / 32;
-constexpr int kMaxTiles = 1024;        // 128-id tiles: vocab <= 131072
 
-struct RowStats {
-  float m;     // max of z * inv_temp   (greedy: max of z)
-  float s;     // sum exp(z * inv_temp - m)
-  int arg;     // first index of the maximum
-};
-
-// Block-wide sum in a fixed order (warp xor-tree, then warps 0..n in order).
-__device__ float block_sum(float v, float* scratch) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  __syncthreads();
-  if (lane == 0) scratch[w] = v;
-  __syncthreads();
-  float t = 0.f;
-  for (int i = 0; i < kSWarps; ++i) t += scratch[i];
-  return t;
-}
-
-__device__ __forceinline__ void stats_update(float raw, int x, bool greedy, float inv_temp,
-                                             float& m, float& s, int& arg) {
-  if (raw > m) {
-    if (!greedy) s = (m == -INFINITY) ? 0.f : s * __expf((m - raw) * inv_temp);
-    m = raw;
-    arg = x;
-  }
-  if (!greedy) s += __expf((raw - m) * inv_temp);
-}
-
-// max / first-argmax / rescaled exp-sum of one row, whole block.
-__device__ RowStats row_stats(const float* z, int V, float inv_temp, bool greedy, float* scr_f,
-                              int* scr_i) {
-  float m = -INFINITY, s = 0.f;
-  int arg = 0x7fffffff;
-  if ((V & 3) == 0 && (reinterpret_cast<uintptr_t>(z) & 15) == 0) {
-    const float4* z4 = reinterpret_cast<const float4*>(z);
-    const int V4 = V >> 2;
-#pragma unroll 4
-    for (int x4 = threadIdx.x; x4 < V4; x4 += kSThreads) {
-      const float4 r = __ldcg(z4 + x4);
-      stats_update(r.x, 4 * x4, greedy, inv_temp, m, s, arg);
-      stats_update(r.y, 4 * x4 + 1, greedy, inv_temp, m, s, arg);
-      stats_update(r.z, 4 * x4 + 2, greedy, inv_temp, m, s, arg);
-      stats_update(r.w, 4 * x4 + 3, greedy, inv_temp, m, s, arg);
-    }
-  } else {
-#pragma unroll 4
-    for (int x = threadIdx.x; x < V; x += kSThreads) stats_update(__ldcg(z + x), x, greedy, inv_temp, m, s, arg);
-  }
-  // block combine: max first (with first index), then sums rescaled to it
-  float bm = m;
-  int ba = arg;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float om = __shfl_xor_sync(0xffffffffu, bm, o);
-    const int oa = __shfl_xor_sync(0xffffffffu, ba, o);
-    if (om > bm || (om == bm && oa < ba)) {
-      bm = om;
-      ba = oa;
-    }
-  }
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  __syncthreads();
-  if (lane == 0) {
-    scr_f[w] = bm;
-    scr_i[w] = ba;
-  }
-  __syncthreads();
-  float M = -INFINITY;
-  int A = 0x7fffffff;
-  for (int i = 0; i < kSWarps; ++i) {
-    if (scr_f[i] > M || (scr_f[i] == M && scr_i[i] < A)) {
-      M = scr_f[i];
-      A = scr_i[i];
-    }
-  }
-  RowStats r;
-  r.m = M * (greedy ? 1.f : inv_temp);
-  r.arg = A;
-  r.s = 0.f;
-  if (!greedy) {
-    const float mine = (m == -INFINITY) ? 0.f : s * __expf((m - M) * inv_temp);
-    r.s = block_sum(mine, scr_f + kSWarps);
-  }
-  return r;
-}
-
-// Smallest id j in [0, V) with sum_{i<=j} w(i) > u * sum w; whole block.
-// w(i) must be >= 0.  Returns -1 if the total weight is zero.  Weights are
-// summed in a fixed order: tiles of 128 consecutive ids (4 per lane, lanes
-// combined by a fixed shuffle tree), tiles combined in id order.
-template <class W>
-__device__ int block_sample(const W& wfun, int V, float u, float* tile_sums, float* scr,
-                            float* total_out) {
-  (void)scr;
-  constexpr int kTile = 128;
-  const int ntiles = (V + kTile - 1) / kTile;
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-#pragma unroll 2
-  for (int tile = w; tile < ntiles; tile += kSWarps) {
-    const int x0 = tile * kTile + lane * 4;
-    float own = 0.f;
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      if (x0 + q < V) own += wfun(x0 + q);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) own += __shfl_xor_sync(0xffffffffu, own, o);
-    if (lane == 0) tile_sums[tile] = own;
-  }
-  __syncthreads();
-  __shared__ int sh_pick;
-  if (w == 0) {
-    // each lane owns a contiguous range of tiles
-    const int tpl = (ntiles + 31) / 32;
-    const int t_lo = min(lane * tpl, ntiles), t_hi = min(t_lo + tpl, ntiles);
-    float ls = 0.f;
-    for (int t = t_lo; t < t_hi; ++t) ls += tile_sums[t];
-    float incl = ls;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const float n = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += n;
-    }
-    float excl = __shfl_up_sync(0xffffffffu, incl, 1);
-    if (lane == 0) excl = 0.f;
-    const float total = __shfl_sync(0xffffffffu, incl, 31);
-    const float target = u * total;
-    int sel = -1;
-    float before = 0.f;
-    if (ls > 0.f && excl <= target && target < incl) {
-      float c = excl;
-      for (int t = t_lo; t < t_hi; ++t) {
-        if (tile_sums[t] > 0.f) {
-          sel = t;
-          before = c;
-          if (c + tile_sums[t] > target) break;
-        }
-        c += tile_sums[t];
-      }
-    }
-    // the claiming lane (at most one: ranges chain exactly); otherwise the last tile with mass
-    unsigned claim = __ballot_sync(0xffffffffu, sel >= 0);
-    int last_lane = 31 - __clz(__ballot_sync(0xffffffffu, ls > 0.f) | 1u);
-    int src = claim ? (__ffs(claim) - 1) : last_lane;
-    if (!claim && lane == src) {   // rounding put the target at/after the end: last tile with mass
-      float c = excl;
-      for (int t = t_lo; t < t_hi; ++t) {
-        if (tile_sums[t] > 0.f) {
-          sel = t;
-          before = c;
-        }
-        c += tile_sums[t];
-      }
-    }
-    sel = __shfl_sync(0xffffffffu, sel, src);
-    before = __shfl_sync(0xffffffffu, before, src);
-    int pick = -1;
-    if (total > 0.f && sel >= 0) {
-      const float r = target - before;
-      const int x0 = sel * kTile + lane * 4;
-      float wv[4], own = 0.f;
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        wv[q] = (x0 + q < V) ? wfun(x0 + q) : 0.f;
-        own += wv[q];
-      }
-      float in2 = own;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const float n = __shfl_up_sync(0xffffffffu, in2, o);
-        if (lane >= o) in2 += n;
-      }
-      float ex2 = __shfl_up_sync(0xffffffffu, in2, 1);
-      if (lane == 0) ex2 = 0.f;
-      int mine = -1;
-      if (own > 0.f && ex2 <= r && r < in2) {
-        float c = ex2;
-        for (int q = 0; q < 4; ++q) {
-          c += wv[q];
-          if (wv[q] > 0.f && c > r) {
-            mine = x0 + q;
-            break;
-          }
-        }
-        if (mine < 0)
-          for (int q = 3; q >= 0; --q)
-            if (wv[q] > 0.f) {
-              mine = x0 + q;
-              break;
-            }
-      }
-      unsigned cl = __ballot_sync(0xffffffffu, mine >= 0);
-      if (cl) {
-        pick = __shfl_sync(0xffffffffu, mine, __ffs(cl) - 1);
-      } else {   // r at/after the tile's scanned mass: its last id with mass
-        int lastq = -1;
-        for (int q = 3; q >= 0; --q)
-          if (wv[q] > 0.f) {
-            lastq = x0 + q;
-            break;
-          }
-        unsigned hm = __ballot_sync(0xffffffffu, lastq >= 0);
-        pick = hm ? __shfl_sync(0xffffffffu, lastq, 31 - __clz(hm)) : -1;
-      }
-    }
-    if (lane == 0) {
-      sh_pick = pick;
-      *total_out = total;
-    }
-  }
-  __syncthreads();
-  return sh_pick;
-}
-
-struct ExpW {  // w(x) = exp(z(x) * it - m)
-  const float* z;
-  float it, m;
-  __device__ float operator()(int x) const { return __expf(z[x] * it - m); }
-};
-
-struct ResidualW {  // w(x) = max(0, p(x) - q(x))
-  const float* zt;
-  const float* zd;
-  float it, mt, st_inv, md, sd_inv;
-  __device__ float operator()(int x) const {
-    const float p = __expf(zt[x] * it - mt) * st_inv;
-    const float q = __expf(zd[x] * it - md) * sd_inv;
-    return fmaxf(p - q, 0.f);
-  }
-};
-
-// ------------------------------------------------------------- draft sampler
-// one CTA per group: x = argmax (T == 0) or inverse-CDF sample of softmax(z/T)
+// one CTA per group
 __global__ void __launch_bounds__(kSThreads) sample_kernel(const __grid_constant__ SampleArgs a) {
-  __shared__ float scr_f[2 * kSWarps];
-  __shared__ int scr_i[kSWarps];
-  __shared__ float tiles[kMaxTiles];
-  __shared__ float total;
+  __shared__ SampleSmem sm;
   pdl_launch_dependents();
   pdl_wait();
-  const int g = blockIdx.x;
-  const float* z = a.logits + g * a.row_stride;
-  const RowStats st = row_stats(z, a.vocab, a.inv_temp, a.greedy != 0, scr_f, scr_i);
-  int tok = st.arg;
-  if (!a.greedy) {
-    float u;
-    if (a.u_explicit != nullptr) {
-      u = a.u_explicit[g];
-    } else {
-      const int step = a.seq_state[g * kStateInts + 2];
-      u = philox_uniform(a.seeds[g], g, step, a.slot);
-    }
-    ExpW wf{z, a.inv_temp, st.m};
-    const int pick = block_sample(wf, a.vocab, u, tiles, scr_f, &total);
-    tok = pick >= 0 ? pick : st.arg;
-  }
-  if (threadIdx.x == 0) a.out_tok[g * a.out_stride] = tok;
+  sample_group<kSThreads>(a, blockIdx.x, sm, threadIdx.x, [] { __syncthreads(); });
 }
 
-// ------------------------------------------------------------- acceptance
-// grid (2K+1 rows, groups): row stats per CTA; the last CTA of a group decides.
+// grid (2K+1 rows, groups): row statistics per CTA; the last CTA of a group decides
 __global__ void __launch_bounds__(kSThreads) accept_kernel(const __grid_constant__ AcceptArgs a) {
-  __shared__ float scr_f[2 * kSWarps];
-  __shared__ int scr_i[kSWarps];
-  __shared__ float tiles[kMaxTiles];
-  __shared__ float total;
-  __shared__ int is_last;
+  __shared__ SampleSmem sm;
   pdl_launch_dependents();
   pdl_wait();
-  const int K = a.K, V = a.vocab;
-  const int rho = blockIdx.x, g = blockIdx.y;
-  const bool greedy = a.greedy != 0;
-  const float* zrow = rho <= K ? a.zt + (static_cast<size_t>(g) * (K + 1) + rho) * V
-                               : a.zd + (static_cast<size_t>(g) * K + (rho - K - 1)) * V;
-  const RowStats st = row_stats(zrow, V, a.inv_temp, greedy, scr_f, scr_i);
-  float* part = a.part + (static_cast<size_t>(g) * (2 * K + 1) + rho) * 4;
-  if (threadIdx.x == 0) {
-    part[0] = st.m;
-    part[1] = st.s;
-    part[2] = __int_as_float(st.arg);
-  }
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0)
-    is_last = (atomicAdd(&a.counters[g], 1) == 2 * K) ? 1 : 0;
-  __syncthreads();
-  if (!is_last) return;
-  __threadfence();
-
-  // ---- decision (whole block reads the shared statistics)
-  const float* pg = a.part + static_cast<size_t>(g) * (2 * K + 1) * 4;
-  int* state = a.seq_state + g * kStateInts;
-  const int L = state[0];
-  const int step = state[2];
-  const int* x = a.draft_tokens + g * a.max_k;
-  __shared__ int sh_n, sh_y;
-  __shared__ float sh_u;
-  float* dbg = a.debug + static_cast<size_t>(g) * (2 * K + 2);
-  if (threadIdx.x == 0) {
-    int n = 0;
-    if (greedy) {
-      while (n < K && x[n] == __float_as_int(ld_cg_f(pg + n * 4 + 2))) ++n;
-    } else {
-      while (n < K) {
-        const int xi = x[n];
-        const float* zt = a.zt + (static_cast<size_t>(g) * (K + 1) + n) * V;
-        const float* zd = a.zd + (static_cast<size_t>(g) * K + n) * V;
-        const float* ptn = pg + n * 4;
-        const float* pdn = pg + (K + 1 + n) * 4;
-        const float p = __expf(ld_cg_f(zt + xi) * a.inv_temp - ld_cg_f(ptn)) / ld_cg_f(ptn + 1);
-        const float q = __expf(ld_cg_f(zd + xi) * a.inv_temp - ld_cg_f(pdn)) / ld_cg_f(pdn + 1);
-        dbg[n] = p;
-        dbg[K + n] = q;
-        const float u = philox_uniform(a.seeds[g], g, step, K + n);
-        if (!(u * q <= p)) break;
-        ++n;
-      }
-    }
-    sh_n = n;
-    sh_u = greedy ? 0.f : philox_uniform(a.seeds[g], g, step, 2 * K);
-    sh_y = greedy ? __float_as_int(ld_cg_f(pg + n * 4 + 2)) : -1;
-  }
-  __syncthreads();
-  const int n = sh_n;
-  int y = sh_y;
-  if (!greedy) {
-    const float u = sh_u;
-    const float* zt = a.zt + (static_cast<size_t>(g) * (K + 1) + n) * V;
-    const float mt = ld_cg_f(pg + n * 4), stn = ld_cg_f(pg + n * 4 + 1);
-    float mass = 1.f;
-    int pick = -1;
-    if (n < K) {
-      const float* zd = a.zd + (static_cast<size_t>(g) * K + n) * V;
-      const float md = ld_cg_f(pg + (K + 1 + n) * 4), sdn = ld_cg_f(pg + (K + 1 + n) * 4 + 1);
-      ResidualW rw{zt, zd, a.inv_temp, mt, 1.f / stn, md, 1.f / sdn};
-      pick = block_sample(rw, V, u, tiles, scr_f, &total);
-      mass = total;
-    }
-    if (pick < 0) {  // n == K (bonus), or a residual without mass: sample p_{n+1}
-      ExpW wf{zt, a.inv_temp, mt};
-      pick = block_sample(wf, V, u, tiles, scr_f, &total);
-      if (n < K) mass = 0.f;
-    }
-    y = pick >= 0 ? pick : __float_as_int(ld_cg_f(pg + n * 4 + 2));
-    if (threadIdx.x == 0) {
-      dbg[2 * K] = mass;
-      dbg[2 * K + 1] = u;
-    }
-  }
-  // ---- commit: append x_1..x_n, y; lengths; KV rollback is the length update
-  if (threadIdx.x == 0) {
-    int* res = a.results + g * (K + 2);
-    res[0] = n;
-    int* toks = a.tokens + static_cast<size_t>(g) * a.max_seq;
-    if (L + n + 1 > a.max_seq) {
-      atomicOr(a.status, 0x4u);
-    } else {
-      for (int i = 0; i < n; ++i) {
-        toks[L + i] = x[i];
-        res[1 + i] = x[i];
-      }
-      toks[L + n] = y;
-      res[1 + n] = y;
-      for (int i = n + 2; i < K + 2; ++i) res[i] = -1;
-      state[0] = L + n + 1;                        // committed length
-      state[1] = L + n;                            // target KV valid below L'-1
-      a.draft_len[g] = L + (n < K - 1 ? n : K - 1);  // draft KV valid below this count
-    }
-    state[2] = step + 1;
-    a.counters[g] = 0;
-  }
+  accept_row<kSThreads>(a, blockIdx.x, blockIdx.y, sm, threadIdx.x, [] { __syncthreads(); });
 }
 
 }  // namespace
