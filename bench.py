@@ -136,7 +136,8 @@ def run_gpu(args, rank: int, world: int):
     max_seq = PREFIX + (steps + warm + 8) * (K + 1) + 16
     t0 = time.time()
     eng = Engine(t, iter_weights(t, 0), max_batch=1, max_seq=max_seq, max_k=K, max_drafts=1,
-                 draft_shape_max=dft, draft_budget_bytes=1 << 30, use_graphs=True, device=dev)
+                 draft_shape_max=dft, draft_budget_bytes=1 << 30, use_graphs=True,
+                 launch_mode=args.launch_mode, device=dev)
     eng.register_draft(0, dft, iter_weights(dft, 1))
     eng.load_draft_async(0)
     eng.set_active_draft(0)
@@ -302,7 +303,8 @@ def run_case(args):
     K = args.k
     max_seq = 512 + (args.steps + args.warmup + 4) * (K + 1) + 16
     eng = Engine(t, iter_weights(t, 0), max_batch=1, max_seq=max_seq, max_k=K, max_drafts=1,
-                 draft_shape_max=d, draft_budget_bytes=512 << 20, use_graphs=True)
+                 draft_shape_max=d, draft_budget_bytes=512 << 20, use_graphs=True,
+                 launch_mode=args.launch_mode, trace=args.trace is not None)
     eng.register_draft(0, d, iter_weights(d, 1))
     eng.load_draft_async(0)
     eng.set_active_draft(0)
@@ -321,6 +323,8 @@ def run_case(args):
     bits = eng.sync()
     L1 = int(eng.seq_state()[0, 0])
     ms = a.elapsed_time(b)
+    if args.trace is not None:      # timestamps of the last persistent launch
+        np.save(args.trace, eng.pass_trace())
     eng.close()
     return {"case": "small", "target": "draft_160m", "draft": "draft_68m", "K": K,
             "ms_per_step": ms / args.steps, "tokens_per_s": (L1 - L0) / ms * 1e3,
@@ -338,6 +342,10 @@ def main():
     ap.add_argument("--case", default="step", choices=["step", "gemm", "small"],
                     help="step: the workload above; gemm / small: diagnostic cases sized for "
                          "profiler captures (one projection GEMM; a 160M target with a 68M draft)")
+    ap.add_argument("--launch-mode", default="per_op", choices=["per_op", "pass"],
+                    help="one launch per op, or one persistent launch per pass")
+    ap.add_argument("--trace", default=None,
+                    help="(--case small, --launch-mode pass) save the last pass's trace (.npy)")
     ap.add_argument("--n", type=int, default=22016)
     ap.add_argument("--kdim", type=int, default=4096)
     ap.add_argument("--rows", type=int, default=5)

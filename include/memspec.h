@@ -137,7 +137,14 @@ typedef struct memspec_init_params {
   void* stream_main;                /* cudaStream_t for all step calls */
   void* stream_side;                /* cudaStream_t for draft loads (may equal main) */
   int32_t use_graphs;               /* 1: capture each step once and replay it */
+  int32_t launch_mode;              /* MEMSPEC_LAUNCH_PER_OP (0): one kernel launch per
+                                       op of a pass; MEMSPEC_LAUNCH_PASS (1): each draft
+                                       step and verify pass as one persistent launch */
+  int32_t trace;                    /* 1: the persistent launch records per-op
+                                       timestamps (MEMSPEC_BUF_PASS_TRACE) */
 } memspec_init_params;
+
+enum { MEMSPEC_LAUNCH_PER_OP = 0, MEMSPEC_LAUNCH_PASS = 1 };
 
 /* Device workspace bytes memspec_init needs for these params. */
 memspec_status memspec_workspace_bytes(const memspec_init_params* p, size_t* bytes);
@@ -236,7 +243,11 @@ typedef enum memspec_buffer {
   MEMSPEC_BUF_TOKENS = 3,        /* int32 [max_batch][max_seq] committed tokens */
   MEMSPEC_BUF_SEQ_STATE = 4,     /* int32 [max_batch][4] = {L, Lt, step, active Ld} */
   MEMSPEC_BUF_ACCEPT_DEBUG = 5,  /* fp32 [batch][2K+2] = {p_i(x_i), q_i(x_i), residual mass, u'} */
-  MEMSPEC_BUF_RESIDUAL = 6       /* fp32 residual stream [rows][d] of the last forward */
+  MEMSPEC_BUF_RESIDUAL = 6,      /* fp32 residual stream [rows][d] of the last forward */
+  MEMSPEC_BUF_PASS_TRACE = 7     /* u64 trace of the last persistent launch (trace = 1):
+                                    {n_ops, grid, then [n_ops][grid][4] globaltimer ns =
+                                    worker start, worker end, activation loads issued,
+                                    first MMA issued}; 2048 ops at most */
 } memspec_buffer;
 
 /* Synchronously copy `bytes` of an internal buffer to host memory (waits for

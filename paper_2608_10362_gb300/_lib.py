@@ -22,7 +22,11 @@ T_TOK_EMB, T_ATTN_NORM, T_WQKV, T_WO, T_FFN_NORM, T_WGATE, T_WUP, T_WDOWN, T_FIN
 
 # buffer ids (memspec_buffer)
 BUF_TARGET_LOGITS, BUF_DRAFT_LOGITS, BUF_DRAFT_TOKENS, BUF_TOKENS, BUF_SEQ_STATE, \
-    BUF_ACCEPT_DEBUG, BUF_RESIDUAL = range(7)
+    BUF_ACCEPT_DEBUG, BUF_RESIDUAL, BUF_PASS_TRACE = range(8)
+
+# launch modes (memspec_init_params.launch_mode)
+LAUNCH_PER_OP, LAUNCH_PASS = 0, 1
+PASS_TRACE_OPS = 2048
 
 DEV_TIMEOUT, DEV_BAD_TOKEN, DEV_BAD_LENGTH = 0x1, 0x2, 0x4
 
@@ -40,7 +44,7 @@ class InitParams(C.Structure):
                 ("max_k", C.c_int32), ("max_drafts", C.c_int32), ("draft_shape_max", ModelCfg),
                 ("draft_arena_dev", C.c_void_p), ("draft_budget_bytes", C.c_size_t),
                 ("stream_main", C.c_void_p), ("stream_side", C.c_void_p),
-                ("use_graphs", C.c_int32)]
+                ("use_graphs", C.c_int32), ("launch_mode", C.c_int32), ("trace", C.c_int32)]
 
 
 EXPORTS = {

@@ -22,6 +22,7 @@
 #include "../../include/memspec.h"
 #include "../../include/memspec_ops.h"
 #include "internal.h"
+#include "pass.h"
 
 using namespace memspec;
 
@@ -91,6 +92,11 @@ bool ensure_func_attrs() {
   e = attention_set_max_smem();
   if (e != cudaSuccess) {
     g_attr_error = std::string("attention smem attribute: ") + cudaGetErrorString(e);
+    return false;
+  }
+  e = pass_set_max_smem();
+  if (e != cudaSuccess) {
+    g_attr_error = std::string("pass kernel smem attribute: ") + cudaGetErrorString(e);
     return false;
   }
   done = true;
@@ -318,6 +324,14 @@ struct memspec_ctx {
   int batch = 1;
   int last_K = 0;
   std::map<GraphKey, cudaGraphExec_t> graphs;
+  // op tables of the pass kernel (workspace areas, bump-allocated per graph)
+  uint8_t* op_area = nullptr;
+  size_t op_area_bytes = 0, op_area_used = 0;
+  int* done_area = nullptr;
+  size_t done_area_ints = 0, done_area_used = 0;
+  bool pass_kernel = false;  // draft / verify passes as one persistent launch
+  bool cooperative = false;
+  unsigned long long* trace = nullptr;   // pass-kernel trace (init param trace = 1)
   std::map<std::tuple<const void*, int, int, int>, CUtensorMap> bmaps;
 };
 
@@ -409,7 +423,15 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   const size_t o_rs64 = w.take(static_cast<size_t>(p->max_seq) * 32 * 4);
   const size_t o_rc128 = w.take(static_cast<size_t>(p->max_seq) * 64 * 4);
   const size_t o_rs128 = w.take(static_cast<size_t>(p->max_seq) * 64 * 4);
+  const size_t op_bytes = static_cast<size_t>(24) << 20;     // pass-kernel op tables
+  const size_t done_ints = static_cast<size_t>(64) << 10;
+  const size_t o_ops = w.take(op_bytes);
+  const size_t o_done = w.take(done_ints * 4);
+  const size_t trace_bytes =
+      p->trace == 1 ? (2 + static_cast<size_t>(kPassTraceOps) * nsm * 4) * 8 : 0;
+  const size_t o_trace = w.take(trace_bytes);
   if (c != nullptr) {
+    c->trace = trace_bytes ? reinterpret_cast<unsigned long long*>(base + o_trace) : nullptr;
     c->h = reinterpret_cast<float*>(base + o_h);
     c->xg = reinterpret_cast<bf16*>(base + o_xg);
     c->xg_lo = reinterpret_cast<bf16*>(base + o_xgl);
@@ -444,6 +466,10 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
     c->rope_sin[0] = reinterpret_cast<float*>(base + o_rs64);
     c->rope_cos[1] = reinterpret_cast<float*>(base + o_rc128);
     c->rope_sin[1] = reinterpret_cast<float*>(base + o_rs128);
+    c->op_area = base + o_ops;
+    c->op_area_bytes = op_bytes;
+    c->done_area = reinterpret_cast<int*>(base + o_done);
+    c->done_area_ints = done_ints;
     c->max_rows = rows;
     c->vocab = V;
   }
@@ -520,20 +546,22 @@ int gemm_grid(int row_tiles, int k_tiles) {
   return std::max(1, std::min({T, sm_count(), T / min_tiles}));
 }
 
-memspec_status run_gemm(memspec_ctx* c, GemmArgs& a, const char* what) {
-  const int grid = gemm_grid(a.row_tiles, a.k_tiles);
+void emit_gemm(memspec_ctx* c, GemmArgs& a, std::vector<PassOp>& ops) {
   const int planes = a.split ? 2 : 1;
   a.stages = gemm_pick_stages(a.n_pad, planes);
   a.partials = c->gemm_part;
   a.counters = c->gemm_cnt;
   a.status = c->status;
-  cudaError_t e =
-      launch_gemm(a, grid, gemm_smem_bytes(a.n_pad, a.stages, planes), c->main, c->pdl);
-  if (e != cudaSuccess) return cuda_fail(c, e, what);
-  return MEMSPEC_OK;
+  PassOp op{};
+  op.type = OP_GEMM;
+  op.grid = gemm_grid(a.row_tiles, a.k_tiles);
+  op.smem = static_cast<int>(gemm_smem_bytes(a.n_pad, a.stages, planes));
+  op.u.g = a;
+  ops.push_back(op);
 }
 
-memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
+memspec_status emit_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f,
+                            std::vector<PassOp>& ops) {
   const memspec_model_cfg& cf = m.cfg;
   const int d = cf.d_model, qd = model_q(cf), kvd = model_kv(cf), F = cf.d_ffn;
   const int rows = f.n_groups * f.R;
@@ -564,8 +592,13 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
   ea.ss_stride = c->ss_stride;
   ea.plan = c->plan;
   ea.status = c->status;
-  cudaError_t e = launch_embed(ea, rows, c->main, c->pdl);
-  if (e != cudaSuccess) return cuda_fail(c, e, "embed launch");
+  {
+    PassOp op{};
+    op.type = OP_EMBED;
+    op.n_units = rows;
+    op.u.e = ea;
+    ops.push_back(op);
+  }
 
   const size_t layer_kv = static_cast<size_t>(c->p.max_batch) * cf.n_kv_heads * c->p.max_seq * cf.head_dim;
   AttnGeo geo = attn_geometry(cf, f.n_groups, f.R, c->p.max_seq);
@@ -608,8 +641,7 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.rope_cos = c->rope_cos[hsel];
       a.rope_sin = c->rope_sin[hsel];
       a.plan = c->plan;
-      memspec_status s = run_gemm(c, a, "qkv gemm launch");
-      if (s != MEMSPEC_OK) return s;
+      emit_gemm(c, a, ops);
     }
     {  // attention
       AttnArgs at{};
@@ -633,8 +665,12 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       at.out_lo = c->o_lo;
       at.plan = c->plan;
       at.status = c->status;
-      e = launch_attention(at, f.n_groups, c->main, c->pdl);
-      if (e != cudaSuccess) return cuda_fail(c, e, "attention launch");
+      PassOp op{};
+      op.type = OP_ATTN;
+      op.n_units = at.n_splits * at.Hkv * at.row_blocks * f.n_groups;
+      op.grid = f.n_groups;
+      op.u.at = at;
+      ops.push_back(op);
     }
     {  // O projection + residual
       GemmArgs a{};
@@ -659,8 +695,7 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.xg_lo_out = c->xg_lo;
       a.ss_stride = c->ss_stride;
       a.plan = c->plan;
-      memspec_status s = run_gemm(c, a, "o gemm launch");
-      if (s != MEMSPEC_OK) return s;
+      emit_gemm(c, a, ops);
       ss_count = ceil_div(d, 128);
     }
     {  // gate/up + SwiGLU
@@ -689,8 +724,7 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.act_lo = c->act_lo;
       a.act_ld = F;
       a.plan = c->plan;
-      memspec_status s = run_gemm(c, a, "gate/up gemm launch");
-      if (s != MEMSPEC_OK) return s;
+      emit_gemm(c, a, ops);
     }
     {  // down projection + residual
       GemmArgs a{};
@@ -716,8 +750,7 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
       a.xg_lo_out = c->xg_lo;
       a.ss_stride = c->ss_stride;
       a.plan = c->plan;
-      memspec_status s = run_gemm(c, a, "down gemm launch");
-      if (s != MEMSPEC_OK) return s;
+      emit_gemm(c, a, ops);
     }
   }
   if (f.logits != nullptr) {  // final RMSNorm + LM head -> fp32 logits
@@ -745,37 +778,144 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
     a.last_only = f.last_only;
     a.out_group_stride = f.out_group_stride;
     a.plan = c->plan;
-    memspec_status s = run_gemm(c, a, "lm head gemm launch");
-    if (s != MEMSPEC_OK) return s;
+    emit_gemm(c, a, ops);
   }
   return MEMSPEC_OK;
 }
 
-// ---------------------------------------------------------------- graphs
-template <class F>
-memspec_status run_maybe_graphed(memspec_ctx* c, const GraphKey& key, F&& enqueue) {
-  if (!c->p.use_graphs) return enqueue();
-  auto it = c->graphs.find(key);
-  if (it == c->graphs.end()) {
-    cudaError_t e = cudaStreamBeginCapture(c->main, cudaStreamCaptureModeThreadLocal);
-    if (e != cudaSuccess) return cuda_fail(c, e, "begin capture");
-    memspec_status s = enqueue();
-    cudaGraph_t g = nullptr;
-    e = cudaStreamEndCapture(c->main, &g);
-    if (s != MEMSPEC_OK) {
-      if (g) cudaGraphDestroy(g);
-      return s;
+// ---------------------------------------------------------------- running op lists
+// Each op as its own kernel launch (programmatic dependent launch between them).
+memspec_status run_ops_separately(memspec_ctx* c, const std::vector<PassOp>& ops) {
+  for (const PassOp& op : ops) {
+    cudaError_t e = cudaSuccess;
+    switch (op.type) {
+      case OP_EMBED: e = launch_embed(op.u.e, op.n_units, c->main, c->pdl); break;
+      case OP_GEMM: e = launch_gemm(op.u.g, op.grid, op.smem, c->main, c->pdl); break;
+      case OP_ATTN: e = launch_attention(op.u.at, op.grid, c->main, c->pdl); break;
+      case OP_SAMPLE: e = launch_sample(op.u.s, c->main, c->pdl); break;
+      case OP_ACCEPT: e = launch_accept(op.u.acc, c->main, false); break;
+      default: return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown op");
     }
-    if (e != cudaSuccess) return cuda_fail(c, e, "end capture");
-    cudaGraphExec_t ex = nullptr;
-    e = cudaGraphInstantiate(&ex, g, 0);
-    cudaGraphDestroy(g);
-    if (e != cudaSuccess) return cuda_fail(c, e, "graph instantiate");
-    it = c->graphs.emplace(key, ex).first;
+    if (e != cudaSuccess) return cuda_fail(c, e, "op launch");
   }
-  cudaError_t e = cudaGraphLaunch(it->second, c->main);
+  return MEMSPEC_OK;
+}
+
+// An op table in the workspace (device copy of the ops + completion counters).
+struct OpTable {
+  PassOp* ops = nullptr;
+  int* done = nullptr;   // [n_ops + 1]: counters, then the exit counter
+  int n_ops = 0;
+  PassArgs args{};
+};
+
+// Place `ops` in the workspace: synchronous copy (the table must be in place
+// before a graph that uses it is captured).
+memspec_status place_table(memspec_ctx* c, const std::vector<PassOp>& ops, OpTable* t) {
+  const size_t bytes = ops.size() * sizeof(PassOp);
+  const size_t ints = ops.size() + 1;
+  if (bytes > c->op_area_bytes || ints > c->done_area_ints)
+    return fail(c, MEMSPEC_ERR_UNSUPPORTED, "pass has more ops than the op-table area holds");
+  if (c->op_area_used + bytes > c->op_area_bytes || c->done_area_used + ints > c->done_area_ints) {
+    // area full: drop every captured graph (their tables go with them)
+    cudaError_t e = cudaStreamSynchronize(c->main);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sync");
+    for (auto& kv : c->graphs) cudaGraphExecDestroy(kv.second);
+    c->graphs.clear();
+    c->op_area_used = 0;
+    c->done_area_used = 0;
+  }
+  t->ops = reinterpret_cast<PassOp*>(c->op_area + c->op_area_used);
+  t->done = c->done_area + c->done_area_used;
+  t->n_ops = static_cast<int>(ops.size());
+  c->op_area_used += (bytes + 255) & ~static_cast<size_t>(255);
+  c->done_area_used += (ints + 63) & ~static_cast<size_t>(63);
+  cudaError_t e = cudaMemcpy(t->ops, ops.data(), bytes, cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(c, e, "op table copy");
+  // shared-memory layout of the pass: deepest activation stage, attention region
+  int b_bytes = 0, hd = 0;
+  uint32_t cols = 32;
+  for (const PassOp& op : ops) {
+    if (op.type == OP_GEMM) {
+      const GemmArgs& a = op.u.g;
+      const int planes = a.split ? 2 : 1;
+      b_bytes = std::max(b_bytes, a.n_pad * 128 * planes);
+      const int acols = (a.split && 2 * a.n_pad <= 256) ? 2 * a.n_pad : a.n_pad;
+      while (cols < static_cast<uint32_t>(2 * acols)) cols <<= 1;
+    } else if (op.type == OP_ATTN) {
+      hd = std::max(hd, op.u.at.hd);
+    }
+  }
+  PassArgs& p = t->args;
+  p.ops = t->ops;
+  p.n_ops = t->n_ops;
+  p.done = t->done;
+  p.exit_cnt = t->done + t->n_ops;
+  p.b_stage_bytes = b_bytes;
+  p.attn_bytes = hd ? static_cast<int>(pass_attn_bytes(hd)) : 0;
+  p.stages = pass_pick_stages(b_bytes, p.attn_bytes);
+  p.tmem_cols = cols;
+  p.status = c->status;
+  p.trace = c->trace;
+  if (p.stages < 2) return fail(c, MEMSPEC_ERR_UNSUPPORTED, "pass kernel: shared memory too small");
+  return MEMSPEC_OK;
+}
+
+memspec_status launch_table(memspec_ctx* c, const OpTable& t) {
+  cudaError_t e = launch_pass(t.args, sm_count(), c->main, c->cooperative);
+  if (e != cudaSuccess) return cuda_fail(c, e, "pass kernel launch");
+  return MEMSPEC_OK;
+}
+
+// Build the op list, then run it: one persistent launch (pass kernel) or one
+// launch per op; captured once as a CUDA graph per key and replayed when graphs
+// are on.  `use_pass` = false always runs separate launches.
+template <class Emit>
+memspec_status run_pass(memspec_ctx* c, const GraphKey& key, bool use_pass, Emit&& emit) {
+  const bool pass = use_pass && c->pass_kernel;
+  if (c->p.use_graphs) {
+    auto it = c->graphs.find(key);
+    if (it != c->graphs.end()) {
+      cudaError_t e = cudaGraphLaunch(it->second, c->main);
+      if (e != cudaSuccess) return cuda_fail(c, e, "graph launch");
+      return MEMSPEC_OK;
+    }
+  }
+  std::vector<PassOp> ops;
+  memspec_status s = emit(ops);
+  if (s != MEMSPEC_OK) return s;
+  OpTable t;
+  if (pass) {
+    s = place_table(c, ops, &t);
+    if (s != MEMSPEC_OK) return s;
+  }
+  if (!c->p.use_graphs) return pass ? launch_table(c, t) : run_ops_separately(c, ops);
+  cudaError_t e = cudaStreamBeginCapture(c->main, cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) return cuda_fail(c, e, "begin capture");
+  s = pass ? launch_table(c, t) : run_ops_separately(c, ops);
+  cudaGraph_t g = nullptr;
+  e = cudaStreamEndCapture(c->main, &g);
+  if (s != MEMSPEC_OK) {
+    if (g) cudaGraphDestroy(g);
+    return s;
+  }
+  if (e != cudaSuccess) return cuda_fail(c, e, "end capture");
+  cudaGraphExec_t ex = nullptr;
+  e = cudaGraphInstantiate(&ex, g, 0);
+  cudaGraphDestroy(g);
+  if (e != cudaSuccess) return cuda_fail(c, e, "graph instantiate");
+  c->graphs.emplace(key, ex);
+  e = cudaGraphLaunch(ex, c->main);
   if (e != cudaSuccess) return cuda_fail(c, e, "graph launch");
   return MEMSPEC_OK;
+}
+
+// A forward pass run with separate launches and no graph (prefill, catch-up).
+memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
+  std::vector<PassOp> ops;
+  memspec_status s = emit_forward(c, m, f, ops);
+  if (s != MEMSPEC_OK) return s;
+  return run_ops_separately(c, ops);
 }
 
 void drop_graphs_of_draft(memspec_ctx* c, int draft) {
@@ -913,6 +1053,11 @@ memspec_status memspec_init(const memspec_init_params* p, void* workspace_dev, m
   // (for measuring what the overlap buys)
   const char* no_pdl = std::getenv("MEMSPEC_NO_PDL");
   c->pdl = !(no_pdl != nullptr && no_pdl[0] == '1');
+  // MEMSPEC_COOPERATIVE=1 launches the pass kernel cooperatively (its grid is
+  // one CTA per SM either way)
+  c->pass_kernel = p->launch_mode == MEMSPEC_LAUNCH_PASS;
+  const char* coop = std::getenv("MEMSPEC_COOPERATIVE");
+  c->cooperative = coop != nullptr && coop[0] == '1';
   c->side = p->stream_side ? static_cast<cudaStream_t>(p->stream_side) : c->main;
   c->ws_bytes = layout_workspace(p, c, static_cast<uint8_t*>(workspace_dev));
   if (!ensure_func_attrs()) {
@@ -1173,7 +1318,7 @@ memspec_status memspec_draft_step(memspec_ctx* c, int32_t K, float T) {
   const int B = c->batch;
   const int id = c->active;
   GraphKey key{0, id, K, fbits(T), B};
-  return run_maybe_graphed(c, key, [&]() -> memspec_status {
+  return run_pass(c, key, true, [&](std::vector<PassOp>& ops) -> memspec_status {
     for (int j = 1; j <= K; ++j) {
       FwdSpec f{};
       f.mode = j == 1 ? PLAN_DRAFT_FIRST : PLAN_DRAFT_NEXT;
@@ -1184,7 +1329,7 @@ memspec_status memspec_draft_step(memspec_ctx* c, int32_t K, float T) {
       f.logits = c->zd + static_cast<size_t>(j - 1) * c->vocab;
       f.last_only = 1;
       f.out_group_stride = static_cast<long long>(K) * c->vocab;
-      memspec_status st = enqueue_forward(c, d.rt, f);
+      memspec_status st = emit_forward(c, d.rt, f, ops);
       if (st != MEMSPEC_OK) return st;
       SampleArgs sa{};
       sa.logits = f.logits;
@@ -1200,8 +1345,11 @@ memspec_status memspec_draft_step(memspec_ctx* c, int32_t K, float T) {
       sa.out_stride = c->p.max_k;
       sa.counters = c->smp_cnt;
       sa.status = c->status;
-      cudaError_t e = launch_sample(sa, c->main, c->pdl);
-      if (e != cudaSuccess) return cuda_fail(c, e, "sample launch");
+      PassOp op{};
+      op.type = OP_SAMPLE;
+      op.n_units = B;
+      op.u.s = sa;
+      ops.push_back(op);
     }
     return MEMSPEC_OK;
   });
@@ -1212,14 +1360,14 @@ memspec_status memspec_verify_step(memspec_ctx* c, int32_t K) {
   if (K < 1 || K > c->p.max_k) return fail(c, MEMSPEC_ERR_INVALID_ARG, "K out of range");
   const int B = c->batch;
   GraphKey key{1, -1, K, 0, B};
-  return run_maybe_graphed(c, key, [&]() -> memspec_status {
+  return run_pass(c, key, true, [&](std::vector<PassOp>& ops) -> memspec_status {
     FwdSpec f{};
     f.mode = PLAN_VERIFY;
     f.n_groups = B;
     f.R = K + 1;
     f.logits = c->zt;
     f.last_only = 0;
-    return enqueue_forward(c, c->target, f);
+    return emit_forward(c, c->target, f, ops);
   });
 }
 
@@ -1231,7 +1379,7 @@ memspec_status memspec_accept_commit(memspec_ctx* c, int32_t K, float T, int32_t
   const int id = c->active;
   if (id < 0) return fail(c, MEMSPEC_ERR_NOT_RESIDENT, "no active draft");
   GraphKey key{2, id, K, fbits(T), B};
-  memspec_status s = run_maybe_graphed(c, key, [&]() -> memspec_status {
+  memspec_status s = run_pass(c, key, false, [&](std::vector<PassOp>& ops) -> memspec_status {
     AcceptArgs a{};
     a.zt = c->zt;
     a.zd = c->zd;
@@ -1252,8 +1400,11 @@ memspec_status memspec_accept_commit(memspec_ctx* c, int32_t K, float T, int32_t
     a.results = c->results;
     a.debug = c->acc_dbg;
     a.status = c->status;
-    cudaError_t e = launch_accept(a, c->main, false);
-    if (e != cudaSuccess) return cuda_fail(c, e, "accept launch");
+    PassOp op{};
+    op.type = OP_ACCEPT;
+    op.n_units = (2 * K + 1) * B;
+    op.u.acc = a;
+    ops.push_back(op);
     return MEMSPEC_OK;
   });
   if (s != MEMSPEC_OK) return s;
@@ -1315,6 +1466,11 @@ static memspec_status buffer_span(memspec_ctx* c, int32_t buf, void** ptr, size_
     case MEMSPEC_BUF_SEQ_STATE: *ptr = c->state; *cap = static_cast<size_t>(B) * kStateInts * 4; break;
     case MEMSPEC_BUF_ACCEPT_DEBUG: *ptr = c->acc_dbg; *cap = static_cast<size_t>(B) * (2 * K + 2) * 4; break;
     case MEMSPEC_BUF_RESIDUAL: *ptr = c->h; *cap = static_cast<size_t>(kMaxRows) * c->p.target.d_model * 4; break;
+    case MEMSPEC_BUF_PASS_TRACE:
+      if (c->trace == nullptr) return fail(c, MEMSPEC_ERR_INVALID_ARG, "tracing is off (init param trace)");
+      *ptr = c->trace;
+      *cap = (2 + static_cast<size_t>(kPassTraceOps) * sm_count() * 4) * 8;
+      break;
     default: return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown buffer id");
   }
   return MEMSPEC_OK;

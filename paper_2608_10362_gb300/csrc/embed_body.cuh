@@ -7,7 +7,7 @@
 namespace memspec {
 namespace emb {
 
-__device__ void compute_group(const EmbedArgs& a, int g, int* req, int* valid, int* pos0) {
+static __device__ void compute_group(const EmbedArgs& a, int g, int* req, int* valid, int* pos0) {
   if (a.mode == PLAN_PREFILL) {
     *req = a.prefill_req;
     *valid = a.prefill_count;
@@ -34,7 +34,7 @@ __device__ void compute_group(const EmbedArgs& a, int g, int* req, int* valid, i
   }
 }
 
-__device__ int row_token(const EmbedArgs& a, int req, int pos, int i) {
+static __device__ int row_token(const EmbedArgs& a, int req, int pos, int i) {
   const int L = a.mode == PLAN_PREFILL ? 0 : a.seq_state[req * kStateInts + 0];
   if (a.mode == PLAN_VERIFY) {
     return i == 0 ? a.tokens[static_cast<size_t>(req) * a.max_seq + L - 1]

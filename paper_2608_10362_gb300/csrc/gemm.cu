@@ -50,6 +50,7 @@ struct SmemCtl {
   uint32_t tmem_base;
   int abort_flag;
   int reduce_flag;
+  int wait_ok;
   float red[4][16];
 };
 
@@ -242,13 +243,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
       const int seg_end = min(t_end, (rt + 1) * KT);
       const int k1 = seg_end - rt * KT;
       const int buf = seg & 1;
-      int ok = 1;
-      if (lane == 0)
-        ok = mbar_wait_bounded(&ctl.acc_full[buf], static_cast<uint32_t>(seg >> 1) & 1u, abort_flag,
-                               a.status)
-                 ? 1
-                 : 0;
-      ok = __shfl_sync(0xffffffffu, ok, 0);   // the warp proceeds (or stops) together
+      // one thread waits; the four epilogue warps follow (or stop) together
+      if (threadIdx.x == 64)
+        ctl.wait_ok = mbar_wait_bounded(&ctl.acc_full[buf], static_cast<uint32_t>(seg >> 1) & 1u,
+                                        abort_flag, a.status)
+                          ? 1
+                          : 0;
+      named_bar_sync(1, 128);
+      const int ok = ctl.wait_ok;
+      named_bar_sync(1, 128);
       if (!ok) break;
       tc_fence_after();
       epilogue_segment(a, layout, acols, tmem_base, buf, seg, c, G, rt, k0, k1, stage, rms,

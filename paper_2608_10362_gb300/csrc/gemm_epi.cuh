@@ -44,7 +44,7 @@ __device__ __forceinline__ bool row_valid(const GemmArgs& a, int r) {
 
 // Epilogue for one 16-row chunk of a finished 128-feature row tile.  Called by
 // the 128 epilogue threads together; et = feature within the tile (= TMEM lane).
-__device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*red)[16], float* stage,
+static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*red)[16], float* stage,
                                             const float* rms, int rt, int chunk, int et,
                                             const float* vin) {
   const int ew = et >> 5, lane = et & 31;

@@ -85,7 +85,13 @@ class Engine:
 
     def __init__(self, target_shape, target_weights, *, max_batch: int = 1, max_seq: int = 1024,
                  max_k: int = 8, max_drafts: int = 4, draft_shape_max=None,
-                 draft_budget_bytes: int = 0, use_graphs: bool = True, device: int = 0):
+                 draft_budget_bytes: int = 0, use_graphs: bool = True,
+                 launch_mode: str = "per_op", trace: bool = False, device: int = 0):
+        """launch_mode "per_op": one kernel launch per op of a pass; "pass": each
+        draft step and verify pass as one persistent launch (``trace`` then
+        records per-op timestamps, see ``pass_trace``)."""
+        if launch_mode not in ("per_op", "pass"):
+            raise ValueError(f"launch_mode must be 'per_op' or 'pass', not {launch_mode!r}")
         self.lib = _lib.load()
         self.device = torch.device("cuda", device)
         torch.cuda.set_device(self.device)
@@ -112,6 +118,8 @@ class Engine:
         p.stream_main = self.stream.cuda_stream
         p.stream_side = self.side.cuda_stream
         p.use_graphs = int(use_graphs)
+        p.launch_mode = _lib.LAUNCH_PASS if launch_mode == "pass" else _lib.LAUNCH_PER_OP
+        p.trace = int(trace)
         self.params = p
         n = C.c_size_t()
         _check(self.lib, self.lib.memspec_workspace_bytes(C.byref(p), C.byref(n)))
@@ -219,6 +227,16 @@ class Engine:
         L = int(self.seq_state()[req, 0])
         toks = self.read_buffer(_lib.BUF_TOKENS, np.int32, self.max_batch * self.max_seq)
         return toks.reshape(self.max_batch, self.max_seq)[req, :L]
+
+    def pass_trace(self) -> np.ndarray:
+        """Timestamps (ns) of the last persistent launch, [n_ops][grid][4] =
+        worker start, worker end, activation loads issued, first MMA issued
+        (entries an op did not take keep older values)."""
+        head = self.read_buffer(_lib.BUF_PASS_TRACE, np.uint64, 2)
+        n_ops, grid = int(head[0]), int(head[1])
+        n = min(n_ops, _lib.PASS_TRACE_OPS)
+        t = self.read_buffer(_lib.BUF_PASS_TRACE, np.uint64, 2 + n * grid * 4)
+        return t[2:].reshape(n, grid, 4)
 
     def target_logits(self, batch: int, K: int) -> np.ndarray:
         n = batch * (K + 1) * self.vocab

@@ -21,32 +21,38 @@ def _run_lockstep(eng, target_o, draft_o, prompt, K, T, seed, steps, use_graphs_
     return rep, sd
 
 
+# (CUDA graphs, launch mode): per-op launches with and without graphs, and the
+# persistent pass kernel
+MODES = [(False, "per_op"), (True, "per_op"), (True, "pass"), (False, "pass")]
+
+
 @pytest.fixture(scope="module")
 def tiny():
     from paper_2608_10362_gb300 import Engine
     t, d = SHAPES["tiny_target"], SHAPES["tiny_draft"]
     wt, wd = gen_weights(t, 0), gen_weights(d, 1)
     engines = {}
-    for graphs in (False, True):
+    for mode in MODES:
+        graphs, launch = mode
         eng = Engine(t, wt, max_batch=1, max_seq=512, max_k=8, max_drafts=1, draft_shape_max=d,
-                     draft_budget_bytes=32 << 20, use_graphs=graphs)
+                     draft_budget_bytes=32 << 20, use_graphs=graphs, launch_mode=launch)
         eng.register_draft(0, d, wd)
         eng.load_draft_async(0)
         eng.set_active_draft(0)
-        engines[graphs] = eng
+        engines[mode] = eng
     yield engines, LlamaOracle(t, wt), LlamaOracle(d, wd)
     for e in engines.values():
         e.close()
 
 
-@pytest.mark.parametrize("graphs", [False, True])
+@pytest.mark.parametrize("mode", MODES, ids=lambda m: f"graphs{int(m[0])}-{m[1]}")
 @pytest.mark.parametrize("T", [0.0, 1.0])
-def test_tiny_pair_lockstep(tiny, T, graphs):
+def test_tiny_pair_lockstep(tiny, T, mode):
     engines, to, do = tiny
-    eng = engines[graphs]
+    eng = engines[mode]
     prompt = gen_prompt(7, 128, 2048)
     rep, sd = _run_lockstep(eng, to, do, prompt, 4, T, seed=3, steps=16)
-    print(f"tiny T={T} graphs={graphs}: steps {rep.steps} tokens {rep.tokens_committed} "
+    print(f"tiny T={T} mode={mode}: steps {rep.steps} tokens {rep.tokens_committed} "
           f"flags {rep.flags}/{rep.decisions} max logit err {rep.max_logit_err_frac:.2e}")
     assert rep.flags <= max(1, rep.decisions // 20)
     assert list(eng.committed_tokens(0)) == sd.tokens
@@ -59,7 +65,7 @@ def test_tiny_greedy_stream_equals_oracle_target_greedy(tiny):
     lock-step tests measure); such a divergence is reported, any other fails."""
     from oracle.speculative import greedy_generate
     engines, to, do = tiny
-    eng = engines[True]
+    eng = engines[(True, "per_op")]
     n_new = 40
     for seed in (8, 9, 10):
         prompt = gen_prompt(seed, 128, 2048)
@@ -84,7 +90,7 @@ def test_tiny_prompt_edge_cases(tiny):
     """Prompt of one token (nothing to prefill) and a prompt crossing the
     128-row prefill chunk boundary by one."""
     engines, to, do = tiny
-    eng = engines[False]
+    eng = engines[(False, "per_op")]
     for n in (1, 129):
         prompt = gen_prompt(9 + n, n, 2048)
         rep, sd = _run_lockstep(eng, to, do, prompt, 3, 1.0, seed=5, steps=4)
