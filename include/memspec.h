@@ -245,9 +245,11 @@ typedef enum memspec_buffer {
   MEMSPEC_BUF_ACCEPT_DEBUG = 5,  /* fp32 [batch][2K+2] = {p_i(x_i), q_i(x_i), residual mass, u'} */
   MEMSPEC_BUF_RESIDUAL = 6,      /* fp32 residual stream [rows][d] of the last forward */
   MEMSPEC_BUF_PASS_TRACE = 7     /* u64 trace of the last persistent launch (trace = 1):
-                                    {n_ops, grid, then [n_ops][grid][4] globaltimer ns =
+                                    {n_ops, grid, then [n_ops][grid][16] globaltimer ns =
                                     worker start, worker end, activation loads issued,
-                                    first MMA issued}; 2048 ops at most */
+                                    first MMA issued, partials stored, arrival counted,
+                                    reduction inputs loaded, reduction done, then
+                                    epilogue-internal points}; 2048 ops at most */
 } memspec_buffer;
 
 /* Synchronously copy `bytes` of an internal buffer to host memory (waits for

@@ -24,7 +24,8 @@ memspec_status memspec_op_linear_scratch_bytes(int32_t rows, int32_t n_out, int3
  * This is the weight-streaming GEMM every projection of the verify and draft
  * passes runs (Q/K/V, O, gate/up, down, LM head): TMA-staged weight tiles,
  * tcgen05 MMA into TMEM, stream-K over all SMs, deterministic split-K
- * reduction.  rows in 1..256, k a multiple of 8, n_out >= 1.
+ * reduction.  rows in 1..256, k a multiple of 8, n_out >= 1, and
+ * ceil(n_out/128) * ceil(k/64) * (SMs + 1) below 2^32.
  * scratch_dev: memspec_op_linear_scratch_bytes bytes, 256-byte aligned; its
  * counters must be zero on entry and are left zero on exit (zero it once).
  * status_dev: uint32 device word, bits set on in-kernel errors (may be NULL).
@@ -41,7 +42,8 @@ memspec_status memspec_op_linear(const void* x_dev, const void* w_dev, float* y_
  * counterpart; this is a property of the library's interface.
  * Instead of a scratch argument it uses one file-scope device array of about
  * 2.6 MB that every GPU loading the library keeps until the process exits.
- * Limits: rows in 1..16, n_out in 1..131072, k a positive multiple of 8; x and w
+ * Limits: rows in 1..16, n_out in 1..131072, k a positive multiple of 8 up to
+ * 2^20; x and w
  * 16-byte aligned.  Larger sizes return MEMSPEC_ERR_INVALID_ARG (message in
  * memspec_op_last_error) and enqueue nothing.  The call allocates nothing; it
  * enqueues a clear of the array's counters and the kernel on `stream`.

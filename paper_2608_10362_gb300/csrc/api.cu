@@ -200,10 +200,10 @@ AttnGeo attn_geometry(const memspec_model_cfg& c, int groups, int R, int max_seq
   want = std::min(want, max_splits);
   g.chunk = round_up(ceil_div(max_seq, want), 64);
   g.n_splits = ceil_div(max_seq, g.chunk);
-  // the combine keeps (n_splits + 1) x qmax floats of split weights in the CTA's
-  // shared memory (3 stages x 64 keys x hd x 2 x 2 bytes, last 16 bytes reserved)
+  // the combine keeps (2 n_splits + 1) x qmax floats of split statistics in the
+  // CTA's shared memory (3 stages x 64 keys x hd x 2 x 2 bytes, last 16 bytes reserved)
   const size_t smem = static_cast<size_t>(3) * 2 * 64 * c.head_dim * 2 - 16;
-  while (static_cast<size_t>(g.n_splits + 1) * g.qmax * 4 > smem) {
+  while (static_cast<size_t>(2 * g.n_splits + 1) * g.qmax * 4 > smem) {
     g.chunk *= 2;
     g.n_splits = ceil_div(max_seq, g.chunk);
   }
@@ -428,7 +428,7 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   const size_t o_ops = w.take(op_bytes);
   const size_t o_done = w.take(done_ints * 4);
   const size_t trace_bytes =
-      p->trace == 1 ? (2 + static_cast<size_t>(kPassTraceOps) * nsm * 4) * 8 : 0;
+      p->trace == 1 ? (2 + static_cast<size_t>(kPassTraceOps) * nsm * kPassTraceSlots) * 8 : 0;
   const size_t o_trace = w.take(trace_bytes);
   if (c != nullptr) {
     c->trace = trace_bytes ? reinterpret_cast<unsigned long long*>(base + o_trace) : nullptr;
@@ -1469,7 +1469,7 @@ static memspec_status buffer_span(memspec_ctx* c, int32_t buf, void** ptr, size_
     case MEMSPEC_BUF_PASS_TRACE:
       if (c->trace == nullptr) return fail(c, MEMSPEC_ERR_INVALID_ARG, "tracing is off (init param trace)");
       *ptr = c->trace;
-      *cap = (2 + static_cast<size_t>(kPassTraceOps) * sm_count() * 4) * 8;
+      *cap = (2 + static_cast<size_t>(kPassTraceOps) * sm_count() * kPassTraceSlots) * 8;
       break;
     default: return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown buffer id");
   }
@@ -1549,8 +1549,10 @@ memspec_status memspec_op_linear(const void* x, const void* w, float* y, int32_t
     g_op_error = "null pointer";
     return MEMSPEC_ERR_INVALID_ARG;
   }
-  if (rows < 1 || rows > kMaxRows || n_out < 1 || k < 8 || k % 8 != 0) {
-    g_op_error = "rows must be in 1..256, n_out >= 1, k a positive multiple of 8";
+  if (rows < 1 || rows > kMaxRows || n_out < 1 || k < 8 || k % 8 != 0 ||
+      !sk_fits(static_cast<long long>(ceil_div(n_out, 128)) * ceil_div(k, 64), sm_count())) {
+    g_op_error = "rows must be in 1..256, n_out >= 1, k a positive multiple of 8, "
+                 "and ceil(n_out/128) * ceil(k/64) below 2^32 / (SMs + 1)";
     return MEMSPEC_ERR_INVALID_ARG;
   }
   if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(w) & 15) ||

@@ -71,7 +71,8 @@ __host__ __device__ constexpr size_t attention_smem_bytes_hd() {
 // threads together, when the unit has no work.
 template <int HD, class Sync>
 __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh, int rb, int split,
-                                              uint8_t* smem_raw, int tid, Sync sync) {
+                                              uint8_t* smem_raw, int tid, Sync sync,
+                                              unsigned long long* ts = nullptr) {
   constexpr int kChunks = HD / 8;                        // 16-byte chunks per row
   constexpr int kTileBytes = kKeyTile * HD * 2;          // one K (or V) tile
   constexpr int kNT = HD / 8;                            // n8 tiles of the output
@@ -316,53 +317,101 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
       a.part_ml[(pbase + v) * 2 + 1] = L;
     }
   }
-  __threadfence();
+  trace_at(ts, 4);
+  // same arrival protocol as the GEMM split-K: the barrier orders this CTA's
+  // partial stores before thread 0's acq_rel arrival; the last split's acquire
+  // and the next barrier order every split's partials before its loads
   sync();
   int* last = reinterpret_cast<int*>(kv + attention_smem_bytes_hd<HD>() - 16);
-  if (tid == 0) *last = (atomicAdd(&a.counters[unit], 1) == n_active - 1) ? 1 : 0;
+  if (tid == 0) *last = (atom_add_acq_rel_gpu(&a.counters[unit], 1) == n_active - 1) ? 1 : 0;
   sync();
+  trace_at(ts, 5);
   if (!*last) return;
-  __threadfence();
   const size_t ubase = static_cast<size_t>(unit) * a.n_splits * a.qmax;
-  // split weights 2^(m_s - M) and 1/L per query vector, computed once in shared memory
-  float* wsm = reinterpret_cast<float*>(kv);                // [n_active][nq]
-  float* linv = wsm + n_active * nq;                        // [nq]
+  const int qmax = a.qmax;
+  const float* part_ml = a.part_ml;
+  const float* part_o = a.part_o;
+  // (m_s, l_s) of every split and query vector, fetched together into shared
+  // memory; then the split weights 2^(m_s - M) (in place of m_s) and 1/L
+  float* msm = reinterpret_cast<float*>(kv);               // [n_active][nq]
+  float* lsm = msm + n_active * nq;                         // [n_active][nq]
+  float* linv = lsm + n_active * nq;                        // [nq]
+  const int n_ml = n_active * nq;
+  for (int i0 = tid; i0 < n_ml; i0 += 4 * kAttThreads) {
+    float2 t[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = i0 + q * kAttThreads;
+      if (i < n_ml) {
+        const int sp = i / nq, v = i - sp * nq;
+        t[q] = ld_cg_f2(part_ml + (ubase + static_cast<size_t>(sp) * qmax + v) * 2);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int i = i0 + q * kAttThreads;
+      if (i < n_ml) {
+        msm[i] = t[q].x;
+        lsm[i] = t[q].y;
+      }
+    }
+  }
+  sync();
   for (int v = tid; v < nq; v += kAttThreads) {
     float M = -INFINITY;
-    for (int s = 0; s < n_active; ++s) M = fmaxf(M, ld_cg_f(a.part_ml + (ubase + s * a.qmax + v) * 2));
+    for (int sp = 0; sp < n_active; ++sp) M = fmaxf(M, msm[sp * nq + v]);
     float L = 0.f;
-    for (int s = 0; s < n_active; ++s) {
-      const size_t pv = ubase + s * a.qmax + v;
-      const float ms = ld_cg_f(a.part_ml + pv * 2);
+    for (int sp = 0; sp < n_active; ++sp) {
+      const float ms = msm[sp * nq + v];
       const float w = ms == -INFINITY ? 0.f : exp2f(ms - M);
-      wsm[s * nq + v] = w;
-      L += w * ld_cg_f(a.part_ml + pv * 2 + 1);
+      msm[sp * nq + v] = w;
+      L += w * lsm[sp * nq + v];
     }
     linv[v] = 1.f / L;
   }
   sync();
-  for (int idx = tid; idx < nq * HD; idx += kAttThreads) {
-    const int v = idx / HD, d = idx - v * HD;
-    float O = 0.f;
-    for (int s0 = 0; s0 < n_active; s0 += 4) {   // four splits fetched at once, summed in order
-      float ov[4];
+  trace_at(ts, 6);
+  // weighted sum of the split outputs, four features per thread, eight splits
+  // fetched at once and added in ascending split order
+  constexpr int kV4 = HD / 4;
+  bf16* out = a.out;
+  bf16* out_lo = a.out_lo;
+  const int H = a.H;
+  for (int idx = tid; idx < nq * kV4; idx += kAttThreads) {
+    const int v = idx / kV4, d = (idx - v * kV4) * 4;
+    float O[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int s0 = 0; s0 < n_active; s0 += 8) {
+      float4 ov[8];
 #pragma unroll
-      for (int q = 0; q < 4; ++q)
-        ov[q] = (s0 + q < n_active) ? ld_cg_f(a.part_o + (ubase + (s0 + q) * a.qmax + v) * HD + d) : 0.f;
+      for (int q = 0; q < 8; ++q)
+        if (s0 + q < n_active)
+          ov[q] = ld_cg_f4(part_o + (ubase + static_cast<size_t>(s0 + q) * qmax + v) * HD + d);
 #pragma unroll
-      for (int q = 0; q < 4; ++q)
-        if (s0 + q < n_active) O += wsm[(s0 + q) * nq + v] * ov[q];
+      for (int q = 0; q < 8; ++q) {
+        if (s0 + q < n_active) {
+          const float w = msm[(s0 + q) * nq + v];
+          O[0] += w * ov[q].x;
+          O[1] += w * ov[q].y;
+          O[2] += w * ov[q].z;
+          O[3] += w * ov[q].w;
+        }
+      }
     }
     const int hl = v / nr, rr = v - hl * nr;
     const int row = g * R + r_lo + rr;
     const int h = kvh * gs + hl;
-    const size_t oi = (static_cast<size_t>(row) * a.H + h) * HD + d;
-    if (a.out_lo != nullptr) {
-      split_bf16(O * linv[v], a.out[oi], a.out_lo[oi]);
-    } else {
-      a.out[oi] = __float2bfloat16_rn(O * linv[v]);
+    const size_t oi = (static_cast<size_t>(row) * H + h) * HD + d;
+    const float li = linv[v];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      if (out_lo != nullptr) {
+        split_bf16(O[e] * li, out[oi + e], out_lo[oi + e]);
+      } else {
+        out[oi + e] = __float2bfloat16_rn(O[e] * li);
+      }
     }
   }
+  trace_at(ts, 7);
   if (tid == 0) a.counters[unit] = 0;
 }
 

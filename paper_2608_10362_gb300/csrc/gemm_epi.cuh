@@ -42,134 +42,238 @@ __device__ __forceinline__ bool row_valid(const GemmArgs& a, int r) {
   return a.plan == nullptr ? true : plan_row_valid(a.plan, r);
 }
 
+// Row metadata of one 8-row group of a chunk, read from the row plan.  Every
+// global value an epilogue reads is loaded before its first global store: the
+// compiler cannot prove that the stores do not alias the loads, so interleaving
+// them would cost one dependent L2 round trip per row.
+struct RowMeta {
+  uint32_t valid;   // bit j: row r0 + j is valid
+  uint32_t last;    // bit j: row r0 + j is the last valid row of its group
+  int grp[8];       // group of the row
+  int pos[8];       // its position (plan rows only)
+  int req[8];       // its request (plan rows only)
+};
+
+__device__ __forceinline__ void row_meta(const GemmArgs& a, int r0, RowMeta& m) {
+  const RowPlan* plan = a.plan;
+  const int rows_total = a.rows_total;
+  m.valid = 0;
+  m.last = 0;
+  if (plan == nullptr) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      m.grp[j] = 0;
+      m.pos[j] = 0;
+      m.req[j] = 0;
+      if (r0 + j < rows_total) m.valid |= 1u << j;
+    }
+    return;
+  }
+  const int R = plan->rows_per_group;
+  int nv[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int r = r0 + j;
+    const int g = r < rows_total ? r / R : 0;
+    m.grp[j] = g;
+    nv[j] = plan->valid[g];
+    m.pos[j] = plan->pos0[g];
+    m.req[j] = plan->req[g];
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int r = r0 + j;
+    const int i = r - m.grp[j] * R;
+    m.pos[j] += i;
+    if (r < rows_total && i < nv[j]) m.valid |= 1u << j;
+    if (r < rows_total && i == nv[j] - 1) m.last |= 1u << j;
+  }
+}
+
 // Epilogue for one 16-row chunk of a finished 128-feature row tile.  Called by
 // the 128 epilogue threads together; et = feature within the tile (= TMEM lane).
 static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*red)[16], float* stage,
-                                            const float* rms, int rt, int chunk, int et,
-                                            const float* vin) {
+                                                   const float* rms, int rt, int chunk, int et,
+                                                   const float* vin,
+                                                   unsigned long long* ts = nullptr) {
   const int ew = et >> 5, lane = et & 31;
+  const int epi = a.epi;
+  const int rows_total = a.rows_total;
+  const int r0 = chunk * 16;
   float v[16];
+  if (a.rms) {
 #pragma unroll
-  for (int j = 0; j < 16; ++j) v[j] = a.rms ? vin[j] * rms[chunk * 16 + j] : vin[j];
-  if (a.epi == EPI_F32) {
+    for (int j = 0; j < 16; ++j) v[j] = vin[j] * rms[r0 + j];
+  } else {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] = vin[j];
+  }
+  if (epi == EPI_F32) {
     const int f = rt * kTileM + et;
-    if (f < a.n_out) {
+    const int n_out = a.n_out, out_ld = a.out_ld, last_only = a.last_only;
+    const long long gstride = a.out_group_stride;
+    float* out = a.out;
+#pragma unroll 1
+    for (int half = 0; half < 2; ++half) {
+      RowMeta m;
+      row_meta(a, r0 + half * 8, m);
+      if (f < n_out) {
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int r = chunk * 16 + j;
-        if (!row_valid(a, r)) continue;
-        if (a.last_only) {
-          const int g = r / a.plan->rows_per_group;
-          const int i = r - g * a.plan->rows_per_group;
-          if (i != a.plan->valid[g] - 1) continue;
-          a.out[g * a.out_group_stride + f] = v[j];
-        } else {
-          a.out[static_cast<size_t>(r) * a.out_ld + f] = v[j];
+        for (int j = 0; j < 8; ++j) {
+          const int r = r0 + half * 8 + j;
+          if (last_only) {
+            if (m.last & (1u << j)) out[m.grp[j] * gstride + f] = v[half * 8 + j];
+          } else if (m.valid & (1u << j)) {
+            out[static_cast<size_t>(r) * out_ld + f] = v[half * 8 + j];
+          }
         }
       }
     }
     return;
   }
-  if (a.epi == EPI_RESIDUAL) {
+  if (epi == EPI_RESIDUAL) {
     const int f = rt * kTileM + et;  // n_out is a multiple of 128 (d_model)
+    float* h = a.h;
+    const int h_ld = a.h_ld;
+    const bf16* gain_next = a.gain_next;
+    bf16* xg_out = a.xg_out;
+    bf16* xg_lo_out = a.xg_lo_out;
+    float* ss_out = a.ss_out;
+    const int ss_stride = a.ss_stride;
+    const float gain = gain_next != nullptr ? __bfloat162float(gain_next[f]) : 0.f;
+    float hn[16], sq[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+      hn[j] = (r0 + j < rows_total) ? h[static_cast<size_t>(r0 + j) * h_ld + f] : 0.f;
+    trace_after(ts, 8, hn[15] + gain);
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
-      const int r = chunk * 16 + j;
-      float sq = 0.f;
-      if (r < a.rows_total) {
-        float* hp = a.h + static_cast<size_t>(r) * a.h_ld + f;
-        const float hn = *hp + v[j];
-        *hp = hn;
-        sq = hn * hn;
-        if (a.gain_next != nullptr) {
-          const float xv = hn * __bfloat162float(a.gain_next[f]);
-          const size_t o = static_cast<size_t>(r) * a.h_ld + f;
-          if (a.xg_lo_out != nullptr) {
-            split_bf16(xv, a.xg_out[o], a.xg_lo_out[o]);
-          } else {
-            a.xg_out[o] = __float2bfloat16_rn(xv);
-          }
+      hn[j] += v[j];
+      sq[j] = (r0 + j < rows_total) ? hn[j] * hn[j] : 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const int r = r0 + j;
+      if (r >= rows_total) continue;
+      const size_t o = static_cast<size_t>(r) * h_ld + f;
+      h[o] = hn[j];
+      if (gain_next != nullptr) {
+        const float xv = hn[j] * gain;
+        if (xg_lo_out != nullptr) {
+          split_bf16(xv, xg_out[o], xg_lo_out[o]);
+        } else {
+          xg_out[o] = __float2bfloat16_rn(xv);
         }
       }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-      if (lane == 0) red[ew][j] = sq;
     }
+    // per-row sums over the warp's 32 features: the 16 butterflies interleaved
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) sq[j] += __shfl_xor_sync(0xffffffffu, sq[j], o);
+    }
+    if (lane == 0) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) red[ew][j] = sq[j];
+    }
+    trace_at(ts, 9);
     named_bar_sync(1, 128);
+    trace_at(ts, 10);
     if (et < 16) {
-      const int r = chunk * 16 + et;
-      if (r < a.rows_total) {
+      const int r = r0 + et;
+      if (r < rows_total) {
         const float s = ((red[0][et] + red[1][et]) + red[2][et]) + red[3][et];
-        a.ss_out[static_cast<size_t>(rt) * a.ss_stride + r] = s;
+        ss_out[static_cast<size_t>(rt) * ss_stride + r] = s;
       }
     }
     named_bar_sync(1, 128);
+    trace_at(ts, 11);
     return;
   }
   // staged epilogues: make the whole 128 x 16 chunk visible to all 128 threads
 #pragma unroll
   for (int j = 0; j < 16; ++j) stage[et * kStagePitch + j] = v[j];
   named_bar_sync(1, 128);
-  if (a.epi == EPI_SWIGLU) {
+  if (epi == EPI_SWIGLU) {
     if (et < 64) {
       const int f = rt * 64 + et;
       if (f < a.n_out) {
+        bf16* act = a.act;
+        bf16* act_lo = a.act_lo;
+        const int act_ld = a.act_ld;
+        float y[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
-          const int r = chunk * 16 + j;
-          if (r >= a.rows_total) continue;
           const float g = stage[et * kStagePitch + j];
           const float u = stage[(et + 64) * kStagePitch + j];
-          const float sg = g / (1.0f + expf(-g));
-          const size_t o = static_cast<size_t>(r) * a.act_ld + f;
-          if (a.act_lo != nullptr) {
-            split_bf16(sg * u, a.act[o], a.act_lo[o]);
+          y[j] = g / (1.0f + expf(-g)) * u;
+        }
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int r = r0 + j;
+          if (r >= rows_total) continue;
+          const size_t o = static_cast<size_t>(r) * act_ld + f;
+          if (act_lo != nullptr) {
+            split_bf16(y[j], act[o], act_lo[o]);
           } else {
-            a.act[o] = __float2bfloat16_rn(sg * u);
+            act[o] = __float2bfloat16_rn(y[j]);
           }
         }
       }
     }
   } else {  // EPI_QKV: RoPE on q and k, K/V appended to the cache
     const int f = rt * kTileM + et;
-    const int hd = a.head_dim, half = hd >> 1;
+    const int q_dim = a.q_dim, kv_dim = a.kv_dim;
+    const int hd = a.head_dim, half_hd = hd >> 1;
+    const int n_kv_heads = a.n_kv_heads, max_seq = a.max_seq;
+    float* q_out = a.q_out;
+    const float* rope_cos = a.rope_cos;
+    const float* rope_sin = a.rope_sin;
     int seg, fs;
-    if (f < a.q_dim) {
+    if (f < q_dim) {
       seg = 0;
       fs = f;
-    } else if (f < a.q_dim + a.kv_dim) {
+    } else if (f < q_dim + kv_dim) {
       seg = 1;
-      fs = f - a.q_dim;
+      fs = f - q_dim;
     } else {
       seg = 2;
-      fs = f - a.q_dim - a.kv_dim;
+      fs = f - q_dim - kv_dim;
     }
     const int head = fs / hd, d = fs - head * hd;
-    const int ip = d < half ? d : d - half;   // rotation pair index
-    const int e1 = et - d + ip;               // staging index of element ip of this head
+    const int ip = d < half_hd ? d : d - half_hd;   // rotation pair index
+    const int e1 = et - d + ip;                     // staging index of element ip of this head
+    bf16* cache = seg == 1 ? a.kcache : a.vcache;
 #pragma unroll 1
-    for (int j = 0; j < 16; ++j) {
-      const int r = chunk * 16 + j;
-      if (!row_valid(a, r)) continue;
-      const int g = r / a.plan->rows_per_group;
-      const int i = r - g * a.plan->rows_per_group;
-      const int pos = a.plan->pos0[g] + i;
-      if (pos < 0 || pos >= a.max_seq) continue;   // flagged by the embedding kernel
-      float val = stage[et * kStagePitch + j];
-      if (seg < 2) {
-        const float x1 = stage[e1 * kStagePitch + j];
-        const float x2 = stage[(e1 + half) * kStagePitch + j];
-        const float c = a.rope_cos[static_cast<size_t>(pos) * half + ip];
-        const float s = a.rope_sin[static_cast<size_t>(pos) * half + ip];
-        val = d < half ? (x1 * c - x2 * s) : (x1 * s + x2 * c);
+    for (int half = 0; half < 2; ++half) {
+      RowMeta m;
+      row_meta(a, r0 + half * 8, m);
+      float y[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int jj = half * 8 + j;
+        // invalid positions were flagged by the embedding kernel: skip the row
+        if (m.pos[j] < 0 || m.pos[j] >= max_seq) m.valid &= ~(1u << j);
+        y[j] = stage[et * kStagePitch + jj];
+        if (seg < 2) {
+          const size_t ri = (m.valid & (1u << j)) ? static_cast<size_t>(m.pos[j]) * half_hd + ip : 0;
+          const float c = rope_cos[ri], sn = rope_sin[ri];
+          const float x1 = stage[e1 * kStagePitch + jj];
+          const float x2 = stage[(e1 + half_hd) * kStagePitch + jj];
+          y[j] = d < half_hd ? (x1 * c - x2 * sn) : (x1 * sn + x2 * c);
+        }
       }
-      if (seg == 0) {
-        a.q_out[static_cast<size_t>(r) * a.q_dim + f] = val;
-      } else {
-        const int req = a.plan->req[g];
-        const size_t off =
-            ((static_cast<size_t>(req) * a.n_kv_heads + head) * a.max_seq + pos) * hd + d;
-        (seg == 1 ? a.kcache : a.vcache)[off] = __float2bfloat16_rn(val);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (!(m.valid & (1u << j))) continue;
+        const int r = r0 + half * 8 + j;
+        if (seg == 0) {
+          q_out[static_cast<size_t>(r) * q_dim + f] = y[j];
+        } else {
+          const size_t off =
+              ((static_cast<size_t>(m.req[j]) * n_kv_heads + head) * max_seq + m.pos[j]) * hd + d;
+          cache[off] = __float2bfloat16_rn(y[j]);
+        }
       }
     }
   }
@@ -208,7 +312,8 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, int layout, 
                                                  int G, int rt, int k0, int k1, float* stage,
                                                  const float* rms, float (*red)[16],
                                                  int* reduce_flag, uint64_t* acc_empty, int et,
-                                                 int ew, int lane) {
+                                                 int ew, int lane,
+                                                 unsigned long long* ts = nullptr) {
   const int KT = a.k_tiles;
   const int T = a.row_tiles * KT;
   const bool full = (k0 == 0 && k1 == KT);
@@ -245,17 +350,21 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, int layout, 
   __syncwarp();
   if (lane == 0) mbar_arrive(&acc_empty[buf]);
   if (full) return;
-  __threadfence();
+  trace_at(ts, 4);
+  // The barrier orders this CTA's partial stores before thread 0's arrival, whose
+  // release (acq_rel, GPU scope) publishes them; the last contributor's acquire
+  // and the second barrier order every other contributor's partials before its
+  // loads (which bypass L1).
   named_bar_sync(1, 128);
   const int c_first = sk_cta_of(rt * KT, T, G);
   const int c_last = sk_cta_of((rt + 1) * KT - 1, T, G);
   if (et == 0) {
-    const int old = atomicAdd(&a.counters[rt], 1);
+    const int old = atom_add_acq_rel_gpu(&a.counters[rt], 1);
     *reduce_flag = (old == c_last - c_first) ? 1 : 0;
   }
   named_bar_sync(1, 128);
+  trace_at(ts, 5);
   if (!*reduce_flag) return;
-  __threadfence();
   for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
 #pragma unroll
     for (int j = 0; j < 16; ++j) v[j] = 0.f;
@@ -286,8 +395,10 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, int layout, 
         }
       }
     }
-    apply_epilogue(a, red, stage, rms, rt, chunk, et, v);
+    if (chunk == 0) trace_after(ts, 6, v[15]);
+    apply_epilogue(a, red, stage, rms, rt, chunk, et, v, ts);
   }
+  trace_at(ts, 7);
   if (et == 0) a.counters[rt] = 0;
 }
 

@@ -234,12 +234,19 @@ __host__ __device__ inline float philox_uniform(unsigned long long seed, int req
 }
 
 // Stream-K schedule: CTA c of G processes global tiles [begin(c), begin(c+1)).
+// 32-bit arithmetic: the host guarantees (T + 1) * (G + 1) < 2^32 for every GEMM
+// (sk_fits).
+inline bool sk_fits(long long T, int G) { return (T + 1) * (G + 1) < (1LL << 32); }
 __host__ __device__ inline int sk_begin(int c, int T, int G) {
-  return static_cast<int>((static_cast<long long>(c) * T) / G);
+  return static_cast<int>((static_cast<unsigned>(c) * static_cast<unsigned>(T)) /
+                          static_cast<unsigned>(G));
 }
 // The CTA whose range contains tile t.
 __host__ __device__ inline int sk_cta_of(int t, int T, int G) {
-  return static_cast<int>(((static_cast<long long>(t) + 1) * G + T - 1) / T) - 1;
+  return static_cast<int>(((static_cast<unsigned>(t) + 1u) * static_cast<unsigned>(G) +
+                           static_cast<unsigned>(T) - 1u) /
+                          static_cast<unsigned>(T)) -
+         1;
 }
 
 }  // namespace memspec

@@ -107,9 +107,9 @@ extern "C" memspec_status memspec_op_linear_noalloc(const void* x, const void* w
     return MEMSPEC_ERR_INVALID_ARG;
   }
   if (rows < 1 || rows > kNoAllocMaxRows || n_out < 1 || n_out > kNoAllocMaxRowTiles * 128 ||
-      k < 8 || k % 8 != 0) {
+      k < 8 || k % 8 != 0 || k > (1 << 20)) {
     set_op_error("sizes beyond this entry point's fixed scratch: rows must be in 1..16, "
-                      "n_out in 1..131072, k a positive multiple of 8");
+                      "n_out in 1..131072, k a positive multiple of 8 up to 2^20");
     return MEMSPEC_ERR_INVALID_ARG;
   }
   if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(w) & 15)) {

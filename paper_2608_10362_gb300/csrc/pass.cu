@@ -47,43 +47,68 @@ struct PassCtl {
   int abort_flag;
   int reduce_flag;
   int wait_ok;
+  int ops_ready;     // highest op whose inputs are complete (workers -> producer)
   float red[4][16];
   float red8[8];
 };
 
-__device__ __forceinline__ int ld_acquire(const int* p) {
+// Completion counters are polled with relaxed loads (they read L2 and leave the
+// SM's L1 alone); one acquire fence follows the successful poll.
+__device__ __forceinline__ int ld_relaxed(const int* p) {
   int v;
-  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  asm volatile("ld.relaxed.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
 
 // Bounded wait until done[n] reaches `target`; false on timeout or abort.
 __device__ bool wait_done(const int* done, int n, int target, volatile int* abort_flag,
                           uint32_t* status) {
-  if (ld_acquire(done + n) >= target) return true;
-  const long long t0 = clock64();
-  while (ld_acquire(done + n) < target) {
-    if (*abort_flag) return false;
-    if (clock64() - t0 > kWaitBudgetCycles) {
-      *abort_flag = 1;
-      atomicOr(status, 0x1u);
-      return false;
+  if (ld_relaxed(done + n) < target) {
+    const long long t0 = clock64();
+    while (ld_relaxed(done + n) < target) {
+      if (*abort_flag) return false;
+      if (clock64() - t0 > kWaitBudgetCycles) {
+        *abort_flag = 1;
+        atomicOr(status, 0x1u);
+        return false;
+      }
+      __nanosleep(32);
     }
-    __nanosleep(64);
   }
+  asm volatile("fence.acq_rel.gpu;" ::: "memory");
   return true;
 }
 
-__device__ __forceinline__ unsigned long long global_ns() {
-  unsigned long long t;
-  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
-  return t;
+// The worker group tells the activation producer of its own CTA that op n may
+// start (ops_ready = n) once it has observed done[n - 1]: one poller per CTA.
+__device__ __forceinline__ void publish_ready(volatile int* ops_ready, int n) {
+  __threadfence_block();
+  *ops_ready = n;
+}
+
+// Bounded wait of the activation producer until ops_ready >= n.
+__device__ bool wait_ready(volatile int* ops_ready, int n, volatile int* abort_flag,
+                           uint32_t* status) {
+  if (*ops_ready < n) {
+    const long long t0 = clock64();
+    while (*ops_ready < n) {
+      if (*abort_flag) return false;
+      if (clock64() - t0 > kWaitBudgetCycles) {
+        *abort_flag = 1;
+        atomicOr(status, 0x1u);
+        return false;
+      }
+      __nanosleep(32);
+    }
+  }
+  __threadfence_block();
+  return true;
 }
 
 // Trace slot of (op n, this CTA, event e), or nullptr when tracing is off.
 __device__ __forceinline__ unsigned long long* trace_slot(const PassArgs& p, int n, int e) {
   if (p.trace == nullptr || n >= kPassTraceOps) return nullptr;
-  return p.trace + 2 + (static_cast<size_t>(n) * gridDim.x + blockIdx.x) * 4 + e;
+  return p.trace + 2 + (static_cast<size_t>(n) * gridDim.x + blockIdx.x) * kPassTraceSlots + e;
 }
 
 __device__ __forceinline__ void fence_proxy_async_global() {
@@ -124,6 +149,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
     mbar_init(&ctl.drain, 1);
     ctl.abort_flag = 0;
     ctl.reduce_flag = 0;
+    ctl.ops_ready = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -156,7 +182,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
         const int plane_bytes = a.n_pad * 128;
         if (!weights) {
           // activations are written by op n-1 (and earlier): wait until it completed
-          if (n > 0 && !wait_done(p.done, n - 1, G, abort_flag, p.status)) {
+          if (n > 0 && !wait_ready(&ctl.ops_ready, n, abort_flag, p.status)) {
             ok = false;
             break;
           }
@@ -280,7 +306,11 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
     for (int n = 0; n < p.n_ops && ok; ++n) {
       const PassOp& op = p.ops[n];
       if (n > 0) {   // everything this op reads was written by op n-1 or earlier
-        if (tid == 0) ctl.wait_ok = wait_done(p.done, n - 1, G, abort_flag, p.status) ? 1 : 0;
+        if (tid == 0) {
+          const bool ok_n = wait_done(p.done, n - 1, G, abort_flag, p.status);
+          ctl.wait_ok = ok_n ? 1 : 0;
+          if (ok_n) publish_ready(&ctl.ops_ready, n);
+        }
         wsync();
         const int wok = ctl.wait_ok;
         wsync();
@@ -324,7 +354,8 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
             }
             tc_fence_after();
             epilogue_segment(a, layout, acols, tmem_base, buf, lseg, c, Gn, rt, k0, k1, stage, rms,
-                             ctl.red, &ctl.reduce_flag, ctl.acc_empty, et, ew, lane);
+                             ctl.red, &ctl.reduce_flag, ctl.acc_empty, et, ew, lane,
+                             tid == 0 ? trace_slot(p, n, 0) : nullptr);
             t = seg_end;
           }
         }
@@ -337,9 +368,11 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
           const int kr = rem / at.n_splits, split = rem - kr * at.n_splits;
           const int kvh = kr / at.row_blocks, rb = kr - kvh * at.row_blocks;
           if (at.hd == 64)
-            attn::attention_cta<64>(at, g, kvh, rb, split, attn_smem, tid, wsync);
+            attn::attention_cta<64>(at, g, kvh, rb, split, attn_smem, tid, wsync,
+                                    tid == 0 ? trace_slot(p, n, 0) : nullptr);
           else
-            attn::attention_cta<128>(at, g, kvh, rb, split, attn_smem, tid, wsync);
+            attn::attention_cta<128>(at, g, kvh, rb, split, attn_smem, tid, wsync,
+                                     tid == 0 ? trace_slot(p, n, 0) : nullptr);
           wsync();
         }
       } else if (op.type == OP_SAMPLE) {

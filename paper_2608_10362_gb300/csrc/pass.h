@@ -34,12 +34,16 @@ struct PassArgs {
   uint32_t tmem_cols;  // TMEM columns allocated (power of two)
   uint32_t* status;
   // nullptr, or per-op timestamps (globaltimer ns) of this launch:
-  // trace[0] = n_ops, trace[1] = grid, then [n_ops][grid][4] = {worker start,
-  // worker end, activation loads issued, first MMA issued} (0 where not taken)
+  // trace[0] = n_ops, trace[1] = grid, then [n_ops][grid][kPassTraceSlots] =
+  // {worker start, worker end, activation loads issued, first MMA issued,
+  //  partials / split outputs stored, arrival counted, reduction inputs loaded,
+  //  reduction epilogue done, then epilogue-internal points 8..15} (slots an op
+  //  does not reach keep older values)
   unsigned long long* trace;
 };
 
 constexpr int kPassTraceOps = 2048;   // ops a trace buffer holds
+constexpr int kPassTraceSlots = 16;
 
 size_t pass_smem_bytes(const PassArgs& p);
 int pass_pick_stages(int b_stage_bytes, int attn_bytes);

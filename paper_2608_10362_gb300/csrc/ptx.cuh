@@ -207,6 +207,35 @@ __device__ __forceinline__ float4 ld_cg_f4(const float* p) {
                : "l"(p));
   return v;
 }
+// Global nanosecond timer (comparable across SMs), for optional tracing.
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Record the time in ts[k] when tracing (ts != nullptr).
+__device__ __forceinline__ void trace_at(unsigned long long* ts, int k) {
+  if (ts != nullptr) ts[k] = global_ns();
+}
+// Same, taken only once `dep` is available (a load it depends on has landed).
+__device__ __forceinline__ void trace_after(unsigned long long* ts, int k, float dep) {
+  if (ts != nullptr) {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t) : "f"(dep));
+    ts[k] = t;
+  }
+}
+__device__ __forceinline__ float2 ld_cg_f2(const float* p) {
+  float2 v;
+  asm volatile("ld.global.cg.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "l"(p));
+  return v;
+}
+// Atomic add with acquire-release semantics at GPU scope; returns the old value.
+__device__ __forceinline__ int atom_add_acq_rel_gpu(int* p, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
 __device__ __forceinline__ float ld_cg_f(const float* p) {
   float v;
   asm volatile("ld.global.cg.f32 %0, [%1];" : "=f"(v) : "l"(p));

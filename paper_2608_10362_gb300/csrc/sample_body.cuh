@@ -298,17 +298,16 @@ __device__ void accept_row(const AcceptArgs& a, int rho, int g, SampleSmem& sm, 
                                : a.zd + (static_cast<size_t>(g) * K + (rho - K - 1)) * V;
   const RowStats st = row_stats<NT>(zrow, V, a.inv_temp, greedy, sm, tid, sync);
   float* part = a.part + (static_cast<size_t>(g) * (2 * K + 1) + rho) * 4;
+  // thread 0 stores this row's statistics and arrives with release semantics; the
+  // block completing the group acquires them all through the same atomic
   if (tid == 0) {
     part[0] = st.m;
     part[1] = st.s;
     part[2] = __int_as_float(st.arg);
+    sm.is_last = (atom_add_acq_rel_gpu(&a.counters[g], 1) == 2 * K) ? 1 : 0;
   }
-  __threadfence();
-  sync();
-  if (tid == 0) sm.is_last = (atomicAdd(&a.counters[g], 1) == 2 * K) ? 1 : 0;
   sync();
   if (!sm.is_last) return;
-  __threadfence();
 
   // ---- decision (the whole block reads the row statistics of group g)
   const float* pg = a.part + static_cast<size_t>(g) * (2 * K + 1) * 4;
@@ -317,29 +316,39 @@ __device__ void accept_row(const AcceptArgs& a, int rho, int g, SampleSmem& sm, 
   const int step = state[2];
   const int* x = a.draft_tokens + g * a.max_k;
   float* dbg = a.debug + static_cast<size_t>(g) * (2 * K + 2);
-  if (tid == 0) {
-    int n = 0;
-    if (greedy) {
-      while (n < K && x[n] == __float_as_int(ld_cg_f(pg + n * 4 + 2))) ++n;
-    } else {
-      while (n < K) {
-        const int xi = x[n];
-        const float* zt = a.zt + (static_cast<size_t>(g) * (K + 1) + n) * V;
-        const float* zd = a.zd + (static_cast<size_t>(g) * K + n) * V;
-        const float* ptn = pg + n * 4;
-        const float* pdn = pg + (K + 1 + n) * 4;
-        const float p = __expf(ld_cg_f(zt + xi) * a.inv_temp - ld_cg_f(ptn)) / ld_cg_f(ptn + 1);
-        const float q = __expf(ld_cg_f(zd + xi) * a.inv_temp - ld_cg_f(pdn)) / ld_cg_f(pdn + 1);
-        dbg[n] = p;
-        dbg[K + n] = q;
-        const float u = philox_uniform(a.seeds[g], g, step, K + n);
-        if (!(u * q <= p)) break;
-        ++n;
+  // draft position i < K is decided by thread i (all loads in flight together);
+  // n = the first rejected position (K if none)
+  if (tid < 32) {
+    bool acc = false;
+    float p = 0.f, q = 0.f;
+    if (tid < K) {
+      const int xi = x[tid];
+      if (greedy) {
+        acc = xi == __float_as_int(ld_cg_f(pg + tid * 4 + 2));
+      } else {
+        const float* zt = a.zt + (static_cast<size_t>(g) * (K + 1) + tid) * V;
+        const float* zd = a.zd + (static_cast<size_t>(g) * K + tid) * V;
+        const float* ptn = pg + tid * 4;
+        const float* pdn = pg + (K + 1 + tid) * 4;
+        const float zx = ld_cg_f(zt + xi), mt = ld_cg_f(ptn), st = ld_cg_f(ptn + 1);
+        const float dx = ld_cg_f(zd + xi), md = ld_cg_f(pdn), sd = ld_cg_f(pdn + 1);
+        p = __expf(zx * a.inv_temp - mt) / st;
+        q = __expf(dx * a.inv_temp - md) / sd;
+        const float u = philox_uniform(a.seeds[g], g, step, K + tid);
+        acc = u * q <= p;
       }
     }
-    sm.n = n;
-    sm.u = greedy ? 0.f : philox_uniform(a.seeds[g], g, step, 2 * K);
-    sm.y = greedy ? __float_as_int(ld_cg_f(pg + n * 4 + 2)) : -1;
+    const unsigned acc_mask = __ballot_sync(0xffffffffu, acc);
+    const int n = min(__ffs(~acc_mask) - 1, K);
+    if (!greedy && tid < K) {
+      dbg[tid] = p;
+      dbg[K + tid] = q;
+    }
+    if (tid == 0) {
+      sm.n = n;
+      sm.u = greedy ? 0.f : philox_uniform(a.seeds[g], g, step, 2 * K);
+      sm.y = greedy ? __float_as_int(ld_cg_f(pg + n * 4 + 2)) : -1;
+    }
   }
   sync();
   const int n = sm.n;
@@ -369,20 +378,28 @@ __device__ void accept_row(const AcceptArgs& a, int rho, int g, SampleSmem& sm, 
     }
   }
   // ---- commit: append x_1..x_n, y; lengths; KV rollback is the length update
+  int* res = a.results + g * (K + 2);
+  int* toks = a.tokens + static_cast<size_t>(g) * a.max_seq;
+  const bool fits = L + n + 1 <= a.max_seq;
+  if (fits && tid < K + 2) {
+    // slot tid of the result row: 0 = n, 1..n = accepted drafts, n + 1 = y, then -1
+    int val = -1;
+    if (tid == 0) {
+      val = n;
+    } else if (tid <= n) {
+      val = x[tid - 1];
+      toks[L + tid - 1] = val;
+    } else if (tid == n + 1) {
+      val = y;
+      toks[L + n] = y;
+    }
+    res[tid] = val;
+  }
   if (tid == 0) {
-    int* res = a.results + g * (K + 2);
-    res[0] = n;
-    int* toks = a.tokens + static_cast<size_t>(g) * a.max_seq;
-    if (L + n + 1 > a.max_seq) {
+    if (!fits) {
+      res[0] = n;
       atomicOr(a.status, 0x4u);
     } else {
-      for (int i = 0; i < n; ++i) {
-        toks[L + i] = x[i];
-        res[1 + i] = x[i];
-      }
-      toks[L + n] = y;
-      res[1 + n] = y;
-      for (int i = n + 2; i < K + 2; ++i) res[i] = -1;
       state[0] = L + n + 1;                          // committed length
       state[1] = L + n;                              // target KV valid below L'-1
       a.draft_len[g] = L + (n < K - 1 ? n : K - 1);  // draft KV valid below this count

@@ -229,14 +229,16 @@ class Engine:
         return toks.reshape(self.max_batch, self.max_seq)[req, :L]
 
     def pass_trace(self) -> np.ndarray:
-        """Timestamps (ns) of the last persistent launch, [n_ops][grid][4] =
-        worker start, worker end, activation loads issued, first MMA issued
-        (entries an op did not take keep older values)."""
+        """Timestamps (ns) of the last persistent launch, [n_ops][grid][16] =
+        worker start, worker end, activation loads issued, first MMA issued,
+        partials stored, arrival counted, reduction inputs loaded, reduction
+        done, then epilogue-internal points (entries an op did not reach keep
+        older values)."""
         head = self.read_buffer(_lib.BUF_PASS_TRACE, np.uint64, 2)
         n_ops, grid = int(head[0]), int(head[1])
         n = min(n_ops, _lib.PASS_TRACE_OPS)
-        t = self.read_buffer(_lib.BUF_PASS_TRACE, np.uint64, 2 + n * grid * 4)
-        return t[2:].reshape(n, grid, 4)
+        t = self.read_buffer(_lib.BUF_PASS_TRACE, np.uint64, 2 + n * grid * 16)
+        return t[2:].reshape(n, grid, 16)
 
     def target_logits(self, batch: int, K: int) -> np.ndarray:
         n = batch * (K + 1) * self.vocab
