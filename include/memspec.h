@@ -140,8 +140,8 @@ typedef struct memspec_init_params {
   int32_t launch_mode;              /* MEMSPEC_LAUNCH_PER_OP (0): one kernel launch per
                                        op of a pass; MEMSPEC_LAUNCH_PASS (1): each draft
                                        step and verify pass as one persistent launch */
-  int32_t trace;                    /* 1: the persistent launch records per-op
-                                       timestamps (MEMSPEC_BUF_PASS_TRACE) */
+  int32_t trace;                    /* per-op timestamps (MEMSPEC_BUF_PASS_TRACE) of
+                                       1: verify passes, 2: draft steps; 0: off */
 } memspec_init_params;
 
 enum { MEMSPEC_LAUNCH_PER_OP = 0, MEMSPEC_LAUNCH_PASS = 1 };
@@ -244,7 +244,7 @@ typedef enum memspec_buffer {
   MEMSPEC_BUF_SEQ_STATE = 4,     /* int32 [max_batch][4] = {L, Lt, step, active Ld} */
   MEMSPEC_BUF_ACCEPT_DEBUG = 5,  /* fp32 [batch][2K+2] = {p_i(x_i), q_i(x_i), residual mass, u'} */
   MEMSPEC_BUF_RESIDUAL = 6,      /* fp32 residual stream [rows][d] of the last forward */
-  MEMSPEC_BUF_PASS_TRACE = 7     /* u64 trace of the last persistent launch (trace = 1):
+  MEMSPEC_BUF_PASS_TRACE = 7     /* u64 trace of the last traced pass (init param trace):
                                     {n_ops, grid, then [n_ops][grid][16] globaltimer ns =
                                     worker start, worker end, activation loads issued,
                                     first MMA issued, partials stored, arrival counted,

@@ -196,7 +196,8 @@ AttnGeo attn_geometry(const memspec_model_cfg& c, int groups, int R, int max_seq
   g.qmax = gs * rpb;
   const int units = groups * c.n_kv_heads * g.row_blocks;
   const int max_splits = ceil_div(max_seq, 64);
-  int want = std::max(1, ceil_div(2 * sm_count(), units));
+  // at most two CTAs per SM in one wave (an extra partial wave would double the time)
+  int want = std::max(1, (2 * sm_count()) / units);
   want = std::min(want, max_splits);
   g.chunk = round_up(ceil_div(max_seq, want), 64);
   g.n_splits = ceil_div(max_seq, g.chunk);
@@ -331,7 +332,7 @@ struct memspec_ctx {
   size_t done_area_ints = 0, done_area_used = 0;
   bool pass_kernel = false;  // draft / verify passes as one persistent launch
   bool cooperative = false;
-  unsigned long long* trace = nullptr;   // pass-kernel trace (init param trace = 1)
+  unsigned long long* trace = nullptr;   // per-op trace (init param trace = 1: verify, 2: draft)
   std::map<std::tuple<const void*, int, int, int>, CUtensorMap> bmaps;
 };
 
@@ -428,7 +429,9 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   const size_t o_ops = w.take(op_bytes);
   const size_t o_done = w.take(done_ints * 4);
   const size_t trace_bytes =
-      p->trace == 1 ? (2 + static_cast<size_t>(kPassTraceOps) * nsm * kPassTraceSlots) * 8 : 0;
+      (p->trace == 1 || p->trace == 2)
+          ? (2 + static_cast<size_t>(kPassTraceOps) * nsm * kPassTraceSlots) * 8
+          : 0;
   const size_t o_trace = w.take(trace_bytes);
   if (c != nullptr) {
     c->trace = trace_bytes ? reinterpret_cast<unsigned long long*>(base + o_trace) : nullptr;
@@ -811,7 +814,8 @@ struct OpTable {
 
 // Place `ops` in the workspace: synchronous copy (the table must be in place
 // before a graph that uses it is captured).
-memspec_status place_table(memspec_ctx* c, const std::vector<PassOp>& ops, OpTable* t) {
+memspec_status place_table(memspec_ctx* c, const std::vector<PassOp>& ops, OpTable* t,
+                           unsigned long long* trace) {
   const size_t bytes = ops.size() * sizeof(PassOp);
   const size_t ints = ops.size() + 1;
   if (bytes > c->op_area_bytes || ints > c->done_area_ints)
@@ -856,8 +860,27 @@ memspec_status place_table(memspec_ctx* c, const std::vector<PassOp>& ops, OpTab
   p.stages = pass_pick_stages(b_bytes, p.attn_bytes);
   p.tmem_cols = cols;
   p.status = c->status;
-  p.trace = c->trace;
+  p.trace = trace;
   if (p.stages < 2) return fail(c, MEMSPEC_ERR_UNSUPPORTED, "pass kernel: shared memory too small");
+  return MEMSPEC_OK;
+}
+
+// Per-op launches record into the trace too: op n's row starts at
+// 2 + n * SMs * 16; the header {n_ops, SMs} is written now (before any capture).
+memspec_status attach_trace(memspec_ctx* c, std::vector<PassOp>& ops) {
+  const int nsm = sm_count();
+  for (size_t n = 0; n < ops.size() && n < static_cast<size_t>(kPassTraceOps); ++n) {
+    unsigned long long* row = c->trace + 2 + n * nsm * kPassTraceSlots;
+    if (ops[n].type == OP_GEMM) ops[n].u.g.trace = row;
+    if (ops[n].type == OP_ATTN) {
+      ops[n].u.at.trace = row;
+      ops[n].u.at.trace_ctas = nsm;
+    }
+  }
+  const unsigned long long head[2] = {static_cast<unsigned long long>(ops.size()),
+                                      static_cast<unsigned long long>(nsm)};
+  cudaError_t e = cudaMemcpy(c->trace, head, sizeof(head), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(c, e, "trace header");
   return MEMSPEC_OK;
 }
 
@@ -884,9 +907,15 @@ memspec_status run_pass(memspec_ctx* c, const GraphKey& key, bool use_pass, Emit
   std::vector<PassOp> ops;
   memspec_status s = emit(ops);
   if (s != MEMSPEC_OK) return s;
+  // tracing: init param trace = 1 records verify passes, 2 draft steps
+  const bool traced = c->trace != nullptr && ((c->p.trace == 1 && key.kind == 1) ||
+                                              (c->p.trace == 2 && key.kind == 0));
   OpTable t;
   if (pass) {
-    s = place_table(c, ops, &t);
+    s = place_table(c, ops, &t, traced ? c->trace : nullptr);
+    if (s != MEMSPEC_OK) return s;
+  } else if (traced) {
+    s = attach_trace(c, ops);
     if (s != MEMSPEC_OK) return s;
   }
   if (!c->p.use_graphs) return pass ? launch_table(c, t) : run_ops_separately(c, ops);

@@ -31,10 +31,16 @@ template <int HD>
 __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant__ AttnArgs a) {
   extern __shared__ __align__(128) uint8_t smem_raw[];
   pdl_launch_dependents();
+  const int lin = (blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
+  unsigned long long* trace =
+      (a.trace != nullptr && threadIdx.x == 0 && lin < a.trace_ctas) ? a.trace + lin * 16 : nullptr;
+  trace_at(trace, 0);
   pdl_wait();
+  trace_at(trace, 13);
   const int kvh = blockIdx.y / a.row_blocks, rb = blockIdx.y - kvh * a.row_blocks;
   attention_cta<HD>(a, blockIdx.z, kvh, rb, blockIdx.x, smem_raw, threadIdx.x,
-                    [] { __syncthreads(); });
+                    [] { __syncthreads(); }, trace);
+  trace_at(trace, 1);
 }
 
 }  // namespace

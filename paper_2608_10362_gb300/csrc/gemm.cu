@@ -54,6 +54,7 @@ struct SmemCtl {
   float red[4][16];
 };
 
+template <int EPI>
 __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_constant__ GemmArgs a) {
   __shared__ SmemCtl ctl;
   extern __shared__ uint8_t dsmem_raw[];
@@ -101,6 +102,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
   tc_fence_after();
   pdl_launch_dependents();
   const uint32_t tmem_base = ctl.tmem_base;
+  // optional trace (16 slots per CTA): 0 entry, 13 dependency released,
+  // 2 activation loads issued, 3 first MMA, 4..11 epilogue, 1 exit
+  unsigned long long* trace = a.trace != nullptr ? a.trace + blockIdx.x * 16 : nullptr;
+  if (threadIdx.x == 64) trace_at(trace, 0);
   volatile int* abort_flag = &ctl.abort_flag;
 
   if (warp == 0) {
@@ -135,6 +140,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
         issued_mask |= 1u << p;
       }
       pdl_wait();
+      trace_at(trace, 2);
       for (int p = 0; p < n_pre; ++p) {
         const int t = t_begin + p;
         const int kt = t - (t / KT) * KT;
@@ -199,6 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
             ok = false;
             break;
           }
+          if (it == 0) trace_at(trace, 3);
           tc_fence_after();
           const uint32_t a_addr = smem_addr(smem_a + static_cast<size_t>(s) * kABytes);
           const uint32_t b_addr = smem_addr(smem_b + static_cast<size_t>(s) * b_bytes);
@@ -235,6 +242,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
     const int ew = warp & 3;
     const int et = ew * 32 + lane;  // tile feature == TMEM lane
     pdl_wait();
+    if (threadIdx.x == 64) trace_at(trace, 13);
     if (a.rms) rms_prologue(a, rms, et);
     int seg = 0;
     for (int t = t_begin; t < t_end; ++seg) {
@@ -254,8 +262,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
       named_bar_sync(1, 128);
       if (!ok) break;
       tc_fence_after();
-      epilogue_segment(a, layout, acols, tmem_base, buf, seg, c, G, rt, k0, k1, stage, rms,
-                       ctl.red, &ctl.reduce_flag, ctl.acc_empty, et, ew, lane);
+      epilogue_segment<EPI>(a, layout, acols, tmem_base, buf, seg, c, G, rt, k0, k1, stage, rms,
+                       ctl.red, &ctl.reduce_flag, ctl.acc_empty, et, ew, lane,
+                       threadIdx.x == 64 ? trace : nullptr);
       t = seg_end;
     }
   }
@@ -267,6 +276,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
     tc_fence_after();
     tmem_dealloc(tmem_base, tmem_cols);
   }
+  if (threadIdx.x == 64) trace_at(trace, 1);
 }
 
 }  // namespace
@@ -302,8 +312,15 @@ size_t gemm_smem_bytes(int n_pad, int stages, int planes) {
 
 cudaError_t gemm_set_max_smem() {
   // 227 KB per block minus the kernel's static shared memory
-  return cudaFuncSetAttribute(gemm_stream_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              220 * 1024);
+  const void* fns[4] = {reinterpret_cast<const void*>(gemm_stream_kernel<EPI_F32>),
+                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_RESIDUAL>),
+                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_SWIGLU>),
+                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_QKV>)};
+  for (const void* f : fns) {
+    cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, 220 * 1024);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s, bool pdl) {
@@ -317,7 +334,13 @@ cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, gemm_stream_kernel, a);
+  switch (a.epi) {
+    case EPI_F32: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_F32>, a);
+    case EPI_RESIDUAL: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_RESIDUAL>, a);
+    case EPI_SWIGLU: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_SWIGLU>, a);
+    case EPI_QKV: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_QKV>, a);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace memspec

@@ -92,12 +92,16 @@ __device__ __forceinline__ void row_meta(const GemmArgs& a, int r0, RowMeta& m) 
 
 // Epilogue for one 16-row chunk of a finished 128-feature row tile.  Called by
 // the 128 epilogue threads together; et = feature within the tile (= TMEM lane).
+// EPI (a GemmEpi) is a template argument so that a kernel carries the code of
+// one epilogue only: the tail of a launch runs this code once, cold, and every
+// instruction-cache miss there sits on the critical path.
+template <int EPI>
 static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*red)[16], float* stage,
                                                    const float* rms, int rt, int chunk, int et,
                                                    const float* vin,
                                                    unsigned long long* ts = nullptr) {
   const int ew = et >> 5, lane = et & 31;
-  const int epi = a.epi;
+  constexpr int epi = EPI;
   const int rows_total = a.rows_total;
   const int r0 = chunk * 16;
   float v[16];
@@ -108,7 +112,7 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*re
 #pragma unroll
     for (int j = 0; j < 16; ++j) v[j] = vin[j];
   }
-  if (epi == EPI_F32) {
+  if constexpr (epi == EPI_F32) {
     const int f = rt * kTileM + et;
     const int n_out = a.n_out, out_ld = a.out_ld, last_only = a.last_only;
     const long long gstride = a.out_group_stride;
@@ -131,7 +135,7 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*re
     }
     return;
   }
-  if (epi == EPI_RESIDUAL) {
+  if constexpr (epi == EPI_RESIDUAL) {
     const int f = rt * kTileM + et;  // n_out is a multiple of 128 (d_model)
     float* h = a.h;
     const int h_ld = a.h_ld;
@@ -190,11 +194,12 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*re
     trace_at(ts, 11);
     return;
   }
+  if constexpr (epi == EPI_SWIGLU || epi == EPI_QKV) {
   // staged epilogues: make the whole 128 x 16 chunk visible to all 128 threads
 #pragma unroll
   for (int j = 0; j < 16; ++j) stage[et * kStagePitch + j] = v[j];
   named_bar_sync(1, 128);
-  if (epi == EPI_SWIGLU) {
+  if constexpr (epi == EPI_SWIGLU) {
     if (et < 64) {
       const int f = rt * 64 + et;
       if (f < a.n_out) {
@@ -278,6 +283,7 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*re
     }
   }
   named_bar_sync(1, 128);  // staging buffer is reused by the next chunk
+  }
 }
 
 // Per-row RMSNorm scale from the partial sums of squares (128 epilogue threads).
@@ -307,6 +313,7 @@ __device__ __forceinline__ void rms_prologue(const GemmArgs& a, float* rms, int 
 // G the op's grid; T = row_tiles * k_tiles.  The caller has waited for the
 // accumulator; this routine reads it (wide layout: adds the hi and lo halves),
 // releases it via acc_empty, and writes the epilogue or a partial.
+template <int EPI>
 __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, int layout, int acols,
                                                  uint32_t tmem_base, int buf, int seg, int c,
                                                  int G, int rt, int k0, int k1, float* stage,
@@ -332,7 +339,7 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, int layout, 
   if (full) {
     for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
       load_chunk(chunk);
-      apply_epilogue(a, red, stage, rms, rt, chunk, et, v);
+      apply_epilogue<EPI>(a, red, stage, rms, rt, chunk, et, v);
     }
   } else {
     // partial sums, feature-major: thread et owns n_pad consecutive floats
@@ -396,7 +403,7 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, int layout, 
       }
     }
     if (chunk == 0) trace_after(ts, 6, v[15]);
-    apply_epilogue(a, red, stage, rms, rt, chunk, et, v, ts);
+    apply_epilogue<EPI>(a, red, stage, rms, rt, chunk, et, v, ts);
   }
   trace_at(ts, 7);
   if (et == 0) a.counters[rt] = 0;

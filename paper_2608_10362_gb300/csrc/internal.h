@@ -113,6 +113,7 @@ struct GemmArgs {
   const float* rope_sin;
   const RowPlan* plan;      // nullptr: rows < rows_total are valid, no positions
   uint32_t* status;
+  unsigned long long* trace;  // nullptr, or this op's trace row (16 slots per CTA)
 };
 
 struct AttnArgs {
@@ -133,6 +134,8 @@ struct AttnArgs {
   bf16* out_lo;             // low-order plane of out
   const RowPlan* plan;
   uint32_t* status;
+  unsigned long long* trace;  // nullptr, or this op's trace row (16 slots per CTA)
+  int trace_ctas;             // CTAs (linear index) that record
 };
 
 struct SampleArgs {         // draft sampling of pass j

@@ -86,10 +86,11 @@ class Engine:
     def __init__(self, target_shape, target_weights, *, max_batch: int = 1, max_seq: int = 1024,
                  max_k: int = 8, max_drafts: int = 4, draft_shape_max=None,
                  draft_budget_bytes: int = 0, use_graphs: bool = True,
-                 launch_mode: str = "per_op", trace: bool = False, device: int = 0):
+                 launch_mode: str = "per_op", trace=None, device: int = 0):
         """launch_mode "per_op": one kernel launch per op of a pass; "pass": each
-        draft step and verify pass as one persistent launch (``trace`` then
-        records per-op timestamps, see ``pass_trace``)."""
+        draft step and verify pass as one persistent launch.  ``trace``
+        ("verify" or "draft") records per-op timestamps of that pass, see
+        ``pass_trace``."""
         if launch_mode not in ("per_op", "pass"):
             raise ValueError(f"launch_mode must be 'per_op' or 'pass', not {launch_mode!r}")
         self.lib = _lib.load()
@@ -119,7 +120,9 @@ class Engine:
         p.stream_side = self.side.cuda_stream
         p.use_graphs = int(use_graphs)
         p.launch_mode = _lib.LAUNCH_PASS if launch_mode == "pass" else _lib.LAUNCH_PER_OP
-        p.trace = int(trace)
+        if trace not in (None, "verify", "draft"):
+            raise ValueError(f"trace must be None, 'verify' or 'draft', not {trace!r}")
+        p.trace = {None: 0, "verify": 1, "draft": 2}[trace]
         self.params = p
         n = C.c_size_t()
         _check(self.lib, self.lib.memspec_workspace_bytes(C.byref(p), C.byref(n)))
@@ -229,7 +232,7 @@ class Engine:
         return toks.reshape(self.max_batch, self.max_seq)[req, :L]
 
     def pass_trace(self) -> np.ndarray:
-        """Timestamps (ns) of the last persistent launch, [n_ops][grid][16] =
+        """Timestamps (ns) of the last traced pass, [n_ops][SMs][16] =
         worker start, worker end, activation loads issued, first MMA issued,
         partials stored, arrival counted, reduction inputs loaded, reduction
         done, then epilogue-internal points (entries an op did not reach keep
