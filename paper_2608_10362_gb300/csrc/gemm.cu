@@ -68,6 +68,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
   uint8_t* smem_b = dsmem + static_cast<size_t>(S) * kABytes;
   float* stage = reinterpret_cast<float*>(smem_b + static_cast<size_t>(S) * b_bytes);
   float* rms = stage + kStageFloats;
+  EpiCtx* ectx = reinterpret_cast<EpiCtx*>(rms + kMaxRows);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int T = a.row_tiles * a.k_tiles;
@@ -244,6 +245,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
     pdl_wait();
     if (threadIdx.x == 64) trace_at(trace, 13);
     if (a.rms) rms_prologue(a, rms, et);
+    epi_prologue<EPI>(a, ectx, et);
+    epilogue_warmup<EPI>(a, ectx, ctl.red, stage, rms, c, G, et);
     int seg = 0;
     for (int t = t_begin; t < t_end; ++seg) {
       const int rt = t / KT;
@@ -262,7 +265,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
       named_bar_sync(1, 128);
       if (!ok) break;
       tc_fence_after();
-      epilogue_segment<EPI>(a, layout, acols, tmem_base, buf, seg, c, G, rt, k0, k1, stage, rms,
+      epilogue_segment<EPI>(a, ectx, layout, acols, tmem_base, buf, seg, c, G, rt, k0, k1, stage, rms,
                        ctl.red, &ctl.reduce_flag, ctl.acc_empty, et, ew, lane,
                        threadIdx.x == 64 ? trace : nullptr);
       t = seg_end;
@@ -298,7 +301,7 @@ static int gemm_budget_bytes(int n_pad) {
 int gemm_pick_stages(int n_pad, int planes) {
   const int stage = kABytes + n_pad * 128 * planes;
   const int budget = gemm_budget_bytes(n_pad);
-  const int fixed = kTileM * kStagePitch * 4 + kMaxRows * 4 + 1024;
+  const int fixed = kTileM * kStagePitch * 4 + kMaxRows * 4 + static_cast<int>(sizeof(EpiCtx)) + 1024;
   int s = (budget - fixed) / stage;
   if (s > kMaxStages) s = kMaxStages;
   if (s < 2) s = 2;
@@ -307,7 +310,7 @@ int gemm_pick_stages(int n_pad, int planes) {
 
 size_t gemm_smem_bytes(int n_pad, int stages, int planes) {
   return static_cast<size_t>(stages) * (kABytes + n_pad * 128 * planes) + kTileM * kStagePitch * 4 +
-         kMaxRows * 4 + 1024;
+         kMaxRows * 4 + sizeof(EpiCtx) + 1024;
 }
 
 cudaError_t gemm_set_max_smem() {

@@ -42,51 +42,71 @@ __device__ __forceinline__ bool row_valid(const GemmArgs& a, int r) {
   return a.plan == nullptr ? true : plan_row_valid(a.plan, r);
 }
 
-// Row metadata of one 8-row group of a chunk, read from the row plan.  Every
-// global value an epilogue reads is loaded before its first global store: the
-// compiler cannot prove that the stores do not alias the loads, so interleaving
-// them would cost one dependent L2 round trip per row.
-struct RowMeta {
-  uint32_t valid;   // bit j: row r0 + j is valid
-  uint32_t last;    // bit j: row r0 + j is the last valid row of its group
-  int grp[8];       // group of the row
-  int pos[8];       // its position (plan rows only)
-  int req[8];       // its request (plan rows only)
+// Per-launch epilogue context in shared memory.  The epilogue warps fill it
+// while the weights stream (epi_prologue), so that the tail of the launch - the
+// split-K reduction and the epilogue - reads no row plan or RoPE table from
+// global memory: each such read would be a dependent L2 round trip there.
+constexpr int kCtxRopeRows = 16;   // rows whose RoPE cos/sin are staged (the first chunk)
+struct EpiCtx {
+  int pos[kMaxRows];               // position of each row (plan rows)
+  int req[kMaxRows];               // its request
+  int grp[kMaxRows];               // its group
+  uint32_t valid[kMaxRows / 32];   // bit r: row r is valid
+  uint32_t last[kMaxRows / 32];    // bit r: row r is the last valid row of its group
+  float rc[kCtxRopeRows][64];      // EPI_QKV: cos / sin at (row, rotation pair)
+  float rs[kCtxRopeRows][64];
 };
 
-__device__ __forceinline__ void row_meta(const GemmArgs& a, int r0, RowMeta& m) {
+__device__ __forceinline__ bool ctx_bit(const uint32_t* w, int r) { return (w[r >> 5] >> (r & 31)) & 1u; }
+
+// Fill the context (the 128 epilogue threads, et = 0..127); ends with a barrier.
+template <int EPI>
+__device__ __forceinline__ void epi_prologue(const GemmArgs& a, EpiCtx* ctx, int et) {
   const RowPlan* plan = a.plan;
-  const int rows_total = a.rows_total;
-  m.valid = 0;
-  m.last = 0;
-  if (plan == nullptr) {
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      m.grp[j] = 0;
-      m.pos[j] = 0;
-      m.req[j] = 0;
-      if (r0 + j < rows_total) m.valid |= 1u << j;
+  const int rows_total = a.rows_total, n_pad = a.n_pad;
+  const int R = plan != nullptr ? plan->rows_per_group : 1;
+  for (int base = 0; base < n_pad; base += 128) {   // uniform trip count: ballots below
+    const int r = base + et;
+    bool valid = false, last = false;
+    int g = 0, pos = 0, req = 0;
+    if (r < rows_total) {
+      if (plan == nullptr) {
+        valid = true;
+      } else {
+        g = r / R;
+        const int i = r - g * R;
+        const int nv = plan->valid[g];
+        valid = i < nv;
+        last = i == nv - 1;
+        pos = plan->pos0[g] + i;
+        req = plan->req[g];
+      }
     }
-    return;
+    if (r < n_pad) {
+      ctx->pos[r] = pos;
+      ctx->req[r] = req;
+      ctx->grp[r] = g;
+    }
+    const uint32_t vb = __ballot_sync(0xffffffffu, valid);
+    const uint32_t lb = __ballot_sync(0xffffffffu, last);
+    if ((et & 31) == 0 && r < kMaxRows) {
+      ctx->valid[r >> 5] = vb;
+      ctx->last[r >> 5] = lb;
+    }
   }
-  const int R = plan->rows_per_group;
-  int nv[8];
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const int r = r0 + j;
-    const int g = r < rows_total ? r / R : 0;
-    m.grp[j] = g;
-    nv[j] = plan->valid[g];
-    m.pos[j] = plan->pos0[g];
-    m.req[j] = plan->req[g];
-  }
-#pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const int r = r0 + j;
-    const int i = r - m.grp[j] * R;
-    m.pos[j] += i;
-    if (r < rows_total && i < nv[j]) m.valid |= 1u << j;
-    if (r < rows_total && i == nv[j] - 1) m.last |= 1u << j;
+  named_bar_sync(1, 128);
+  if constexpr (EPI == EPI_QKV) {
+    const int half = a.head_dim >> 1;
+    const int nr = min(n_pad, kCtxRopeRows);
+    for (int idx = et; idx < nr * half; idx += 128) {
+      const int j = idx / half, ip = idx - j * half;
+      const int pos = ctx->pos[j];
+      const bool ok = ctx_bit(ctx->valid, j) && pos >= 0 && pos < a.max_seq;
+      const size_t ri = ok ? static_cast<size_t>(pos) * half + ip : 0;
+      ctx->rc[j][ip] = a.rope_cos[ri];
+      ctx->rs[j][ip] = a.rope_sin[ri];
+    }
+    named_bar_sync(1, 128);
   }
 }
 
@@ -96,10 +116,11 @@ __device__ __forceinline__ void row_meta(const GemmArgs& a, int r0, RowMeta& m) 
 // one epilogue only: the tail of a launch runs this code once, cold, and every
 // instruction-cache miss there sits on the critical path.
 template <int EPI>
-static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*red)[16], float* stage,
+static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, const EpiCtx* ctx,
+                                                   float (*red)[16], float* stage,
                                                    const float* rms, int rt, int chunk, int et,
-                                                   const float* vin,
-                                                   unsigned long long* ts = nullptr) {
+                                                   const float* vin, unsigned long long* ts,
+                                                   bool dry) {
   const int ew = et >> 5, lane = et & 31;
   constexpr int epi = EPI;
   const int rows_total = a.rows_total;
@@ -117,19 +138,14 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*re
     const int n_out = a.n_out, out_ld = a.out_ld, last_only = a.last_only;
     const long long gstride = a.out_group_stride;
     float* out = a.out;
-#pragma unroll 1
-    for (int half = 0; half < 2; ++half) {
-      RowMeta m;
-      row_meta(a, r0 + half * 8, m);
-      if (f < n_out) {
+    if (f < n_out) {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const int r = r0 + half * 8 + j;
-          if (last_only) {
-            if (m.last & (1u << j)) out[m.grp[j] * gstride + f] = v[half * 8 + j];
-          } else if (m.valid & (1u << j)) {
-            out[static_cast<size_t>(r) * out_ld + f] = v[half * 8 + j];
-          }
+      for (int j = 0; j < 16; ++j) {
+        const int r = r0 + j;
+        if (last_only) {
+          if (ctx_bit(ctx->last, r) && !dry) out[ctx->grp[r] * gstride + f] = v[j];
+        } else if (ctx_bit(ctx->valid, r) && !dry) {
+          out[static_cast<size_t>(r) * out_ld + f] = v[j];
         }
       }
     }
@@ -158,7 +174,7 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*re
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
       const int r = r0 + j;
-      if (r >= rows_total) continue;
+      if (r >= rows_total || dry) continue;
       const size_t o = static_cast<size_t>(r) * h_ld + f;
       h[o] = hn[j];
       if (gain_next != nullptr) {
@@ -185,7 +201,7 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*re
     trace_at(ts, 10);
     if (et < 16) {
       const int r = r0 + et;
-      if (r < rows_total) {
+      if (r < rows_total && !dry) {
         const float s = ((red[0][et] + red[1][et]) + red[2][et]) + red[3][et];
         ss_out[static_cast<size_t>(rt) * ss_stride + r] = s;
       }
@@ -195,94 +211,119 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, float (*re
     return;
   }
   if constexpr (epi == EPI_SWIGLU || epi == EPI_QKV) {
-  // staged epilogues: make the whole 128 x 16 chunk visible to all 128 threads
+    // staged epilogues: make the whole 128 x 16 chunk visible to all 128 threads
 #pragma unroll
-  for (int j = 0; j < 16; ++j) stage[et * kStagePitch + j] = v[j];
-  named_bar_sync(1, 128);
-  if constexpr (epi == EPI_SWIGLU) {
-    if (et < 64) {
-      const int f = rt * 64 + et;
-      if (f < a.n_out) {
-        bf16* act = a.act;
-        bf16* act_lo = a.act_lo;
-        const int act_ld = a.act_ld;
-        float y[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const float g = stage[et * kStagePitch + j];
-          const float u = stage[(et + 64) * kStagePitch + j];
-          y[j] = g / (1.0f + expf(-g)) * u;
+    for (int j = 0; j < 16; ++j) stage[et * kStagePitch + j] = v[j];
+    named_bar_sync(1, 128);
+    if constexpr (epi == EPI_SWIGLU) {
+      if (et < 64) {
+        const int f = rt * 64 + et;
+        if (f < a.n_out) {
+          bf16* act = a.act;
+          bf16* act_lo = a.act_lo;
+          const int act_ld = a.act_ld;
+          // rolled: the inputs are in shared memory, and a launch runs this once,
+          // with a cold instruction cache
+#pragma unroll 1
+          for (int j = 0; j < 16; ++j) {
+            const int r = r0 + j;
+            if (r >= rows_total) break;
+            const float g = stage[et * kStagePitch + j];
+            const float u = stage[(et + 64) * kStagePitch + j];
+            const float y = g / (1.0f + expf(-g)) * u;
+            if (dry) continue;
+            const size_t o = static_cast<size_t>(r) * act_ld + f;
+            if (act_lo != nullptr) {
+              split_bf16(y, act[o], act_lo[o]);
+            } else {
+              act[o] = __float2bfloat16_rn(y);
+            }
+          }
         }
+      }
+    } else {  // EPI_QKV: RoPE on q and k, K/V appended to the cache
+      const int f = rt * kTileM + et;
+      const int q_dim = a.q_dim, kv_dim = a.kv_dim;
+      const int hd = a.head_dim, half_hd = hd >> 1;
+      const int n_kv_heads = a.n_kv_heads, max_seq = a.max_seq;
+      float* q_out = a.q_out;
+      const float* rope_cos = a.rope_cos;
+      const float* rope_sin = a.rope_sin;
+      int seg, fs;
+      if (f < q_dim) {
+        seg = 0;
+        fs = f;
+      } else if (f < q_dim + kv_dim) {
+        seg = 1;
+        fs = f - q_dim;
+      } else {
+        seg = 2;
+        fs = f - q_dim - kv_dim;
+      }
+      const int head = fs / hd, d = fs - head * hd;
+      const int ip = d < half_hd ? d : d - half_hd;   // rotation pair index
+      const int e1 = et - d + ip;                     // staging index of element ip of this head
+      bf16* cache = seg == 1 ? a.kcache : a.vcache;
+      if (chunk == 0) {
+        // rolled (see SwiGLU): every input of the first chunk is in shared memory
+#pragma unroll 1
+        for (int j = 0; j < 16; ++j) {
+          const int r = j;
+          const int pos = ctx->pos[r];
+          // invalid positions were flagged by the embedding kernel: skip the row
+          if (!(ctx_bit(ctx->valid, r) && pos >= 0 && pos < max_seq)) continue;
+          float y = stage[et * kStagePitch + j];
+          if (seg < 2) {
+            const float c = ctx->rc[j][ip], sn = ctx->rs[j][ip];
+            const float x1 = stage[e1 * kStagePitch + j];
+            const float x2 = stage[(e1 + half_hd) * kStagePitch + j];
+            y = d < half_hd ? (x1 * c - x2 * sn) : (x1 * sn + x2 * c);
+          }
+          if (dry) continue;
+          if (seg == 0) {
+            q_out[static_cast<size_t>(r) * q_dim + f] = y;
+          } else {
+            const size_t off =
+                ((static_cast<size_t>(ctx->req[r]) * n_kv_heads + head) * max_seq + pos) * hd + d;
+            cache[off] = __float2bfloat16_rn(y);
+          }
+        }
+      } else {
+        // later chunks (batched and prefill passes): the sixteen rows' cos / sin
+        // are loaded together, before any store
+        float y[16];
+        uint32_t ok_mask = 0;
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
           const int r = r0 + j;
-          if (r >= rows_total) continue;
-          const size_t o = static_cast<size_t>(r) * act_ld + f;
-          if (act_lo != nullptr) {
-            split_bf16(y[j], act[o], act_lo[o]);
+          const int pos = ctx->pos[r];
+          const bool ok = ctx_bit(ctx->valid, r) && pos >= 0 && pos < max_seq;
+          if (ok) ok_mask |= 1u << j;
+          y[j] = stage[et * kStagePitch + j];
+          if (seg < 2) {
+            const size_t ri = ok ? static_cast<size_t>(pos) * half_hd + ip : 0;
+            const float c = rope_cos[ri], sn = rope_sin[ri];
+            const float x1 = stage[e1 * kStagePitch + j];
+            const float x2 = stage[(e1 + half_hd) * kStagePitch + j];
+            y[j] = d < half_hd ? (x1 * c - x2 * sn) : (x1 * sn + x2 * c);
+          }
+        }
+        if (dry) ok_mask = 0;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          if (!(ok_mask & (1u << j))) continue;
+          const int r = r0 + j;
+          if (seg == 0) {
+            q_out[static_cast<size_t>(r) * q_dim + f] = y[j];
           } else {
-            act[o] = __float2bfloat16_rn(y[j]);
+            const size_t off =
+                ((static_cast<size_t>(ctx->req[r]) * n_kv_heads + head) * max_seq + ctx->pos[r]) * hd + d;
+            cache[off] = __float2bfloat16_rn(y[j]);
           }
         }
       }
     }
-  } else {  // EPI_QKV: RoPE on q and k, K/V appended to the cache
-    const int f = rt * kTileM + et;
-    const int q_dim = a.q_dim, kv_dim = a.kv_dim;
-    const int hd = a.head_dim, half_hd = hd >> 1;
-    const int n_kv_heads = a.n_kv_heads, max_seq = a.max_seq;
-    float* q_out = a.q_out;
-    const float* rope_cos = a.rope_cos;
-    const float* rope_sin = a.rope_sin;
-    int seg, fs;
-    if (f < q_dim) {
-      seg = 0;
-      fs = f;
-    } else if (f < q_dim + kv_dim) {
-      seg = 1;
-      fs = f - q_dim;
-    } else {
-      seg = 2;
-      fs = f - q_dim - kv_dim;
-    }
-    const int head = fs / hd, d = fs - head * hd;
-    const int ip = d < half_hd ? d : d - half_hd;   // rotation pair index
-    const int e1 = et - d + ip;                     // staging index of element ip of this head
-    bf16* cache = seg == 1 ? a.kcache : a.vcache;
-#pragma unroll 1
-    for (int half = 0; half < 2; ++half) {
-      RowMeta m;
-      row_meta(a, r0 + half * 8, m);
-      float y[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int jj = half * 8 + j;
-        // invalid positions were flagged by the embedding kernel: skip the row
-        if (m.pos[j] < 0 || m.pos[j] >= max_seq) m.valid &= ~(1u << j);
-        y[j] = stage[et * kStagePitch + jj];
-        if (seg < 2) {
-          const size_t ri = (m.valid & (1u << j)) ? static_cast<size_t>(m.pos[j]) * half_hd + ip : 0;
-          const float c = rope_cos[ri], sn = rope_sin[ri];
-          const float x1 = stage[e1 * kStagePitch + jj];
-          const float x2 = stage[(e1 + half_hd) * kStagePitch + jj];
-          y[j] = d < half_hd ? (x1 * c - x2 * sn) : (x1 * sn + x2 * c);
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        if (!(m.valid & (1u << j))) continue;
-        const int r = r0 + half * 8 + j;
-        if (seg == 0) {
-          q_out[static_cast<size_t>(r) * q_dim + f] = y[j];
-        } else {
-          const size_t off =
-              ((static_cast<size_t>(m.req[j]) * n_kv_heads + head) * max_seq + m.pos[j]) * hd + d;
-          cache[off] = __float2bfloat16_rn(y[j]);
-        }
-      }
-    }
-  }
-  named_bar_sync(1, 128);  // staging buffer is reused by the next chunk
+    named_bar_sync(1, 128);  // staging buffer is reused by the next chunk
   }
 }
 
@@ -308,13 +349,66 @@ __device__ __forceinline__ void rms_prologue(const GemmArgs& a, float* rms, int 
   named_bar_sync(1, 128);
 }
 
+// Sum of the split-K partials of row tile rt, chunk `chunk`, for feature et:
+// contributors in ascending CTA order, four fetched at once.
+__device__ __forceinline__ void reduce_partials(const GemmArgs& a, int rt, int c_first, int c_last,
+                                                int chunk, int et, int T, int G, float* v) {
+  const int KT = a.k_tiles;
+#pragma unroll
+  for (int j = 0; j < 16; ++j) v[j] = 0.f;
+  for (int cc0 = c_first; cc0 <= c_last; cc0 += 4) {
+    float4 tmp[4][4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int cc = cc0 + q;
+      if (cc <= c_last) {
+        const int sl = (sk_begin(cc, T, G) >= rt * KT) ? 0 : 1;
+        const float* pp = a.partials + static_cast<size_t>(2 * cc + sl) * a.n_pad * kTileM +
+                          static_cast<size_t>(et) * a.n_pad + chunk * 16;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) tmp[q][e] = ld_cg_f4(pp + 4 * e);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (cc0 + q <= c_last) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          v[4 * e] += tmp[q][e].x;
+          v[4 * e + 1] += tmp[q][e].y;
+          v[4 * e + 2] += tmp[q][e].z;
+          v[4 * e + 3] += tmp[q][e].w;
+        }
+      }
+    }
+  }
+}
+
+// Dry run of the tail - the partial reduction and the epilogue of this CTA's
+// first row tile, with every global store off - by the 128 epilogue threads
+// while the weights stream.  The tail runs once per launch; without this its
+// instructions are fetched cold, one miss after another, on the critical path.
+template <int EPI>
+__device__ __forceinline__ void epilogue_warmup(const GemmArgs& a, const EpiCtx* ctx,
+                                                float (*red)[16], float* stage, const float* rms,
+                                                int c, int G, int et) {
+  const int KT = a.k_tiles, T = a.row_tiles * KT;
+  const int rt = sk_begin(c, T, G) / KT;
+  const int c_first = sk_cta_of(rt * KT, T, G);
+  const int c_last = sk_cta_of((rt + 1) * KT - 1, T, G);
+  float v[16];
+  reduce_partials(a, rt, c_first, c_last, 0, et, T, G, v);
+  apply_epilogue<EPI>(a, ctx, red, stage, rms, rt, 0, et, v, nullptr, true);
+}
+
 // Epilogue of one accumulated segment [k0, k1) of row tile rt, run by the 128
 // epilogue threads (et = TMEM lane = tile feature).  `c` is this CTA's index and
 // G the op's grid; T = row_tiles * k_tiles.  The caller has waited for the
 // accumulator; this routine reads it (wide layout: adds the hi and lo halves),
 // releases it via acc_empty, and writes the epilogue or a partial.
 template <int EPI>
-__device__ __forceinline__ void epilogue_segment(const GemmArgs& a, int layout, int acols,
+__device__ __forceinline__ void epilogue_segment(const GemmArgs& a, const EpiCtx* ctx, int layout,
+                                                 int acols,
                                                  uint32_t tmem_base, int buf, int seg, int c,
                                                  int G, int rt, int k0, int k1, float* stage,
                                                  const float* rms, float (*red)[16],
@@ -339,7 +433,7 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, int layout, 
   if (full) {
     for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
       load_chunk(chunk);
-      apply_epilogue<EPI>(a, red, stage, rms, rt, chunk, et, v);
+      apply_epilogue<EPI>(a, ctx, red, stage, rms, rt, chunk, et, v, nullptr, false);
     }
   } else {
     // partial sums, feature-major: thread et owns n_pad consecutive floats
@@ -373,37 +467,9 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, int layout, 
   trace_at(ts, 5);
   if (!*reduce_flag) return;
   for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
-#pragma unroll
-    for (int j = 0; j < 16; ++j) v[j] = 0.f;
-    // contributors are summed in ascending CTA order; four are fetched at once
-    for (int cc0 = c_first; cc0 <= c_last; cc0 += 4) {
-      float4 tmp[4][4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int cc = cc0 + q;
-        if (cc <= c_last) {
-          const int sl = (sk_begin(cc, T, G) >= rt * KT) ? 0 : 1;
-          const float* pp = a.partials + static_cast<size_t>(2 * cc + sl) * a.n_pad * kTileM +
-                            static_cast<size_t>(et) * a.n_pad + chunk * 16;
-#pragma unroll
-          for (int e = 0; e < 4; ++e) tmp[q][e] = ld_cg_f4(pp + 4 * e);
-        }
-      }
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        if (cc0 + q <= c_last) {
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            v[4 * e] += tmp[q][e].x;
-            v[4 * e + 1] += tmp[q][e].y;
-            v[4 * e + 2] += tmp[q][e].z;
-            v[4 * e + 3] += tmp[q][e].w;
-          }
-        }
-      }
-    }
+    reduce_partials(a, rt, c_first, c_last, chunk, et, T, G, v);
     if (chunk == 0) trace_after(ts, 6, v[15]);
-    apply_epilogue<EPI>(a, red, stage, rms, rt, chunk, et, v, ts);
+    apply_epilogue<EPI>(a, ctx, red, stage, rms, rt, chunk, et, v, ts, false);
   }
   trace_at(ts, 7);
   if (et == 0) a.counters[rt] = 0;

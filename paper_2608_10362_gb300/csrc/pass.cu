@@ -130,7 +130,8 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
   uint8_t* attn_smem = ring_b + static_cast<size_t>(S) * p.b_stage_bytes;
   float* stage = reinterpret_cast<float*>(attn_smem + p.attn_bytes);
   float* rms = stage + kStageFloats;
-  smp::SampleSmem* ssm = reinterpret_cast<smp::SampleSmem*>(rms + kMaxRows);
+  EpiCtx* ectx = reinterpret_cast<EpiCtx*>(rms + kMaxRows);
+  smp::SampleSmem* ssm = reinterpret_cast<smp::SampleSmem*>(ectx + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = gridDim.x, c = blockIdx.x;
@@ -332,6 +333,12 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
           const int layout = op_layout(a);
           const int acols = acc_cols(a, layout);
           if (a.rms) rms_prologue(a, rms, et);
+          switch (a.epi) {
+            case EPI_F32: epi_prologue<EPI_F32>(a, ectx, et); break;
+            case EPI_RESIDUAL: epi_prologue<EPI_RESIDUAL>(a, ectx, et); break;
+            case EPI_SWIGLU: epi_prologue<EPI_SWIGLU>(a, ectx, et); break;
+            default: epi_prologue<EPI_QKV>(a, ectx, et); break;
+          }
           int lseg = 0;   // segment index within this op (partial slot choice)
           for (int t = t_begin; t < t_end; ++seg, ++lseg) {
             const int rt = t / KT;
@@ -355,7 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
             tc_fence_after();
             unsigned long long* ts = tid == 0 ? trace_slot(p, n, 0) : nullptr;
 #define MEMSPEC_PASS_EPI(E)                                                                  \
-  epilogue_segment<E>(a, layout, acols, tmem_base, buf, lseg, c, Gn, rt, k0, k1, stage, rms, \
+  epilogue_segment<E>(a, ectx, layout, acols, tmem_base, buf, lseg, c, Gn, rt, k0, k1, stage, rms, \
                       ctl.red, &ctl.reduce_flag, ctl.acc_empty, et, ew, lane, ts)
             switch (a.epi) {
               case EPI_F32: MEMSPEC_PASS_EPI(EPI_F32); break;
@@ -428,11 +435,12 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
 
 size_t pass_smem_bytes(const PassArgs& p) {
   return static_cast<size_t>(p.stages) * (kABytes + p.b_stage_bytes) + p.attn_bytes +
-         kStageFloats * 4 + kMaxRows * 4 + sizeof(smp::SampleSmem) + 1024;
+         kStageFloats * 4 + kMaxRows * 4 + sizeof(EpiCtx) + sizeof(smp::SampleSmem) + 1024;
 }
 
 int pass_pick_stages(int b_stage_bytes, int attn_bytes) {
   const int budget = 226 * 1024 - attn_bytes - kStageFloats * 4 - kMaxRows * 4 -
+                     static_cast<int>(sizeof(EpiCtx)) -
                      static_cast<int>(sizeof(smp::SampleSmem)) - 1024 - 1024;
   int s = budget / (kABytes + b_stage_bytes);
   if (s > kMaxStages) s = kMaxStages;
