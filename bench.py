@@ -157,6 +157,7 @@ def run_gpu(args, rank: int, world: int):
         dist.barrier()
     torch.cuda.synchronize()
     with ClockSampler(dev) as clk:
+        torch.cuda.nvtx.range_push("timed")   # for profilers: --nvtx --nvtx-include "timed/"
         start.record(s)
         for i in range(steps):
             eng.draft_step(K, TEMP)
@@ -165,6 +166,7 @@ def run_gpu(args, rank: int, world: int):
             ev[i][1].record(s)
             eng.accept_commit(K, TEMP)
         stop.record(s)
+        torch.cuda.nvtx.range_pop()
         torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
@@ -302,6 +304,36 @@ def run_case(args):
         return {"case": "gemm", "n_out": args.n, "k": args.kdim, "rows": args.rows,
                 "us_per_launch": ms * 1e3, "GB/s": nbytes / ms / 1e6}
     from paper_2608_10362_gb300 import Engine
+    if args.case == "verify":
+        # the 7B verify pass alone, one launch per op and no graph, inside an NVTX
+        # range "verify" (for profilers: ncu --nvtx --nvtx-include "verify/")
+        t = SHAPES[TARGET]
+        K = args.k
+        max_seq = PREFIX + (args.steps + args.warmup + 2) * (K + 1) + 16
+        eng = Engine(t, iter_weights(t, 0), max_batch=1, max_seq=max_seq, max_k=K, max_drafts=0,
+                     use_graphs=False, launch_mode=args.launch_mode)
+        from paper_2608_10362_gb300 import _lib
+        eng.prefill(0, gen_prompt(3, PREFIX, t.vocab), seed=1)
+        dt = np.zeros((1, eng.max_k), dtype=np.int32)
+        dt[0, :K] = gen_prompt(4, K, t.vocab)
+        eng.write_buffer(_lib.BUF_DRAFT_TOKENS, dt)
+        for _ in range(args.warmup):
+            eng.verify_step(K)
+        eng.sync()
+        s = eng.stream
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.nvtx.range_push("verify")
+        a.record(s)
+        for _ in range(args.steps):
+            eng.verify_step(K)
+        b.record(s)
+        torch.cuda.nvtx.range_pop()
+        torch.cuda.synchronize()
+        bits = eng.sync()
+        ms = a.elapsed_time(b) / args.steps
+        eng.close()
+        return {"case": "verify", "target": TARGET, "K": K, "prefix": PREFIX, "graphs": False,
+                "ms_per_verify": ms, "device_status": bits}
     t, d = SHAPES["draft_160m"], SHAPES["draft_68m"]
     K = args.k
     max_seq = 512 + (args.steps + args.warmup + 4) * (K + 1) + 16
@@ -335,6 +367,42 @@ def run_case(args):
             "device_status": bits}
 
 
+TRAFFIC_PROFILE = os.path.join(ROOT, "profiles", "verify_7b_k4_ctx2048_dram.md")
+
+
+def kernel_sources_hash() -> str:
+    """sha256 over the CUDA sources (name + content, sorted by name)."""
+    import glob
+    import hashlib
+    csrc = os.path.join(ROOT, "paper_2608_10362_gb300", "csrc")
+    files = sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh")) +
+                   glob.glob(os.path.join(csrc, "*.h")))
+    h = hashlib.sha256()
+    for f in files:
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def recorded_traffic():
+    """DRAM bytes of one verify pass from the committed ncu summary, if it was
+    taken on the kernel sources as they are now (else None)."""
+    try:
+        with open(TRAFFIC_PROFILE) as fh:
+            text = fh.read()
+    except OSError:
+        return None
+    vals = {}
+    for ln in text.splitlines():
+        if ":" in ln and ln.split(":")[0] in ("traffic_bytes_per_verify", "kernel_sources_sha256"):
+            k, v = ln.split(":", 1)
+            vals[k.strip()] = v.strip()
+    if vals.get("kernel_sources_sha256") != kernel_sources_hash():
+        return None
+    return int(vals["traffic_bytes_per_verify"]) if "traffic_bytes_per_verify" in vals else None
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -343,7 +411,7 @@ def main():
     ap.add_argument("--k", type=int, default=K_DRAFT)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", default="step", choices=["step", "gemm", "small"],
+    ap.add_argument("--case", default="step", choices=["step", "gemm", "small", "verify"],
                     help="step: the workload above; gemm / small: diagnostic cases sized for "
                          "profiler captures (one projection GEMM; a 160M target with a 68M draft)")
     ap.add_argument("--launch-mode", default="per_op", choices=["per_op", "pass"],
@@ -414,7 +482,11 @@ def main():
         "roofline": {"kernel": "verify pass (one CUDA graph of the target forward)",
                      "bound": "hbm", "achieved": achieved, "peak": peak,
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
-                     "traffic": None, "verify_ms": r["verify_ms"],
+                     "traffic": recorded_traffic(),
+                     "traffic_source": "ncu dram__bytes_read+write of one verify pass "
+                                       "(profiles/verify_7b_k4_ctx2048_dram.md); null when the "
+                                       "kernels changed since",
+                     "verify_ms": r["verify_ms"],
                      "algorithmic_bytes": r["verify_bytes"],
                      "frac_of_8000": achieved / 8000.0},
         "e2e": {"value": r["generated"] / r["e2e_s"], "unit": "tokens/s",

@@ -151,6 +151,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     *reinterpret_cast<uint4*>(qs + kTileBytes + swz<HD>(v, ch)) = *reinterpret_cast<const uint4*>(el);
   }
   sync();
+  trace_at(ts, 8);
 
   // Q fragments (hi and lo) of this warp's m-tile stay in registers
   uint32_t qa[HD / 16][4], ql[HD / 16][4];
@@ -180,6 +181,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   for (int t = 0; t < n_tiles; ++t) {
     cp_async_wait<kStages - 2>();
     sync();
+    if (t == 0) trace_at(ts, 10);
     if (t + kStages - 1 < n_tiles) load_tile(t + kStages - 1);
     cp_async_commit();
     if (!active) continue;
@@ -274,6 +276,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   }
   cp_async_wait<0>();
   sync();
+  trace_at(ts, 9);
 
   // merge the key groups of each m-tile (shared memory reuses the K/V stages)
   float* mo = reinterpret_cast<float*>(kv);                 // [4 warps][16][HD]
