@@ -85,13 +85,23 @@ typedef struct memspec_model_cfg {
 
 /* ---- weight blob layout ------------------------------------------------
  * A model's weights live in ONE contiguous blob (device memory for the
- * target, pinned host memory for drafts that get loaded into the arena).
- * Every tensor is bf16, row-major, 256-byte aligned inside the blob:
- *   TOK_EMB [vocab][d]            LM_HEAD [vocab][d] (absent if tied)
- *   per layer: ATTN_NORM [d], WQKV [(H + 2 Hkv) hd][d] (q rows, then k, then v),
- *   WO [d][H hd], FFN_NORM [d], WGATE [F][d], WUP [F][d], WDOWN [d][F]
- *   FINAL_NORM [d]
- * Linear weights are [out][in], i.e. y = x W^T. */
+ * target, pinned host memory for drafts that get loaded into the arena), every
+ * tensor 256-byte aligned inside it:
+ *   TOK_EMB [vocab][d] bf16 row-major; ATTN_NORM, FFN_NORM, FINAL_NORM [d] bf16;
+ *   projection matrices in PACKED TILES (below): per layer WQKV (n = (H + 2 Hkv)
+ *   hd rows: q, then k, then v; k = d), WO (n = d, k = H hd), WGATE (the gate/up
+ *   pair, n = F, k = d; WUP reports 0 bytes at WGATE's offset), WDOWN (n = d,
+ *   k = F); LM_HEAD (n = vocab, k = d; absent if tied: the LM head then reads
+ *   TOK_EMB).  Linear weights are [out][in], i.e. y = x W^T.
+ * Packed tiles: the [n][k] matrix is cut into tiles of 128 rows x 64 columns;
+ * tile (rt, kt) is 16384 contiguous bytes at (rt * ceil(k/64) + kt) * 16384;
+ * row r of a tile starts at byte 128 r and its 16-byte column chunk c (columns
+ * 64 kt + 8c .. + 7) is stored at chunk position c ^ (r % 8); entries beyond n
+ * or k are zero.  For the gate/up pair a tile's rows 0..63 are gate rows
+ * 64 rt .. 64 rt + 63 and rows 64..127 the same rows of up (ceil(F/64) row
+ * tiles).  This is the shared-memory image the tensor cores read, in the order
+ * the GEMM streams it, so weights move by 1-D bulk copies of whole tiles.
+ * memspec_pack_matrix writes a packed tensor from row-major device arrays. */
 typedef enum memspec_tensor {
   MEMSPEC_T_TOK_EMB = 0,
   MEMSPEC_T_ATTN_NORM = 1,
@@ -113,6 +123,15 @@ memspec_status memspec_weights_bytes(const memspec_model_cfg* cfg, size_t* bytes
  * Errors: INVALID_ARG (bad tensor id / layer). */
 memspec_status memspec_weights_offset(const memspec_model_cfg* cfg, int32_t tensor,
                                       int32_t layer, size_t* offset, size_t* bytes);
+
+/* Pack row-major bf16 src [n][k] (device) into packed tiles at dst (device,
+ * dst_bytes >= ceil(n/128) * ceil(k/64) * 16384); with src2 non-NULL, src and
+ * src2 are the gate and up matrices of a pair (dst_bytes >= ceil(n/64) *
+ * ceil(k/64) * 16384).  k a positive multiple of 8; all pointers 16-byte
+ * aligned.  Enqueued on `stream` (cudaStream_t).  Errors (message in
+ * memspec_op_last_error): INVALID_ARG, CUDA. */
+memspec_status memspec_pack_matrix(const void* src_dev, const void* src2_dev, int32_t n,
+                                   int32_t k, void* dst_dev, size_t dst_bytes, void* stream);
 
 /* Bytes of one model's KV cache: n_layers * 2 * max_batch * n_kv_heads *
  * max_seq * head_dim bf16, layout [layer][K|V][request][kv_head][pos][hd]. */

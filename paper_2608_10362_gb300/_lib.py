@@ -82,6 +82,8 @@ EXPORTS = {
     "memspec_op_sample": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_float, C.c_void_p,
                                     C.c_void_p, C.c_void_p]),
     "memspec_op_last_error": (C.c_char_p, []),
+    "memspec_pack_matrix": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p,
+                                      C.c_size_t, C.c_void_p]),
 }
 
 _lib = None

@@ -155,23 +155,28 @@ Layout make_layout(const memspec_model_cfg& c) {
   const size_t d = c.d_model, q = static_cast<size_t>(c.n_heads) * c.head_dim,
                kv = static_cast<size_t>(c.n_kv_heads) * c.head_dim, f = c.d_ffn, v = c.vocab;
   size_t off = 0;
-  auto take = [&](size_t elems) {
+  auto take = [&](size_t elems) {   // row-major bf16
     const size_t o = off;
     off = align256(off + elems * 2);
+    return o;
+  };
+  auto take_packed = [&](size_t n, size_t k, bool pair) {
+    const size_t o = off;
+    off = align256(off + packed_bytes(static_cast<long long>(n), static_cast<long long>(k), pair));
     return o;
   };
   L.emb = take(v * d);
   for (int l = 0; l < c.n_layers; ++l) {
     L.attn_norm.push_back(take(d));
-    L.wqkv.push_back(take((q + 2 * kv) * d));
-    L.wo.push_back(take(d * q));
+    L.wqkv.push_back(take_packed(q + 2 * kv, d, false));
+    L.wo.push_back(take_packed(d, q, false));
     L.ffn_norm.push_back(take(d));
-    L.wgate.push_back(take(f * d));
-    L.wup.push_back(take(f * d));
-    L.wdown.push_back(take(d * f));
+    L.wgate.push_back(take_packed(f, d, true));   // gate/up pair tiles
+    L.wup.push_back(L.wgate.back());
+    L.wdown.push_back(take_packed(d, f, false));
   }
   L.final_norm = take(d);
-  L.lm_head = c.tied_embeddings ? L.emb : take(v * d);
+  L.lm_head = c.tied_embeddings ? L.emb : take_packed(v, d, false);
   L.total = off;
   return L;
 }
@@ -225,8 +230,7 @@ struct ModelRT {
   Layout lay;
   const uint8_t* w = nullptr;  // device blob
   bf16* kv = nullptr;
-  std::vector<CUtensorMap> m_qkv, m_o, m_gate, m_up, m_down;
-  CUtensorMap m_lm{};
+  CUtensorMap m_lm{};   // tied LM head: the row-major embedding
   int l2_hint = L2_EVICT_FIRST;
   bool ready = false;
 };
@@ -235,20 +239,13 @@ bool build_maps(ModelRT& m, std::string* why) {
   const memspec_model_cfg& c = m.cfg;
   const int d = c.d_model, q = c.n_heads * c.head_dim, kv = c.n_kv_heads * c.head_dim,
             f = c.d_ffn;
-  m.m_qkv.resize(c.n_layers);
-  m.m_o.resize(c.n_layers);
-  m.m_gate.resize(c.n_layers);
-  m.m_up.resize(c.n_layers);
-  m.m_down.resize(c.n_layers);
+  (void)q;
+  (void)kv;
+  (void)f;
+  // projection weights are packed tiles (bulk copies, no tensor map); only a
+  // tied LM head reads the row-major embedding through a tensor map
   bool ok = true;
-  for (int l = 0; l < c.n_layers; ++l) {
-    ok &= encode_map(&m.m_qkv[l], m.w + m.lay.wqkv[l], q + 2 * kv, d, 128);
-    ok &= encode_map(&m.m_o[l], m.w + m.lay.wo[l], d, q, 128);
-    ok &= encode_map(&m.m_gate[l], m.w + m.lay.wgate[l], f, d, 64);
-    ok &= encode_map(&m.m_up[l], m.w + m.lay.wup[l], f, d, 64);
-    ok &= encode_map(&m.m_down[l], m.w + m.lay.wdown[l], d, f, 128);
-  }
-  ok &= encode_map(&m.m_lm, m.w + m.lay.lm_head, c.vocab, d, 128);
+  if (c.tied_embeddings) ok = encode_map(&m.m_lm, m.w + m.lay.lm_head, c.vocab, d, 128);
   if (!ok) *why = "cuTensorMapEncodeTiled failed (driver entry point or alignment)";
   m.ready = ok;
   return ok;
@@ -614,7 +611,7 @@ memspec_status emit_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f,
     bf16* vl = kl + layer_kv;
     {  // QKV + RoPE + KV append, RMSNorm fused into the activation producer
       GemmArgs a{};
-      a.map_a = m.m_qkv[l];
+      a.a_packed = m.w + m.lay.wqkv[l];
       a.n_out = qd + 2 * kvd;
       a.k_in = d;
       a.pair = 0;
@@ -677,7 +674,7 @@ memspec_status emit_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f,
     }
     {  // O projection + residual
       GemmArgs a{};
-      a.map_a = m.m_o[l];
+      a.a_packed = m.w + m.lay.wo[l];
       a.n_out = d;
       a.k_in = qd;
       a.rows_total = rows;
@@ -703,8 +700,7 @@ memspec_status emit_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f,
     }
     {  // gate/up + SwiGLU
       GemmArgs a{};
-      a.map_a = m.m_gate[l];
-      a.map_a2 = m.m_up[l];
+      a.a_packed = m.w + m.lay.wgate[l];
       a.pair = 1;
       a.n_out = F;
       a.k_in = d;
@@ -731,7 +727,7 @@ memspec_status emit_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f,
     }
     {  // down projection + residual
       GemmArgs a{};
-      a.map_a = m.m_down[l];
+      a.a_packed = m.w + m.lay.wdown[l];
       a.n_out = d;
       a.k_in = F;
       a.rows_total = rows;
@@ -758,7 +754,10 @@ memspec_status emit_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f,
   }
   if (f.logits != nullptr) {  // final RMSNorm + LM head -> fp32 logits
     GemmArgs a{};
-    a.map_a = m.m_lm;
+    if (cf.tied_embeddings)
+      a.map_a = m.m_lm;
+    else
+      a.a_packed = m.w + m.lay.lm_head;
     a.n_out = cf.vocab;
     a.k_in = d;
     a.rows_total = rows;
@@ -1029,14 +1028,17 @@ memspec_status memspec_weights_offset(const memspec_model_cfg* cfg, int32_t tens
   switch (tensor) {
     case MEMSPEC_T_TOK_EMB: *offset = L.emb; *bytes = v * d * 2; break;
     case MEMSPEC_T_ATTN_NORM: *offset = L.attn_norm[layer]; *bytes = d * 2; break;
-    case MEMSPEC_T_WQKV: *offset = L.wqkv[layer]; *bytes = (q + 2 * kv) * d * 2; break;
-    case MEMSPEC_T_WO: *offset = L.wo[layer]; *bytes = d * q * 2; break;
+    case MEMSPEC_T_WQKV: *offset = L.wqkv[layer]; *bytes = packed_bytes(q + 2 * kv, d, false); break;
+    case MEMSPEC_T_WO: *offset = L.wo[layer]; *bytes = packed_bytes(d, q, false); break;
     case MEMSPEC_T_FFN_NORM: *offset = L.ffn_norm[layer]; *bytes = d * 2; break;
-    case MEMSPEC_T_WGATE: *offset = L.wgate[layer]; *bytes = f * d * 2; break;
-    case MEMSPEC_T_WUP: *offset = L.wup[layer]; *bytes = f * d * 2; break;
-    case MEMSPEC_T_WDOWN: *offset = L.wdown[layer]; *bytes = d * f * 2; break;
+    case MEMSPEC_T_WGATE: *offset = L.wgate[layer]; *bytes = packed_bytes(f, d, true); break;
+    case MEMSPEC_T_WUP: *offset = L.wup[layer]; *bytes = 0; break;   // inside WGATE's pair tiles
+    case MEMSPEC_T_WDOWN: *offset = L.wdown[layer]; *bytes = packed_bytes(d, f, false); break;
     case MEMSPEC_T_FINAL_NORM: *offset = L.final_norm; *bytes = d * 2; break;
-    case MEMSPEC_T_LM_HEAD: *offset = L.lm_head; *bytes = v * d * 2; break;
+    case MEMSPEC_T_LM_HEAD:
+      *offset = L.lm_head;
+      *bytes = cfg->tied_embeddings ? v * d * 2 : packed_bytes(v, d, false);
+      break;
     default: return MEMSPEC_ERR_INVALID_ARG;
   }
   return MEMSPEC_OK;
@@ -1568,6 +1570,34 @@ static size_t op_linear_scratch(int rows, int n_out, int k) {
 memspec_status memspec_op_linear_scratch_bytes(int32_t rows, int32_t n_out, int32_t k, size_t* bytes) {
   if (bytes == nullptr || rows < 1 || rows > kMaxRows || n_out < 1 || k < 8) return MEMSPEC_ERR_INVALID_ARG;
   *bytes = op_linear_scratch(rows, n_out, k);
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_pack_matrix(const void* src, const void* src2, int32_t n, int32_t k,
+                                   void* dst, size_t dst_bytes, void* stream) {
+  if (src == nullptr || dst == nullptr) {
+    g_op_error = "null pointer";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (n < 1 || k < 8 || k % 8 != 0) {
+    g_op_error = "n >= 1 and k a positive multiple of 8";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if ((reinterpret_cast<uintptr_t>(src) & 15) || (reinterpret_cast<uintptr_t>(src2) & 15) ||
+      (reinterpret_cast<uintptr_t>(dst) & 15)) {
+    g_op_error = "src, src2 and dst must be 16-byte aligned";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (dst_bytes < packed_bytes(n, k, src2 != nullptr)) {
+    g_op_error = "dst smaller than the packed size";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  cudaError_t e = launch_pack(static_cast<const bf16*>(src), static_cast<const bf16*>(src2), n, k,
+                              static_cast<uint8_t*>(dst), static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) {
+    g_op_error = std::string("pack launch: ") + cudaGetErrorString(e);
+    return MEMSPEC_ERR_CUDA;
+  }
   return MEMSPEC_OK;
 }
 

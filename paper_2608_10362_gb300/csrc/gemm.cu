@@ -114,8 +114,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
     // Weight tiles do not depend on earlier kernels: the first S of them are
     // requested before griddepcontrol.wait.  Activation tiles are requested after.
     if (lane == 0) {
-      tma_prefetch_desc(&a.map_a);
-      if (a.pair) tma_prefetch_desc(&a.map_a2);
+      if (a.a_packed == nullptr) {
+        tma_prefetch_desc(&a.map_a);
+        if (a.pair) tma_prefetch_desc(&a.map_a2);
+      }
       tma_prefetch_desc(&a.map_b);
       if (a.split) tma_prefetch_desc(&a.map_b2);
       const uint64_t pol = a.l2_hint == L2_EVICT_FIRST  ? l2_policy_evict_first()
@@ -123,58 +125,70 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
                                                         : l2_policy_evict_normal();
       const uint64_t pol_b = l2_policy_evict_last();   // activations are re-read by every CTA
       uint32_t issued_mask = 0, last_par = 0;
-      int it = 0;
       bool ok = true;
       const int n_pre = min(S, t_end - t_begin);
-      // weights of the first n_pre tiles (the ring is empty: no wait needed)
-      for (int p = 0; p < n_pre; ++p) {
-        const int t = t_begin + p;
-        const int rt = t / KT, kt = t - rt * KT;
-        uint8_t* dst = smem_a + static_cast<size_t>(p) * kABytes;
-        mbar_arrive_expect_tx(&ctl.full[p], stage_tx);
-        if (a.pair) {
-          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * 64, &ctl.full[p], pol);
-          tma_load_2d(dst + kABytes / 2, &a.map_a2, kt * kTileK, rt * 64, &ctl.full[p], pol);
+      // One thread issues every copy, so the loop is lean: the ring position and
+      // the tile coordinates advance incrementally (no division per tile).
+      const uint8_t* wsrc = a.a_packed != nullptr
+                                ? a.a_packed + static_cast<size_t>(t_begin) * kABytes : nullptr;
+      int rt = t_begin / KT, kt = t_begin - rt * KT;
+      auto load_a = [&](int slot) {
+        uint8_t* dst = smem_a + static_cast<size_t>(slot) * kABytes;
+        if (wsrc != nullptr) {
+          bulk_load(dst, wsrc, kABytes, &ctl.full[slot], pol);
+          wsrc += kABytes;
+        } else if (a.pair) {
+          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * 64, &ctl.full[slot], pol);
+          tma_load_2d(dst + kABytes / 2, &a.map_a2, kt * kTileK, rt * 64, &ctl.full[slot], pol);
         } else {
-          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * kTileM, &ctl.full[p], pol);
+          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * kTileM, &ctl.full[slot], pol);
         }
+      };
+      auto load_b = [&](int slot, int k_tile) {
+        uint8_t* dst = smem_b + static_cast<size_t>(slot) * b_bytes;
+        tma_load_2d(dst, &a.map_b, k_tile * kTileK, 0, &ctl.full[slot], pol_b);
+        if (a.split) tma_load_2d(dst + plane_bytes, &a.map_b2, k_tile * kTileK, 0, &ctl.full[slot], pol_b);
+      };
+      // weights of the first n_pre tiles (the ring is empty: no wait needed)
+      const int kt_first = kt;
+      for (int p = 0; p < n_pre; ++p) {
+        mbar_arrive_expect_tx(&ctl.full[p], stage_tx);
+        load_a(p);
         issued_mask |= 1u << p;
+        if (++kt == KT) {
+          kt = 0;
+          ++rt;
+        }
       }
       pdl_wait();
       trace_at(trace, 2);
-      for (int p = 0; p < n_pre; ++p) {
-        const int t = t_begin + p;
-        const int kt = t - (t / KT) * KT;
-        tma_load_2d(smem_b + static_cast<size_t>(p) * b_bytes, &a.map_b, kt * kTileK, 0,
-                    &ctl.full[p], pol_b);
-        if (a.split)
-          tma_load_2d(smem_b + static_cast<size_t>(p) * b_bytes + plane_bytes, &a.map_b2,
-                      kt * kTileK, 0, &ctl.full[p], pol_b);
+      {
+        int k2 = kt_first;
+        for (int p = 0; p < n_pre; ++p) {
+          load_b(p, k2);
+          if (++k2 == KT) k2 = 0;
+        }
       }
-      it = n_pre;
-      for (int t = t_begin + n_pre; t < t_end; ++t, ++it) {
-        const int rt = t / KT, kt = t - rt * KT;
-        const int s = it % S;
-        const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
+      int s = n_pre == S ? 0 : n_pre;
+      uint32_t ph = n_pre == S ? 1u : 0u;   // phase of the fill the next wait is for
+      for (int t = t_begin + n_pre; t < t_end; ++t) {
         if (!mbar_wait_bounded(&ctl.empty[s], ph ^ 1u, abort_flag, a.status)) {
           ok = false;
           break;
         }
-        uint8_t* dst = smem_a + static_cast<size_t>(s) * kABytes;
         mbar_arrive_expect_tx(&ctl.full[s], stage_tx);
-        if (a.pair) {
-          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * 64, &ctl.full[s], pol);
-          tma_load_2d(dst + kABytes / 2, &a.map_a2, kt * kTileK, rt * 64, &ctl.full[s], pol);
-        } else {
-          tma_load_2d(dst, &a.map_a, kt * kTileK, rt * kTileM, &ctl.full[s], pol);
-        }
-        tma_load_2d(smem_b + static_cast<size_t>(s) * b_bytes, &a.map_b, kt * kTileK, 0,
-                    &ctl.full[s], pol_b);
-        if (a.split)
-          tma_load_2d(smem_b + static_cast<size_t>(s) * b_bytes + plane_bytes, &a.map_b2,
-                      kt * kTileK, 0, &ctl.full[s], pol_b);
+        load_a(s);
+        load_b(s, kt);
         issued_mask |= 1u << s;
         last_par = (last_par & ~(1u << s)) | (ph << s);
+        if (++kt == KT) {
+          kt = 0;
+          ++rt;
+        }
+        if (++s == S) {
+          s = 0;
+          ph ^= 1u;
+        }
       }
       if (!ok) {  // tear-down: let every copy still in flight land before exit
         for (int s = 0; s < S; ++s)
@@ -185,8 +199,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idesc = make_idesc_bf16_f32(kTileM, layout == kWide ? 2 * a.n_pad : a.n_pad);
-      int it = 0, seg = 0;
-      bool ok = true;
+      // descriptors of stage 0; a stage's (and a k-step's) are offsets in the
+      // start-address field (address >> 4, 14 bits: shared memory < 256 KB)
+      const uint64_t adesc0 = make_smem_desc_sw128(smem_addr(smem_a));
+      const uint64_t bdesc0 = make_smem_desc_sw128(smem_addr(smem_b));
+      const uint32_t a_step = kABytes >> 4, b_step = static_cast<uint32_t>(b_bytes) >> 4;
+      const uint32_t p_step = static_cast<uint32_t>(plane_bytes) >> 4;
+      int s = 0, seg = 0;
+      uint32_t ph = 0;
+      bool ok = true, first = true;
       for (int t = t_begin; t < t_end && ok; ++seg) {
         const int rt = t / KT;
         const int seg_end = min(t_end, (rt + 1) * KT);
@@ -199,34 +220,35 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * acols);
-        for (int tt = t; tt < seg_end; ++tt, ++it) {
-          const int s = it % S;
-          const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
+        for (int tt = t; tt < seg_end; ++tt) {
           if (!mbar_wait_bounded(&ctl.full[s], ph, abort_flag, a.status)) {
             ok = false;
             break;
           }
-          if (it == 0) trace_at(trace, 3);
+          if (first) {
+            trace_at(trace, 3);
+            first = false;
+          }
           tc_fence_after();
-          const uint32_t a_addr = smem_addr(smem_a + static_cast<size_t>(s) * kABytes);
-          const uint32_t b_addr = smem_addr(smem_b + static_cast<size_t>(s) * b_bytes);
+          const uint64_t ad = adesc0 + static_cast<uint32_t>(s) * a_step;
+          const uint64_t bd = bdesc0 + static_cast<uint32_t>(s) * b_step;
+          const uint32_t acc0 = tt > t ? 1u : 0u;
           if (layout != kTwice) {   // one MMA per k-step (N = n_pad or 2 n_pad)
 #pragma unroll
             for (int kk = 0; kk < kTileK / 16; ++kk)
-              tc_mma_bf16(d_tmem, make_smem_desc_sw128(a_addr + kk * 32),
-                          make_smem_desc_sw128(b_addr + kk * 32), idesc,
-                          (tt > t || kk > 0) ? 1u : 0u);
+              tc_mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, kk > 0 ? 1u : acc0);
           } else {                  // hi then lo plane into the same accumulator
 #pragma unroll
             for (int kk = 0; kk < kTileK / 16; ++kk) {
-              const uint64_t adesc = make_smem_desc_sw128(a_addr + kk * 32);
-              tc_mma_bf16(d_tmem, adesc, make_smem_desc_sw128(b_addr + kk * 32), idesc,
-                          (tt > t || kk > 0) ? 1u : 0u);
-              tc_mma_bf16(d_tmem, adesc, make_smem_desc_sw128(b_addr + plane_bytes + kk * 32),
-                          idesc, 1u);
+              tc_mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, kk > 0 ? 1u : acc0);
+              tc_mma_bf16(d_tmem, ad + 2 * kk, bd + p_step + 2 * kk, idesc, 1u);
             }
           }
           tc_commit(&ctl.empty[s]);
+          if (++s == S) {
+            s = 0;
+            ph ^= 1u;
+          }
         }
         if (!ok) break;
         tc_commit(&ctl.acc_full[buf]);

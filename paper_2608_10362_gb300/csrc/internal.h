@@ -71,6 +71,8 @@ enum L2Hint : int { L2_EVICT_FIRST = 0, L2_EVICT_NORMAL = 1, L2_EVICT_LAST = 2 }
 struct GemmArgs {
   CUtensorMap map_a;        // weights [n_out][k] bf16, box {64, 128} (or {64, 64} for pairs)
   CUtensorMap map_a2;       // second matrix of a SwiGLU pair (up), box {64, 64}
+  const uint8_t* a_packed;  // non-null: weights as packed 16 KB tiles in stream-K order
+                            // (tile t at a_packed + t * 16384; map_a, map_a2 unused)
   CUtensorMap map_b;        // activations [rows_total][k] bf16, box {64, n_pad}
   CUtensorMap map_b2;       // low-order plane of the activations (split), same shape
   int split;                // 1: activations = hi + lo bf16 planes, two MMAs per k-step
@@ -237,6 +239,19 @@ __host__ __device__ inline float philox_uniform(unsigned long long seed, int req
 }
 
 // Stream-K schedule: CTA c of G processes global tiles [begin(c), begin(c+1)).
+// Packed weight tiles: a [n][k] matrix as tiles of 128 rows x 64 columns, tile
+// (rt, kt) = 16384 contiguous bytes at (rt * ceil(k/64) + kt) * 16384; row r of a
+// tile at byte 128 r, its 16-byte column chunk c at chunk position c ^ (r % 8)
+// (the 128-byte-swizzled K-major image the tensor cores read); zero beyond n, k.
+// Pairs (gate/up): tile rows 0..63 from the first matrix, 64..127 from the second.
+constexpr int kPackTileBytes = 16384;
+inline size_t packed_bytes(long long n, long long k, bool pair) {
+  const long long rt = pair ? (n + 63) / 64 : (n + 127) / 128;
+  return static_cast<size_t>(rt * ((k + 63) / 64)) * kPackTileBytes;
+}
+cudaError_t launch_pack(const bf16* src, const bf16* src2, int n, int k, uint8_t* dst,
+                        cudaStream_t s);
+
 // 32-bit arithmetic: the host guarantees (T + 1) * (G + 1) < 2^32 for every GEMM
 // (sk_fits).
 inline bool sk_fits(long long T, int G) { return (T + 1) * (G + 1) < (1LL << 32); }

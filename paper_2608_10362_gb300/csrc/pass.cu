@@ -201,7 +201,10 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
           if (weights) {
             uint8_t* dst = ring_a + static_cast<size_t>(s) * kABytes;
             mbar_arrive_expect_tx(&ctl.full_a[s], kABytes);
-            if (a.pair) {
+            if (a.a_packed != nullptr) {
+              bulk_load(dst, a.a_packed + static_cast<size_t>(t) * kABytes, kABytes, &ctl.full_a[s],
+                        pol_w);
+            } else if (a.pair) {
               tma_load_2d(dst, &a.map_a, kt * kTileK, rt * 64, &ctl.full_a[s], pol_w);
               tma_load_2d(dst + kABytes / 2, &a.map_a2, kt * kTileK, rt * 64, &ctl.full_a[s], pol_w);
             } else {

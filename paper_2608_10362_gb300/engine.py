@@ -57,27 +57,74 @@ def kv_bytes(shape, max_batch: int, max_seq: int) -> int:
     return n.value
 
 
-_SIMPLE = {"tok_emb": _lib.T_TOK_EMB, "attn_norm": _lib.T_ATTN_NORM, "wo": _lib.T_WO,
-           "ffn_norm": _lib.T_FFN_NORM, "w_gate": _lib.T_WGATE, "w_up": _lib.T_WUP,
-           "w_down": _lib.T_WDOWN, "final_norm": _lib.T_FINAL_NORM, "lm_head": _lib.T_LM_HEAD}
+_ROW_MAJOR = {"tok_emb": _lib.T_TOK_EMB, "attn_norm": _lib.T_ATTN_NORM,
+              "ffn_norm": _lib.T_FFN_NORM, "final_norm": _lib.T_FINAL_NORM}
+_PACKED = {"wo": _lib.T_WO, "w_down": _lib.T_WDOWN, "lm_head": _lib.T_LM_HEAD}
 
 
-def fill_blob(shape, blob: torch.Tensor, tensors: Iterable) -> None:
+def _bf16(arr, device) -> torch.Tensor:
+    t = arr if isinstance(arr, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(arr))
+    return t.to(device=device, dtype=torch.bfloat16).contiguous()
+
+
+def pack_matrix(src: torch.Tensor, dst: torch.Tensor, src2: torch.Tensor = None,
+                stream=None) -> None:
+    """Pack row-major bf16 device matrices (src [n][k], and src2 for a gate/up
+    pair) into the blob's packed-tile format at dst (a uint8 device view)."""
+    lib = _lib.load()
+    n, k = src.shape
+    s = stream.cuda_stream if stream is not None else torch.cuda.current_stream(src.device).cuda_stream
+    _check(lib, lib.memspec_pack_matrix(C.c_void_p(src.data_ptr()),
+                                        C.c_void_p(src2.data_ptr() if src2 is not None else 0),
+                                        int(n), int(k), C.c_void_p(dst.data_ptr()), dst.numel(),
+                                        C.c_void_p(s)))
+
+
+def fill_blob(shape, blob: torch.Tensor, tensors: Iterable, device=None) -> None:
     """Copy (name, layer, array) weights (float32 arrays holding bf16 values, or
-    bf16 torch tensors) into a uint8 blob at the library's offsets."""
-    q_bytes = shape.n_heads * shape.head_dim * shape.d_model * 2
-    kv_b = shape.n_kv_heads * shape.head_dim * shape.d_model * 2
+    bf16 torch tensors) into a uint8 blob at the library's offsets: norms and the
+    embedding row-major, projection matrices packed on the GPU (memspec_pack_matrix).
+    A host blob (pinned) is packed on `device` and copied back."""
+    dev = blob.device if blob.device.type == "cuda" else torch.device(device or "cuda")
+    pending = {}   # (layer, group) -> {name: device tensor}
+
+    def place(tensor_id, layer, fill):
+        off, nb = tensor_offset(shape, tensor_id, max(layer, 0))
+        if blob.device.type == "cuda":
+            fill(blob[off:off + nb])
+        else:   # pack into a device buffer, then copy to the host blob
+            tmp = torch.empty(nb, dtype=torch.uint8, device=dev)
+            fill(tmp)
+            blob[off:off + nb].copy_(tmp.cpu())
+
     for name, layer, arr in tensors:
-        t = arr if isinstance(arr, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(arr))
-        t = t.to(torch.bfloat16).contiguous().view(-1)
-        if name in ("wq", "wk", "wv"):
-            off, _ = tensor_offset(shape, _lib.T_WQKV, layer)
-            off += {"wq": 0, "wk": q_bytes, "wv": q_bytes + kv_b}[name]
-        else:
-            off, nb = tensor_offset(shape, _SIMPLE[name], max(layer, 0))
+        if name in _ROW_MAJOR:
+            off, nb = tensor_offset(shape, _ROW_MAJOR[name], max(layer, 0))
+            t = _bf16(arr, blob.device).view(-1)
             assert nb == t.numel() * 2, (name, nb, t.numel())
-        view = blob[off:off + t.numel() * 2].view(torch.bfloat16)
-        view.copy_(t.to(blob.device), non_blocking=False)
+            blob[off:off + nb].view(torch.bfloat16).copy_(t)
+        elif name in _PACKED:
+            t = _bf16(arr, dev)
+            place(_PACKED[name], layer, lambda view, t=t: pack_matrix(t, view))
+        elif name in ("wq", "wk", "wv"):
+            g = pending.setdefault((layer, "qkv"), {})
+            g[name] = _bf16(arr, dev)
+            if len(g) == 3:
+                w = torch.cat([g["wq"], g["wk"], g["wv"]], dim=0)
+                place(_lib.T_WQKV, layer, lambda view, w=w: pack_matrix(w, view))
+                del pending[(layer, "qkv")]
+        elif name in ("w_gate", "w_up"):
+            g = pending.setdefault((layer, "ffn"), {})
+            g[name] = _bf16(arr, dev)
+            if len(g) == 2:
+                gt, up = g["w_gate"], g["w_up"]
+                place(_lib.T_WGATE, layer, lambda view, gt=gt, up=up: pack_matrix(gt, view, up))
+                del pending[(layer, "ffn")]
+        else:
+            raise KeyError(f"unknown tensor {name}")
+    if pending:
+        raise ValueError(f"incomplete matrix groups: {sorted(pending)}")
+    torch.cuda.synchronize(dev)
 
 
 class Engine:
@@ -157,7 +204,7 @@ class Engine:
     # -------------------------------------------------------------- drafts
     def register_draft(self, draft_id: int, shape, weights):
         blob = torch.empty(weights_bytes(shape), dtype=torch.uint8, pin_memory=True)
-        fill_blob(shape, blob, _as_triples(weights))
+        fill_blob(shape, blob, _as_triples(weights), device=self.device)
         kv = torch.empty(kv_bytes(shape, self.max_batch, self.max_seq), dtype=torch.uint8,
                          device=self.device)
         cfg = model_cfg(shape)

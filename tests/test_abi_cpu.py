@@ -59,6 +59,16 @@ def test_weight_blob_layout(lib):
         cfg = model_cfg(s)
         total = C.c_size_t()
         assert lib.memspec_weights_bytes(C.byref(cfg), C.byref(total)) == 0
+        # documented sizes: row-major bf16, or packed 16 KB tiles of 128 (pairs:
+        # 64 + 64) rows x 64 columns, zero-padded
+        def packed(n, k, pair=False):
+            rows = 64 if pair else 128
+            return -(-n // rows) * -(-k // 64) * 16384
+        d, q, kv, f, v = s.d_model, s.n_heads * s.head_dim, s.n_kv_heads * s.head_dim, s.d_ffn, s.vocab
+        expect = {_lib.T_TOK_EMB: v * d * 2, _lib.T_ATTN_NORM: d * 2, _lib.T_WQKV: packed(q + 2 * kv, d),
+                  _lib.T_WO: packed(d, q), _lib.T_FFN_NORM: d * 2, _lib.T_WGATE: packed(f, d, True),
+                  _lib.T_WUP: 0, _lib.T_WDOWN: packed(d, f), _lib.T_FINAL_NORM: d * 2,
+                  _lib.T_LM_HEAD: v * d * 2 if s.tied else packed(v, d)}
         spans = []
         for t in range(10):
             layers = range(s.n_layers) if 1 <= t <= 7 else [0]
@@ -66,14 +76,18 @@ def test_weight_blob_layout(lib):
                 off, nb = C.c_size_t(), C.c_size_t()
                 assert lib.memspec_weights_offset(C.byref(cfg), t, l, C.byref(off), C.byref(nb)) == 0
                 assert off.value % 256 == 0
-                if not (t == _lib.T_LM_HEAD and s.tied):
-                    spans.append((off.value, nb.value))
+                assert nb.value == expect[t], (name, t, nb.value, expect[t])
+                if t == _lib.T_WUP:   # inside the gate/up pair tiles
+                    g = C.c_size_t()
+                    lib.memspec_weights_offset(C.byref(cfg), _lib.T_WGATE, l, C.byref(g), C.byref(nb))
+                    assert g.value == off.value
+                elif not (t == _lib.T_LM_HEAD and s.tied):
+                    spans.append((off.value, expect[t]))
         spans.sort()
         for (o1, n1), (o2, _) in zip(spans, spans[1:]):
             assert o1 + n1 <= o2
         assert spans[-1][0] + spans[-1][1] <= total.value
-        assert total.value >= 2 * s.n_params()
-        assert total.value - 2 * s.n_params() < 256 * len(spans)
+        assert total.value - sum(n for _, n in spans) < 256 * len(spans)
         if s.tied:
             a, b, n = C.c_size_t(), C.c_size_t(), C.c_size_t()
             lib.memspec_weights_offset(C.byref(cfg), _lib.T_LM_HEAD, 0, C.byref(a), C.byref(n))

@@ -52,6 +52,52 @@ def test_linear_full_7b_shapes_sampled(n_out, k):
     assert np.all(np.abs(y[:, cols] - ref) <= 1e-4 * bound + 1e-6)
 
 
+def _pack_reference(a, b=None):
+    """Packed-tile bytes (as bf16 bit patterns) written out from the documented
+    format: 128-row (pairs: 64 + 64) x 64-column tiles, row-major tiles in
+    (row tile, k tile) order, 16-byte chunk c of row r stored at c ^ (r % 8)."""
+    n, k = a.shape
+    rows = 64 if b is not None else 128
+    RT, KT = -(-n // rows), -(-k // 64)
+    bits = lambda x: (np.ascontiguousarray(x, dtype=np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    out = np.zeros((RT, KT, 128, 64), dtype=np.uint16)
+    for rt in range(RT):
+        for kt in range(KT):
+            tile = np.zeros((128, 64), dtype=np.uint16)
+            for r in range(128):
+                if b is not None:
+                    src, row = (a, rt * 64 + r) if r < 64 else (b, rt * 64 + r - 64)
+                else:
+                    src, row = a, rt * 128 + r
+                if row >= n:
+                    continue
+                cols = src[row, kt * 64:kt * 64 + 64]
+                vals = np.zeros(64, dtype=np.uint16)
+                vals[:len(cols)] = bits(cols)
+                for c in range(8):
+                    pos = c ^ (r % 8)
+                    tile[r, pos * 8:pos * 8 + 8] = vals[c * 8:c * 8 + 8]
+            out[rt, kt] = tile
+    return out.reshape(-1)
+
+
+@pytest.mark.parametrize("n,k,pair", [(300, 200, False), (130, 136, True), (128, 64, False),
+                                      (256, 8, True)])
+def test_pack_matrix_matches_documented_layout(n, k, pair):
+    from paper_2608_10362_gb300 import pack_matrix
+    rng = np.random.default_rng(n * 7 + k)
+    a = bf16_round(rng.standard_normal((n, k), dtype=np.float32))
+    b = bf16_round(rng.standard_normal((n, k), dtype=np.float32)) if pair else None
+    ref = _pack_reference(a, b)
+    dst = torch.full((ref.size * 2,), 0xAB, dtype=torch.uint8, device="cuda")   # non-zero fill
+    ta = torch.from_numpy(a).to(torch.bfloat16).cuda()
+    tb = torch.from_numpy(b).to(torch.bfloat16).cuda() if pair else None
+    pack_matrix(ta, dst, tb)
+    torch.cuda.synchronize()
+    got = dst.cpu().numpy().view(np.uint16)
+    assert np.array_equal(got, ref)
+
+
 @pytest.mark.parametrize("T", [0.0, 1.0, 0.8])
 @pytest.mark.parametrize("vocab", [2048, 32000, 128256, 97])
 def test_sampler_matches_inverse_cdf(T, vocab):
