@@ -384,9 +384,29 @@ __device__ __forceinline__ void reduce_partials(const GemmArgs& a, int rt, int c
   }
 }
 
+// Synthetic context for the dry run (below): every row valid, position and
+// request 0, so every address the dry run forms is in bounds.  Ends with a barrier.
+__device__ __forceinline__ void epi_ctx_dry(EpiCtx* ctx, int n_pad, int et) {
+  for (int r = et; r < n_pad; r += 128) {
+    ctx->pos[r] = 0;
+    ctx->req[r] = 0;
+    ctx->grp[r] = 0;
+  }
+  if (et < kMaxRows / 32) {
+    ctx->valid[et] = 0xffffffffu;
+    ctx->last[et] = 0u;
+  }
+  for (int i = et; i < kCtxRopeRows * 64; i += 128) {
+    ctx->rc[i / 64][i % 64] = 1.f;
+    ctx->rs[i / 64][i % 64] = 0.f;
+  }
+  named_bar_sync(1, 128);
+}
+
 // Dry run of the tail - the partial reduction and the epilogue of this CTA's
 // first row tile, with every global store off - by the 128 epilogue threads
-// while the weights stream.  The tail runs once per launch; without this its
+// before the launch waits for its predecessor (griddepcontrol.wait): it only
+// reads scratch and weights, with the synthetic context of epi_ctx_dry.  The tail runs once per launch; without this its
 // instructions are fetched cold, one miss after another, on the critical path.
 template <int EPI>
 __device__ __forceinline__ void epilogue_warmup(const GemmArgs& a, const EpiCtx* ctx,
