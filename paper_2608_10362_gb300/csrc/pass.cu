@@ -170,7 +170,8 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
       const uint64_t pol_w = l2_policy_evict_first();
       const uint64_t pol_b = l2_policy_evict_last();
       uint32_t issued = 0, last_par = 0;
-      int it = 0;
+      int s = 0;                // ring position of the next tile (incremental: no division)
+      uint32_t ph = 0;
       bool ok = true;
       for (int n = 0; n < p.n_ops && ok; ++n) {
         const PassOp& op = p.ops[n];
@@ -181,6 +182,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
         const int T = a.row_tiles * a.k_tiles, KT = a.k_tiles;
         const int t_begin = sk_begin(c, T, Gn), t_end = sk_begin(c + 1, T, Gn);
         const int plane_bytes = a.n_pad * 128;
+        int rt = t_begin / KT, kt = t_begin - rt * KT;
         if (!weights) {
           // activations are written by op n-1 (and earlier): wait until it completed
           if (n > 0 && !wait_ready(&ctl.ops_ready, n, abort_flag, p.status)) {
@@ -190,10 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
           fence_proxy_async_global();
           if (unsigned long long* ts = trace_slot(p, n, 2)) *ts = global_ns();
         }
-        for (int t = t_begin; t < t_end; ++t, ++it) {
-          const int rt = t / KT, kt = t - rt * KT;
-          const int s = it % S;
-          const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
+        for (int t = t_begin; t < t_end; ++t) {
           if (!mbar_wait_bounded(&ctl.empty[s], ph ^ 1u, abort_flag, p.status)) {
             ok = false;
             break;
@@ -218,6 +217,14 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
           }
           issued |= 1u << s;
           last_par = (last_par & ~(1u << s)) | (ph << s);
+          if (++kt == KT) {
+            kt = 0;
+            ++rt;
+          }
+          if (++s == S) {
+            s = 0;
+            ph ^= 1u;
+          }
         }
       }
       if (!ok) {   // tear-down: let the copies in flight land before exit
@@ -229,8 +236,12 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
   } else if (warp == 1) {
     // ---------------------------------------------------- MMA issuer
     if (lane == 0) {
-      int it = 0, seg = 0;
+      int seg = 0, s = 0;
+      uint32_t ph = 0;
       bool ok = true;
+      const uint64_t adesc0 = make_smem_desc_sw128(smem_addr(ring_a));
+      const uint64_t bdesc0 = make_smem_desc_sw128(smem_addr(ring_b));
+      const uint32_t a_step = kABytes >> 4, b_step = static_cast<uint32_t>(p.b_stage_bytes) >> 4;
       for (int n = 0; n < p.n_ops && ok; ++n) {
         const PassOp& op = p.ops[n];
         if (op.type != OP_GEMM) continue;
@@ -256,9 +267,8 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
           }
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * acols);
-          for (int tt = t; tt < seg_end; ++tt, ++it) {
-            const int s = it % S;
-            const uint32_t ph = static_cast<uint32_t>(it / S) & 1u;
+          const uint32_t p_step = static_cast<uint32_t>(plane_bytes) >> 4;
+          for (int tt = t; tt < seg_end; ++tt) {
             if (!mbar_wait_bounded(&ctl.full_a[s], ph, abort_flag, p.status) ||
                 !mbar_wait_bounded(&ctl.full_b[s], ph, abort_flag, p.status)) {
               ok = false;
@@ -269,25 +279,25 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
               ts_mma = nullptr;
             }
             tc_fence_after();
-            const uint32_t a_addr = smem_addr(ring_a + static_cast<size_t>(s) * kABytes);
-            const uint32_t b_addr = smem_addr(ring_b + static_cast<size_t>(s) * p.b_stage_bytes);
+            const uint64_t ad = adesc0 + static_cast<uint32_t>(s) * a_step;
+            const uint64_t bd = bdesc0 + static_cast<uint32_t>(s) * b_step;
+            const uint32_t acc0 = tt > t ? 1u : 0u;
             if (layout != kTwice) {
 #pragma unroll
               for (int kk = 0; kk < kTileK / 16; ++kk)
-                tc_mma_bf16(d_tmem, make_smem_desc_sw128(a_addr + kk * 32),
-                            make_smem_desc_sw128(b_addr + kk * 32), idesc,
-                            (tt > t || kk > 0) ? 1u : 0u);
+                tc_mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, kk > 0 ? 1u : acc0);
             } else {
 #pragma unroll
               for (int kk = 0; kk < kTileK / 16; ++kk) {
-                const uint64_t adesc = make_smem_desc_sw128(a_addr + kk * 32);
-                tc_mma_bf16(d_tmem, adesc, make_smem_desc_sw128(b_addr + kk * 32), idesc,
-                            (tt > t || kk > 0) ? 1u : 0u);
-                tc_mma_bf16(d_tmem, adesc, make_smem_desc_sw128(b_addr + plane_bytes + kk * 32),
-                            idesc, 1u);
+                tc_mma_bf16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, kk > 0 ? 1u : acc0);
+                tc_mma_bf16(d_tmem, ad + 2 * kk, bd + p_step + 2 * kk, idesc, 1u);
               }
             }
             tc_commit(&ctl.empty[s]);
+            if (++s == S) {
+              s = 0;
+              ph ^= 1u;
+            }
           }
           if (!ok) break;
           tc_commit(&ctl.acc_full[buf]);
