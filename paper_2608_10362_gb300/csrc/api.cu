@@ -202,7 +202,8 @@ AttnGeo attn_geometry(const memspec_model_cfg& c, int groups, int R, int max_seq
   const int units = groups * c.n_kv_heads * g.row_blocks;
   const int max_splits = ceil_div(max_seq, 64);
   // at most two CTAs per SM in one wave (an extra partial wave would double the time)
-  int want = std::max(1, (2 * sm_count()) / units);
+  // (and at most 16 splits: the combine fetches 16 splits' outputs per round trip)
+  int want = std::max(1, std::min(16, (2 * sm_count()) / units));
   want = std::min(want, max_splits);
   g.chunk = round_up(ceil_div(max_seq, want), 64);
   g.n_splits = ceil_div(max_seq, g.chunk);
@@ -546,8 +547,29 @@ int gemm_grid(int row_tiles, int k_tiles) {
   return std::max(1, std::min({T, sm_count(), T / min_tiles}));
 }
 
+// Whether a GEMM launch dry-runs its tail before griddepcontrol.wait: worth it
+// when the launch starts early (while its predecessor's CTAs drain); the down
+// projection follows gate/up, whose CTAs nearly all reduce and leave late.
+// MEMSPEC_WARM_DOWN / MEMSPEC_WARM_OTHER = 0 or 1 override (measurement).
+int warm_default(const char* env, int dflt) {
+  const char* e = std::getenv(env);
+  return e != nullptr ? (e[0] == '1') : dflt;
+}
+int warm_down() {
+  static int v = -1;
+  if (v < 0) v = warm_default("MEMSPEC_WARM_DOWN", 1);
+  return v;
+}
+int warm_other() {
+  static int v = -1;
+  if (v < 0) v = warm_default("MEMSPEC_WARM_OTHER", 1);
+  return v;
+}
+
 void emit_gemm(memspec_ctx* c, GemmArgs& a, std::vector<PassOp>& ops) {
   const int planes = a.split ? 2 : 1;
+  if (a.warm < 0) a.warm = warm_down();   // the down projection marks itself with -1
+  else a.warm = warm_other();
   a.stages = gemm_pick_stages(a.n_pad, planes);
   a.partials = c->gemm_part;
   a.counters = c->gemm_cnt;
@@ -727,6 +749,7 @@ memspec_status emit_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f,
     }
     {  // down projection + residual
       GemmArgs a{};
+      a.warm = -1;
       a.a_packed = m.w + m.lay.wdown[l];
       a.n_out = d;
       a.k_in = F;

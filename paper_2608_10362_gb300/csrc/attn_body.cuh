@@ -69,17 +69,28 @@ __host__ __device__ constexpr size_t attention_smem_bytes_hd() {
 // (tid 0..127); `sync` is a barrier over exactly those threads; smem_raw is the
 // CTA's attention shared memory (attention_smem_bytes).  Returns early, all
 // threads together, when the unit has no work.
+// dry: a run of the same code on one synthetic tile that reads only scratch and
+// writes no global memory (no output, no partials, no counters): launched
+// before griddepcontrol.wait, it brings this code into the instruction cache
+// while the previous kernel finishes.  Callers pass g = kvh = rb = split = 0.
 template <int HD, class Sync>
 __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh, int rb, int split,
                                               uint8_t* smem_raw, int tid, Sync sync,
-                                              unsigned long long* ts = nullptr) {
+                                              unsigned long long* ts = nullptr, bool dry = false) {
   constexpr int kChunks = HD / 8;                        // 16-byte chunks per row
   constexpr int kTileBytes = kKeyTile * HD * 2;          // one K (or V) tile
   constexpr int kNT = HD / 8;                            // n8 tiles of the output
   const RowPlan* plan = a.plan;
-  if (g >= plan->n_groups) return;
-  const int R = plan->rows_per_group;
-  const int req = plan->req[g], valid = plan->valid[g], pos0 = plan->pos0[g];
+  // every plan field in one round trip (g < kMaxGroups: in bounds before the check)
+  int n_groups = 1, R = a.rows_per_block, req = 0, valid = a.rows_per_block, pos0 = 0;
+  if (!dry) {
+    n_groups = plan->n_groups;
+    R = plan->rows_per_group;
+    req = plan->req[g];
+    valid = plan->valid[g];
+    pos0 = plan->pos0[g];
+  }
+  if (g >= n_groups) return;
   const int r_lo = rb * a.rows_per_block;
   const int r_hi = min(r_lo + a.rows_per_block, valid);
   if (r_lo >= r_hi) return;
@@ -118,7 +129,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     const int kt0 = k0 + t * kKeyTile;
     for (int c = tid; c < kKeyTile * kChunks; c += kAttThreads) {
       const int row = c / kChunks, ch = c - row * kChunks;
-      const bool ok = kt0 + row < k1;
+      const bool ok = kt0 + row < k1 && !dry;   // dry: zero-fill, no global read
       const size_t off = ok ? static_cast<size_t>(kt0 + row) * HD + ch * 8 : 0;
       cp_async16_zfill(ks + swz<HD>(row, ch), kc + off, ok);
       cp_async16_zfill(vs + swz<HD>(row, ch), vc + off, ok);
@@ -133,7 +144,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   for (int c = tid; c < kMaxQ * kChunks; c += kAttThreads) {
     const int v = c / kChunks, ch = c - v * kChunks;
     __nv_bfloat16 e[8], el[8];
-    if (v < nq) {
+    if (v < nq && !dry) {
       const int hl = v / nr, rr = v - hl * nr;
       const int row = g * R + r_lo + rr;
       const int h = kvh * gs + hl;
@@ -314,6 +325,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
       L += f * ml[(ww * 16 + r) * 2 + 1];
       O += f * mo[(ww * 16 + r) * HD + d];
     }
+    if (dry) continue;
     a.part_o[(pbase + v) * HD + d] = O;
     if (d == 0) {
       a.part_ml[(pbase + v) * 2 + 0] = M;
@@ -326,7 +338,8 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   // and the next barrier order every split's partials before its loads
   sync();
   int* last = reinterpret_cast<int*>(kv + attention_smem_bytes_hd<HD>() - 16);
-  if (tid == 0) *last = (atom_add_acq_rel_gpu(&a.counters[unit], 1) == n_active - 1) ? 1 : 0;
+  if (tid == 0)
+    *last = dry ? 1 : ((atom_add_acq_rel_gpu(&a.counters[unit], 1) == n_active - 1) ? 1 : 0);
   sync();
   trace_at(ts, 5);
   if (!*last) return;
@@ -374,8 +387,9 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   }
   sync();
   trace_at(ts, 6);
-  // weighted sum of the split outputs, four features per thread, eight splits
-  // fetched at once and added in ascending split order
+  // weighted sum of the split outputs, four features per thread, sixteen splits
+  // fetched at once (one round trip for up to 16 splits) and added in ascending
+  // split order
   constexpr int kV4 = HD / 4;
   bf16* out = a.out;
   bf16* out_lo = a.out_lo;
@@ -383,14 +397,14 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   for (int idx = tid; idx < nq * kV4; idx += kAttThreads) {
     const int v = idx / kV4, d = (idx - v * kV4) * 4;
     float O[4] = {0.f, 0.f, 0.f, 0.f};
-    for (int s0 = 0; s0 < n_active; s0 += 8) {
-      float4 ov[8];
+    for (int s0 = 0; s0 < n_active; s0 += 16) {
+      float4 ov[16];
 #pragma unroll
-      for (int q = 0; q < 8; ++q)
+      for (int q = 0; q < 16; ++q)
         if (s0 + q < n_active)
           ov[q] = ld_cg_f4(part_o + (ubase + static_cast<size_t>(s0 + q) * qmax + v) * HD + d);
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
+      for (int q = 0; q < 16; ++q) {
         if (s0 + q < n_active) {
           const float w = msm[(s0 + q) * nq + v];
           O[0] += w * ov[q].x;
@@ -405,6 +419,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     const int h = kvh * gs + hl;
     const size_t oi = (static_cast<size_t>(row) * H + h) * HD + d;
     const float li = linv[v];
+    if (dry) continue;
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       if (out_lo != nullptr) {
@@ -415,7 +430,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     }
   }
   trace_at(ts, 7);
-  if (tid == 0) a.counters[unit] = 0;
+  if (tid == 0 && !dry) a.counters[unit] = 0;
 }
 
 

@@ -265,8 +265,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
     const int ew = warp & 3;
     const int et = ew * 32 + lane;  // tile feature == TMEM lane
     // the dry run overlaps the previous launch's tail; the real context follows
-    epi_ctx_dry(ectx, a.n_pad, et);
-    epilogue_warmup<EPI>(a, ectx, ctl.red, stage, rms, c, G, et);
+    if (a.warm) {
+      epi_ctx_dry(ectx, a.n_pad, et);
+      epilogue_warmup<EPI>(a, ectx, ctl.red, stage, rms, c, G, et);
+    }
     pdl_wait();
     if (threadIdx.x == 64) trace_at(trace, 13);
     if (a.rms) rms_prologue(a, rms, et);

@@ -186,11 +186,14 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, const EpiC
         }
       }
     }
-    // per-row sums over the warp's 32 features: the 16 butterflies interleaved
+    // per-row sums over the warp's 32 features, valid rows only (a decode pass
+    // has 1 to a few rows of the 16)
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
+    for (int j = 0; j < 16; ++j) {
+      if (r0 + j < rows_total) {
 #pragma unroll
-      for (int j = 0; j < 16; ++j) sq[j] += __shfl_xor_sync(0xffffffffu, sq[j], o);
+        for (int o = 16; o > 0; o >>= 1) sq[j] += __shfl_xor_sync(0xffffffffu, sq[j], o);
+      }
     }
     if (lane == 0) {
 #pragma unroll

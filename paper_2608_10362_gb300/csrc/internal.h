@@ -116,6 +116,7 @@ struct GemmArgs {
   const RowPlan* plan;      // nullptr: rows < rows_total are valid, no positions
   uint32_t* status;
   unsigned long long* trace;  // nullptr, or this op's trace row (16 slots per CTA)
+  int warm;                 // 1: dry run of the tail before griddepcontrol.wait
 };
 
 struct AttnArgs {
