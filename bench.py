@@ -304,6 +304,33 @@ def run_case(args):
         return {"case": "gemm", "n_out": args.n, "k": args.kdim, "rows": args.rows,
                 "us_per_launch": ms * 1e3, "GB/s": nbytes / ms / 1e6}
     from paper_2608_10362_gb300 import Engine
+    if args.case == "prefill":
+        # a whole-prompt prefill of the 7B target (chunks of up to 128 rows), timed,
+        # inside an NVTX range "prefill"
+        t = SHAPES[TARGET]
+        eng = Engine(t, iter_weights(t, 0), max_batch=1, max_seq=PREFIX + 64, max_k=args.k,
+                     max_drafts=0, use_graphs=True,
+                     trace="prefill" if args.trace is not None else None)
+        prompt = gen_prompt(3, PREFIX, t.vocab)
+        for _ in range(args.warmup):
+            eng.prefill(0, prompt, seed=1)
+        eng.sync()
+        s = eng.stream
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.nvtx.range_push("prefill")
+        a.record(s)
+        for _ in range(args.steps):
+            eng.prefill(0, prompt, seed=1)
+        b.record(s)
+        torch.cuda.nvtx.range_pop()
+        torch.cuda.synchronize()
+        bits = eng.sync()
+        ms = a.elapsed_time(b) / args.steps
+        if args.trace is not None:
+            np.save(args.trace, eng.pass_trace())
+        eng.close()
+        return {"case": "prefill", "target": TARGET, "tokens": PREFIX, "ms": ms,
+                "tokens_per_s": PREFIX / ms * 1e3, "device_status": bits}
     if args.case == "verify":
         # the 7B verify pass alone, one launch per op and no graph, inside an NVTX
         # range "verify" (for profilers: ncu --nvtx --nvtx-include "verify/")
@@ -411,7 +438,7 @@ def main():
     ap.add_argument("--k", type=int, default=K_DRAFT)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", default="step", choices=["step", "gemm", "small", "verify"],
+    ap.add_argument("--case", default="step", choices=["step", "gemm", "small", "verify", "prefill"],
                     help="step: the workload above; gemm / small: diagnostic cases sized for "
                          "profiler captures (one projection GEMM; a 160M target with a 68M draft)")
     ap.add_argument("--launch-mode", default="per_op", choices=["per_op", "pass"],
@@ -419,7 +446,8 @@ def main():
     ap.add_argument("--trace", default=None,
                     help="save per-op timestamps of the last traced pass (.npy); diagnostic, "
                          "not for the headline number")
-    ap.add_argument("--trace-pass", default="verify", choices=["verify", "draft"])
+    ap.add_argument("--trace-pass", default="verify", choices=["verify", "draft"],
+                    help="(--case step) the pass to trace; --case prefill traces prefill chunks")
     ap.add_argument("--n", type=int, default=22016)
     ap.add_argument("--kdim", type=int, default=4096)
     ap.add_argument("--rows", type=int, default=5)

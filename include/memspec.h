@@ -160,7 +160,8 @@ typedef struct memspec_init_params {
                                        op of a pass; MEMSPEC_LAUNCH_PASS (1): each draft
                                        step and verify pass as one persistent launch */
   int32_t trace;                    /* per-op timestamps (MEMSPEC_BUF_PASS_TRACE) of
-                                       1: verify passes, 2: draft steps; 0: off */
+                                       1: verify passes, 2: draft steps, 3: prefill
+                                       chunks (the last one); 0: off */
 } memspec_init_params;
 
 enum { MEMSPEC_LAUNCH_PER_OP = 0, MEMSPEC_LAUNCH_PASS = 1 };

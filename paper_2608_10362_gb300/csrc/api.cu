@@ -293,6 +293,7 @@ struct memspec_ctx {
   bf16* act = nullptr;
   float* gemm_part = nullptr;
   int* gemm_cnt = nullptr;
+  size_t gemm_cnt_bytes = 0;
   float* att_po = nullptr;
   float* att_pml = nullptr;
   int* att_cnt = nullptr;
@@ -400,7 +401,7 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   const size_t o_act = w.take(static_cast<size_t>(kMaxRows) * fmax * 2);
   const size_t o_actl = w.take(static_cast<size_t>(kMaxRows) * fmax * 2);
   const size_t o_gp = w.take(static_cast<size_t>(2) * nsm * kMaxRows * 128 * 4);
-  const size_t o_gc = w.take(static_cast<size_t>(max_rt) * 4);
+  const size_t o_gc = w.take(static_cast<size_t>(max_rt) * 4);   // split-K arrival counters
   const size_t o_apo = w.take(po * 4);
   const size_t o_apml = w.take(po / 64 * 2 * 4 + 1024);
   const size_t o_acnt = w.take(cnt * 4);
@@ -427,7 +428,7 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   const size_t o_ops = w.take(op_bytes);
   const size_t o_done = w.take(done_ints * 4);
   const size_t trace_bytes =
-      (p->trace == 1 || p->trace == 2)
+      (p->trace >= 1 && p->trace <= 3)
           ? (2 + static_cast<size_t>(kPassTraceOps) * nsm * kPassTraceSlots) * 8
           : 0;
   const size_t o_trace = w.take(trace_bytes);
@@ -444,6 +445,7 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
     c->act = reinterpret_cast<bf16*>(base + o_act);
     c->gemm_part = reinterpret_cast<float*>(base + o_gp);
     c->gemm_cnt = reinterpret_cast<int*>(base + o_gc);
+    c->gemm_cnt_bytes = static_cast<size_t>(max_rt) * 4;
     c->att_po = reinterpret_cast<float*>(base + o_apo);
     c->att_pml = reinterpret_cast<float*>(base + o_apml);
     c->att_cnt = reinterpret_cast<int*>(base + o_acnt);
@@ -966,6 +968,10 @@ memspec_status enqueue_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f) {
   std::vector<PassOp> ops;
   memspec_status s = emit_forward(c, m, f, ops);
   if (s != MEMSPEC_OK) return s;
+  if (c->trace != nullptr && c->p.trace == 3 && f.mode == PLAN_PREFILL) {   // each chunk overwrites
+    s = attach_trace(c, ops);
+    if (s != MEMSPEC_OK) return s;
+  }
   return run_ops_separately(c, ops);
 }
 
@@ -1504,7 +1510,10 @@ memspec_status memspec_sync(memspec_ctx* c, int32_t timeout_ms, uint32_t* bits) 
     // a kernel gave up part-way: clear the status and the arrival counters so the
     // context can be used again
     cudaMemset(c->status, 0, 4);
-    cudaMemset(c->gemm_cnt, 0, 4);
+    cudaMemset(c->gemm_cnt, 0, c->gemm_cnt_bytes);
+    cudaMemset(c->att_cnt, 0, c->att_cnt_cap * 4);
+    cudaMemset(c->acc_cnt, 0, static_cast<size_t>(c->p.max_batch) * 4);
+    cudaMemset(c->smp_cnt, 0, static_cast<size_t>(c->p.max_batch) * 4);
     return fail(c, MEMSPEC_ERR_DEVICE_STATUS, "device status word set");
   }
   return MEMSPEC_OK;
@@ -1587,7 +1596,9 @@ static size_t op_linear_scratch(int rows, int n_out, int k) {
   const int n_pad = round_up(rows, 16);
   const int rt = ceil_div(n_out, 128);
   (void)k;
-  return align256(static_cast<size_t>(2) * sm_count() * n_pad * 128 * 4) + align256(static_cast<size_t>(rt) * 4) + 256;
+  // partials, then one arrival counter per row tile
+  return align256(static_cast<size_t>(2) * sm_count() * n_pad * 128 * 4) +
+         align256(static_cast<size_t>(rt) * 4) + 256;
 }
 
 memspec_status memspec_op_linear_scratch_bytes(int32_t rows, int32_t n_out, int32_t k, size_t* bytes) {

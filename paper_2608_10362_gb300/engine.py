@@ -136,7 +136,7 @@ class Engine:
                  launch_mode: str = "per_op", trace=None, device: int = 0):
         """launch_mode "per_op": one kernel launch per op of a pass; "pass": each
         draft step and verify pass as one persistent launch.  ``trace``
-        ("verify" or "draft") records per-op timestamps of that pass, see
+        ("verify", "draft" or "prefill") records per-op timestamps of that pass, see
         ``pass_trace``."""
         if launch_mode not in ("per_op", "pass"):
             raise ValueError(f"launch_mode must be 'per_op' or 'pass', not {launch_mode!r}")
@@ -167,9 +167,9 @@ class Engine:
         p.stream_side = self.side.cuda_stream
         p.use_graphs = int(use_graphs)
         p.launch_mode = _lib.LAUNCH_PASS if launch_mode == "pass" else _lib.LAUNCH_PER_OP
-        if trace not in (None, "verify", "draft"):
-            raise ValueError(f"trace must be None, 'verify' or 'draft', not {trace!r}")
-        p.trace = {None: 0, "verify": 1, "draft": 2}[trace]
+        if trace not in (None, "verify", "draft", "prefill"):
+            raise ValueError(f"trace must be None, 'verify', 'draft' or 'prefill', not {trace!r}")
+        p.trace = {None: 0, "verify": 1, "draft": 2, "prefill": 3}[trace]
         self.params = p
         n = C.c_size_t()
         _check(self.lib, self.lib.memspec_workspace_bytes(C.byref(p), C.byref(n)))
