@@ -277,6 +277,154 @@ def oracle_sample(tokens_per_iter: float, K: int, reps: int = 1):
     }
 
 
+def verify_bytes_batch(t, ctxs, K: int) -> int:
+    """verify_bytes for a batch: weights once, each request's KV at its context."""
+    L, kv = t.n_layers, t.kv_dim
+    weights = verify_bytes(t, 0, 0) - L * 2 * 1 * kv * 2 - t.vocab * 4
+    B = len(ctxs)
+    return (weights + sum(L * 2 * int(c) * kv * 2 for c in ctxs) + B * L * 2 * (K + 1) * kv * 2
+            + B * (K + 1) * t.vocab * 4)
+
+
+def run_pair_case(args, tname: str, dname: str, prefixes, K: int, T: float, seed: int = 0):
+    """Steady-state decoding of len(prefixes) requests with a target/draft pair:
+    aggregate committed tokens/s, and the verify pass against the HBM roofline."""
+    import numpy as np
+    import torch
+
+    from paper_2608_10362_gb300 import Engine, weights_bytes
+    from seeded_inputs import SHAPES, gen_prompt, iter_weights
+    t, d = SHAPES[tname], SHAPES[dname]
+    B = len(prefixes)
+    steps, warm = args.steps, args.warmup
+    max_seq = int(max(prefixes)) + (steps + warm + 4) * (K + 1) + 16
+    eng = Engine(t, iter_weights(t, seed), max_batch=B, max_seq=max_seq, max_k=K, max_drafts=1,
+                 draft_shape_max=d, draft_budget_bytes=weights_bytes(d) + (1 << 20), use_graphs=True)
+    eng.register_draft(0, d, iter_weights(d, seed + 1))
+    eng.load_draft_async(0)
+    eng.set_active_draft(0)
+    for b, n in enumerate(prefixes):
+        eng.prefill(b, gen_prompt(100 + b, int(n), t.vocab), seed=1 + b)
+    eng.set_batch(B)
+    for _ in range(warm):
+        eng.step(K, T)
+    eng.sync()
+    L0 = eng.seq_state()[:B, 0].astype(np.int64)
+    s = eng.stream
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)]
+    a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(s)
+    for i in range(steps):
+        eng.draft_step(K, T)
+        ev[i][0].record(s)
+        eng.verify_step(K)
+        ev[i][1].record(s)
+        eng.accept_commit(K, T)
+    b_.record(s)
+    torch.cuda.synchronize()
+    bits = eng.sync()
+    L1 = eng.seq_state()[:B, 0].astype(np.int64)
+    ms = a.elapsed_time(b_)
+    v_ms = sum(x.elapsed_time(y) for x, y in ev) / steps
+    vb = verify_bytes_batch(t, (L0 + L1) // 2, K)
+    eng.close()
+    peak, peak_kind = measured_peaks()
+    gbs = vb / (v_ms * 1e-3) / 1e9
+    return {"target": tname, "draft": dname, "batch": B, "K": K, "T": T,
+            "tokens_per_s": float((L1 - L0).sum()) / (ms * 1e-3), "ms_per_step": ms / steps,
+            "tokens_per_step": float((L1 - L0).sum()) / steps, "verify_ms": v_ms,
+            "verify_GBps": gbs, "verify_frac": gbs / peak, "peak": peak, "peak_kind": peak_kind,
+            "algorithmic_bytes": vb, "device_status": bits}
+
+
+def run_switching_case(args):
+    """Draft switching under a 2 GiB draft budget: the 7B target with a pool of
+    drafts (68M, 160M, tied 1.1B) in pinned host memory; every 64 committed tokens
+    the active draft changes by a seeded schedule, and the next scheduled draft is
+    loaded asynchronously (side stream) while the current one decodes."""
+    import numpy as np
+    import torch
+
+    from paper_2608_10362_gb300 import Engine, weights_bytes
+    from seeded_inputs import SHAPES, gen_prompt, iter_weights
+    t = SHAPES[TARGET]
+    pool = {0: SHAPES["draft_68m"], 1: SHAPES["draft_160m"], 2: SHAPES["draft_1b1_tied"]}
+    K, T, prefix, budget = 4, 1.0, 1024, 2 << 30
+    rng = np.random.default_rng(3)
+    n_switch = max(2, args.steps)
+    sched = [int(x) for x in rng.integers(0, 3, n_switch + 1)]
+    sched[0] = 0   # start on the smallest draft (the tied 1.1B, 2.07 GB, fits only alone)
+    for i in range(1, len(sched)):
+        if sched[i] == sched[i - 1]:
+            sched[i] = (sched[i] + 1) % 3
+    max_seq = prefix + (n_switch + 2) * 64 * 2 + 256
+    eng = Engine(t, iter_weights(t, 0), max_batch=1, max_seq=max_seq, max_k=K, max_drafts=3,
+                 draft_shape_max=pool[2], draft_budget_bytes=budget, use_graphs=True)
+    for i, sh in pool.items():
+        eng.register_draft(i, sh, iter_weights(sh, 10 + i))
+    eng.prefill(0, gen_prompt(5, prefix, t.vocab), seed=2)
+    resident = []
+
+    def ensure_loaded(i):
+        """Make draft i resident (evicting non-active drafts first); False when it
+        cannot fit beside the active draft (the active draft is never evicted)."""
+        if i in resident:
+            return True
+        need = weights_bytes(pool[i])
+        others = [j for j in resident if j != active[0]]
+        if need + sum(weights_bytes(pool[j]) for j in resident if j == active[0]) > budget:
+            return False
+        while sum(weights_bytes(pool[j]) for j in resident) + need > budget:
+            victim = others.pop(0)
+            eng.evict_draft(victim)
+            resident.remove(victim)
+        eng.load_draft_async(i)
+        resident.append(i)
+        return True
+
+    active = [sched[0]]
+    ensure_loaded(sched[0])
+    eng.set_active_draft(sched[0])
+    eng.sync()
+    s = eng.stream
+    load_ms, tokens, step_ms, fallbacks = [], 0, [], 0
+    L = int(eng.seq_state()[0, 0])
+    torch.cuda.synchronize()
+    wall0 = time.perf_counter()
+    for k in range(n_switch):
+        if k + 1 < len(sched):
+            ensure_loaded(sched[k + 1])          # prefetch the next draft (side stream)
+        start = L
+        while L - start < 64:
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(s)
+            eng.step(K, T)
+            b.record(s)
+            b.synchronize()
+            step_ms.append(a.elapsed_time(b))
+            L = int(eng.seq_state()[0, 0])
+        tokens += L - start
+        if k + 1 < len(sched):
+            if not ensure_loaded(sched[k + 1]):
+                fallbacks += 1                       # stays on the resident draft
+                continue
+            t0 = time.perf_counter()
+            active[0] = sched[k + 1]
+            eng.set_active_draft(sched[k + 1])   # waits on the GPU for the copy, catches up
+            eng.sync()
+            load_ms.append((time.perf_counter() - t0) * 1e3)
+    wall = time.perf_counter() - wall0
+    bits = eng.sync()
+    eng.close()
+    return {"case": "switching", "target": TARGET, "pool": ["68M", "160M", "1.1B tied"],
+            "budget_GiB": 2, "switch_every_tokens": 64, "switches": n_switch,
+            "schedule": sched[:n_switch + 1], "tokens_per_s": tokens / wall,
+            "step_ms_median": float(np.median(step_ms)),
+            "switch_ms_median": float(np.median(load_ms)) if load_ms else None,
+            "fallbacks": fallbacks, "device_status": bits}
+
+
 def run_case(args):
     """Diagnostic cases (not the headline metric)."""
     import numpy as np
@@ -304,6 +452,14 @@ def run_case(args):
         return {"case": "gemm", "n_out": args.n, "k": args.kdim, "rows": args.rows,
                 "us_per_launch": ms * 1e3, "GB/s": nbytes / ms / 1e6}
     from paper_2608_10362_gb300 import Engine
+    if args.case == "edge":
+        return {"case": "edge", **run_pair_case(args, "target_1b1", "draft_68m", [512], 5, args.temp)}
+    if args.case == "batched":
+        from seeded_inputs import gen_prompt_lengths
+        ctx = [int(c) for c in gen_prompt_lengths(11, 16, 512, 4096)]
+        return {"case": "batched", **run_pair_case(args, "target_8b", "draft_1b1_v128k", ctx, 8, 1.0)}
+    if args.case == "switching":
+        return run_switching_case(args)
     if args.case == "prefill":
         # a whole-prompt prefill of the 7B target (chunks of up to 128 rows), timed,
         # inside an NVTX range "prefill"
@@ -438,9 +594,11 @@ def main():
     ap.add_argument("--k", type=int, default=K_DRAFT)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", default="step", choices=["step", "gemm", "small", "verify", "prefill"],
+    ap.add_argument("--case", default="step", choices=["step", "gemm", "small", "verify", "prefill", "edge", "batched",
+                                                          "switching"],
                     help="step: the workload above; gemm / small: diagnostic cases sized for "
                          "profiler captures (one projection GEMM; a 160M target with a 68M draft)")
+    ap.add_argument("--temp", type=float, default=0.8, help="(--case edge) temperature")
     ap.add_argument("--launch-mode", default="per_op", choices=["per_op", "pass"],
                     help="one launch per op, or one persistent launch per pass")
     ap.add_argument("--trace", default=None,
