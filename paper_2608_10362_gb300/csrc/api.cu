@@ -543,9 +543,15 @@ struct FwdSpec {
 // CTA so that a row tile is shared by at most ~4 CTAs (the last of them sums the
 // partials; more contributors lengthen that serial tail more than they add
 // bandwidth on small matrices).
+int env_int(const char* name, int dflt) {
+  const char* e = std::getenv(name);
+  return e != nullptr ? std::atoi(e) : dflt;
+}
+// MEMSPEC_SK_MAXC overrides the contributor limit (measurement).
 int gemm_grid(int row_tiles, int k_tiles) {
+  static const int max_contrib = std::max(1, env_int("MEMSPEC_SK_MAXC", 4));
   const int T = row_tiles * k_tiles;
-  const int min_tiles = std::max(1, (k_tiles + 3) / 4);
+  const int min_tiles = std::max(1, (k_tiles + max_contrib - 1) / max_contrib);
   return std::max(1, std::min({T, sm_count(), T / min_tiles}));
 }
 
@@ -568,18 +574,81 @@ int warm_other() {
   return v;
 }
 
+// Cluster exchange for decode GEMMs (16 padded rows): a grid of Q clusters of C
+// CTAs whose stream-K ranges put every split row tile inside one cluster, so that
+// the split-K partials move through distributed shared memory instead of global
+// memory (no store, counter or reload on the critical tail).  Taken when its
+// largest range is at most kCskTailTiles - 1 tiles longer than plain stream-K's:
+// a global-memory exchange costs about as much as streaming that many tiles
+// (~1.5 us, measured).  Clusters of at most four CTAs: larger ones (fewer ring
+// stages for the receive slots, longer sums) made the draft step slower, measured.
+// MEMSPEC_CSK=0 disables it; MEMSPEC_CSK_MAX sets the largest C (measurement).
+constexpr int kCskTailTiles = 4;
+bool sk_split_free(int T, int KT, int G) {   // no row tile is shared by two CTAs
+  for (int c = 1; c < G; ++c)
+    if (sk_begin(c, T, G) % KT != 0) return false;
+  return true;
+}
+bool csk_aligned(int R, int KT, int G, int C) {
+  const int T = R * KT;
+  for (int rt = 0; rt < R; ++rt)
+    if (sk_cta_of(rt * KT, T, G) / C != sk_cta_of(rt * KT + KT - 1, T, G) / C) return false;
+  return true;
+}
+struct CskPick {
+  int grid, csk;
+};
+CskPick pick_csk(const GemmArgs& a, int planes, int g0) {
+  static const int enabled = env_int("MEMSPEC_CSK", 1);
+  static const int c_max = std::min(8, env_int("MEMSPEC_CSK_MAX", 4));
+  const int R = a.row_tiles, KT = a.k_tiles, T = R * KT;
+  CskPick best{g0, 0};
+  if (!enabled || a.n_pad != 16 || sk_split_free(T, KT, g0)) return best;
+  int best_cost = ceil_div(T, g0) + kCskTailTiles;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  static std::map<std::tuple<int, int, int, size_t>, int> fit;   // (device, epi, C, smem) -> clusters
+  static std::mutex fit_mu;
+  std::lock_guard<std::mutex> lock(fit_mu);
+  for (int C = 2; C <= c_max; ++C) {
+    const size_t smem = gemm_smem_bytes(a.n_pad, gemm_pick_stages(a.n_pad, planes, C), planes, C);
+    const auto key = std::make_tuple(dev, a.epi, C, smem);
+    auto it = fit.find(key);
+    if (it == fit.end()) it = fit.emplace(key, gemm_max_active_clusters(a.epi, C, smem)).first;
+    const int q_max = std::min({it->second, sm_count() / C, T / C});
+    for (int Q = q_max; Q >= 1; --Q) {
+      const int G = Q * C;
+      if (!sk_fits(T, G)) continue;
+      const int cost = ceil_div(T, G);
+      if (cost >= best_cost) break;   // smaller grids only cost more
+      if (!csk_aligned(R, KT, G, C)) continue;
+      best = {G, C};
+      best_cost = cost;
+      break;
+    }
+  }
+  return best;
+}
+
 void emit_gemm(memspec_ctx* c, GemmArgs& a, std::vector<PassOp>& ops) {
   const int planes = a.split ? 2 : 1;
   if (a.warm < 0) a.warm = warm_down();   // the down projection marks itself with -1
   else a.warm = warm_other();
-  a.stages = gemm_pick_stages(a.n_pad, planes);
+  int grid = gemm_grid(a.row_tiles, a.k_tiles);
+  a.csk = 0;
+  if (!c->pass_kernel) {   // the persistent kernel runs every op on its own grid
+    const CskPick pk = pick_csk(a, planes, grid);
+    grid = pk.grid;
+    a.csk = pk.csk;
+  }
+  a.stages = gemm_pick_stages(a.n_pad, planes, a.csk);
   a.partials = c->gemm_part;
   a.counters = c->gemm_cnt;
   a.status = c->status;
   PassOp op{};
   op.type = OP_GEMM;
-  op.grid = gemm_grid(a.row_tiles, a.k_tiles);
-  op.smem = static_cast<int>(gemm_smem_bytes(a.n_pad, a.stages, planes));
+  op.grid = grid;
+  op.smem = static_cast<int>(gemm_smem_bytes(a.n_pad, a.stages, planes, a.csk));
   op.u.g = a;
   ops.push_back(op);
 }

@@ -288,6 +288,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   cp_async_wait<0>();
   sync();
   trace_at(ts, 9);
+  if (ts != nullptr) trace_after(ts, 12, o[0][0] + o[kNT - 1][3]);   // last MMAs retired
 
   // merge the key groups of each m-tile (shared memory reuses the K/V stages)
   float* mo = reinterpret_cast<float*>(kv);                 // [4 warps][16][HD]
@@ -310,6 +311,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     }
   }
   sync();
+  trace_at(ts, 11);
   const int unit = (g * a.Hkv + kvh) * a.row_blocks + rb;
   const size_t pbase = (static_cast<size_t>(unit) * a.n_splits + split) * a.qmax;
   for (int idx = tid; idx < nq * HD; idx += kAttThreads) {

@@ -52,9 +52,13 @@ struct SmemCtl {
   int reduce_flag;
   int wait_ok;
   float red[4][16];
+  uint64_t recv;        // cluster exchange: partials pushed by peers (one phase)
+  int recv_pending;     // this CTA expects pushed partials it has not yet consumed
 };
 
-template <int EPI>
+// CSK: launched in clusters of a.csk CTAs with the cluster exchange of split row
+// tiles (epilogue_segment); the plain kernel carries none of that code.
+template <int EPI, bool CSK>
 __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_constant__ GemmArgs a) {
   __shared__ SmemCtl ctl;
   extern __shared__ uint8_t dsmem_raw[];
@@ -69,6 +73,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
   float* stage = reinterpret_cast<float*>(smem_b + static_cast<size_t>(S) * b_bytes);
   float* rms = stage + kStageFloats;
   EpiCtx* ectx = reinterpret_cast<EpiCtx*>(rms + kMaxRows);
+  float* recv = reinterpret_cast<float*>(
+      (reinterpret_cast<uintptr_t>(ectx + 1) + 15) & ~static_cast<uintptr_t>(15));
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int T = a.row_tiles * a.k_tiles;
@@ -89,6 +95,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
       mbar_init(&ctl.acc_empty[b], 4);
     }
     mbar_init(&ctl.drain, 1);
+    if constexpr (CSK) {
+      mbar_init(&ctl.recv, 1);
+      ctl.recv_pending = 0;
+    }
     ctl.abort_flag = 0;
     ctl.reduce_flag = 0;
     fence_mbar_init();
@@ -101,6 +111,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // cluster exchange: the barriers above are initialised before any peer pushes
+  // (every thread arrives here; a thread waits before its first push)
+  if constexpr (CSK) cluster_arrive_release();
   pdl_launch_dependents();
   const uint32_t tmem_base = ctl.tmem_base;
   // optional trace (16 slots per CTA): 0 entry, 13 dependency released,
@@ -264,12 +277,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
     // a warp may only read TMEM lanes 32*(warp % 4) .. +31: that is its feature block
     const int ew = warp & 3;
     const int et = ew * 32 + lane;  // tile feature == TMEM lane
+    // cluster exchange: the first contributor of the row tile this range ends in
+    // expects its peers' partials (arrival count 1: this arrive; bytes may land first)
+    bool csk_reducer = false;
+    if (CSK && t_end > t_begin) {
+      const int rt_last = (t_end - 1) / KT;
+      const int cf = sk_cta_of(rt_last * KT, T, G), cl = sk_cta_of((rt_last + 1) * KT - 1, T, G);
+      csk_reducer = cf == c && cl > c && cf / a.csk == cl / a.csk;
+      if (csk_reducer && threadIdx.x == 64) {
+        mbar_arrive_expect_tx(&ctl.recv, static_cast<uint32_t>((cl - cf) * kTileM * 16 * 4));
+        ctl.recv_pending = 1;
+      }
+    }
     // the dry run overlaps the previous launch's tail; the real context follows
     if (a.warm) {
       epi_ctx_dry(ectx, a.n_pad, et);
-      epilogue_warmup<EPI>(a, ectx, ctl.red, stage, rms, c, G, et);
+      epilogue_warmup<EPI, CSK>(a, ectx, ctl.red, stage, rms, c, G, et, recv, csk_reducer);
     }
     pdl_wait();
+    if constexpr (CSK) cluster_wait_acquire();
     if (threadIdx.x == 64) trace_at(trace, 13);
     if (a.rms) rms_prologue(a, rms, et);
     epi_prologue<EPI>(a, ectx, et);
@@ -291,13 +317,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
       named_bar_sync(1, 128);
       if (!ok) break;
       tc_fence_after();
-      epilogue_segment<EPI>(a, ectx, layout, acols, tmem_base, buf, seg, c, G, rt, k0, k1, stage, rms,
-                       ctl.red, &ctl.reduce_flag, ctl.acc_empty, et, ew, lane,
-                       threadIdx.x == 64 ? trace : nullptr);
+      epilogue_segment<EPI, CSK>(a, ectx, layout, acols, tmem_base, buf, seg, c, G, rt, k0, k1, stage, rms,
+                       ctl.red, &ctl.reduce_flag, ctl.acc_empty, et, ew, lane, recv, &ctl.recv,
+                       abort_flag, threadIdx.x == 64 ? trace : nullptr);
       t = seg_end;
     }
   }
 
+  // a CTA that expects pushed partials leaves only after they landed (they do at
+  // once unless a peer stopped early; the wait is bounded)
+  if constexpr (CSK) {
+    if (threadIdx.x == 64 && ctl.recv_pending) mbar_wait_drain(&ctl.recv, 0);
+  }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -324,32 +355,74 @@ static int gemm_budget_bytes(int n_pad) {
   return n_pad <= 32 ? 200 * 1024 : 200 * 1024;
 }
 
-int gemm_pick_stages(int n_pad, int planes) {
+// Shared memory that receives the partials pushed by cluster peers: csk - 1
+// slots of one 128 x 16 fp32 accumulator each.
+static int csk_recv_bytes(int csk) { return csk > 1 ? (csk - 1) * kTileM * 16 * 4 + 16 : 0; }
+
+int gemm_pick_stages(int n_pad, int planes, int csk) {
   const int stage = kABytes + n_pad * 128 * planes;
   const int budget = gemm_budget_bytes(n_pad);
-  const int fixed = kTileM * kStagePitch * 4 + kMaxRows * 4 + static_cast<int>(sizeof(EpiCtx)) + 1024;
+  const int fixed = kTileM * kStagePitch * 4 + kMaxRows * 4 + static_cast<int>(sizeof(EpiCtx)) + 1024 +
+                    csk_recv_bytes(csk);
   int s = (budget - fixed) / stage;
   if (s > kMaxStages) s = kMaxStages;
   if (s < 2) s = 2;
   return s;
 }
 
-size_t gemm_smem_bytes(int n_pad, int stages, int planes) {
+size_t gemm_smem_bytes(int n_pad, int stages, int planes, int csk) {
   return static_cast<size_t>(stages) * (kABytes + n_pad * 128 * planes) + kTileM * kStagePitch * 4 +
-         kMaxRows * 4 + sizeof(EpiCtx) + 1024;
+         kMaxRows * 4 + sizeof(EpiCtx) + 1024 + csk_recv_bytes(csk);
 }
 
 cudaError_t gemm_set_max_smem() {
   // 227 KB per block minus the kernel's static shared memory
-  const void* fns[4] = {reinterpret_cast<const void*>(gemm_stream_kernel<EPI_F32>),
-                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_RESIDUAL>),
-                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_SWIGLU>),
-                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_QKV>)};
+  const void* fns[8] = {reinterpret_cast<const void*>(gemm_stream_kernel<EPI_F32, false>),
+                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_RESIDUAL, false>),
+                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_SWIGLU, false>),
+                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_QKV, false>),
+                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_F32, true>),
+                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_RESIDUAL, true>),
+                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_SWIGLU, true>),
+                        reinterpret_cast<const void*>(gemm_stream_kernel<EPI_QKV, true>)};
   for (const void* f : fns) {
     cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, 220 * 1024);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
+}
+
+template <bool CSK>
+static const void* gemm_kernel_for(int epi) {
+  switch (epi) {
+    case EPI_F32: return reinterpret_cast<const void*>(gemm_stream_kernel<EPI_F32, CSK>);
+    case EPI_RESIDUAL: return reinterpret_cast<const void*>(gemm_stream_kernel<EPI_RESIDUAL, CSK>);
+    case EPI_SWIGLU: return reinterpret_cast<const void*>(gemm_stream_kernel<EPI_SWIGLU, CSK>);
+    case EPI_QKV: return reinterpret_cast<const void*>(gemm_stream_kernel<EPI_QKV, CSK>);
+    default: return nullptr;
+  }
+}
+
+int gemm_max_active_clusters(int epi, int csk, size_t smem) {
+  const void* fn = gemm_kernel_for<true>(epi);
+  if (fn == nullptr || csk < 2 || csk > 8) return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(csk);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = csk;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return 0;
+  }
+  return n;
 }
 
 cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s, bool pdl) {
@@ -358,16 +431,37 @@ cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  int n_attr = 0;
+  if (pdl) {
+    attr[n_attr].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n_attr].val.programmaticStreamSerializationAllowed = 1;
+    ++n_attr;
+  }
+  if (a.csk > 1) {
+    if (a.csk > 8 || grid % a.csk != 0 || a.n_pad != 16) return cudaErrorInvalidValue;
+    attr[n_attr].id = cudaLaunchAttributeClusterDimension;
+    attr[n_attr].val.clusterDim.x = a.csk;
+    attr[n_attr].val.clusterDim.y = 1;
+    attr[n_attr].val.clusterDim.z = 1;
+    ++n_attr;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = n_attr;
+  if (a.csk > 1) {
+    switch (a.epi) {
+      case EPI_F32: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_F32, true>, a);
+      case EPI_RESIDUAL: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_RESIDUAL, true>, a);
+      case EPI_SWIGLU: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_SWIGLU, true>, a);
+      case EPI_QKV: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_QKV, true>, a);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   switch (a.epi) {
-    case EPI_F32: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_F32>, a);
-    case EPI_RESIDUAL: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_RESIDUAL>, a);
-    case EPI_SWIGLU: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_SWIGLU>, a);
-    case EPI_QKV: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_QKV>, a);
+    case EPI_F32: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_F32, false>, a);
+    case EPI_RESIDUAL: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_RESIDUAL, false>, a);
+    case EPI_SWIGLU: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_SWIGLU, false>, a);
+    case EPI_QKV: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_QKV, false>, a);
     default: return cudaErrorInvalidValue;
   }
 }

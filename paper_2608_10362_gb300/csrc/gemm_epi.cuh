@@ -165,7 +165,7 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, const EpiC
 #pragma unroll
     for (int j = 0; j < 16; ++j)
       hn[j] = (r0 + j < rows_total) ? h[static_cast<size_t>(r0 + j) * h_ld + f] : 0.f;
-    trace_after(ts, 8, hn[15] + gain);
+    trace_after(ts, 8, hn[0] + gain);
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
       hn[j] += v[j];
@@ -186,6 +186,7 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, const EpiC
         }
       }
     }
+    trace_at(ts, 12);
     // per-row sums over the warp's 32 features, valid rows only (a decode pass
     // has 1 to a few rows of the 16)
 #pragma unroll
@@ -195,6 +196,7 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, const EpiC
         for (int o = 16; o > 0; o >>= 1) sq[j] += __shfl_xor_sync(0xffffffffu, sq[j], o);
       }
     }
+    trace_after(ts, 14, sq[0]);
     if (lane == 0) {
 #pragma unroll
       for (int j = 0; j < 16; ++j) red[ew][j] = sq[j];
@@ -406,20 +408,58 @@ __device__ __forceinline__ void epi_ctx_dry(EpiCtx* ctx, int n_pad, int et) {
   named_bar_sync(1, 128);
 }
 
+// Cluster exchange, first contributor: its own accumulator plus the n_recv
+// pushed partials in contributor order, then the epilogue (dry: nothing stored).
+template <int EPI>
+static __device__ __noinline__ void csk_reduce(const GemmArgs& a, const EpiCtx* ctx,
+                                               float (*red)[16], float* stage, const float* rms,
+                                               int rt, int et, const float* own, const float* recv,
+                                               int n_recv, unsigned long long* ts, bool dry) {
+  float sum[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) sum[j] = 0.f + own[j];
+  for (int k = 0; k < n_recv; ++k) {
+    const float4* src = reinterpret_cast<const float4*>(recv + (static_cast<size_t>(k) * kTileM + et) * 16);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4 x = src[q];
+      sum[4 * q] += x.x;
+      sum[4 * q + 1] += x.y;
+      sum[4 * q + 2] += x.z;
+      sum[4 * q + 3] += x.w;
+    }
+  }
+  trace_after(ts, 6, sum[15]);
+  apply_epilogue<EPI>(a, ctx, red, stage, rms, rt, 0, et, sum, ts, dry);
+}
+
 // Dry run of the tail - the partial reduction and the epilogue of this CTA's
 // first row tile, with every global store off - by the 128 epilogue threads
 // before the launch waits for its predecessor (griddepcontrol.wait): it only
-// reads scratch and weights, with the synthetic context of epi_ctx_dry.  The tail runs once per launch; without this its
-// instructions are fetched cold, one miss after another, on the critical path.
-template <int EPI>
+// reads scratch and weights, with the synthetic context of epi_ctx_dry.  The
+// tail runs once per launch; without this its instructions are fetched cold,
+// one miss after another, on the critical path.  With the cluster exchange, a
+// CTA that sums pushed partials warms that path instead (on whatever its
+// receive slots hold; nothing is stored).
+template <int EPI, bool CSK>
 __device__ __forceinline__ void epilogue_warmup(const GemmArgs& a, const EpiCtx* ctx,
                                                 float (*red)[16], float* stage, const float* rms,
-                                                int c, int G, int et) {
+                                                int c, int G, int et, const float* recv,
+                                                bool csk_reducer) {
   const int KT = a.k_tiles, T = a.row_tiles * KT;
+  float v[16];
+  if constexpr (CSK) {
+    if (csk_reducer) {
+      const int rt = (sk_begin(c + 1, T, G) - 1) / KT;
+#pragma unroll
+      for (int j = 0; j < 16; ++j) v[j] = 0.f;
+      csk_reduce<EPI>(a, ctx, red, stage, rms, rt, et, v, recv, a.csk - 1, nullptr, true);
+      return;
+    }
+  }
   const int rt = sk_begin(c, T, G) / KT;
   const int c_first = sk_cta_of(rt * KT, T, G);
   const int c_last = sk_cta_of((rt + 1) * KT - 1, T, G);
-  float v[16];
   reduce_partials(a, rt, c_first, c_last, 0, et, T, G, v);
   apply_epilogue<EPI>(a, ctx, red, stage, rms, rt, 0, et, v, nullptr, true);
 }
@@ -429,18 +469,31 @@ __device__ __forceinline__ void epilogue_warmup(const GemmArgs& a, const EpiCtx*
 // G the op's grid; T = row_tiles * k_tiles.  The caller has waited for the
 // accumulator; this routine reads it (wide layout: adds the hi and lo halves),
 // releases it via acc_empty, and writes the epilogue or a partial.
-template <int EPI>
+//
+// Cluster exchange (CSK: a kernel launched in clusters, a.csk > 1, n_pad == 16;
+// kernels without it carry none of this code): when every contributor of row tile
+// rt sits in this CTA's cluster, the contributors after the first push their
+// accumulator into slot (c - c_first - 1) of the first contributor's `recv`
+// (st.async, completing bytes on its `recv_bar`) and are done; the first
+// contributor - for which rt is the last row tile of its range, so `recv` is
+// used once per launch - waits for the bytes and adds the slots to its own
+// accumulator in contributor order, the order of the global-memory path.
+template <int EPI, bool CSK>
 __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, const EpiCtx* ctx, int layout,
                                                  int acols,
                                                  uint32_t tmem_base, int buf, int seg, int c,
                                                  int G, int rt, int k0, int k1, float* stage,
                                                  const float* rms, float (*red)[16],
                                                  int* reduce_flag, uint64_t* acc_empty, int et,
-                                                 int ew, int lane,
+                                                 int ew, int lane, float* recv, uint64_t* recv_bar,
+                                                 volatile int* abort_flag,
                                                  unsigned long long* ts = nullptr) {
   const int KT = a.k_tiles;
   const int T = a.row_tiles * KT;
   const bool full = (k0 == 0 && k1 == KT);
+  const int c_first = sk_cta_of(rt * KT, T, G);
+  const int c_last = sk_cta_of((rt + 1) * KT - 1, T, G);
+  const bool dsm = CSK && !full && c_first / a.csk == c_last / a.csk;
   const uint32_t tbase = tmem_base + (static_cast<uint32_t>(ew * 32) << 16) +
                          static_cast<uint32_t>(buf * acols);
   float v[16];
@@ -457,6 +510,17 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, const EpiCtx
     for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
       load_chunk(chunk);
       apply_epilogue<EPI>(a, ctx, red, stage, rms, rt, chunk, et, v, nullptr, false);
+    }
+  } else if (CSK && dsm) {
+    load_chunk(0);   // n_pad == 16: the whole accumulator
+    if (c != c_first) {
+      const uint32_t rank = static_cast<uint32_t>(c_first % a.csk);
+      const uint32_t slot = smem_addr(recv + (static_cast<size_t>(c - c_first - 1) * kTileM + et) * 16);
+      const uint32_t raddr = mapa_shared(slot, rank);
+      const uint32_t rbar = mapa_shared(smem_addr(recv_bar), rank);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        st_async_f4(raddr + 16 * q, v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3], rbar);
     }
   } else {
     // partial sums, feature-major: thread et owns n_pad consecutive floats
@@ -475,13 +539,26 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, const EpiCtx
   if (lane == 0) mbar_arrive(&acc_empty[buf]);
   if (full) return;
   trace_at(ts, 4);
+  if (CSK && dsm) {
+    if (c != c_first) return;
+    // one thread waits; the epilogue threads follow (or stop) together, then each
+    // acquires the peers' bytes itself (the phase is complete: no wait)
+    if (et == 0) *reduce_flag = mbar_wait_cluster_bounded(recv_bar, 0, abort_flag, a.status) ? 1 : 0;
+    named_bar_sync(1, 128);
+    const int ok = *reduce_flag;
+    named_bar_sync(1, 128);
+    if (!ok) return;
+    mbar_wait_cluster_bounded(recv_bar, 0, nullptr, nullptr);
+    trace_at(ts, 5);
+    csk_reduce<EPI>(a, ctx, red, stage, rms, rt, et, v, recv, c_last - c_first, ts, false);
+    trace_at(ts, 7);
+    return;
+  }
   // The barrier orders this CTA's partial stores before thread 0's arrival, whose
   // release (acq_rel, GPU scope) publishes them; the last contributor's acquire
   // and the second barrier order every other contributor's partials before its
   // loads (which bypass L1).
   named_bar_sync(1, 128);
-  const int c_first = sk_cta_of(rt * KT, T, G);
-  const int c_last = sk_cta_of((rt + 1) * KT - 1, T, G);
   if (et == 0) {
     const int old = atom_add_acq_rel_gpu(&a.counters[rt], 1);
     *reduce_flag = (old == c_last - c_first) ? 1 : 0;

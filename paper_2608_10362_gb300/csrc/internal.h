@@ -92,6 +92,10 @@ struct GemmArgs {
   // split-K scratch
   float* partials;          // [2 * grid][n_pad * 128]
   int* counters;            // [row_tiles], zero on entry, left zero
+  int csk;                  // > 1: launched in clusters of csk CTAs (n_pad == 16 only); a
+                            // row tile whose contributors share a cluster is summed by
+                            // its first contributor from partials the others push into
+                            // its shared memory (no global partials, no counter)
   // epilogue
   int epi;
   float* out;               // EPI_F32
@@ -184,8 +188,11 @@ struct AcceptArgs {
 // launchers (each returns the launch's cudaError_t)
 cudaError_t launch_embed(const EmbedArgs& a, int rows, cudaStream_t s, bool pdl);
 cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s, bool pdl);
-size_t gemm_smem_bytes(int n_pad, int stages, int planes = 1);
-int gemm_pick_stages(int n_pad, int planes = 1);
+size_t gemm_smem_bytes(int n_pad, int stages, int planes = 1, int csk = 0);
+int gemm_pick_stages(int n_pad, int planes = 1, int csk = 0);
+// Thread-block clusters of `csk` CTAs of the GEMM kernel with epilogue `epi` and
+// `smem` bytes of dynamic shared memory that can be resident at once (0: none).
+int gemm_max_active_clusters(int epi, int csk, size_t smem);
 cudaError_t gemm_set_max_smem();
 cudaError_t launch_attention(const AttnArgs& a, int n_groups, cudaStream_t s, bool pdl);
 size_t attention_smem_bytes(const AttnArgs& a);

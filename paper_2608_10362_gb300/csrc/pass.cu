@@ -375,8 +375,9 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
             tc_fence_after();
             unsigned long long* ts = tid == 0 ? trace_slot(p, n, 0) : nullptr;
 #define MEMSPEC_PASS_EPI(E)                                                                  \
-  epilogue_segment<E>(a, ectx, layout, acols, tmem_base, buf, lseg, c, Gn, rt, k0, k1, stage, rms, \
-                      ctl.red, &ctl.reduce_flag, ctl.acc_empty, et, ew, lane, ts)
+  epilogue_segment<E, false>(a, ectx, layout, acols, tmem_base, buf, lseg, c, Gn, rt, k0, k1, stage, rms, \
+                      ctl.red, &ctl.reduce_flag, ctl.acc_empty, et, ew, lane, nullptr, nullptr, \
+                      nullptr, ts)
             switch (a.epi) {
               case EPI_F32: MEMSPEC_PASS_EPI(EPI_F32); break;
               case EPI_RESIDUAL: MEMSPEC_PASS_EPI(EPI_RESIDUAL); break;

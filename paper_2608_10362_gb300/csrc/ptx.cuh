@@ -253,4 +253,64 @@ __device__ __forceinline__ float ld_cg_f(const float* p) {
   return v;
 }
 
+// ---------------------------------------------------------------- clusters
+// Rank of this CTA in its thread-block cluster.
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Shared-memory address of the same variable in cluster CTA `rank`.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+// Cluster barrier, split: every thread arrives (release: this CTA's mbarrier
+// initialisation becomes visible cluster-wide); a thread that will touch another
+// CTA's shared memory waits (acquire) first.  Both CTAs are co-scheduled.
+__device__ __forceinline__ void cluster_arrive_release() {
+  asm volatile("barrier.cluster.arrive.release;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+  asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
+}
+// 16-byte store into a cluster peer's shared memory that completes 16 bytes of
+// transaction count on the peer's mbarrier `rbar` (both shared::cluster addresses).
+__device__ __forceinline__ void st_async_f4(uint32_t raddr, float x, float y, float z, float w,
+                                            uint32_t rbar) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];"
+      ::"r"(raddr), "f"(x), "f"(y), "f"(z), "f"(w), "r"(rbar)
+      : "memory");
+}
+// Wait for phase `parity` of a local mbarrier completed by cluster peers
+// (acquire at cluster scope), bounded like mbar_wait_bounded.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_cluster_bounded(uint64_t* bar, uint32_t parity,
+                                                          volatile int* abort_flag,
+                                                          uint32_t* status) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try_wait_cluster(bar, parity)) {
+    if (abort_flag != nullptr && *abort_flag) return false;
+    if (clock64() - t0 > kWaitBudgetCycles) {
+      if (abort_flag != nullptr) *abort_flag = 1;
+      if (status != nullptr) atomicOr(status, 0x1u);
+      return false;
+    }
+  }
+  return true;
+}
+
 }  // namespace memspec
