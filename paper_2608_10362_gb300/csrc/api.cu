@@ -550,9 +550,11 @@ int env_int(const char* name, int dflt) {
 // MEMSPEC_SK_MAXC overrides the contributor limit (measurement).
 int gemm_grid(int row_tiles, int k_tiles) {
   static const int max_contrib = std::max(1, env_int("MEMSPEC_SK_MAXC", 4));
+  static const int max_grid = env_int("MEMSPEC_GEMM_MAXG", 0);   // 0: the SM count (measurement)
   const int T = row_tiles * k_tiles;
   const int min_tiles = std::max(1, (k_tiles + max_contrib - 1) / max_contrib);
-  return std::max(1, std::min({T, sm_count(), T / min_tiles}));
+  const int sms = max_grid > 0 ? std::min(max_grid, sm_count()) : sm_count();
+  return std::max(1, std::min({T, sms, T / min_tiles}));
 }
 
 // Whether a GEMM launch dry-runs its tail before griddepcontrol.wait: worth it
@@ -653,8 +655,24 @@ void emit_gemm(memspec_ctx* c, GemmArgs& a, std::vector<PassOp>& ops) {
   ops.push_back(op);
 }
 
+// Launches as separate kernels: the op after the embedding kernel (which writes
+// the row plan) waits for every earlier kernel (no programmatic dependent
+// launch), so every later op starts after the plan - and the KV cache of earlier
+// positions - is final and may read them before griddepcontrol.wait (ctx_early).
+// MEMSPEC_CTX_EARLY=0 turns this off (measurement).
+void mark_ctx_early(std::vector<PassOp>& ops, size_t first) {
+  static const int enabled = env_int("MEMSPEC_CTX_EARLY", 1);
+  if (!enabled || ops.size() < first + 2 || ops[first].type != OP_EMBED) return;
+  ops[first + 1].full_dep = 1;
+  for (size_t i = first + 2; i < ops.size(); ++i) {
+    if (ops[i].type == OP_GEMM) ops[i].u.g.ctx_early = 1;
+    if (ops[i].type == OP_ATTN) ops[i].u.at.ctx_early = 1;
+  }
+}
+
 memspec_status emit_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f,
                             std::vector<PassOp>& ops) {
+  const size_t first_op = ops.size();
   const memspec_model_cfg& cf = m.cfg;
   const int d = cf.d_model, qd = model_q(cf), kvd = model_kv(cf), F = cf.d_ffn;
   const int rows = f.n_groups * f.R;
@@ -876,6 +894,7 @@ memspec_status emit_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f,
     a.plan = c->plan;
     emit_gemm(c, a, ops);
   }
+  if (!c->pass_kernel) mark_ctx_early(ops, first_op);
   return MEMSPEC_OK;
 }
 
@@ -886,8 +905,8 @@ memspec_status run_ops_separately(memspec_ctx* c, const std::vector<PassOp>& ops
     cudaError_t e = cudaSuccess;
     switch (op.type) {
       case OP_EMBED: e = launch_embed(op.u.e, op.n_units, c->main, c->pdl); break;
-      case OP_GEMM: e = launch_gemm(op.u.g, op.grid, op.smem, c->main, c->pdl); break;
-      case OP_ATTN: e = launch_attention(op.u.at, op.grid, c->main, c->pdl); break;
+      case OP_GEMM: e = launch_gemm(op.u.g, op.grid, op.smem, c->main, c->pdl && !op.full_dep); break;
+      case OP_ATTN: e = launch_attention(op.u.at, op.grid, c->main, c->pdl && !op.full_dep); break;
       case OP_SAMPLE: e = launch_sample(op.u.s, c->main, c->pdl); break;
       case OP_ACCEPT: e = launch_accept(op.u.acc, c->main, false); break;
       default: return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown op");

@@ -38,12 +38,15 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
   auto sync = [] { __syncthreads(); };
   // dry run while the previous kernel finishes: warms this code, writes no
   // global memory (see attention_cta)
-  attention_cta<HD>(a, 0, 0, 0, 0, smem_raw, threadIdx.x, sync, nullptr, true);
+  attention_cta<HD>(a, 0, 0, 0, 0, smem_raw, threadIdx.x, sync, [] {}, false, nullptr, true);
   __syncthreads();
-  pdl_wait();
-  trace_at(trace, 13);
+  auto wait = [&] {
+    pdl_wait();
+    trace_at(trace, 13);
+  };
   const int kvh = blockIdx.y / a.row_blocks, rb = blockIdx.y - kvh * a.row_blocks;
-  attention_cta<HD>(a, blockIdx.z, kvh, rb, blockIdx.x, smem_raw, threadIdx.x, sync, trace);
+  attention_cta<HD>(a, blockIdx.z, kvh, rb, blockIdx.x, smem_raw, threadIdx.x, sync, wait,
+                    a.ctx_early != 0, trace);
   trace_at(trace, 1);
 }
 

@@ -58,11 +58,12 @@ __device__ __forceinline__ uint32_t swz(int row, int ch) {
 
 template <int HD>
 __host__ __device__ constexpr size_t attention_smem_bytes_hd() {
-  // kStages x (K tile + V tile); the merge buffers reuse it; the last 16 bytes hold a flag
+  // kStages x (K tile + V tile); the merge buffers (o, (m, l), weights, (M, L))
+  // reuse it; the last 16 bytes hold a flag
   return static_cast<size_t>(kStages) * 2 * kKeyTile * HD * 2 >
-                 static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + 16
+                 static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + kMaxQ * 6 * 4 + 16
              ? static_cast<size_t>(kStages) * 2 * kKeyTile * HD * 2
-             : static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + 16;
+             : static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + kMaxQ * 6 * 4 + 16;
 }
 
 // One CTA of split-KV attention for unit (g, kvh, rb, split), run by 128 threads
@@ -73,13 +74,20 @@ __host__ __device__ constexpr size_t attention_smem_bytes_hd() {
 // writes no global memory (no output, no partials, no counters): launched
 // before griddepcontrol.wait, it brings this code into the instruction cache
 // while the previous kernel finishes.  Callers pass g = kvh = rb = split = 0.
-template <int HD, class Sync>
+// wait: called once by every thread before the first read of the previous
+// kernel's output (the kernel passes griddepcontrol.wait).  early: the row plan
+// and the cached keys / values before the group's first new position are final
+// before wait() (see AttnArgs::ctx_early): the plan is read, and the first tiles
+// that hold only such keys are requested, before it.
+template <int HD, class Sync, class Wait>
 __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh, int rb, int split,
-                                              uint8_t* smem_raw, int tid, Sync sync,
-                                              unsigned long long* ts = nullptr, bool dry = false) {
+                                              uint8_t* smem_raw, int tid, Sync sync, Wait wait,
+                                              bool early, unsigned long long* ts = nullptr,
+                                              bool dry = false) {
   constexpr int kChunks = HD / 8;                        // 16-byte chunks per row
   constexpr int kTileBytes = kKeyTile * HD * 2;          // one K (or V) tile
   constexpr int kNT = HD / 8;                            // n8 tiles of the output
+  if (!early) wait();
   const RowPlan* plan = a.plan;
   // every plan field in one round trip (g < kMaxGroups: in bounds before the check)
   int n_groups = 1, R = a.rows_per_block, req = 0, valid = a.rows_per_block, pos0 = 0;
@@ -98,7 +106,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   const int gs = a.H / a.Hkv;
   const int nq = gs * nr;
   const int kmax = pos0 + r_hi - 1;
-  if (pos0 < 0 || kmax >= a.max_seq || nq > kMaxQ) {   // reported, never read
+  if (pos0 < 0 || kmax >= a.max_seq || nq > kMaxQ || a.n_splits > 16) {   // reported, never read
     if (threadIdx.x == 0 && split == 0) atomicOr(a.status, 0x4u);
     return;
   }
@@ -136,8 +144,17 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     }
   };
 
-  // prologue: start the first kStages-1 tiles, then stage Q (fp32 -> bf16, scaled)
-  for (int s = 0; s < kStages - 1; ++s) {
+  // prologue: start the first kStages-1 tiles (early: those below pos0 before the
+  // wait), then stage Q (fp32 -> bf16, scaled)
+  int s_pre = 0;
+  if (early) {
+    for (; s_pre < kStages - 1 && s_pre < n_tiles && k0 + (s_pre + 1) * kKeyTile <= pos0; ++s_pre) {
+      load_tile(s_pre);
+      cp_async_commit();
+    }
+    wait();
+  }
+  for (int s = s_pre; s < kStages - 1; ++s) {
     if (s < n_tiles) load_tile(s);
     cp_async_commit();
   }
@@ -290,18 +307,23 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   trace_at(ts, 9);
   if (ts != nullptr) trace_after(ts, 12, o[0][0] + o[kNT - 1][3]);   // last MMAs retired
 
-  // merge the key groups of each m-tile (shared memory reuses the K/V stages)
+  // merge the key groups of each m-tile (shared memory reuses the K/V stages):
+  // the query vectors' rows of o go to shared memory (padding rows are not
+  // written or read), one thread per vector computes M = max_w m_w, the group
+  // weights f_w = 2^(m_w - M) and L = sum_w f_w l_w, then four features per
+  // thread: o = sum_w f_w o_w (groups in ascending order)
   float* mo = reinterpret_cast<float*>(kv);                 // [4 warps][16][HD]
   float* ml = mo + 4 * 16 * HD;                             // [4 warps][16][2]
+  float* mf = ml + 4 * 16 * 2;                              // [kMaxQ][4] weights
+  float* mml = mf + kMaxQ * 4;                              // [kMaxQ][2] M, L
   if (active) {
     const int r0 = lane >> 2, cc = (lane & 3) << 1;
+    const bool lo_ok = mt * 16 + r0 < nq, hi_ok = mt * 16 + r0 + 8 < nq;
 #pragma unroll
     for (int i = 0; i < kNT; ++i) {
       float* dst = mo + (warp * 16) * HD + i * 8 + cc;
-      dst[r0 * HD] = o[i][0];
-      dst[r0 * HD + 1] = o[i][1];
-      dst[(r0 + 8) * HD] = o[i][2];
-      dst[(r0 + 8) * HD + 1] = o[i][3];
+      if (lo_ok) *reinterpret_cast<float2*>(dst + r0 * HD) = make_float2(o[i][0], o[i][1]);
+      if (hi_ok) *reinterpret_cast<float2*>(dst + (r0 + 8) * HD) = make_float2(o[i][2], o[i][3]);
     }
     if ((lane & 3) == 0) {
       ml[(warp * 16 + r0) * 2] = m_run[0];
@@ -311,28 +333,41 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     }
   }
   sync();
-  trace_at(ts, 11);
-  const int unit = (g * a.Hkv + kvh) * a.row_blocks + rb;
-  const size_t pbase = (static_cast<size_t>(unit) * a.n_splits + split) * a.qmax;
-  for (int idx = tid; idx < nq * HD; idx += kAttThreads) {
-    const int v = idx / HD, d = idx - v * HD;
+  for (int v = tid; v < nq; v += kAttThreads) {
     const int m_t = v >> 4, r = v & 15;
     float M = -INFINITY;
     for (int w = 0; w < kg; ++w) M = fmaxf(M, ml[((m_t * kg + w) * 16 + r) * 2]);
-    float L = 0.f, O = 0.f;
+    float L = 0.f;
     for (int w = 0; w < kg; ++w) {
       const int ww = m_t * kg + w;
       const float mw = ml[(ww * 16 + r) * 2];
       const float f = mw == -INFINITY ? 0.f : exp2f(mw - M);
+      mf[v * 4 + w] = f;
       L += f * ml[(ww * 16 + r) * 2 + 1];
-      O += f * mo[(ww * 16 + r) * HD + d];
+    }
+    mml[v * 2] = M;
+    mml[v * 2 + 1] = L;
+  }
+  sync();
+  trace_at(ts, 11);
+  const int unit = (g * a.Hkv + kvh) * a.row_blocks + rb;
+  const size_t pbase = (static_cast<size_t>(unit) * a.n_splits + split) * a.qmax;
+  constexpr int kMV4 = HD / 4;
+  for (int idx = tid; idx < nq * kMV4; idx += kAttThreads) {
+    const int v = idx / kMV4, d = (idx - v * kMV4) * 4;
+    const int m_t = v >> 4, r = v & 15;
+    float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int w = 0; w < kg; ++w) {
+      const float f = mf[v * 4 + w];
+      const float4 x = *reinterpret_cast<const float4*>(mo + ((m_t * kg + w) * 16 + r) * HD + d);
+      O.x += f * x.x;
+      O.y += f * x.y;
+      O.z += f * x.z;
+      O.w += f * x.w;
     }
     if (dry) continue;
-    a.part_o[(pbase + v) * HD + d] = O;
-    if (d == 0) {
-      a.part_ml[(pbase + v) * 2 + 0] = M;
-      a.part_ml[(pbase + v) * 2 + 1] = L;
-    }
+    *reinterpret_cast<float4*>(a.part_o + (pbase + v) * HD + d) = O;
+    if (d == 0) *reinterpret_cast<float2*>(a.part_ml + (pbase + v) * 2) = *reinterpret_cast<const float2*>(mml + v * 2);
   }
   trace_at(ts, 4);
   // same arrival protocol as the GEMM split-K: the barrier orders this CTA's
@@ -349,78 +384,50 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   const int qmax = a.qmax;
   const float* part_ml = a.part_ml;
   const float* part_o = a.part_o;
-  // (m_s, l_s) of every split and query vector, fetched together into shared
-  // memory; then the split weights 2^(m_s - M) (in place of m_s) and 1/L
-  float* msm = reinterpret_cast<float*>(kv);               // [n_active][nq]
-  float* lsm = msm + n_active * nq;                         // [n_active][nq]
-  float* linv = lsm + n_active * nq;                        // [nq]
-  const int n_ml = n_active * nq;
-  for (int i0 = tid; i0 < n_ml; i0 += 4 * kAttThreads) {
-    float2 t[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int i = i0 + q * kAttThreads;
-      if (i < n_ml) {
-        const int sp = i / nq, v = i - sp * nq;
-        t[q] = ld_cg_f2(part_ml + (ubase + static_cast<size_t>(sp) * qmax + v) * 2);
-      }
-    }
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int i = i0 + q * kAttThreads;
-      if (i < n_ml) {
-        msm[i] = t[q].x;
-        lsm[i] = t[q].y;
-      }
-    }
-  }
-  sync();
-  for (int v = tid; v < nq; v += kAttThreads) {
-    float M = -INFINITY;
-    for (int sp = 0; sp < n_active; ++sp) M = fmaxf(M, msm[sp * nq + v]);
-    float L = 0.f;
-    for (int sp = 0; sp < n_active; ++sp) {
-      const float ms = msm[sp * nq + v];
-      const float w = ms == -INFINITY ? 0.f : exp2f(ms - M);
-      msm[sp * nq + v] = w;
-      L += w * lsm[sp * nq + v];
-    }
-    linv[v] = 1.f / L;
-  }
-  sync();
-  trace_at(ts, 6);
-  // weighted sum of the split outputs, four features per thread, sixteen splits
-  // fetched at once (one round trip for up to 16 splits) and added in ascending
-  // split order
+  // One round trip: each thread fetches, for its query vector v and its four
+  // features, every split's (m_s, l_s) (the 32 threads of a vector read the same
+  // words: one transaction) together with its o_s (n_active <= 16: the geometry
+  // caps the splits), then M = max m_s, weights 2^(m_s - M), L and the weighted
+  // sum, all in ascending split order.
   constexpr int kV4 = HD / 4;
   bf16* out = a.out;
   bf16* out_lo = a.out_lo;
   const int H = a.H;
   for (int idx = tid; idx < nq * kV4; idx += kAttThreads) {
     const int v = idx / kV4, d = (idx - v * kV4) * 4;
-    float O[4] = {0.f, 0.f, 0.f, 0.f};
-    for (int s0 = 0; s0 < n_active; s0 += 16) {
-      float4 ov[16];
+    float2 mlv[16];
+    float4 ov[16];
 #pragma unroll
-      for (int q = 0; q < 16; ++q)
-        if (s0 + q < n_active)
-          ov[q] = ld_cg_f4(part_o + (ubase + static_cast<size_t>(s0 + q) * qmax + v) * HD + d);
-#pragma unroll
-      for (int q = 0; q < 16; ++q) {
-        if (s0 + q < n_active) {
-          const float w = msm[(s0 + q) * nq + v];
-          O[0] += w * ov[q].x;
-          O[1] += w * ov[q].y;
-          O[2] += w * ov[q].z;
-          O[3] += w * ov[q].w;
-        }
+    for (int q = 0; q < 16; ++q) {
+      if (q < n_active) {
+        const size_t pv = ubase + static_cast<size_t>(q) * qmax + v;
+        mlv[q] = ld_cg_f2(part_ml + pv * 2);
+        ov[q] = ld_cg_f4(part_o + pv * HD + d);
       }
     }
+    if (idx == tid) trace_after(ts, 6, mlv[0].x + ov[0].x);
+    float M = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < 16; ++q)
+      if (q < n_active) M = fmaxf(M, mlv[q].x);
+    float L = 0.f;
+    float O[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int q = 0; q < 16; ++q) {
+      if (q < n_active) {
+        const float w = mlv[q].x == -INFINITY ? 0.f : exp2f(mlv[q].x - M);
+        L += w * mlv[q].y;
+        O[0] += w * ov[q].x;
+        O[1] += w * ov[q].y;
+        O[2] += w * ov[q].z;
+        O[3] += w * ov[q].w;
+      }
+    }
+    const float li = 1.f / L;
     const int hl = v / nr, rr = v - hl * nr;
     const int row = g * R + r_lo + rr;
     const int h = kvh * gs + hl;
     const size_t oi = (static_cast<size_t>(row) * H + h) * HD + d;
-    const float li = linv[v];
     if (dry) continue;
 #pragma unroll
     for (int e = 0; e < 4; ++e) {

@@ -290,7 +290,12 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
       }
     }
     // the dry run overlaps the previous launch's tail; the real context follows
-    if (a.warm) {
+    // (ctx_early: the row plan is final before the wait, so the real context is
+    // built there and the dry run uses it)
+    if (a.ctx_early) {
+      epi_prologue<EPI>(a, ectx, et);
+      if (a.warm) epilogue_warmup<EPI, CSK>(a, ectx, ctl.red, stage, rms, c, G, et, recv, csk_reducer);
+    } else if (a.warm) {
       epi_ctx_dry(ectx, a.n_pad, et);
       epilogue_warmup<EPI, CSK>(a, ectx, ctl.red, stage, rms, c, G, et, recv, csk_reducer);
     }
@@ -298,7 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
     if constexpr (CSK) cluster_wait_acquire();
     if (threadIdx.x == 64) trace_at(trace, 13);
     if (a.rms) rms_prologue(a, rms, et);
-    epi_prologue<EPI>(a, ectx, et);
+    if (!a.ctx_early) epi_prologue<EPI>(a, ectx, et);
     int seg = 0;
     for (int t = t_begin; t < t_end; ++seg) {
       const int rt = t / KT;

@@ -121,6 +121,10 @@ struct GemmArgs {
   uint32_t* status;
   unsigned long long* trace;  // nullptr, or this op's trace row (16 slots per CTA)
   int warm;                 // 1: dry run of the tail before griddepcontrol.wait
+  int ctx_early;            // 1: every kernel before the previous one has completed when
+                            // this one starts (an earlier launch of the pass had a full
+                            // dependency after the row-plan writer), so the row plan
+                            // may be read before griddepcontrol.wait
 };
 
 struct AttnArgs {
@@ -143,6 +147,9 @@ struct AttnArgs {
   uint32_t* status;
   unsigned long long* trace;  // nullptr, or this op's trace row (16 slots per CTA)
   int trace_ctas;             // CTAs (linear index) that record
+  int ctx_early;              // 1: as GemmArgs::ctx_early; the row plan and the cached
+                              // keys / values of positions before this pass's first
+                              // new position may be read before griddepcontrol.wait
 };
 
 struct SampleArgs {         // draft sampling of pass j

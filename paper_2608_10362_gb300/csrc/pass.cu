@@ -397,10 +397,10 @@ __global__ void __launch_bounds__(kThreads, 1) pass_kernel(const __grid_constant
           const int kr = rem / at.n_splits, split = rem - kr * at.n_splits;
           const int kvh = kr / at.row_blocks, rb = kr - kvh * at.row_blocks;
           if (at.hd == 64)
-            attn::attention_cta<64>(at, g, kvh, rb, split, attn_smem, tid, wsync,
+            attn::attention_cta<64>(at, g, kvh, rb, split, attn_smem, tid, wsync, [] {}, false,
                                     tid == 0 ? trace_slot(p, n, 0) : nullptr);
           else
-            attn::attention_cta<128>(at, g, kvh, rb, split, attn_smem, tid, wsync,
+            attn::attention_cta<128>(at, g, kvh, rb, split, attn_smem, tid, wsync, [] {}, false,
                                      tid == 0 ? trace_slot(p, n, 0) : nullptr);
           wsync();
         }

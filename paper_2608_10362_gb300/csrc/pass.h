@@ -13,7 +13,9 @@ struct alignas(64) PassOp {
   int grid;       // OP_GEMM: stream-K grid (CTAs with tiles)
   int n_units;    // OP_EMBED rows, OP_ATTN units, OP_SAMPLE groups, OP_ACCEPT rows x groups
   int smem;       // OP_GEMM as its own launch: dynamic shared memory bytes
-  int pad[12];
+  int full_dep;   // as its own launch: without programmatic dependent launch, so it
+                  // starts after every earlier kernel has completed
+  int pad[11];
   union U {
     GemmArgs g;
     AttnArgs at;
