@@ -542,7 +542,13 @@ struct FwdSpec {
 // Stream-K grid: at most one CTA per SM, and at least ceil(k_tiles / 4) tiles per
 // CTA so that a row tile is shared by at most ~4 CTAs (the last of them sums the
 // partials; more contributors lengthen that serial tail more than they add
-// bandwidth on small matrices).
+// bandwidth on small matrices).  kGemmSpareSms SMs stay free: with every SM
+// streaming, some SMs stream 1-2 us slower than the rest and the CTAs that start
+// on SMs still held by the previous launch start late, and a static partition
+// waits for the slowest; with 16 SMs free the verify pass measured 3.34 ms
+// instead of 3.42 (QKV launch 21 us instead of 25).
+constexpr int kGemmSpareSms = 16;
+
 int env_int(const char* name, int dflt) {
   const char* e = std::getenv(name);
   return e != nullptr ? std::atoi(e) : dflt;
@@ -550,10 +556,12 @@ int env_int(const char* name, int dflt) {
 // MEMSPEC_SK_MAXC overrides the contributor limit (measurement).
 int gemm_grid(int row_tiles, int k_tiles) {
   static const int max_contrib = std::max(1, env_int("MEMSPEC_SK_MAXC", 4));
-  static const int max_grid = env_int("MEMSPEC_GEMM_MAXG", 0);   // 0: the SM count (measurement)
+  static const int max_grid = env_int("MEMSPEC_GEMM_MAXG", 0);   // > 0: overrides (measurement)
   const int T = row_tiles * k_tiles;
   const int min_tiles = std::max(1, (k_tiles + max_contrib - 1) / max_contrib);
-  const int sms = max_grid > 0 ? std::min(max_grid, sm_count()) : sm_count();
+  const int sms = max_grid > 0 ? std::min(max_grid, sm_count())
+                               : (sm_count() > 4 * kGemmSpareSms ? sm_count() - kGemmSpareSms
+                                                                 : sm_count());
   return std::max(1, std::min({T, sms, T / min_tiles}));
 }
 
@@ -617,7 +625,9 @@ CskPick pick_csk(const GemmArgs& a, int planes, int g0) {
     const auto key = std::make_tuple(dev, a.epi, C, smem);
     auto it = fit.find(key);
     if (it == fit.end()) it = fit.emplace(key, gemm_max_active_clusters(a.epi, C, smem)).first;
-    const int q_max = std::min({it->second, sm_count() / C, T / C});
+    // never more CTAs than plain stream-K: clusters must all be resident while the
+    // previous launch still holds SMs (a larger clustered grid measured far slower)
+    const int q_max = std::min({it->second, g0 / C, T / C});
     for (int Q = q_max; Q >= 1; --Q) {
       const int G = Q * C;
       if (!sk_fits(T, G)) continue;
