@@ -429,14 +429,12 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     const int h = kvh * gs + hl;
     const size_t oi = (static_cast<size_t>(row) * H + h) * HD + d;
     if (dry) continue;
+    // four features: one 8-byte store per plane (oi is a multiple of 4)
+    __nv_bfloat16 hv[4], lv[4];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      if (out_lo != nullptr) {
-        split_bf16(O[e] * li, out[oi + e], out_lo[oi + e]);
-      } else {
-        out[oi + e] = __float2bfloat16_rn(O[e] * li);
-      }
-    }
+    for (int e = 0; e < 4; ++e) split_bf16(O[e] * li, hv[e], lv[e]);
+    *reinterpret_cast<uint2*>(out + oi) = *reinterpret_cast<const uint2*>(hv);
+    if (out_lo != nullptr) *reinterpret_cast<uint2*>(out_lo + oi) = *reinterpret_cast<const uint2*>(lv);
   }
   trace_at(ts, 7);
   if (tid == 0 && !dry) a.counters[unit] = 0;

@@ -177,14 +177,8 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, const EpiC
       if (r >= rows_total || dry) continue;
       const size_t o = static_cast<size_t>(r) * h_ld + f;
       h[o] = hn[j];
-      if (gain_next != nullptr) {
-        const float xv = hn[j] * gain;
-        if (xg_lo_out != nullptr) {
-          split_bf16(xv, xg_out[o], xg_lo_out[o]);
-        } else {
-          xg_out[o] = __float2bfloat16_rn(xv);
-        }
-      }
+      if (gain_next != nullptr)
+        store_split_bf16(xg_out + o, xg_lo_out != nullptr ? xg_lo_out + o : nullptr, hn[j] * gain);
     }
     trace_at(ts, 12);
     // per-row sums over the warp's 32 features, valid rows only (a decode pass
@@ -238,11 +232,7 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, const EpiC
             const float y = g / (1.0f + expf(-g)) * u;
             if (dry) continue;
             const size_t o = static_cast<size_t>(r) * act_ld + f;
-            if (act_lo != nullptr) {
-              split_bf16(y, act[o], act_lo[o]);
-            } else {
-              act[o] = __float2bfloat16_rn(y);
-            }
+            store_split_bf16(act + o, act_lo != nullptr ? act_lo + o : nullptr, y);
           }
         }
       }

@@ -211,9 +211,19 @@ cudaError_t launch_rope_table(float* cos_t, float* sin_t, int max_seq, int half,
 
 // x ~= hi + lo with hi = bf16(x), lo = bf16(x - hi): two bf16 planes carry about
 // 16 significant bits, so bf16 tensor-core products see (almost) fp32 inputs.
+// x = hi + lo in two bf16 planes.  The references must be registers or shared
+// memory: with global references the compiler re-read hi from memory (a round
+// trip per call, measured); use store_split_bf16 for global outputs.
 __device__ __forceinline__ void split_bf16(float x, bf16& hi, bf16& lo) {
-  hi = __float2bfloat16_rn(x);
-  lo = __float2bfloat16_rn(x - __bfloat162float(hi));
+  const bf16 h = __float2bfloat16_rn(x);
+  hi = h;
+  lo = __float2bfloat16_rn(x - __bfloat162float(h));
+}
+// Store x as bf16 at hi_p and (lo_p != nullptr) its low-order part at lo_p.
+__device__ __forceinline__ void store_split_bf16(bf16* hi_p, bf16* lo_p, float x) {
+  const bf16 h = __float2bfloat16_rn(x);
+  *hi_p = h;
+  if (lo_p != nullptr) *lo_p = __float2bfloat16_rn(x - __bfloat162float(h));
 }
 
 // Message returned by memspec_op_last_error() on this host thread.
