@@ -38,6 +38,14 @@ sys.path.insert(0, ROOT)
 TARGET, DRAFT = "target_7b", "draft_160m"
 PREFIX, K_DRAFT, TEMP = 2048, 4, 1.0
 WORKLOAD = "7B-shape target + 160M draft, prefix 2048, K=4, T=1.0, batch 1"
+METRIC = "accepted tokens/s (batch 1, 7B-shape, K=4); verify-step HBM GB/s vs peak"
+
+
+def workload_config(k: int, world: int) -> dict:
+    """The workload keys both arms report in `config`."""
+    return {"workload": WORKLOAD, "target": TARGET, "draft": DRAFT, "prefix": PREFIX,
+            "K": k, "temperature": TEMP, "global_batch": world,
+            "parallelism": f"replicas x{world}"}
 
 
 def measured_peaks():
@@ -212,6 +220,73 @@ def run_gpu(args, rank: int, world: int):
                 e2e_s=e2e_s, generated=generated, h2d=h2d / e2e_steps, d2h=d2h,
                 setup_s=setup_s, bits=bits, steps=steps, tokens_per_step=tokens / steps / world,
                 launches=launches_per_step(t, dft, K) * steps)
+
+
+def oracle_step_timer(K: int):
+    """The reference arm's step: the oracle's time for one draft-then-verify
+    iteration, estimated from five parts - a target layer (alternating between
+    two; 5 rows at context 2048), the target LM head, a draft layer (1 row), the
+    draft LM head, one acceptance - each weighted by how often an iteration runs
+    it.  Every part is timed once at setup; each call re-times one part (in turn),
+    so a step is a bounded sample.  The sampled layers are built once."""
+    import numpy as np
+
+    from oracle.llama import LlamaOracle
+    from oracle.speculative import accept
+    from seeded_inputs import SHAPES, gen_kv, gen_logits, gen_tensor
+
+    t, dft = SHAPES[TARGET], SHAPES[DRAFT]
+
+    def build(shape, seed, rows):
+        w = {}
+        for li in (0, 1):
+            for n in ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate", "w_up", "w_down"):
+                w[(n, li)] = gen_tensor(shape, seed, n, li)
+        w[("final_norm", -1)] = gen_tensor(shape, seed, "final_norm")
+        w[("lm_head", -1)] = gen_tensor(shape, seed, "lm_head")
+        model = LlamaOracle(shape, w)
+        cache = model.new_cache(PREFIX + rows)
+        kvs = gen_kv(3, (2, PREFIX, shape.n_kv_heads, shape.head_dim), 1.0)
+        cache.k[:2, :PREFIX] = kvs
+        cache.v[:2, :PREFIX] = kvs[::-1]
+        h = np.random.default_rng(0).standard_normal((rows, shape.d_model))
+        return model, cache, h, np.arange(PREFIX, PREFIX + rows)
+
+    tgt = build(t, 0, K + 1)
+    drf = build(dft, 1, 1)
+    zt = gen_logits(5, K + 1, t.vocab).astype(np.float64)
+    zd = gen_logits(6, K, t.vocab).astype(np.float64)
+    n = [0]
+
+    def t_layer():
+        tgt[0].layer(n[0] & 1, tgt[2], tgt[1], tgt[3])
+
+    def d_layer():
+        drf[0].layer(n[0] & 1, drf[2], drf[1], drf[3])
+
+    parts = [t_layer, lambda: tgt[0].logits(tgt[2]), d_layer, lambda: drf[0].logits(drf[2]),
+             lambda: accept(zt, zd, [1] * K, TEMP, [0.5] * K, 0.5)]
+    weight = [t.n_layers, 1, K * dft.n_layers, K, 1]   # times per iteration
+    last = [0.0] * len(parts)
+
+    def run_part(i):
+        a = time.perf_counter()
+        parts[i]()
+        last[i] = time.perf_counter() - a
+
+    for i in range(len(parts)):   # every part timed once before the first step
+        run_part(i)
+
+    def one() -> float:
+        # a step times one part afresh (in turn) and returns the iteration estimate
+        run_part(n[0] % len(parts))
+        n[0] += 1
+        return sum(w * x for w, x in zip(weight, last))
+
+    desc = (f"fp64 numpy oracle: iteration = {t.n_layers} x one target layer (5 rows, context "
+            f"{PREFIX}) + LM head + {K} x ({dft.n_layers} x one draft layer (1 row) + LM head) + "
+            f"one acceptance (V={t.vocab}); each step re-times one of these five parts in turn")
+    return one, desc
 
 
 def oracle_sample(tokens_per_iter: float, K: int, reps: int = 1):
@@ -621,25 +696,30 @@ def main():
     if args.impl == "reference":
         if rank != 0:
             return
-        steps = max(1, min(args.steps, 3))
-        vals = []
-        # The oracle cannot run enough full-depth 7B iterations within the time
-        # bound to measure its own acceptance; every iteration commits at least one
-        # token, so the reference arm counts 1 token per iteration (a lower bound,
-        # stated in the sample description).
+        # The oracle cannot run full-depth 7B iterations fast enough to measure its
+        # own acceptance; every iteration commits at least one token, so the
+        # reference arm counts 1 token per iteration (a lower bound, stated in the
+        # sample description).  W untimed steps, then K timed ones (one part each).
         tok_iter = 1.0
-        for _ in range(steps):
-            r = oracle_sample(tok_iter, args.k)
-            vals.append(r["value"])
-        v = statistics.median(vals)
-        line = {"impl": "reference", "metric": "accepted tokens/s", "value": v,
-                "unit": "tokens/s", "n_gpus": args.gpus, "steps": steps, "warmup": 0,
-                "ms_per_step": 1000.0 * r["iter_s"], "higher_is_better": True,
+        a0 = time.perf_counter()
+        one, desc = oracle_step_timer(args.k)
+        for _ in range(args.warmup):
+            one()
+        iters = [one() for _ in range(args.steps)]
+        it = statistics.median(iters)
+        v = tok_iter / it
+        wall = time.perf_counter() - a0
+        cfg = workload_config(args.k, world)
+        cfg["timing"] = "oracle on host cores"
+        line = {"impl": "reference", "metric": METRIC, "value": v,
+                "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": 1000.0 * it, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-                "config": {"workload": WORKLOAD, "timing": "oracle on host cores"},
-                "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": r["cores"],
+                "config": cfg,
+                "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": os.cpu_count(),
                                  "kind": "oracle",
-                                 "sample": r["sample"] + "; tokens/iteration counted as 1 "
+                                 "sample": desc + f"; median of {args.steps} steps, wall "
+                                           f"{wall:.1f} s; tokens/iteration counted as 1 "
                                            "(lower bound: acceptance not measured by the oracle)"},
                 "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}}
@@ -656,13 +736,11 @@ def main():
     achieved = r["verify_bytes"] / (r["verify_ms"] * 1e-3) / 1e9
     value = r["tokens"] / (r["ms"] * 1e-3)
     line = {
-        "metric": "accepted tokens/s (batch 1, 7B-shape, K=4); verify-step HBM GB/s vs peak",
+        "metric": METRIC,
         "value": value, "unit": "tokens/s", "n_gpus": world, "steps": r["steps"],
         "warmup": args.warmup, "ms_per_step": r["ms"] / r["steps"], "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "target": TARGET, "draft": DRAFT, "prefix": PREFIX,
-                   "K": args.k, "temperature": TEMP, "global_batch": world,
-                   "parallelism": f"replicas x{world}",
+        "config": {**workload_config(args.k, world),
                    "l2": "inputs larger than L2 (13.5 GB of target weights streamed per verify)",
                    "tokens_per_step": r["tokens_per_step"]},
         "roofline": {"kernel": "verify pass (one CUDA graph of the target forward)",
