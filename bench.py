@@ -128,6 +128,25 @@ def launches_per_step(t, dft, K: int) -> int:
     return K * (per_fwd(dft, True) + 1) + per_fwd(t, True) + 1
 
 
+def combine_rank_stats(stats, world: int, device):
+    """One rank's [ms, tokens, e2e_s, generated, verify_ms] -> the job's: the
+    times (ms, e2e_s, verify_ms) are the maximum over ranks, the counts (tokens,
+    generated) the sum.  torch.distributed is initialised when world > 1; the
+    collective runs on `device` ("cuda" for NCCL, "cpu" for gloo)."""
+    import torch
+    import torch.distributed as dist
+
+    if world <= 1:
+        return stats.clone()
+    mx = stats.clone().to(device)
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    sm = stats.clone().to(device)
+    dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+    out = mx.cpu().clone()
+    out[1], out[3] = sm[1].cpu(), sm[3].cpu()
+    return out
+
+
 def run_gpu(args, rank: int, world: int):
     import numpy as np
     import torch
@@ -209,12 +228,8 @@ def run_gpu(args, rank: int, world: int):
 
     stats = torch.tensor([ms, float(tokens), e2e_s, float(generated), v_avg], dtype=torch.float64)
     if world > 1:
-        mx = stats.clone().cuda()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        sm = stats.clone().cuda()
-        dist.all_reduce(sm, op=dist.ReduceOp.SUM)
-        ms, e2e_s, v_avg = float(mx[0]), float(mx[2]), float(mx[4])
-        tokens, generated = float(sm[1]), float(sm[3])
+        job = combine_rank_stats(stats, world, "cuda")
+        ms, tokens, e2e_s, generated, v_avg = (float(x) for x in job)
     eng.close()
     return dict(ms=ms, tokens=tokens, verify_ms=v_avg, verify_bytes=vb, clocks=clk.summary(),
                 e2e_s=e2e_s, generated=generated, h2d=h2d / e2e_steps, d2h=d2h,
