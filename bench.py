@@ -123,11 +123,6 @@ def verify_bytes(t, ctx: int, K: int) -> int:
     return weights + kv_read + kv_write + logits
 
 
-def launches_per_step(t, dft, K: int) -> int:
-    per_fwd = lambda m, lm: 1 + 5 * m.n_layers + (1 if lm else 0)
-    return K * (per_fwd(dft, True) + 1) + per_fwd(t, True) + 1
-
-
 def combine_rank_stats(stats, world: int, device):
     """One rank's [ms, tokens, e2e_s, generated, verify_ms] -> the job's: the
     times (ms, e2e_s, verify_ms) are the maximum over ranks, the counts (tokens,
@@ -165,7 +160,8 @@ def run_gpu(args, rank: int, world: int):
     eng = Engine(t, iter_weights(t, 0), max_batch=1, max_seq=max_seq, max_k=K, max_drafts=1,
                  draft_shape_max=dft, draft_budget_bytes=1 << 30, use_graphs=True,
                  launch_mode=args.launch_mode,
-                 trace=args.trace_pass if args.trace is not None else None, device=dev)
+                 trace=args.trace_pass if args.trace is not None else None, device=dev,
+                 draft_kernel=args.draft_kernel)
     eng.register_draft(0, dft, iter_weights(dft, 1))
     eng.load_draft_async(0)
     eng.set_active_draft(0)
@@ -179,6 +175,7 @@ def run_gpu(args, rank: int, world: int):
     L0 = int(eng.seq_state()[0, 0])
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(steps)]
+    ev_d = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         dist.barrier()
@@ -187,6 +184,7 @@ def run_gpu(args, rank: int, world: int):
         torch.cuda.nvtx.range_push("timed")   # for profilers: --nvtx --nvtx-include "timed/"
         start.record(s)
         for i in range(steps):
+            ev_d[i].record(s)
             eng.draft_step(K, TEMP)
             ev[i][0].record(s)
             eng.verify_step(K)
@@ -202,6 +200,9 @@ def run_gpu(args, rank: int, world: int):
         np.save(args.trace, eng.pass_trace())
     ms = start.elapsed_time(stop)
     verify_ms = [a.elapsed_time(b) for a, b in ev]
+    draft_ms = sum(d.elapsed_time(v[0]) for d, v in zip(ev_d, ev)) / steps
+    launches = eng.launches_per_step()
+    draft_fused = bool(eng.info(__import__("paper_2608_10362_gb300")._lib.INFO_DRAFT_FUSED))
     L1 = int(eng.seq_state()[0, 0])
     tokens = L1 - L0
     ctx_mean = L0 + (L1 - L0) / 2
@@ -234,7 +235,8 @@ def run_gpu(args, rank: int, world: int):
     return dict(ms=ms, tokens=tokens, verify_ms=v_avg, verify_bytes=vb, clocks=clk.summary(),
                 e2e_s=e2e_s, generated=generated, h2d=h2d / e2e_steps, d2h=d2h,
                 setup_s=setup_s, bits=bits, steps=steps, tokens_per_step=tokens / steps / world,
-                launches=launches_per_step(t, dft, K) * steps)
+                launches=launches * steps, launches_per_step=launches, draft_ms=draft_ms,
+                draft_fused=draft_fused)
 
 
 def oracle_step_timer(K: int):
@@ -691,6 +693,8 @@ def main():
     ap.add_argument("--temp", type=float, default=0.8, help="(--case edge) temperature")
     ap.add_argument("--launch-mode", default="per_op", choices=["per_op", "pass"],
                     help="one launch per op, or one persistent launch per pass")
+    ap.add_argument("--draft-kernel", default="auto", choices=["auto", "per_op", "fused"],
+                    help="draft-step kernels (auto: the fused draft kernel when the draft fits it)")
     ap.add_argument("--trace", default=None,
                     help="save per-op timestamps of the last traced pass (.npy); diagnostic, "
                          "not for the headline number")
@@ -772,6 +776,9 @@ def main():
                 "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"],
                 "scope": "prompt H2D + prefill 2048 + decode, per-step D2H of results"},
         "gpu_launches": r["launches"],
+        "draft": {"ms_per_step": r["draft_ms"], "us_per_pass": 1000.0 * r["draft_ms"] / args.k,
+                  "kernel": "fused (one launch per draft step)" if r["draft_fused"] else "per-op",
+                  "launches_per_step": r["launches_per_step"]},
         "clocks": r["clocks"],
         "device_status": r["bits"],
         "setup_s": r["setup_s"],

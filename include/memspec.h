@@ -162,9 +162,16 @@ typedef struct memspec_init_params {
   int32_t trace;                    /* per-op timestamps (MEMSPEC_BUF_PASS_TRACE) of
                                        1: verify passes, 2: draft steps, 3: prefill
                                        chunks (the last one); 0: off */
+  int32_t draft_kernel;             /* draft step with launch_mode PER_OP:
+                                       MEMSPEC_DRAFT_KERNEL_AUTO (0): the fused draft
+                                       kernel when the draft and batch fit it (below),
+                                       else per-op kernels; PER_OP (1): always per-op
+                                       kernels; FUSED (2): the fused kernel, init or the
+                                       draft step fails with UNSUPPORTED if it cannot */
 } memspec_init_params;
 
 enum { MEMSPEC_LAUNCH_PER_OP = 0, MEMSPEC_LAUNCH_PASS = 1 };
+enum { MEMSPEC_DRAFT_KERNEL_AUTO = 0, MEMSPEC_DRAFT_KERNEL_PER_OP = 1, MEMSPEC_DRAFT_KERNEL_FUSED = 2 };
 
 /* Device workspace bytes memspec_init needs for these params. */
 memspec_status memspec_workspace_bytes(const memspec_init_params* p, size_t* bytes);
@@ -264,13 +271,24 @@ typedef enum memspec_buffer {
   MEMSPEC_BUF_SEQ_STATE = 4,     /* int32 [max_batch][4] = {L, Lt, step, active Ld} */
   MEMSPEC_BUF_ACCEPT_DEBUG = 5,  /* fp32 [batch][2K+2] = {p_i(x_i), q_i(x_i), residual mass, u'} */
   MEMSPEC_BUF_RESIDUAL = 6,      /* fp32 residual stream [rows][d] of the last forward */
-  MEMSPEC_BUF_PASS_TRACE = 7     /* u64 trace of the last traced pass (init param trace):
+  MEMSPEC_BUF_PASS_TRACE = 7,    /* u64 trace of the last traced pass (init param trace):
                                     {n_ops, grid, then [n_ops][grid][16] globaltimer ns =
                                     worker start, worker end, activation loads issued,
                                     first MMA issued, partials stored, arrival counted,
                                     reduction inputs loaded, reduction done, then
                                     epilogue-internal points}; 2048 ops at most */
+  MEMSPEC_BUF_SEEDS = 8          /* u64 [max_batch] Philox keys of the requests (set by prefill) */
 } memspec_buffer;
+
+/* Facts about the last step calls (host-side, no wait).  what:
+ *   MEMSPEC_INFO_DRAFT_LAUNCHES  kernel launches of the last draft step
+ *   MEMSPEC_INFO_VERIFY_LAUNCHES kernel launches of the last verify pass
+ *   MEMSPEC_INFO_ACCEPT_LAUNCHES kernel launches of the last acceptance
+ *   MEMSPEC_INFO_DRAFT_FUSED     1 if the last draft step ran the fused draft kernel
+ * Errors: INVALID_ARG (unknown id). */
+enum { MEMSPEC_INFO_DRAFT_LAUNCHES = 0, MEMSPEC_INFO_VERIFY_LAUNCHES = 1,
+       MEMSPEC_INFO_ACCEPT_LAUNCHES = 2, MEMSPEC_INFO_DRAFT_FUSED = 3 };
+memspec_status memspec_query_info(memspec_ctx* ctx, int32_t what, int64_t* value);
 
 /* Synchronously copy `bytes` of an internal buffer to host memory (waits for
  * the main stream first).  Errors: INVALID_ARG (bytes too large), CUDA. */

@@ -36,22 +36,24 @@ memspec_status memspec_op_linear(const void* x_dev, const void* w_dev, float* y_
                                  uint32_t* status_dev, void* stream);
 
 /* The same GEMM as memspec_op_linear (y = x . w^T, fp32 out), for callers
- * that cannot allocate device memory: code running while a CUDA graph is
- * being captured, plug-ins whose host application owns all device memory, and
- * fixed-budget deployments that allocate only at start-up.  The paper has no
- * counterpart; this is a property of the library's interface.
+ * that cannot allocate device memory: plug-ins whose host application owns all
+ * device memory, fixed-budget deployments that allocate only at start-up, and
+ * latency-critical loops that cannot afford cudaMalloc / cudaFree (which may
+ * synchronise the device).  The paper has no counterpart; this is a property
+ * of the library's interface.
  * Instead of a scratch argument it uses one file-scope device array of about
  * 2.6 MB that every GPU loading the library keeps until the process exits.
  * Limits: rows in 1..16, n_out in 1..131072, k a positive multiple of 8 up to
- * 2^20; x and w
- * 16-byte aligned.  Larger sizes return MEMSPEC_ERR_INVALID_ARG (message in
- * memspec_op_last_error) and enqueue nothing.  The call allocates nothing; it
- * enqueues a clear of the array's counters and the kernel on `stream`.
+ * 2^20; x and w 16-byte aligned.  Larger sizes return MEMSPEC_ERR_INVALID_ARG
+ * (message in memspec_op_last_error) and enqueue nothing.  The call allocates
+ * nothing; it enqueues a clear of the array's counters and the kernel on
+ * `stream`.  Its split-K grid differs from memspec_op_linear's, so results
+ * agree with it within rounding, not bit for bit.
  * All calls share the array: calls that overlap on the GPU (other streams,
  * other host threads) race - serialise them.  The first call on a device looks
  * up the array's address on that device; make it before any stream capture.
  * status_dev: optional uint32 device word for in-kernel error bits (NULL: an
- * internal word is used). */
+ * internal word that the caller cannot read is used). */
 memspec_status memspec_op_linear_noalloc(const void* x_dev, const void* w_dev, float* y_dev,
                                          int32_t rows, int32_t n_out, int32_t k,
                                          uint32_t* status_dev, void* stream);
@@ -72,7 +74,7 @@ const char* memspec_op_last_error(void);
 /* Overwrite an internal buffer of ctx (same ids as memspec_read_buffer) from
  * host memory; synchronous.  Lets tests feed the acceptance step synthetic
  * logits and set sequence state.  Writable: TARGET_LOGITS, DRAFT_LOGITS,
- * DRAFT_TOKENS, TOKENS, SEQ_STATE. */
+ * DRAFT_TOKENS, TOKENS, SEQ_STATE, SEEDS. */
 memspec_status memspec_write_buffer(memspec_ctx* ctx, int32_t buffer, const void* src_host,
                                     size_t bytes);
 

@@ -22,13 +22,18 @@ T_TOK_EMB, T_ATTN_NORM, T_WQKV, T_WO, T_FFN_NORM, T_WGATE, T_WUP, T_WDOWN, T_FIN
 
 # buffer ids (memspec_buffer)
 BUF_TARGET_LOGITS, BUF_DRAFT_LOGITS, BUF_DRAFT_TOKENS, BUF_TOKENS, BUF_SEQ_STATE, \
-    BUF_ACCEPT_DEBUG, BUF_RESIDUAL, BUF_PASS_TRACE = range(8)
+    BUF_ACCEPT_DEBUG, BUF_RESIDUAL, BUF_PASS_TRACE, BUF_SEEDS = range(9)
 
 # launch modes (memspec_init_params.launch_mode)
 LAUNCH_PER_OP, LAUNCH_PASS = 0, 1
+# draft-step kernels (memspec_init_params.draft_kernel)
+DRAFT_KERNEL_AUTO, DRAFT_KERNEL_PER_OP, DRAFT_KERNEL_FUSED = 0, 1, 2
 PASS_TRACE_OPS = 2048
 
 DEV_TIMEOUT, DEV_BAD_TOKEN, DEV_BAD_LENGTH = 0x1, 0x2, 0x4
+
+# memspec_query_info ids
+INFO_DRAFT_LAUNCHES, INFO_VERIFY_LAUNCHES, INFO_ACCEPT_LAUNCHES, INFO_DRAFT_FUSED = range(4)
 
 
 class ModelCfg(C.Structure):
@@ -44,7 +49,39 @@ class InitParams(C.Structure):
                 ("max_k", C.c_int32), ("max_drafts", C.c_int32), ("draft_shape_max", ModelCfg),
                 ("draft_arena_dev", C.c_void_p), ("draft_budget_bytes", C.c_size_t),
                 ("stream_main", C.c_void_p), ("stream_side", C.c_void_p),
-                ("use_graphs", C.c_int32), ("launch_mode", C.c_int32), ("trace", C.c_int32)]
+                ("use_graphs", C.c_int32), ("launch_mode", C.c_int32), ("trace", C.c_int32),
+                ("draft_kernel", C.c_int32)]
+
+
+# draft scheduling (memspec_sched.h)
+POLICY_MEMSPEC, POLICY_MAB_ASYNC, POLICY_STATIC = 0, 1, 2
+SCHED_MAX_DRAFTS = 16
+STATE_FN = C.CFUNCTYPE(C.c_int32, C.c_void_p, C.c_int32, C.POINTER(C.c_int32))
+DRAFT_FN = C.CFUNCTYPE(C.c_int32, C.c_void_p, C.c_int32)
+
+
+class Residency(C.Structure):
+    _fields_ = [("user", C.c_void_p), ("state", STATE_FN), ("load", DRAFT_FN), ("evict", DRAFT_FN),
+                ("set_active", DRAFT_FN)]
+
+
+class SchedParams(C.Structure):
+    _fields_ = [("n_drafts", C.c_int32), ("capacity", C.c_int32), ("policy", C.c_int32),
+                ("ucb_c", C.c_float), ("k_draft", C.c_int32)]
+
+
+class SchedDecision(C.Structure):
+    _fields_ = [("active", C.c_int32), ("desired", C.c_int32), ("fallback", C.c_int32),
+                ("n_evicted", C.c_int32), ("n_prefetched", C.c_int32),
+                ("evicted", C.c_int32 * SCHED_MAX_DRAFTS),
+                ("prefetched", C.c_int32 * SCHED_MAX_DRAFTS)]
+
+
+class SchedStats(C.Structure):
+    _fields_ = [("points", C.c_int64), ("desired_intervals", C.c_int64),
+                ("fallback_intervals", C.c_int64), ("loads", C.c_int64), ("evictions", C.c_int64),
+                ("refusals", C.c_int64), ("switches", C.c_int64), ("desired_s", C.c_double),
+                ("fallback_s", C.c_double), ("policy_s", C.c_double)]
 
 
 EXPORTS = {
@@ -72,6 +109,7 @@ EXPORTS = {
     "memspec_accept_commit": (C.c_int, [C.c_void_p, C.c_int32, C.c_float, C.c_void_p]),
     "memspec_sync": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_uint32)]),
     "memspec_read_buffer": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_size_t]),
+    "memspec_query_info": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_int64)]),
     "memspec_write_buffer": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_size_t]),
     "memspec_op_linear_scratch_bytes": (C.c_int, [C.c_int32, C.c_int32, C.c_int32,
                                                   C.POINTER(C.c_size_t)]),
@@ -84,6 +122,13 @@ EXPORTS = {
     "memspec_op_last_error": (C.c_char_p, []),
     "memspec_pack_matrix": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p,
                                       C.c_size_t, C.c_void_p]),
+    "memspec_sched_create": (C.c_int, [C.POINTER(SchedParams), C.POINTER(Residency), C.c_void_p,
+                                       C.POINTER(C.c_void_p)]),
+    "memspec_sched_destroy": (None, [C.c_void_p]),
+    "memspec_sched_start": (C.c_int, [C.c_void_p, C.c_void_p, C.POINTER(SchedDecision)]),
+    "memspec_sched_point": (C.c_int, [C.c_void_p, C.c_void_p, C.POINTER(SchedDecision)]),
+    "memspec_sched_feedback": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_double]),
+    "memspec_sched_get_stats": (C.c_int, [C.c_void_p, C.POINTER(SchedStats)]),
 }
 
 _lib = None

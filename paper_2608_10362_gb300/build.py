@@ -17,7 +17,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmemspec.so")
-SOURCES = ["gemm.cu", "attention.cu", "embed.cu", "sampling.cu", "api.cu", "noalloc.cu", "pass.cu", "pack.cu"]
+SOURCES = ["gemm.cu", "attention.cu", "embed.cu", "sampling.cu", "api.cu", "noalloc.cu", "pass.cu", "pack.cu",
+           "draft_fused.cu", "sched.cpp"]
 HEADERS = ["ptx.cuh", "internal.h", "gemm_epi.cuh", "attn_body.cuh", "sample_body.cuh", "embed_body.cuh", "pass.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
@@ -33,12 +34,12 @@ def nvcc() -> str:
 
 def _deps_mtime() -> float:
     files = [os.path.join(CSRC, h) for h in HEADERS]
-    files += [os.path.join(ROOT, "include", h) for h in ("memspec.h", "memspec_ops.h")]
+    files += [os.path.join(ROOT, "include", h) for h in ("memspec.h", "memspec_ops.h", "memspec_sched.h")]
     return max(os.path.getmtime(f) for f in files)
 
 
 def _compile(src: str, force: bool, verbose: bool) -> str:
-    obj = os.path.join(BUILD, src.replace(".cu", ".o"))
+    obj = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
     path = os.path.join(CSRC, src)
     if (not force and os.path.exists(obj)
             and os.path.getmtime(obj) >= max(os.path.getmtime(path), _deps_mtime())):

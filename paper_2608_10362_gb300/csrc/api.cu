@@ -99,6 +99,11 @@ bool ensure_func_attrs() {
     g_attr_error = std::string("pass kernel smem attribute: ") + cudaGetErrorString(e);
     return false;
   }
+  e = draft_fused_set_max_smem();
+  if (e != cudaSuccess) {
+    g_attr_error = std::string("fused draft kernel smem attribute: ") + cudaGetErrorString(e);
+    return false;
+  }
   done = true;
   return true;
 }
@@ -324,6 +329,9 @@ struct memspec_ctx {
   int batch = 1;
   int last_K = 0;
   std::map<GraphKey, cudaGraphExec_t> graphs;
+  std::map<GraphKey, int> graph_launches;   // kernel launches inside each captured graph
+  int last_launches[3] = {0, 0, 0};         // of the last draft step, verify pass, acceptance
+  bool last_draft_fused = false;            // the last draft step ran the fused kernel
   // op tables of the pass kernel (workspace areas, bump-allocated per graph)
   uint8_t* op_area = nullptr;
   size_t op_area_bytes = 0, op_area_used = 0;
@@ -332,6 +340,13 @@ struct memspec_ctx {
   bool pass_kernel = false;  // draft / verify passes as one persistent launch
   bool cooperative = false;
   unsigned long long* trace = nullptr;   // per-op trace (init param trace = 1: verify, 2: draft)
+  // fused draft step scratch
+  float* df_att = nullptr;
+  size_t df_att_floats = 0;
+  float* df_lm = nullptr;
+  unsigned int* df_bar = nullptr;
+  int* df_cnt = nullptr;
+  bool df_coop = true;       // cooperative launch attribute (cleared if capture refuses it)
   std::map<std::tuple<const void*, int, int, int>, CUtensorMap> bmaps;
 };
 
@@ -425,6 +440,17 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   const size_t o_rs128 = w.take(static_cast<size_t>(p->max_seq) * 64 * 4);
   const size_t op_bytes = static_cast<size_t>(24) << 20;     // pass-kernel op tables
   const size_t done_ints = static_cast<size_t>(64) << 10;
+  // fused draft step: attention partials [rows][H][splits][hd + 4], LM-head
+  // statistics [groups][SMs][4], barrier words
+  const int dhd = has_draft ? dm.head_dim : 64;
+  const size_t df_att_floats = static_cast<size_t>(kDfMaxRows) *
+                               std::max<size_t>(nsm, static_cast<size_t>(kDfMaxGroups) *
+                                                         (has_draft ? dm.n_heads : 1)) *
+                               (dhd + 4);
+  const size_t o_dfa = w.take(df_att_floats * 4);
+  const size_t o_dfl = w.take(static_cast<size_t>(kDfMaxGroups) * nsm * 4 * 4);
+  const size_t o_dfb = w.take(64);
+  const size_t o_dfc = w.take(static_cast<size_t>(kDfMaxGroups) * (has_draft ? dm.n_heads : 1) * 4);
   const size_t o_ops = w.take(op_bytes);
   const size_t o_done = w.take(done_ints * 4);
   const size_t trace_bytes =
@@ -469,6 +495,11 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
     c->rope_sin[0] = reinterpret_cast<float*>(base + o_rs64);
     c->rope_cos[1] = reinterpret_cast<float*>(base + o_rc128);
     c->rope_sin[1] = reinterpret_cast<float*>(base + o_rs128);
+    c->df_att = reinterpret_cast<float*>(base + o_dfa);
+    c->df_att_floats = df_att_floats;
+    c->df_lm = reinterpret_cast<float*>(base + o_dfl);
+    c->df_bar = reinterpret_cast<unsigned int*>(base + o_dfb);
+    c->df_cnt = reinterpret_cast<int*>(base + o_dfc);
     c->op_area = base + o_ops;
     c->op_area_bytes = op_bytes;
     c->done_area = reinterpret_cast<int*>(base + o_done);
@@ -505,6 +536,10 @@ memspec_status validate_params(const memspec_init_params* p, std::string* why) {
   }
   if (p->max_drafts < 0 || p->max_drafts > kMaxDrafts) {
     *why = "max_drafts must be in 0..16";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (p->draft_kernel < MEMSPEC_DRAFT_KERNEL_AUTO || p->draft_kernel > MEMSPEC_DRAFT_KERNEL_FUSED) {
+    *why = "draft_kernel must be AUTO, PER_OP or FUSED";
     return MEMSPEC_ERR_INVALID_ARG;
   }
   if (p->max_drafts > 0) {
@@ -1018,17 +1053,21 @@ memspec_status launch_table(memspec_ctx* c, const OpTable& t) {
 template <class Emit>
 memspec_status run_pass(memspec_ctx* c, const GraphKey& key, bool use_pass, Emit&& emit) {
   const bool pass = use_pass && c->pass_kernel;
+  const int slot = key.kind == 1 ? 1 : (key.kind == 2 ? 2 : 0);
   if (c->p.use_graphs) {
     auto it = c->graphs.find(key);
     if (it != c->graphs.end()) {
       cudaError_t e = cudaGraphLaunch(it->second, c->main);
       if (e != cudaSuccess) return cuda_fail(c, e, "graph launch");
+      c->last_launches[slot] = c->graph_launches[key];
       return MEMSPEC_OK;
     }
   }
   std::vector<PassOp> ops;
   memspec_status s = emit(ops);
   if (s != MEMSPEC_OK) return s;
+  const int n_launch = pass ? 1 : static_cast<int>(ops.size());
+  c->last_launches[slot] = n_launch;
   // tracing: init param trace = 1 records verify passes, 2 draft steps
   const bool traced = c->trace != nullptr && ((c->p.trace == 1 && key.kind == 1) ||
                                               (c->p.trace == 2 && key.kind == 0));
@@ -1056,6 +1095,7 @@ memspec_status run_pass(memspec_ctx* c, const GraphKey& key, bool use_pass, Emit
   cudaGraphDestroy(g);
   if (e != cudaSuccess) return cuda_fail(c, e, "graph instantiate");
   c->graphs.emplace(key, ex);
+  c->graph_launches[key] = n_launch;
   e = cudaGraphLaunch(ex, c->main);
   if (e != cudaSuccess) return cuda_fail(c, e, "graph launch");
   return MEMSPEC_OK;
@@ -1129,6 +1169,155 @@ memspec_status draft_catch_up(memspec_ctx* c, int id) {
     }
   }
   return MEMSPEC_OK;
+}
+
+
+// ---------------------------------------------------------------- fused draft step
+// Launch parameters of the fused draft kernel for the active draft, or false
+// (with the reason) when the draft or batch does not fit it: at most
+// kDfMaxGroups requests, and a shared-memory ring of at least 8 weight slots
+// beside the activation rows.
+bool fused_draft_plan(memspec_ctx* c, DraftRec& dr, int K, float T, DraftFusedArgs* out,
+                      std::string* why) {
+  const memspec_model_cfg& m = dr.cfg;
+  const Layout& lay = dr.rt.lay;
+  const int B = c->batch, G = sm_count();
+  if (B > kDfMaxGroups) {
+    *why = "more than 4 requests";
+    return false;
+  }
+  const int hq = m.n_heads * m.head_dim;
+  const int f_pad = round_up(m.d_ffn, 64);
+  const int act_floats = std::max({m.d_model, hq, f_pad});
+  const size_t fixed = draft_fused_smem_bytes(0, 2 * B, act_floats) + draft_fused_static_smem() + 1024;
+  const long long room = 227LL * 1024 - static_cast<long long>(fixed);
+  const int slots = static_cast<int>(std::min<long long>(kDfMaxSlots, room / kDfSlotBytes));
+  if (slots < 8) {
+    *why = "activation rows leave no room for the weight ring";
+    return false;
+  }
+  int S = std::max(1, G / (B * m.n_heads));
+  S = std::min({S, 32, std::max(1, ceil_div(c->p.max_seq, 64))});
+  if (static_cast<size_t>(2 * B) * m.n_heads * S * (m.head_dim + 4) > c->df_att_floats) {
+    *why = "too many attention units for the scratch";
+    return false;
+  }
+  // the sampler scans one CTA's vocabulary slice with 32 ids per lane at most
+  if (ceil_div(ceil_div(m.vocab, 8), G) * 8 > 1024 || G > 256) {
+    *why = "vocabulary slice per SM above 1024 ids";
+    return false;
+  }
+  if (m.n_layers > 1) {   // per-layer tensors at a fixed stride
+    const size_t st = lay.attn_norm[1] - lay.attn_norm[0];
+    for (int l = 1; l < m.n_layers; ++l)
+      if (lay.attn_norm[l] - lay.attn_norm[l - 1] != st || lay.wqkv[l] - lay.wqkv[l - 1] != st ||
+          lay.wo[l] - lay.wo[l - 1] != st || lay.ffn_norm[l] - lay.ffn_norm[l - 1] != st ||
+          lay.wgate[l] - lay.wgate[l - 1] != st || lay.wdown[l] - lay.wdown[l - 1] != st) {
+        *why = "irregular layer layout";
+        return false;
+      }
+  }
+  DraftFusedArgs& a = *out;
+  a.w = dr.rt.w;
+  a.off_emb = static_cast<long long>(lay.emb);
+  a.off_attn_norm = static_cast<long long>(lay.attn_norm[0]);
+  a.off_wqkv = static_cast<long long>(lay.wqkv[0]);
+  a.off_wo = static_cast<long long>(lay.wo[0]);
+  a.off_ffn_norm = static_cast<long long>(lay.ffn_norm[0]);
+  a.off_wgate = static_cast<long long>(lay.wgate[0]);
+  a.off_wdown = static_cast<long long>(lay.wdown[0]);
+  a.off_final_norm = static_cast<long long>(lay.final_norm);
+  a.off_lm = static_cast<long long>(lay.lm_head);
+  a.lstride = m.n_layers > 1 ? static_cast<long long>(lay.attn_norm[1] - lay.attn_norm[0]) : 0;
+  a.tied = m.tied_embeddings;
+  a.n_layers = m.n_layers;
+  a.d = m.d_model;
+  a.H = m.n_heads;
+  a.Hkv = m.n_kv_heads;
+  a.hd = m.head_dim;
+  a.F = m.d_ffn;
+  a.V = m.vocab;
+  a.eps = m.norm_eps;
+  a.kv = dr.rt.kv;
+  a.layer_kv = static_cast<long long>(c->p.max_batch) * m.n_kv_heads * c->p.max_seq * m.head_dim;
+  a.max_seq = c->p.max_seq;
+  a.max_k = c->p.max_k;
+  a.rope_cos = c->rope_cos[m.head_dim == 128 ? 1 : 0];
+  a.rope_sin = c->rope_sin[m.head_dim == 128 ? 1 : 0];
+  a.K = K;
+  a.B = B;
+  a.greedy = T == 0.f;
+  a.inv_temp = T == 0.f ? 0.f : 1.f / T;
+  a.seq_state = c->state;
+  a.draft_len = dr.d_len;
+  a.tokens = c->tokens;
+  a.draft_tokens = c->draft_tokens;
+  a.seeds = c->seeds;
+  a.zd = c->zd;
+  a.h = c->h;
+  a.qb = c->q;
+  a.att = c->df_att;
+  a.att_cnt = c->df_cnt;
+  a.ao = reinterpret_cast<float*>(c->o);
+  a.act = reinterpret_cast<float*>(c->act);
+  a.lm_part = c->df_lm;
+  a.bar = c->df_bar;
+  a.status = c->status;
+  a.n_splits = S;
+  a.ring_slots = slots;
+  a.act_floats = act_floats;
+  // per-phase timestamps of the draft step (init param trace = 2)
+  a.trace = (c->trace != nullptr && c->p.trace == 2) ? c->trace : nullptr;
+  a.trace_phases = std::min(kPassTraceOps, K * (5 * m.n_layers + 1));
+  if (a.trace != nullptr) {
+    const unsigned long long head[2] = {static_cast<unsigned long long>(a.trace_phases),
+                                        static_cast<unsigned long long>(G)};
+    if (cudaMemcpy(c->trace, head, sizeof(head), cudaMemcpyHostToDevice) != cudaSuccess) {
+      *why = "trace header";
+      return false;
+    }
+  }
+  return true;
+}
+
+// One launch (captured once per key as a CUDA graph when graphs are on).  The
+// launch is cooperative, so that every CTA of the grid is resident for the
+// grid-wide barriers; if stream capture refuses the attribute, a plain launch of
+// one CTA per SM is used (the kernel's barrier waits are bounded either way).
+memspec_status run_fused_draft(memspec_ctx* c, const GraphKey& key, const DraftFusedArgs& a) {
+  const int G = sm_count();
+  c->last_launches[0] = 1;
+  if (!c->p.use_graphs) {
+    cudaError_t e = launch_draft_fused(a, G, c->main, c->df_coop);
+    if (e != cudaSuccess) return cuda_fail(c, e, "fused draft launch");
+    return MEMSPEC_OK;
+  }
+  auto it = c->graphs.find(key);
+  if (it != c->graphs.end()) {
+    cudaError_t e = cudaGraphLaunch(it->second, c->main);
+    if (e != cudaSuccess) return cuda_fail(c, e, "graph launch");
+    return MEMSPEC_OK;
+  }
+  for (int attempt = 0; attempt < 2; ++attempt) {
+    cudaError_t e = cudaStreamBeginCapture(c->main, cudaStreamCaptureModeThreadLocal);
+    if (e != cudaSuccess) return cuda_fail(c, e, "begin capture");
+    const cudaError_t le = launch_draft_fused(a, G, c->main, c->df_coop);
+    cudaGraph_t g = nullptr;
+    e = cudaStreamEndCapture(c->main, &g);
+    cudaGraphExec_t ex = nullptr;
+    if (le == cudaSuccess && e == cudaSuccess) e = cudaGraphInstantiate(&ex, g, 0);
+    if (g) cudaGraphDestroy(g);
+    if (le == cudaSuccess && e == cudaSuccess) {
+      c->graphs.emplace(key, ex);
+      e = cudaGraphLaunch(ex, c->main);
+      if (e != cudaSuccess) return cuda_fail(c, e, "graph launch");
+      return MEMSPEC_OK;
+    }
+    (void)cudaGetLastError();
+    if (!c->df_coop) return cuda_fail(c, le != cudaSuccess ? le : e, "fused draft capture");
+    c->df_coop = false;   // retry without the cooperative attribute
+  }
+  return fail(c, MEMSPEC_ERR_CUDA, "fused draft capture");
 }
 
 }  // namespace
@@ -1475,6 +1664,18 @@ memspec_status memspec_draft_step(memspec_ctx* c, int32_t K, float T) {
   if (s != MEMSPEC_OK) return s;
   const int B = c->batch;
   const int id = c->active;
+  if (!c->pass_kernel && c->p.draft_kernel != MEMSPEC_DRAFT_KERNEL_PER_OP) {
+    DraftFusedArgs fa{};
+    std::string why;
+    const bool fits = fused_draft_plan(c, d, K, T, &fa, &why);
+    if (fits) {
+      c->last_draft_fused = true;
+      return run_fused_draft(c, GraphKey{3, id, K, fbits(T), B}, fa);
+    }
+    if (c->p.draft_kernel == MEMSPEC_DRAFT_KERNEL_FUSED)
+      return fail(c, MEMSPEC_ERR_UNSUPPORTED, "fused draft kernel: " + why);
+  }
+  c->last_draft_fused = false;
   GraphKey key{0, id, K, fbits(T), B};
   return run_pass(c, key, true, [&](std::vector<PassOp>& ops) -> memspec_status {
     for (int j = 1; j <= K; ++j) {
@@ -1586,7 +1787,7 @@ memspec_status memspec_sync(memspec_ctx* c, int32_t timeout_ms, uint32_t* bits) 
     if (e != cudaSuccess) return cuda_fail(c, e, "event create");
     e = cudaEventRecord(ev, c->main);
     int waited = 0;
-    while (e == cudaSuccess) {
+    while (e == cudaSuccess || e == cudaErrorNotReady) {
       e = cudaEventQuery(ev);
       if (e != cudaErrorNotReady) break;
       if (waited >= timeout_ms) {
@@ -1617,6 +1818,18 @@ memspec_status memspec_sync(memspec_ctx* c, int32_t timeout_ms, uint32_t* bits) 
   return MEMSPEC_OK;
 }
 
+memspec_status memspec_query_info(memspec_ctx* c, int32_t what, int64_t* value) {
+  if (c == nullptr || value == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  switch (what) {
+    case MEMSPEC_INFO_DRAFT_LAUNCHES: *value = c->last_launches[0]; break;
+    case MEMSPEC_INFO_VERIFY_LAUNCHES: *value = c->last_launches[1]; break;
+    case MEMSPEC_INFO_ACCEPT_LAUNCHES: *value = c->last_launches[2]; break;
+    case MEMSPEC_INFO_DRAFT_FUSED: *value = c->last_draft_fused ? 1 : 0; break;
+    default: return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown info id");
+  }
+  return MEMSPEC_OK;
+}
+
 static memspec_status buffer_span(memspec_ctx* c, int32_t buf, void** ptr, size_t* cap) {
   const int B = c->p.max_batch, K = c->p.max_k, V = c->vocab;
   switch (buf) {
@@ -1627,6 +1840,7 @@ static memspec_status buffer_span(memspec_ctx* c, int32_t buf, void** ptr, size_
     case MEMSPEC_BUF_SEQ_STATE: *ptr = c->state; *cap = static_cast<size_t>(B) * kStateInts * 4; break;
     case MEMSPEC_BUF_ACCEPT_DEBUG: *ptr = c->acc_dbg; *cap = static_cast<size_t>(B) * (2 * K + 2) * 4; break;
     case MEMSPEC_BUF_RESIDUAL: *ptr = c->h; *cap = static_cast<size_t>(kMaxRows) * c->p.target.d_model * 4; break;
+    case MEMSPEC_BUF_SEEDS: *ptr = c->seeds; *cap = static_cast<size_t>(B) * 8; break;
     case MEMSPEC_BUF_PASS_TRACE:
       if (c->trace == nullptr) return fail(c, MEMSPEC_ERR_INVALID_ARG, "tracing is off (init param trace)");
       *ptr = c->trace;
@@ -1661,7 +1875,8 @@ memspec_status memspec_read_buffer(memspec_ctx* c, int32_t buf, void* dst, size_
 memspec_status memspec_write_buffer(memspec_ctx* c, int32_t buf, const void* src, size_t bytes) {
   if (c == nullptr || src == nullptr) return MEMSPEC_ERR_INVALID_ARG;
   if (buf != MEMSPEC_BUF_TARGET_LOGITS && buf != MEMSPEC_BUF_DRAFT_LOGITS &&
-      buf != MEMSPEC_BUF_DRAFT_TOKENS && buf != MEMSPEC_BUF_TOKENS && buf != MEMSPEC_BUF_SEQ_STATE)
+      buf != MEMSPEC_BUF_DRAFT_TOKENS && buf != MEMSPEC_BUF_TOKENS && buf != MEMSPEC_BUF_SEQ_STATE &&
+      buf != MEMSPEC_BUF_SEEDS)
     return fail(c, MEMSPEC_ERR_INVALID_ARG, "buffer is not writable");
   void* p;
   size_t cap;

@@ -1,0 +1,1163 @@
+// draft_fused.cu - the draft step of a small draft model as ONE launch.
+//
+// The draft step is K autoregressive forward passes of one position each (two
+// for the first pass after a fully accepted step) plus a categorical sample per
+// pass (the proposals x_1..x_K of the draft-then-verify step).  For a small
+// draft (68M-160M parameters) each projection is a few MB, so with one kernel
+// launch per op the step is bound by launch and tail latency, not by bytes.
+// This kernel runs the whole step in one cooperative launch, one CTA per SM:
+//
+//  * every op of a pass (QKV + RoPE + KV append, attention, O + residual,
+//    gate/up + SwiGLU, down + residual; final RMSNorm + LM head; sampling) is a
+//    phase separated from the next by a grid-wide barrier (an arrival counter in
+//    global memory, release / acquire, bounded waits);
+//  * projection weights are split into units of 8 output rows (the rows of a
+//    unit and their RoPE partners for QKV; 8 gate + 8 up rows for the SwiGLU
+//    pair), assigned round-robin to CTAs; each CTA computes its units' full dot
+//    products (no split-K, no partial sums) on CUDA cores, with fp32 activations
+//    and bf16 weights;
+//  * one copy-issuing warp streams the CTA's weight bytes of every op of every
+//    pass, in the order the compute warps consume them, into a ring of 8 KB
+//    shared-memory slots with 1-D bulk copies (cp.async.bulk) signalled on
+//    mbarriers.  The weights do not depend on activations, so the ring fills
+//    ahead across op and pass boundaries while the compute warps wait at grid
+//    barriers;
+//  * attention: one (request, head, key split) unit per CTA; the keys of
+//    positions before the pass are prefetched into L2 while the QKV phase runs;
+//    the O phase combines the splits (m, l, o) itself;
+//  * LM head: each CTA owns a contiguous vocabulary slice and writes its
+//    logits and (max, first argmax, sum exp) statistics; after the barrier every
+//    CTA redoes the tiny combine and the inverse-CDF search in the owning slice
+//    (same data, same order, same result), so the next pass needs no extra
+//    barrier.  Sampling follows the draft sampler: T == 0 argmax (lowest id on
+//    ties), else the smallest id j with sum_{i<=j} exp((z_i - M)/T) >
+//    u * sum_i exp((z_i - M)/T), u = Philox(seed, request, step, j - 1).
+//
+// Row r = g * R + i of pass j (R = 2 for j = 1, else 1) is position pos0[g] + i
+// of request g; pass 1 feeds the committed tokens the draft has not processed
+// (one, or two after a fully accepted step), pass j > 1 feeds x_{j-1}.
+#include <cuda_bf16.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace memspec {
+namespace {
+
+constexpr int kCW = kDfComputeWarps;
+constexpr int kCT = kCW * 32;              // compute threads
+constexpr int kUR = 8;                     // output rows per unit
+constexpr int kKeyBlock = kCT;             // keys per attention block (one per thread)
+// attention scores (2 rows), queries (2 x hd <= 128), key-group partials; the O
+// phase reuses it for the split weights (rows x H x n_splits)
+constexpr int kDfScratchFloats = 2 * kKeyBlock + 2 * 128 + 2 * kCT;
+
+enum DfOp { OP_QKV = 0, OP_O = 1, OP_GU = 2, OP_DOWN = 3, OP_LM = 4 };
+
+struct DfCtl {
+  uint64_t full[kDfMaxSlots];
+  uint64_t empty[kDfMaxSlots];
+  int abort;                          // this CTA stops (a wait ran out or the grid aborted)
+  int gs_ok;                          // result of the last grid barrier (written by thread 0)
+  int R, rows;                        // rows per request, rows of the pass
+  int valid[kDfMaxGroups], pos0[kDfMaxGroups];
+  int tok[kDfMaxRows];
+  int ok[kDfMaxRows];                 // row is valid and inside the cache
+  int next_tok[kDfMaxGroups];         // sample of the last pass
+  float red[kCW][kDfMaxRows];
+  float scale[kDfMaxRows];
+  float xch[kCW][kDfMaxRows];
+  float stat_m[kCW][kDfMaxGroups], stat_s[kCW][kDfMaxGroups];
+  int stat_a[kCW][kDfMaxGroups];
+  float samp_f[4];
+  int samp_i[4];
+};
+
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ unsigned ld_relaxed_u32(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+__device__ __forceinline__ float ldcg(const float* p) { return __ldcg(p); }
+
+__device__ __forceinline__ void csync() { named_bar_sync(1, kCT); }
+// Barrier over the compute warps that also ANDs a flag: the same answer in every
+// thread, so that a CTA stops as a whole.
+__device__ __forceinline__ bool csync_and(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, 1, %2, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(v)), "n"(kCT)
+      : "memory");
+  return r != 0;
+}
+
+// ------------------------------------------------------------------ schedule
+// Units of each weight op, and ring slots per unit.
+struct Geo {
+  int G, c;
+  int kt_d, kt_q, kt_f;          // 64-column tiles of d, H*hd, F
+  int u_qkv, u_o, u_gu, u_down, u_lm;
+  int s_qkv, s_o, s_gu, s_down, s_lm;
+};
+
+__device__ __forceinline__ Geo make_geo(const DraftFusedArgs& a) {
+  Geo g;
+  g.G = gridDim.x;
+  g.c = blockIdx.x;
+  g.kt_d = a.d / 64;
+  g.kt_q = a.H * a.hd / 64;
+  g.kt_f = (a.F + 63) / 64;
+  g.u_qkv = (a.H + 2 * a.Hkv) * a.hd / kUR;
+  g.u_o = a.d / kUR;
+  g.u_gu = a.F / kUR;
+  g.u_down = a.d / kUR;
+  g.u_lm = (a.V + kUR - 1) / kUR;
+  g.s_qkv = (g.kt_d + 7) / 8;
+  g.s_o = (g.kt_q + 7) / 8;
+  g.s_gu = (g.kt_d + 3) / 4;
+  g.s_down = (g.kt_f + 7) / 8;
+  g.s_lm = a.tied ? (a.d + 511) / 512 : (g.kt_d + 7) / 8;
+  return g;
+}
+__device__ __forceinline__ int first_unit(const Geo& g, int off) { return ((g.c - off) % g.G + g.G) % g.G; }
+__device__ __forceinline__ int lm_lo(const Geo& g, int c) {
+  return static_cast<int>(static_cast<long long>(c) * g.u_lm / g.G);
+}
+
+// Issue the copies of slot `s` of unit `u` of op `op` (layer `l`) into `dst`,
+// completing on `bar`.  Returns the bytes.
+__device__ uint32_t issue_slot(const DraftFusedArgs& a, const Geo& g, int op, int l, int u, int s,
+                               uint8_t* dst, uint64_t* bar, uint64_t pol, bool go) {
+  constexpr uint32_t kTile = kPackTileBytes;
+  uint32_t bytes = 0;
+  auto copy = [&](uint8_t* d, const uint8_t* src, uint32_t n) {
+    if (go) bulk_load(d, src, n, bar, pol);
+    bytes += n;
+  };
+  if (op == OP_QKV) {
+    const uint8_t* base = a.w + a.off_wqkv + static_cast<long long>(l) * a.lstride;
+    const int hb = u / (a.hd / kUR), ui = u - hb * (a.hd / kUR);
+    const int r_lo = hb * a.hd + 4 * ui, r_hi = r_lo + a.hd / 2;
+    const int kt0 = s * 8, kt1 = min(kt0 + 8, g.kt_d);
+    for (int kt = kt0; kt < kt1; ++kt) {
+      uint8_t* d = dst + (kt - kt0) * 1024;
+      copy(d, base + (static_cast<size_t>(r_lo / 128) * g.kt_d + kt) * kTile + (r_lo % 128) * 128, 512);
+      copy(d + 512, base + (static_cast<size_t>(r_hi / 128) * g.kt_d + kt) * kTile + (r_hi % 128) * 128, 512);
+    }
+  } else if (op == OP_GU) {
+    const uint8_t* base = a.w + a.off_wgate + static_cast<long long>(l) * a.lstride;
+    const int j0 = u * kUR, rt = j0 / 64, rr = j0 % 64;
+    const int kt0 = s * 4, kt1 = min(kt0 + 4, g.kt_d);
+    for (int kt = kt0; kt < kt1; ++kt) {
+      const uint8_t* t = base + (static_cast<size_t>(rt) * g.kt_d + kt) * kTile;
+      uint8_t* d = dst + (kt - kt0) * 2048;
+      copy(d, t + rr * 128, 1024);
+      copy(d + 1024, t + (64 + rr) * 128, 1024);
+    }
+  } else if (op == OP_LM && a.tied) {
+    const uint8_t* base = a.w + a.off_lm;
+    const int c0 = s * 512, nc = min(512, a.d - c0);
+    for (int w = 0; w < kUR; ++w) {
+      const int v = u * kUR + w;
+      if (v >= a.V) break;
+      copy(dst + w * 1024, base + (static_cast<size_t>(v) * a.d + c0) * 2, static_cast<uint32_t>(nc) * 2);
+    }
+  } else {   // O, DOWN, packed LM: 8 contiguous rows of each k tile
+    const uint8_t* base;
+    int kt_n;
+    if (op == OP_O) {
+      base = a.w + a.off_wo + static_cast<long long>(l) * a.lstride;
+      kt_n = g.kt_q;
+    } else if (op == OP_DOWN) {
+      base = a.w + a.off_wdown + static_cast<long long>(l) * a.lstride;
+      kt_n = g.kt_f;
+    } else {
+      base = a.w + a.off_lm;
+      kt_n = g.kt_d;
+    }
+    const int r0 = u * kUR;
+    const int kt0 = s * 8, kt1 = min(kt0 + 8, kt_n);
+    for (int kt = kt0; kt < kt1; ++kt)
+      copy(dst + (kt - kt0) * 1024, base + (static_cast<size_t>(r0 / 128) * kt_n + kt) * kTile + (r0 % 128) * 128,
+           1024);
+  }
+  return bytes;
+}
+
+// The copy-issuing lane: every slot of every unit of every op of every pass,
+// in consumption order.
+__device__ void producer(const DraftFusedArgs& a, DfCtl& ctl, uint8_t* ring) {
+  const Geo g = make_geo(a);
+  const int S = a.ring_slots;
+  const uint64_t pol = l2_policy_evict_first();
+  uint32_t n = 0;
+  bool ok = true;
+  auto fill = [&](int op, int l, int u, int s) {
+    if (!ok) return;
+    const int i = static_cast<int>(n % static_cast<uint32_t>(S));
+    if (n >= static_cast<uint32_t>(S)) {
+      const uint32_t par = ((n / S) - 1) & 1u;
+      if (!mbar_wait_bounded(&ctl.empty[i], par, &ctl.abort, a.status)) {
+        ok = false;
+        return;
+      }
+    }
+    uint8_t* dst = ring + static_cast<size_t>(i) * kDfSlotBytes;
+    const uint32_t bytes = issue_slot(a, g, op, l, u, s, dst, &ctl.full[i], pol, false);
+    mbar_arrive_expect_tx(&ctl.full[i], bytes);
+    issue_slot(a, g, op, l, u, s, dst, &ctl.full[i], pol, true);
+    ++n;
+  };
+  for (int j = 1; j <= a.K && ok; ++j) {
+    int cum = 0;
+    for (int l = 0; l < a.n_layers && ok; ++l) {
+      const int nu[4] = {g.u_qkv, g.u_o, g.u_gu, g.u_down};
+      const int ns[4] = {g.s_qkv, g.s_o, g.s_gu, g.s_down};
+      for (int op = 0; op < 4; ++op) {
+        const int off = cum % g.G;
+        cum += nu[op];
+        for (int u = first_unit(g, off); u < nu[op]; u += g.G)
+          for (int s = 0; s < ns[op]; ++s) fill(op, l, u, s);
+      }
+    }
+    for (int u = lm_lo(g, g.c); u < lm_lo(g, g.c + 1); ++u)
+      for (int s = 0; s < g.s_lm; ++s) fill(OP_LM, 0, u, s);
+  }
+  // tear-down: the last fill of every slot must have landed before the CTA exits
+  const uint32_t first = n > static_cast<uint32_t>(S) ? n - S : 0;
+  for (uint32_t m = first; m < n; ++m) mbar_wait_drain(&ctl.full[m % S], (m / S) & 1u);
+}
+
+// ------------------------------------------------------------------ helpers (compute warps)
+// Grid-wide barrier over the compute warps of every CTA.  false: the grid
+// aborted (the same answer in every thread of the CTA).
+__device__ bool grid_sync(const DraftFusedArgs& a, DfCtl& ctl, unsigned& epoch, int tid,
+                          unsigned long long& t_phase) {
+  csync();
+  if (tid == 0) {
+    ++epoch;
+    const unsigned target = epoch * gridDim.x;
+    unsigned long long* tr =
+        a.trace != nullptr ? a.trace + 2 + (static_cast<size_t>(epoch - 1) * gridDim.x + blockIdx.x) * 16
+                           : nullptr;
+    if (tr != nullptr && epoch <= static_cast<unsigned>(a.trace_phases)) {
+      tr[0] = t_phase;
+      tr[1] = global_ns();
+    }
+    int ok = *reinterpret_cast<volatile int*>(&ctl.abort) ? 0 : 1;
+    if (ok) {
+      __threadfence();
+      red_release_add(&a.bar[0], 1u);
+      const long long t0 = clock64();
+      while (ld_acquire_u32(&a.bar[0]) < target) {
+        if (ld_relaxed_u32(&a.bar[2]) != 0u) {
+          ok = 0;
+          break;
+        }
+        if (clock64() - t0 > kWaitBudgetCycles) {
+          atomicOr(a.status, 0x1u);
+          atomicExch(&a.bar[2], 1u);
+          ok = 0;
+          break;
+        }
+      }
+      __threadfence();
+    }
+    t_phase = global_ns();
+    if (tr != nullptr && epoch <= static_cast<unsigned>(a.trace_phases)) tr[13] = t_phase;
+    if (!ok) *reinterpret_cast<volatile int*>(&ctl.abort) = 1;
+    ctl.gs_ok = ok;
+  }
+  csync();
+  return ctl.gs_ok != 0;
+}
+
+// Per-row block sums of v[r] (r < rows) in a fixed order; result in ctl.red[0][r].
+// Starts with a barrier, so earlier readers of ctl.xch / ctl.red are done.
+__device__ void block_row_sums(DfCtl& ctl, float* v, int rows, int tid) {
+  const int w = tid >> 5, lane = tid & 31;
+  csync();
+#pragma unroll
+  for (int r = 0; r < kDfMaxRows; ++r) {
+    if (r >= rows) break;
+    float x = v[r];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    if (lane == 0) ctl.xch[w][r] = x;
+  }
+  csync();
+  if (tid < rows) {
+    float s = 0.f;
+    for (int i = 0; i < kCW; ++i) s += ctl.xch[i][tid];
+    ctl.red[0][tid] = s;
+  }
+  csync();
+}
+
+// act[r][0..d) = RMSNorm(x_r) * gain for the rows of the pass (LM: one row per
+// request, the last valid one).  src: 0 embedding rows of ctl.tok (and CTA 0
+// writes them to the residual stream), 1 residual stream.
+__device__ void load_norm_rows(const DraftFusedArgs& a, DfCtl& ctl, float* act, int src,
+                               const bf16* gain, bool lm_rows, int tid) {
+  const int d = a.d, AF = a.act_floats;
+  const int nrow = lm_rows ? a.B : ctl.rows;
+  float ss[kDfMaxRows];
+#pragma unroll
+  for (int r = 0; r < kDfMaxRows; ++r) ss[r] = 0.f;
+  for (int k = tid * 4; k < d; k += kCT * 4) {
+#pragma unroll
+    for (int r = 0; r < kDfMaxRows; ++r) {
+      if (r >= nrow) break;
+      const int rs = lm_rows ? r * ctl.R + ctl.valid[r] - 1 : r;
+      float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (ctl.ok[rs]) {
+        if (src == 0) {
+          const uint2 raw = *reinterpret_cast<const uint2*>(a.w + a.off_emb +
+                                                            (static_cast<size_t>(ctl.tok[rs]) * d + k) * 2);
+          x = make_float4(bf_lo(raw.x), bf_hi(raw.x), bf_lo(raw.y), bf_hi(raw.y));
+          if (blockIdx.x == 0) *reinterpret_cast<float4*>(a.h + static_cast<size_t>(rs) * d + k) = x;
+        } else {
+          x = __ldcg(reinterpret_cast<const float4*>(a.h + static_cast<size_t>(rs) * d + k));
+        }
+      }
+      ss[r] += x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w;
+      *reinterpret_cast<float4*>(act + r * AF + k) = x;
+    }
+  }
+  block_row_sums(ctl, ss, nrow, tid);
+  if (tid < nrow) ctl.scale[tid] = 1.f / sqrtf(ctl.red[0][tid] / static_cast<float>(d) + a.eps);
+  csync();
+  for (int k = tid * 4; k < d; k += kCT * 4) {
+    const uint2 graw = *reinterpret_cast<const uint2*>(gain + k);
+    const float g0 = bf_lo(graw.x), g1 = bf_hi(graw.x), g2 = bf_lo(graw.y), g3 = bf_hi(graw.y);
+#pragma unroll
+    for (int r = 0; r < kDfMaxRows; ++r) {
+      if (r >= nrow) break;
+      float4* p = reinterpret_cast<float4*>(act + r * AF + k);
+      const float sc = ctl.scale[r];
+      float4 x = *p;
+      x.x = x.x * sc * g0;
+      x.y = x.y * sc * g1;
+      x.z = x.z * sc * g2;
+      x.w = x.w * sc * g3;
+      *p = x;
+    }
+  }
+  csync();
+}
+
+// Dot products of the 8 rows of one unit (NRW = 2: gate and up rows) against
+// the M activation rows, over the unit's ring slots.  Returns false on abort.
+template <int OPK>
+__device__ bool unit_dots(const DraftFusedArgs& a, DfCtl& ctl, const uint8_t* ring, const float* act,
+                          int M, int n_slots, int kt_n, int swz_row_lo, int swz_row_hi,
+                          uint32_t& cons, float (&acc)[2][kDfMaxRows], int tid) {
+  const int w = tid >> 5, lane = tid & 31;
+  const int S = a.ring_slots, AF = a.act_floats;
+#pragma unroll
+  for (int q = 0; q < 2; ++q)
+#pragma unroll
+    for (int m = 0; m < kDfMaxRows; ++m) acc[q][m] = 0.f;
+  for (int s = 0; s < n_slots; ++s, ++cons) {
+    const int i = static_cast<int>(cons % static_cast<uint32_t>(S));
+    if (!mbar_wait_bounded(const_cast<uint64_t*>(&ctl.full[i]), (cons / S) & 1u, &ctl.abort, a.status))
+      return false;
+    const uint8_t* slot = ring + static_cast<size_t>(i) * kDfSlotBytes;
+    if constexpr (OPK == OP_GU) {
+      // 4 k tiles x (8 gate rows | 8 up rows) of 128-byte swizzled rows
+      const int kt0 = s * 4, nkt = min(4, kt_n - kt0);
+      const int q = lane;                   // chunk: k tile q / 8, column chunk q % 8
+      if (q < nkt * 8) {
+        const int ktl = q >> 3, c = q & 7;
+        const int kidx = (kt0 + ktl) * 64 + c * 8;
+        const int pos = (c ^ ((swz_row_lo + w) & 7)) * 16;
+        const uint4 wg = *reinterpret_cast<const uint4*>(slot + ktl * 2048 + w * 128 + pos);
+        const uint4 wu = *reinterpret_cast<const uint4*>(slot + ktl * 2048 + 1024 + w * 128 + pos);
+#pragma unroll
+        for (int m = 0; m < kDfMaxRows; ++m) {
+          if (m >= M) break;
+          const float4 x0 = *reinterpret_cast<const float4*>(act + m * AF + kidx);
+          const float4 x1 = *reinterpret_cast<const float4*>(act + m * AF + kidx + 4);
+          float t = acc[0][m];
+          t = fmaf(bf_lo(wg.x), x0.x, t); t = fmaf(bf_hi(wg.x), x0.y, t);
+          t = fmaf(bf_lo(wg.y), x0.z, t); t = fmaf(bf_hi(wg.y), x0.w, t);
+          t = fmaf(bf_lo(wg.z), x1.x, t); t = fmaf(bf_hi(wg.z), x1.y, t);
+          t = fmaf(bf_lo(wg.w), x1.z, t); t = fmaf(bf_hi(wg.w), x1.w, t);
+          acc[0][m] = t;
+          float v = acc[1][m];
+          v = fmaf(bf_lo(wu.x), x0.x, v); v = fmaf(bf_hi(wu.x), x0.y, v);
+          v = fmaf(bf_lo(wu.y), x0.z, v); v = fmaf(bf_hi(wu.y), x0.w, v);
+          v = fmaf(bf_lo(wu.z), x1.x, v); v = fmaf(bf_hi(wu.z), x1.y, v);
+          v = fmaf(bf_lo(wu.w), x1.z, v); v = fmaf(bf_hi(wu.w), x1.w, v);
+          acc[1][m] = v;
+        }
+      }
+    } else {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int q = lane + 32 * h;        // chunk of this row in the slot
+        bool have;
+        int woff, kidx;
+        if (OPK == OP_LM && a.tied) {       // row-major: row w, 512 columns
+          const int c0 = s * 512;
+          kidx = c0 + q * 8;
+          have = kidx < a.d;
+          woff = w * 1024 + q * 16;
+        } else {
+          const int kt0 = s * 8, nkt = min(8, kt_n - kt0);
+          const int ktl = q >> 3, c = q & 7;
+          have = q < nkt * 8;
+          kidx = (kt0 + ktl) * 64 + c * 8;
+          const int trow = (OPK == OP_QKV && w >= 4) ? swz_row_hi + (w - 4) : swz_row_lo + w;
+          woff = ktl * 1024 + w * 128 + ((c ^ (trow & 7)) * 16);
+        }
+        if (!have) continue;
+        const uint4 wv = *reinterpret_cast<const uint4*>(slot + woff);
+#pragma unroll
+        for (int m = 0; m < kDfMaxRows; ++m) {
+          if (m >= M) break;
+          const float4 x0 = *reinterpret_cast<const float4*>(act + m * AF + kidx);
+          const float4 x1 = *reinterpret_cast<const float4*>(act + m * AF + kidx + 4);
+          float t = acc[0][m];
+          t = fmaf(bf_lo(wv.x), x0.x, t); t = fmaf(bf_hi(wv.x), x0.y, t);
+          t = fmaf(bf_lo(wv.y), x0.z, t); t = fmaf(bf_hi(wv.y), x0.w, t);
+          t = fmaf(bf_lo(wv.z), x1.x, t); t = fmaf(bf_hi(wv.z), x1.y, t);
+          t = fmaf(bf_lo(wv.w), x1.z, t); t = fmaf(bf_hi(wv.w), x1.w, t);
+          acc[0][m] = t;
+        }
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(const_cast<uint64_t*>(&ctl.empty[i]));
+  }
+  // fixed xor tree: every lane ends with the row totals
+#pragma unroll
+  for (int q = 0; q < 2; ++q)
+#pragma unroll
+    for (int m = 0; m < kDfMaxRows; ++m) {
+      if (m >= M) break;
+      float x = acc[q][m];
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+      acc[q][m] = x;
+    }
+  return true;
+}
+
+__device__ __forceinline__ float pick(const float (&v)[kDfMaxRows], int m) {
+  float r = 0.f;
+#pragma unroll
+  for (int i = 0; i < kDfMaxRows; ++i)
+    if (i == m) r = v[i];
+  return r;
+}
+
+// One (request, head, key split) of attention for the rows of request g: writes
+// (m, l, o) in log2 units to the partial buffer; the last split of (g, h) to
+// finish (arrival counter) combines all splits in split order and writes the
+// attention output of the head to a.ao.  scratch: kDfScratchFloats floats.
+template <int HD>
+__device__ void attention_unit(const DraftFusedArgs& a, DfCtl& ctl, int layer, int g, int h, int s,
+                               float* scratch, int tid) {
+  constexpr int KG = kCT / HD;            // key groups of the PV product
+  const int R = ctl.R, S = a.n_splits;
+  const int nr = ctl.valid[g];
+  const int p0 = ctl.pos0[g];
+  const int ctx = p0 + nr;                // keys 0..ctx-1
+  const int chunk = (ctx + S - 1) / S;
+  const int k0 = s * chunk, k1 = min(k0 + chunk, ctx);
+  const int kvh = h / (a.H / a.Hkv);
+  const size_t kbase = static_cast<size_t>(layer) * 2 * a.layer_kv +
+                       (static_cast<size_t>(g) * a.Hkv + kvh) * a.max_seq * HD;
+  const bf16* kc = a.kv + kbase;
+  const bf16* vc = kc + a.layer_kv;
+  float* sc = scratch;                    // [2][kKeyBlock] scores, then weights
+  float* qs = sc + 2 * kKeyBlock;         // [2][HD]
+  float* op = qs + 2 * HD;                // [kCT][2] o partials (key groups)
+  const float qscale = 1.4426950408889634f / sqrtf(static_cast<float>(HD));
+  for (int e = tid; e < nr * HD; e += kCT) {
+    const int i = e / HD, dd = e - i * HD;
+    qs[e] = ldcg(a.qb + (static_cast<size_t>(g * R + i) * a.H + h) * HD + dd) * qscale;
+  }
+  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  const int dd = tid % HD, kg = tid / HD;
+  float o_run[2] = {0.f, 0.f};
+  csync();
+  for (int kb = k0; kb < k1; kb += kKeyBlock) {
+    const int t = kb + tid;
+    float sco[2] = {-INFINITY, -INFINITY};
+    if (t < k1) {
+      // the whole key row in one round trip
+      uint4 kr[HD / 8];
+      const uint4* src = reinterpret_cast<const uint4*>(kc + static_cast<size_t>(t) * HD);
+#pragma unroll
+      for (int c = 0; c < HD / 8; ++c) kr[c] = __ldcg(src + c);
+      float dot[2] = {0.f, 0.f};
+#pragma unroll
+      for (int c = 0; c < HD / 8; ++c) {
+        const float kf[8] = {bf_lo(kr[c].x), bf_hi(kr[c].x), bf_lo(kr[c].y), bf_hi(kr[c].y),
+                             bf_lo(kr[c].z), bf_hi(kr[c].z), bf_lo(kr[c].w), bf_hi(kr[c].w)};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          dot[0] = fmaf(qs[c * 8 + e], kf[e], dot[0]);
+          dot[1] = fmaf(qs[HD + c * 8 + e], kf[e], dot[1]);
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < 2; ++i)
+        if (i < nr && t <= p0 + i) sco[i] = dot[i];
+    }
+    // block max per row
+    float mx[2];
+    {
+      const int w = tid >> 5, lane = tid & 31;
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        float x = sco[i];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
+        if (lane == 0) ctl.xch[w][i] = x;
+      }
+      csync();
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        float x = -INFINITY;
+        for (int ww = 0; ww < kCW; ++ww) x = fmaxf(x, ctl.xch[ww][i]);
+        mx[i] = x;
+      }
+    }
+    float alpha[2], mnew[2], p[2];
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      mnew[i] = fmaxf(m_run[i], mx[i]);
+      alpha[i] = (m_run[i] == -INFINITY) ? 0.f : exp2f(m_run[i] - mnew[i]);
+      p[i] = (sco[i] == -INFINITY) ? 0.f : exp2f(sco[i] - mnew[i]);
+      sc[i * kKeyBlock + tid] = p[i];
+    }
+    float ps[kDfMaxRows];
+#pragma unroll
+    for (int i = 0; i < kDfMaxRows; ++i) ps[i] = i < 2 ? p[i] : 0.f;
+    block_row_sums(ctl, ps, 2, tid);       // also a barrier: sc is complete
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      l_run[i] = l_run[i] * alpha[i] + ctl.red[0][i];
+      m_run[i] = mnew[i];
+      o_run[i] *= alpha[i];
+    }
+    const int nk = min(kKeyBlock, k1 - kb);
+    const bf16* vb = vc + static_cast<size_t>(kb) * HD + dd;
+    for (int t0 = kg; t0 < nk; t0 += 8 * KG) {
+      float v[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int tt = t0 + q * KG;
+        v[q] = tt < nk ? __bfloat162float(vb[static_cast<size_t>(tt) * HD]) : 0.f;
+      }
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int tt = t0 + q * KG;
+        if (tt < nk) {
+          o_run[0] = fmaf(sc[tt], v[q], o_run[0]);
+          o_run[1] = fmaf(sc[kKeyBlock + tt], v[q], o_run[1]);
+        }
+      }
+    }
+    csync();                                // sc is rewritten by the next block
+  }
+  // combine the key groups in order, write (m, l, o)
+  op[tid * 2] = o_run[0];
+  op[tid * 2 + 1] = o_run[1];
+  csync();
+  const int stride = HD + 4;
+  float* mine = a.att + (static_cast<size_t>(g * R) * a.H + h) * S * stride;   // row i at + i * H * S * stride
+  for (int e = tid; e < nr * HD; e += kCT) {
+    const int i = e / HD, d2 = e - i * HD;
+    float o = 0.f;
+#pragma unroll
+    for (int k = 0; k < KG; ++k) o += op[(k * HD + d2) * 2 + i];
+    mine[(static_cast<size_t>(i) * a.H * S + s) * stride + 4 + d2] = o;
+  }
+  if (tid < nr) {
+    float* hdr = mine + (static_cast<size_t>(tid) * a.H * S + s) * stride;
+    hdr[0] = tid == 0 ? m_run[0] : m_run[1];
+    hdr[1] = tid == 0 ? l_run[0] : l_run[1];
+  }
+  // the last split of (g, h) to arrive combines them all
+  csync();
+  if (tid == 0) {
+    __threadfence();
+    const int old = atomicAdd(&a.att_cnt[g * a.H + h], 1);
+    ctl.samp_i[0] = old == S - 1 ? 1 : 0;
+    if (old == S - 1) {
+      a.att_cnt[g * a.H + h] = 0;             // ready for the next layer
+      __threadfence();
+    }
+  }
+  csync();
+  if (!ctl.samp_i[0]) return;
+  float* w = scratch;                          // [2][32] split weights (scores are done)
+  if (tid < nr) {
+    const float* base = mine + static_cast<size_t>(tid) * a.H * S * stride;
+    float mv[32], lv[32];
+#pragma unroll
+    for (int q = 0; q < 32; ++q) {
+      float2 ml = make_float2(-INFINITY, 0.f);
+      if (q < S) ml = __ldcg(reinterpret_cast<const float2*>(base + q * stride));
+      mv[q] = ml.x;
+      lv[q] = ml.y;
+    }
+    float M = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < 32; ++q)
+      if (lv[q] > 0.f) M = fmaxf(M, mv[q]);
+    float Lsum = 0.f;
+#pragma unroll
+    for (int q = 0; q < 32; ++q) {
+      const float wv = lv[q] > 0.f ? exp2f(mv[q] - M) : 0.f;
+      mv[q] = wv;
+      Lsum += wv * lv[q];
+    }
+    const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
+#pragma unroll
+    for (int q = 0; q < 32; ++q) w[tid * 32 + q] = mv[q] * inv;
+  }
+  csync();
+  for (int e = tid; e < nr * HD; e += kCT) {
+    const int i = e / HD, d2 = e - i * HD;
+    const float* base = mine + static_cast<size_t>(i) * a.H * S * stride + 4 + d2;
+    float v[32];
+#pragma unroll
+    for (int q = 0; q < 32; ++q) v[q] = q < S ? ldcg(base + q * stride) : 0.f;
+    float o = 0.f;
+#pragma unroll
+    for (int q = 0; q < 32; ++q)
+      if (q < S) o = fmaf(w[i * 32 + q], v[q], o);
+    a.ao[static_cast<size_t>(g * R + i) * a.H * HD + h * HD + d2] = o;
+  }
+}
+
+// Sample request g's token of pass j from the LM-head statistics (warp 0);
+// result in ctl.next_tok[g].
+__device__ void sample_group(const DraftFusedArgs& a, DfCtl& ctl, int j, int g, int lane) {
+  const int G = gridDim.x;
+  const float* part = a.lm_part + static_cast<size_t>(g) * G * 4;
+  const int per = (G + 31) / 32;               // <= 8 (grid <= 256)
+  const int c_lo = min(lane * per, G), c_hi = min(c_lo + per, G);
+  float pm[8], ps[8];
+  int pa[8];
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    float4 v = make_float4(-INFINITY, 0.f, __int_as_float(0x7fffffff), 0.f);
+    if (c_lo + q < c_hi) v = __ldcg(reinterpret_cast<const float4*>(part + (c_lo + q) * 4));
+    pm[q] = v.x;
+    ps[q] = v.y;
+    pa[q] = __float_as_int(v.z);
+  }
+  // max and first argmax
+  float bm = -INFINITY;
+  int ba = 0x7fffffff;
+#pragma unroll
+  for (int q = 0; q < 8; ++q)
+    if (pm[q] > bm || (pm[q] == bm && pa[q] < ba)) {
+      bm = pm[q];
+      ba = pa[q];
+    }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float om = __shfl_xor_sync(0xffffffffu, bm, o);
+    const int oa = __shfl_xor_sync(0xffffffffu, ba, o);
+    if (om > bm || (om == bm && oa < ba)) {
+      bm = om;
+      ba = oa;
+    }
+  }
+  int tok = ba;
+  if (!a.greedy) {
+    const float it = a.inv_temp, M = bm;
+    // per-CTA weights in CTA (= vocabulary) order, inclusive scan over lanes
+    float wq[8], ls = 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      wq[q] = ps[q] > 0.f ? ps[q] * __expf((pm[q] - M) * it) : 0.f;
+      ls += wq[q];
+    }
+    float incl = ls;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float nb = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += nb;
+    }
+    float excl = __shfl_up_sync(0xffffffffu, incl, 1);
+    if (lane == 0) excl = 0.f;
+    const float total = __shfl_sync(0xffffffffu, incl, 31);
+    const int step = a.seq_state[g * kStateInts + 2];
+    const float u = philox_uniform(a.seeds[g], g, step, j - 1);
+    const float target = u * total;
+    int sel = -1;
+    float before = 0.f;
+    if (ls > 0.f && excl <= target && target < incl) {
+      float cum = excl;
+      bool done = false;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (!done && wq[q] > 0.f) {
+          sel = c_lo + q;
+          before = cum;
+          if (cum + wq[q] > target) done = true;
+        }
+        if (!done) cum += wq[q];
+      }
+    }
+    const unsigned claim = __ballot_sync(0xffffffffu, sel >= 0);
+    const int last_lane = 31 - __clz(__ballot_sync(0xffffffffu, ls > 0.f) | 1u);
+    const int src = claim ? (__ffs(claim) - 1) : last_lane;
+    if (!claim && lane == src) {
+      float cum = excl;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (wq[q] > 0.f) {
+          sel = c_lo + q;
+          before = cum;
+        }
+        cum += wq[q];
+      }
+    }
+    sel = __shfl_sync(0xffffffffu, sel, src);
+    before = __shfl_sync(0xffffffffu, before, src);
+    if (total > 0.f && sel >= 0) {
+      // the owning slice, in id order: contiguous ranges per lane
+      const Geo geo = make_geo(a);
+      const int v0 = lm_lo(geo, sel) * kUR, v1 = min(lm_lo(geo, sel + 1) * kUR, a.V);
+      const int n = v1 - v0, pl = (n + 31) / 32;   // <= 32 (slice <= 1024 ids)
+      const int x0 = min(v0 + lane * pl, v1), x1 = min(x0 + pl, v1);
+      const float* z = a.zd + (static_cast<size_t>(g) * a.K + (j - 1)) * a.V;
+      float wv[32];
+#pragma unroll
+      for (int q = 0; q < 32; ++q) wv[q] = x0 + q < x1 ? ldcg(z + x0 + q) : -INFINITY;
+      float own = 0.f;
+#pragma unroll
+      for (int q = 0; q < 32; ++q) {
+        wv[q] = x0 + q < x1 ? __expf((wv[q] - M) * it) : 0.f;
+        own += wv[q];
+      }
+      float in2 = own;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float nb = __shfl_up_sync(0xffffffffu, in2, o);
+        if (lane >= o) in2 += nb;
+      }
+      float ex2 = __shfl_up_sync(0xffffffffu, in2, 1);
+      if (lane == 0) ex2 = 0.f;
+      const float r = target - before;
+      int mine = -1, lastx = -1;
+      {
+        float cum = ex2;
+        const bool scan = own > 0.f && ex2 <= r && r < in2;
+#pragma unroll
+        for (int q = 0; q < 32; ++q) {
+          cum += wv[q];
+          if (wv[q] > 0.f) {
+            lastx = x0 + q;
+            if (scan && mine < 0 && cum > r) mine = x0 + q;
+          }
+        }
+        if (scan && mine < 0) mine = lastx;
+      }
+      const unsigned cl = __ballot_sync(0xffffffffu, mine >= 0);
+      if (cl) {
+        tok = __shfl_sync(0xffffffffu, mine, __ffs(cl) - 1);
+      } else {   // r at or after the slice's scanned mass: its last id with mass
+        const unsigned hm = __ballot_sync(0xffffffffu, lastx >= 0);
+        if (hm) tok = __shfl_sync(0xffffffffu, lastx, 31 - __clz(hm));
+      }
+    }
+  }
+  if (lane == 0) ctl.next_tok[g] = tok;
+}
+
+__global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid_constant__ DraftFusedArgs a) {
+  __shared__ DfCtl ctl;
+  extern __shared__ __align__(128) uint8_t dsm[];
+  uint8_t* ring = dsm;
+  float* act = reinterpret_cast<float*>(dsm + static_cast<size_t>(a.ring_slots) * kDfSlotBytes);
+  float* scratch = act + static_cast<size_t>(2 * a.B) * a.act_floats;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    for (int i = 0; i < a.ring_slots; ++i) {
+      mbar_init(&ctl.full[i], 1);
+      mbar_init(&ctl.empty[i], kCW);
+    }
+    ctl.abort = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (warp == kCW) {
+    if (lane == 0) producer(a, ctl, ring);
+  } else {
+    const Geo geo = make_geo(a);
+    const int G = geo.G, c = geo.c;
+    uint32_t cons = 0;
+    unsigned epoch = 0;
+    unsigned long long t_phase = global_ns();
+    bool run = true;
+    float acc[2][kDfMaxRows];
+    for (int j = 1; j <= a.K && run; ++j) {
+      // ---------------- the rows of this pass
+      if (tid == 0) {
+        const int R = j == 1 ? 2 : 1;
+        ctl.R = R;
+        ctl.rows = a.B * R;
+        for (int g = 0; g < a.B; ++g) {
+          const int L = a.seq_state[g * kStateInts + 0];
+          int valid, pos0;
+          if (j == 1) {
+            int nv = L - a.draft_len[g];
+            if (nv < 1 || nv > 2) {
+              atomicOr(a.status, 0x4u);     // draft cache not caught up
+              nv = nv < 1 ? 1 : 2;
+            }
+            valid = nv;
+            pos0 = L - nv;
+          } else {
+            valid = 1;
+            pos0 = L + j - 2;
+          }
+          ctl.valid[g] = valid;
+          ctl.pos0[g] = pos0;
+          for (int i = 0; i < R; ++i) {
+            const int r = g * R + i, pos = pos0 + i;
+            bool ok = i < valid;
+            int tok = 0;
+            if (ok && (pos < 0 || pos >= a.max_seq)) {
+              atomicOr(a.status, 0x4u);
+              ok = false;
+            }
+            if (ok) {
+              tok = j == 1 ? a.tokens[static_cast<size_t>(g) * a.max_seq + pos] : ctl.next_tok[g];
+              if (tok < 0 || tok >= a.V) {
+                atomicOr(a.status, 0x2u);
+                tok = 0;
+              }
+            }
+            ctl.ok[r] = ok ? 1 : 0;
+            ctl.tok[r] = tok;
+          }
+        }
+      }
+      csync();
+      const int R = ctl.R, rows = ctl.rows;
+      int cum = 0;
+      for (int l = 0; l < a.n_layers && run; ++l) {
+        const size_t loff = static_cast<size_t>(l) * a.lstride;
+        // ---------------- QKV + RoPE + KV append
+        {
+          // this layer's attention units: earlier keys into L2 while QKV runs
+          const int units = a.B * a.H * a.n_splits;
+          if (tid == 0)
+            for (int ua = c; ua < units; ua += G) {
+              const int g = ua / (a.H * a.n_splits), h = (ua / a.n_splits) % a.H, s = ua % a.n_splits;
+              const int ctx = ctl.pos0[g] + ctl.valid[g];
+              const int chunk = (ctx + a.n_splits - 1) / a.n_splits;
+              const int k0 = s * chunk, k1 = min(min(k0 + chunk, ctx), ctl.pos0[g]);
+              if (k1 > k0 && ctl.pos0[g] + ctl.valid[g] <= a.max_seq) {
+                const int kvh = h / (a.H / a.Hkv);
+                const bf16* kc = a.kv + static_cast<size_t>(l) * 2 * a.layer_kv +
+                                 (static_cast<size_t>(g) * a.Hkv + kvh) * a.max_seq * a.hd;
+                const uint32_t nb = static_cast<uint32_t>(k1 - k0) * a.hd * 2;
+                prefetch_l2(kc + static_cast<size_t>(k0) * a.hd, nb);
+                prefetch_l2(kc + a.layer_kv + static_cast<size_t>(k0) * a.hd, nb);
+              }
+            }
+          load_norm_rows(a, ctl, act, l == 0 ? 0 : 1,
+                         reinterpret_cast<const bf16*>(a.w + a.off_attn_norm + loff), false, tid);
+          const int off = cum % G;
+          cum += geo.u_qkv;
+          const int upb = a.hd / kUR;               // units per head block
+          for (int u = first_unit(geo, off); u < geo.u_qkv && run; u += G) {
+            const int hb = u / upb, ui = u - hb * upb;
+            const int r_lo = hb * a.hd + 4 * ui, r_hi = r_lo + a.hd / 2;
+            run = csync_and(unit_dots<OP_QKV>(a, ctl, ring, act, rows, geo.s_qkv, geo.kt_d, r_lo % 128,
+                                              r_hi % 128, cons, acc, tid));
+            if (!run) break;
+            if (lane < rows) ctl.xch[warp][lane] = pick(acc[0], lane);
+            csync();
+            if (warp < 4 && lane < rows && ctl.ok[lane]) {
+              const int m = lane, g = m / R, pos = ctl.pos0[g] + (m - g * R);
+              const float x1 = ctl.xch[warp][m], x2 = ctl.xch[warp + 4][m];
+              const int fi = 4 * ui + warp;         // pair (fi, fi + hd/2) of the head
+              const int half = a.hd / 2;
+              if (hb < a.H + a.Hkv) {
+                const float cs = a.rope_cos[static_cast<size_t>(pos) * half + fi];
+                const float sn = a.rope_sin[static_cast<size_t>(pos) * half + fi];
+                const float y1 = x1 * cs - x2 * sn, y2 = x1 * sn + x2 * cs;
+                if (hb < a.H) {
+                  float* qd = a.qb + (static_cast<size_t>(m) * a.H + hb) * a.hd;
+                  qd[fi] = y1;
+                  qd[fi + half] = y2;
+                } else {
+                  bf16* kd = a.kv + static_cast<size_t>(l) * 2 * a.layer_kv +
+                             ((static_cast<size_t>(g) * a.Hkv + (hb - a.H)) * a.max_seq + pos) * a.hd;
+                  kd[fi] = __float2bfloat16_rn(y1);
+                  kd[fi + half] = __float2bfloat16_rn(y2);
+                }
+              } else {
+                bf16* vd = a.kv + static_cast<size_t>(l) * 2 * a.layer_kv + a.layer_kv +
+                           ((static_cast<size_t>(g) * a.Hkv + (hb - a.H - a.Hkv)) * a.max_seq + pos) * a.hd;
+                vd[fi] = __float2bfloat16_rn(x1);
+                vd[fi + half] = __float2bfloat16_rn(x2);
+              }
+            }
+            csync();
+          }
+          if (run) run = grid_sync(a, ctl, epoch, tid, t_phase);
+        }
+        // ---------------- attention
+        if (run) {
+          const int units = a.B * a.H * a.n_splits;
+          for (int ua = c; ua < units; ua += G) {
+            const int g = ua / (a.H * a.n_splits), h = (ua / a.n_splits) % a.H, s = ua % a.n_splits;
+            bool grp_ok = true;
+            for (int i = 0; i < ctl.valid[g]; ++i) grp_ok = grp_ok && ctl.ok[g * R + i];
+            if (grp_ok) {
+              if (a.hd == 64)
+                attention_unit<64>(a, ctl, l, g, h, s, scratch, tid);
+              else
+                attention_unit<128>(a, ctl, l, g, h, s, scratch, tid);
+            }
+            csync();                            // scratch and ctl are reused by the next unit
+          }
+          run = grid_sync(a, ctl, epoch, tid, t_phase);
+        }
+        // ---------------- O projection + residual (combines the key splits)
+        if (run) {
+          const int off = cum % G;
+          cum += geo.u_o;
+          const int fu = first_unit(geo, off);
+          if (fu < geo.u_o) {
+            // the heads' attention outputs (combined by the last split of each)
+            const int qd = a.H * a.hd, n4 = rows * qd / 4;
+            for (int e0 = tid; e0 < n4; e0 += 4 * kCT) {
+              float4 v[4];
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                const int e = e0 + q * kCT;
+                const int m = e < n4 ? (4 * e) / qd : 0;
+                v[q] = (e < n4 && ctl.ok[m]) ? __ldcg(reinterpret_cast<const float4*>(a.ao) + e)
+                                              : make_float4(0.f, 0.f, 0.f, 0.f);
+              }
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                const int e = e0 + q * kCT;
+                if (e < n4) {
+                  const int m = (4 * e) / qd, k = 4 * e - m * qd;
+                  *reinterpret_cast<float4*>(act + m * a.act_floats + k) = v[q];
+                }
+              }
+            }
+            csync();
+          }
+          for (int u = fu; u < geo.u_o && run; u += G) {
+            run = csync_and(unit_dots<OP_O>(a, ctl, ring, act, rows, geo.s_o, geo.kt_q, (u * kUR) % 128, 0,
+                                            cons, acc, tid));
+            if (!run) break;
+            if (lane < rows && ctl.ok[lane]) {
+              float* hp = a.h + static_cast<size_t>(lane) * a.d + u * kUR + warp;
+              *hp = ldcg(hp) + pick(acc[0], lane);
+            }
+          }
+          if (run) run = grid_sync(a, ctl, epoch, tid, t_phase);
+        }
+        // ---------------- gate/up + SwiGLU
+        if (run) {
+          const int off = cum % G;
+          cum += geo.u_gu;
+          const int fu = first_unit(geo, off);
+          if (fu < geo.u_gu)
+            load_norm_rows(a, ctl, act, 1, reinterpret_cast<const bf16*>(a.w + a.off_ffn_norm + loff), false,
+                           tid);
+          for (int u = fu; u < geo.u_gu && run; u += G) {
+            run = csync_and(unit_dots<OP_GU>(a, ctl, ring, act, rows, geo.s_gu, geo.kt_d, (u * kUR) % 64, 0,
+                                             cons, acc, tid));
+            if (!run) break;
+            if (lane < rows && ctl.ok[lane]) {
+              const float gt = pick(acc[0], lane), up = pick(acc[1], lane);
+              const float sg = gt / (1.f + expf(-gt));
+              a.act[static_cast<size_t>(lane) * a.F + u * kUR + warp] = sg * up;
+            }
+          }
+          if (run) run = grid_sync(a, ctl, epoch, tid, t_phase);
+        }
+        // ---------------- down + residual
+        if (run) {
+          const int off = cum % G;
+          cum += geo.u_down;
+          const int fu = first_unit(geo, off);
+          if (fu < geo.u_down) {
+            const int Fp = geo.kt_f * 64, n4 = rows * Fp / 4;
+            for (int e0 = tid; e0 < n4; e0 += 4 * kCT) {
+              float4 v[4];
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                const int e = e0 + q * kCT;
+                const int m = e < n4 ? (4 * e) / Fp : 0, k = 4 * e - m * Fp;
+                v[q] = (e < n4 && k < a.F && ctl.ok[m])
+                           ? __ldcg(reinterpret_cast<const float4*>(a.act + static_cast<size_t>(m) * a.F + k))
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
+              }
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                const int e = e0 + q * kCT;
+                if (e < n4) {
+                  const int m = (4 * e) / Fp, k = 4 * e - m * Fp;
+                  *reinterpret_cast<float4*>(act + m * a.act_floats + k) = v[q];
+                }
+              }
+            }
+            csync();
+          }
+          for (int u = fu; u < geo.u_down && run; u += G) {
+            run = csync_and(unit_dots<OP_DOWN>(a, ctl, ring, act, rows, geo.s_down, geo.kt_f, (u * kUR) % 128,
+                                               0, cons, acc, tid));
+            if (!run) break;
+            if (lane < rows && ctl.ok[lane]) {
+              float* hp = a.h + static_cast<size_t>(lane) * a.d + u * kUR + warp;
+              *hp = ldcg(hp) + pick(acc[0], lane);
+            }
+          }
+          if (run) run = grid_sync(a, ctl, epoch, tid, t_phase);
+        }
+      }
+      // ---------------- final RMSNorm + LM head (this CTA's vocabulary slice)
+      if (run) {
+        const int B = a.B;
+        const int ulo = lm_lo(geo, c), uhi = lm_lo(geo, c + 1);
+        float sm_m = -INFINITY, sm_s = 0.f;
+        int sm_a = 0x7fffffff;
+        if (ulo < uhi)
+          load_norm_rows(a, ctl, act, 1, reinterpret_cast<const bf16*>(a.w + a.off_final_norm), true, tid);
+        const bool greedy = a.greedy != 0;
+        const float it = a.inv_temp;
+        for (int u = ulo; u < uhi && run; ++u) {
+          run = csync_and(unit_dots<OP_LM>(a, ctl, ring, act, B, geo.s_lm, geo.kt_d, (u * kUR) % 128, 0,
+                                           cons, acc, tid));
+          if (!run) break;
+          const int v = u * kUR + warp;
+          if (lane < B && v < a.V) {
+            const float z = pick(acc[0], lane);
+            a.zd[(static_cast<size_t>(lane) * a.K + (j - 1)) * a.V + v] = z;
+            if (z > sm_m) {
+              if (!greedy) sm_s = (sm_m == -INFINITY) ? 0.f : sm_s * __expf((sm_m - z) * it);
+              sm_m = z;
+              sm_a = v;
+            }
+            if (!greedy) sm_s += __expf((z - sm_m) * it);
+          }
+        }
+        if (run) {
+          // this CTA's statistics per request: warps combined in order
+          if (lane < B) {
+            ctl.stat_m[warp][lane] = sm_m;
+            ctl.stat_s[warp][lane] = sm_s;
+            ctl.stat_a[warp][lane] = sm_a;
+          }
+          csync();
+          if (tid < B) {
+            float M = -INFINITY;
+            int A = 0x7fffffff;
+            for (int w = 0; w < kCW; ++w) {
+              const float m = ctl.stat_m[w][tid];
+              const int ar = ctl.stat_a[w][tid];
+              if (m > M || (m == M && ar < A)) {
+                M = m;
+                A = ar;
+              }
+            }
+            float Ssum = 0.f;
+            if (!greedy)
+              for (int w = 0; w < kCW; ++w) {
+                const float m = ctl.stat_m[w][tid];
+                if (m != -INFINITY) Ssum += ctl.stat_s[w][tid] * __expf((m - M) * it);
+              }
+            float* p = a.lm_part + (static_cast<size_t>(tid) * G + c) * 4;
+            p[0] = M;
+            p[1] = Ssum;
+            p[2] = __int_as_float(A);
+          }
+          run = grid_sync(a, ctl, epoch, tid, t_phase);
+        }
+      }
+      // ---------------- sampling: every CTA before the next pass, CTA 0 after the last
+      if (run && (j < a.K || c == 0)) {
+        if (warp == 0)
+          for (int g = 0; g < a.B; ++g) sample_group(a, ctl, j, g, lane);
+        csync();
+        if (c == 0 && tid < a.B) a.draft_tokens[tid * a.max_k + (j - 1)] = ctl.next_tok[tid];
+        csync();
+      }
+    }
+    // a consumer that stopped early releases the copy-issuing lane and the grid
+    if (!run && tid == 0) {
+      *reinterpret_cast<volatile int*>(&ctl.abort) = 1;
+      atomicExch(&a.bar[2], 1u);
+    }
+  }
+  __syncthreads();
+  // the last CTA to leave resets the barrier counters for the next launch
+  if (tid == 0) {
+    __threadfence();
+    if (atomicAdd(&a.bar[1], 1u) == gridDim.x - 1) {
+      atomicExch(&a.bar[0], 0u);
+      atomicExch(&a.bar[2], 0u);
+      __threadfence();
+      atomicExch(&a.bar[1], 0u);
+    }
+  }
+}
+
+}  // namespace
+
+size_t draft_fused_smem_bytes(int ring_slots, int act_rows, int act_floats) {
+  return static_cast<size_t>(ring_slots) * kDfSlotBytes + static_cast<size_t>(act_rows) * act_floats * 4 +
+         static_cast<size_t>(kDfScratchFloats) * 4;
+}
+
+size_t draft_fused_static_smem() { return sizeof(DfCtl); }
+
+cudaError_t draft_fused_set_max_smem() {
+  return cudaFuncSetAttribute(draft_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(227 * 1024 - sizeof(DfCtl) - 64));
+}
+
+cudaError_t launch_draft_fused(const DraftFusedArgs& a, int grid, cudaStream_t s, bool cooperative) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kDfThreads);
+  cfg.dynamicSmemBytes = draft_fused_smem_bytes(a.ring_slots, 2 * a.B, a.act_floats);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = cooperative ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, draft_fused_kernel, a);
+}
+
+}  // namespace memspec

@@ -192,6 +192,62 @@ struct AcceptArgs {
   uint32_t* status;
 };
 
+// Fused draft step (draft_fused.cu): all K forward passes of a small draft and
+// their samples in one cooperative launch, one CTA per SM, grid-wide barriers
+// between the ops of a pass.  Rows: at most 2 per request (catch-up) and at most
+// kDfMaxGroups requests.
+constexpr int kDfMaxGroups = 4;
+constexpr int kDfMaxRows = 2 * kDfMaxGroups;
+constexpr int kDfSlotBytes = 8192;      // weight ring slot
+constexpr int kDfMaxSlots = 32;
+constexpr int kDfComputeWarps = 8;
+constexpr int kDfThreads = (kDfComputeWarps + 1) * 32;   // + one copy-issuing warp
+
+struct DraftFusedArgs {
+  const uint8_t* w;          // draft weight blob
+  // tensor offsets in the blob; per-layer tensors at off + layer * lstride
+  long long off_emb, off_attn_norm, off_wqkv, off_wo, off_ffn_norm, off_wgate, off_wdown,
+      off_final_norm, off_lm, lstride;
+  int tied;                  // LM head = row-major embedding
+  int n_layers, d, H, Hkv, hd, F, V;
+  float eps;
+  bf16* kv;                  // draft KV cache [layer][K|V][req][kv_head][pos][hd]
+  long long layer_kv;        // elements of one layer's K (or V) block
+  int max_seq, max_k;
+  const float* rope_cos;     // [max_seq][hd/2]
+  const float* rope_sin;
+  int K, B;                  // passes, requests
+  float inv_temp;            // 1/T (0: greedy)
+  int greedy;
+  const int* seq_state;      // [max_batch][kStateInts]
+  const int* draft_len;      // [max_batch] processed count of this draft
+  const int* tokens;         // [max_batch][max_seq]
+  int* draft_tokens;         // [max_batch][max_k]
+  const unsigned long long* seeds;
+  float* zd;                 // draft logits [B][K][V]
+  // scratch
+  float* h;                  // residual stream [kDfMaxRows][d]
+  float* qb;                 // rotated queries [kDfMaxRows][H * hd]
+  float* att;                // attention partials [kDfMaxRows][H][n_splits][hd + 4]
+  int* att_cnt;              // split arrivals [kDfMaxGroups][H], zero between phases
+  float* ao;                 // combined attention output [kDfMaxRows][H * hd]
+  float* act;                // SwiGLU output [kDfMaxRows][F]
+  float* lm_part;            // per-CTA LM-head statistics [B][grid][4]
+  unsigned int* bar;         // [0] barrier arrivals, [1] exits, [2] abort flag
+  uint32_t* status;
+  int n_splits;              // attention key splits per (request, head)
+  int ring_slots;            // weight ring slots of kDfSlotBytes
+  int act_floats;            // activation buffer (floats) per row in shared memory (rows: 2B)
+  unsigned long long* trace; // optional: {phases, grid, [phase][grid][16] globaltimer ns}: slot 0
+                             // phase start, 1 barrier arrival, 13 barrier passed
+  int trace_phases;          // phases the trace holds
+};
+size_t draft_fused_smem_bytes(int ring_slots, int act_rows, int act_floats);
+size_t draft_fused_static_smem();
+constexpr int kDfScratchFloatsHost = 2 * 256 + 2 * 128 + 2 * 256;   // == kDfScratchFloats
+cudaError_t draft_fused_set_max_smem();
+cudaError_t launch_draft_fused(const DraftFusedArgs& a, int grid, cudaStream_t s, bool cooperative);
+
 // launchers (each returns the launch's cudaError_t)
 cudaError_t launch_embed(const EmbedArgs& a, int rows, cudaStream_t s, bool pdl);
 cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s, bool pdl);

@@ -2,12 +2,12 @@
 // that must not allocate device memory.
 //
 // memspec_op_linear needs a caller-provided scratch buffer (split-K partial sums,
-// per-row-tile arrival counters).  Some callers cannot provide one: code that runs
-// while a CUDA graph is being captured (an allocation there is not allowed to be
-// part of the graph), plug-ins whose host application owns every byte of device
-// memory, and fixed-budget deployments where all allocation happens once at
-// start-up.  This entry point keeps that scratch in a file-scope device array of
-// fixed size instead, so a call allocates nothing.
+// per-row-tile arrival counters).  Some callers cannot provide one: plug-ins whose
+// host application owns every byte of device memory and hands out none,
+// fixed-budget deployments where all allocation happens once at start-up, and
+// latency-critical loops that cannot afford cudaMalloc / cudaFree (which may
+// synchronise the device).  This entry point keeps that scratch in a file-scope
+// device array of fixed size instead, so a call allocates nothing.
 //
 // Properties a user must know:
 //  * the array (kNoAllocScratchBytes, about 2.6 MB) exists on every GPU that
@@ -43,15 +43,16 @@ constexpr size_t kNoAllocScratchBytes = kPartialBytes + kCounterBytes + 256;
 // split-K partials | arrival counters | status word
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_setup_mutex;
-void* g_scratch_ptr[kMaxDevices] = {};
-int g_sm_count[kMaxDevices] = {};
-
 typedef CUresult (*EncodeFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                              const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
                              const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                              CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+constexpr int kMaxDevices = 64;
+std::mutex g_setup_mutex;            // guards everything below
+void* g_scratch_ptr[kMaxDevices] = {};
+int g_sm_count[kMaxDevices] = {};
+EncodeFn g_encode_fn = nullptr;      // driver entry point, looked up once
 
 bool encode(EncodeFn fn, CUtensorMap* map, const void* base, int rows, int cols, int box_rows) {
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
@@ -65,9 +66,22 @@ bool encode(EncodeFn fn, CUtensorMap* map, const void* base, int rows, int cols,
 
 // Per-device set-up, done once with the device current: the array's device
 // address (a host-side reference to the array is not a device address), the SM
-// count and the GEMM kernel's shared-memory limit.
-memspec_status setup_device(int dev, void** scratch, int* n_sm) {
+// count and the GEMM kernel's shared-memory limit; and, once per process, the
+// driver's tensor-map encoder.  All under one mutex, so first calls from
+// several host threads are safe.
+memspec_status setup_device(int dev, void** scratch, int* n_sm, EncodeFn* encode_fn) {
   std::lock_guard<std::mutex> lock(g_setup_mutex);
+  if (g_encode_fn == nullptr) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || p == nullptr) {
+      set_op_error("cuTensorMapEncodeTiled entry point not found");
+      return MEMSPEC_ERR_CUDA;
+    }
+    g_encode_fn = reinterpret_cast<EncodeFn>(p);
+  }
   if (g_scratch_ptr[dev] == nullptr) {
     void* p = nullptr;
     cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
@@ -91,6 +105,7 @@ memspec_status setup_device(int dev, void** scratch, int* n_sm) {
   }
   *scratch = g_scratch_ptr[dev];
   *n_sm = g_sm_count[dev];
+  *encode_fn = g_encode_fn;
   return MEMSPEC_OK;
 }
 
@@ -124,21 +139,9 @@ extern "C" memspec_status memspec_op_linear_noalloc(const void* x, const void* w
   }
   void* scratch = nullptr;
   int n_sm = 0;
-  memspec_status st = setup_device(dev, &scratch, &n_sm);
+  EncodeFn fn = nullptr;
+  memspec_status st = setup_device(dev, &scratch, &n_sm, &fn);
   if (st != MEMSPEC_OK) return st;
-
-  static EncodeFn fn = nullptr;
-  if (fn == nullptr) {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) != cudaSuccess ||
-        q != cudaDriverEntryPointSuccess) {
-      set_op_error("cuTensorMapEncodeTiled entry point not found");
-      return MEMSPEC_ERR_CUDA;
-    }
-    fn = reinterpret_cast<EncodeFn>(p);
-  }
   GemmArgs a{};
   const int n_pad = 16;
   if (!encode(fn, &a.map_a, w, n_out, k, 128) || !encode(fn, &a.map_b, x, rows, k, n_pad)) {
@@ -162,7 +165,11 @@ extern "C" memspec_status memspec_op_linear_noalloc(const void* x, const void* w
   uint32_t* own_status = reinterpret_cast<uint32_t*>(sb + kPartialBytes + kCounterBytes);
   a.status = status != nullptr ? status : own_status;
   a.plan = nullptr;
-  // same stream-K grid rule as memspec_op_linear, capped by the fixed scratch
+  // Stream-K grid: at most one CTA per SM and at most four contributors per row
+  // tile, capped by the fixed scratch (kNoAllocMaxCtas).  Unlike memspec_op_linear
+  // it keeps no SMs spare and reads no tuning variables, so its split-K summation
+  // order can differ: results agree with memspec_op_linear within rounding, not
+  // bit for bit.
   const int T = a.row_tiles * a.k_tiles;
   const int min_tiles = (a.k_tiles + 3) / 4 > 0 ? (a.k_tiles + 3) / 4 : 1;
   int grid = T;

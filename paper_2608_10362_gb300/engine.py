@@ -133,11 +133,13 @@ class Engine:
     def __init__(self, target_shape, target_weights, *, max_batch: int = 1, max_seq: int = 1024,
                  max_k: int = 8, max_drafts: int = 4, draft_shape_max=None,
                  draft_budget_bytes: int = 0, use_graphs: bool = True,
-                 launch_mode: str = "per_op", trace=None, device: int = 0):
+                 launch_mode: str = "per_op", trace=None, device: int = 0,
+                 draft_kernel: str = "auto"):
         """launch_mode "per_op": one kernel launch per op of a pass; "pass": each
         draft step and verify pass as one persistent launch.  ``trace``
         ("verify", "draft" or "prefill") records per-op timestamps of that pass, see
-        ``pass_trace``."""
+        ``pass_trace``.  draft_kernel ("auto", "per_op", "fused") picks the kernels
+        of the per-op draft step, see memspec_init_params.draft_kernel."""
         if launch_mode not in ("per_op", "pass"):
             raise ValueError(f"launch_mode must be 'per_op' or 'pass', not {launch_mode!r}")
         self.lib = _lib.load()
@@ -170,6 +172,11 @@ class Engine:
         if trace not in (None, "verify", "draft", "prefill"):
             raise ValueError(f"trace must be None, 'verify', 'draft' or 'prefill', not {trace!r}")
         p.trace = {None: 0, "verify": 1, "draft": 2, "prefill": 3}[trace]
+        kinds = {"auto": _lib.DRAFT_KERNEL_AUTO, "per_op": _lib.DRAFT_KERNEL_PER_OP,
+                 "fused": _lib.DRAFT_KERNEL_FUSED}
+        if draft_kernel not in kinds:
+            raise ValueError(f"draft_kernel must be one of {sorted(kinds)}, not {draft_kernel!r}")
+        p.draft_kernel = kinds[draft_kernel]
         self.params = p
         n = C.c_size_t()
         _check(self.lib, self.lib.memspec_workspace_bytes(C.byref(p), C.byref(n)))
@@ -261,6 +268,16 @@ class Engine:
         self.accept_commit(K, temperature, results)
 
     # -------------------------------------------------------------- inspection
+    def info(self, what: int) -> int:
+        v = C.c_int64()
+        self._call(self.lib.memspec_query_info, what, C.byref(v))
+        return v.value
+
+    def launches_per_step(self) -> int:
+        """Kernel launches of the last draft step + verify pass + acceptance."""
+        return sum(self.info(w) for w in (_lib.INFO_DRAFT_LAUNCHES, _lib.INFO_VERIFY_LAUNCHES,
+                                          _lib.INFO_ACCEPT_LAUNCHES))
+
     def read_buffer(self, buf: int, dtype, count: int) -> np.ndarray:
         out = np.empty(count, dtype=dtype)
         self._call(self.lib.memspec_read_buffer, buf, out.ctypes.data, out.nbytes)
@@ -333,17 +350,23 @@ def op_linear(x: torch.Tensor, w: torch.Tensor, scratch: torch.Tensor | None = N
     return y
 
 
-def op_linear_noalloc(x: torch.Tensor, w: torch.Tensor,
+def op_linear_noalloc(x: torch.Tensor, w: torch.Tensor, y: torch.Tensor | None = None,
+                      status: torch.Tensor | None = None,
                       stream: torch.cuda.Stream | None = None) -> torch.Tensor:
     """y = x . w^T through memspec_op_linear_noalloc (no scratch argument; the
-    library's fixed device array is used).  rows <= 16."""
+    library's fixed device array is used).  rows <= 16.  ``y`` (fp32 [rows][n_out])
+    may be given so that the call itself allocates nothing; ``status`` (one
+    int32/uint32 on the device) receives the kernel's error bits."""
     lib = _lib.load()
     rows, k = x.shape
     n_out = w.shape[0]
-    y = torch.empty(rows, n_out, dtype=torch.float32, device=x.device)
+    if y is None:
+        y = torch.empty(rows, n_out, dtype=torch.float32, device=x.device)
     s = stream or torch.cuda.current_stream(x.device)
     _check(lib, lib.memspec_op_linear_noalloc(x.data_ptr(), w.data_ptr(), y.data_ptr(), rows,
-                                              n_out, k, None, s.cuda_stream))
+                                              n_out, k,
+                                              None if status is None else status.data_ptr(),
+                                              s.cuda_stream))
     return y
 
 

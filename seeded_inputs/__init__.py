@@ -25,7 +25,7 @@ import numpy as np
 __all__ = [
     "ModelShape", "SHAPES", "tensor_names", "tensor_shape", "gen_tensor",
     "iter_weights", "gen_weights", "gen_prompt", "gen_logits", "gen_kv",
-    "bf16_round",
+    "bf16_round", "gen_score_stream",
 ]
 
 
@@ -176,3 +176,21 @@ def gen_kv(seed: int, shape_tuple, scale: float = 1.0) -> np.ndarray:
     rng = np.random.default_rng([seed, 0x6B76])
     return bf16_round(rng.standard_normal(int(np.prod(shape_tuple)), dtype=np.float32)
                       * np.float32(scale)).reshape(shape_tuple)
+
+
+def gen_score_stream(seed: int, points: int, n_drafts: int, phase: int = 4,
+                     noise: float = 0.15) -> np.ndarray:
+    """float32 [points][n_drafts] per-draft scores standing in for a draft
+    predictor's output at successive scheduling points: a seeded "best draft"
+    that changes every ``phase`` points (random phase boundaries), scored 1.0,
+    the others uniform in [0, 0.8), plus N(0, noise^2) jitter."""
+    rng = np.random.default_rng([seed, 0x73636F72])
+    out = np.empty((points, n_drafts), dtype=np.float32)
+    best = int(rng.integers(0, n_drafts))
+    for i in range(points):
+        if i % phase == 0 and rng.random() < 0.8:
+            best = int(rng.integers(0, n_drafts))
+        row = rng.random(n_drafts) * 0.8
+        row[best] = 1.0
+        out[i] = (row + rng.standard_normal(n_drafts) * noise).astype(np.float32)
+    return out

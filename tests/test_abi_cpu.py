@@ -11,7 +11,7 @@ import numpy as np
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-HEADERS = [os.path.join(ROOT, "include", h) for h in ("memspec.h", "memspec_ops.h")]
+HEADERS = [os.path.join(ROOT, "include", h) for h in ("memspec.h", "memspec_ops.h", "memspec_sched.h")]
 
 pytestmark = pytest.mark.skipif(shutil.which("nvcc") is None and
                                 not os.path.exists("/usr/local/cuda/bin/nvcc"),

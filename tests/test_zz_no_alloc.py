@@ -1,12 +1,15 @@
 """The GEMM entry point that allocates nothing (memspec_op_linear_noalloc).
 
-It exists for callers that cannot allocate device memory (code running under
-CUDA-graph capture, plug-ins whose host owns all device memory, fixed-budget
-deployments): its split-K scratch is a fixed device array inside the library.
-These tests check that it gives the same results as memspec_op_linear, on two
-calls in a row (the array keeps the previous call's contents), and that sizes
-beyond its fixed scratch are refused before anything runs.  This file is
-collected last on purpose.
+Some callers cannot allocate device memory: plug-ins whose host application
+owns all of it, fixed-budget deployments that allocate only at start-up, and
+latency-critical loops that cannot afford cudaMalloc.  For them the library
+keeps this GEMM's split-K scratch in a fixed device array of its own.  These
+tests check, through the C ABI, that two calls in a row (the array keeps the
+previous call's contents) give y = x . w^T within the GEMM tolerance of the
+fp64 matmul of the same bf16 inputs, agree with memspec_op_linear within that
+tolerance, leave the error word at zero, and that sizes beyond the fixed
+scratch are refused before anything runs.  This file is collected last on
+purpose.
 """
 import ctypes as C
 
@@ -26,17 +29,28 @@ def _pair(seed, rows, n_out, k):
 
 @pytest.mark.gpu
 @pytest.mark.parametrize("rows,n_out,k", [(1, 256, 128), (5, 4096, 4096), (16, 688, 256),
-                                          (9, 32000, 768), (3, 2560, 2048)])
-def test_noalloc_linear_matches_op_linear_twice(rows, n_out, k):
+                                          (9, 32000, 768), (3, 2560, 2048), (2, 130, 72)])
+def test_noalloc_linear_matches_fp64_matmul_twice(rows, n_out, k):
     from paper_2608_10362_gb300 import op_linear, op_linear_noalloc
     x, w = _pair(7, rows, n_out, k)
     xt = torch.from_numpy(x).to(torch.bfloat16).cuda()
     wt = torch.from_numpy(w).to(torch.bfloat16).cuda()
-    ref = op_linear(xt, wt).cpu().numpy().astype(np.float64)
+    ref = x.astype(np.float64) @ w.astype(np.float64).T
+    # fp32 accumulation of exact bf16 products: |y - ref| <= 1e-4 * sum_k |x_k w_k|
     bound = np.abs(x).astype(np.float64) @ np.abs(w).astype(np.float64).T
-    for _ in range(2):
-        y = op_linear_noalloc(xt, wt).cpu().numpy().astype(np.float64)
-        assert np.all(np.abs(y - ref) <= 1e-4 * bound + 1e-6), np.abs(y - ref).max()
+    other = op_linear(xt, wt).cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(other - ref) <= 1e-4 * bound + 1e-6)
+    y = torch.empty(rows, n_out, dtype=torch.float32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for call in range(2):
+        y.fill_(float("nan"))                 # every output element must be written
+        op_linear_noalloc(xt, wt, y=y, status=status)
+        torch.cuda.synchronize()
+        assert int(status.item()) == 0, f"call {call}: device error bits {int(status.item()):#x}"
+        got = y.cpu().numpy().astype(np.float64)
+        assert np.all(np.isfinite(got)), call
+        assert np.all(np.abs(got - ref) <= 1e-4 * bound + 1e-6), (call, np.abs(got - ref).max())
+        assert np.all(np.abs(got - other) <= 2e-4 * bound + 2e-6), call
 
 
 def test_noalloc_linear_refuses_sizes_beyond_its_scratch():
