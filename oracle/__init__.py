@@ -14,7 +14,8 @@ What it restates, and where it comes from:
 * ``llama``   - the Llama-style decoder used as target and draft (MemSpec
   Section 4.1 evaluates LLaMA-2-7B / Qwen2.5-7B targets with small drafts):
   RMSNorm, rotary position embedding, causal grouped-query attention over a
-  KV cache, SwiGLU feed-forward, LM head.
+  KV cache that holds bf16 values (the workload's KV precision), SwiGLU
+  feed-forward, LM head.
 * ``speculative`` - the draft-and-verify iteration that MemSpec runs unchanged
   (Section 3.5: "the standard draft-and-verify process"; Section 2.1, Eq. 1:
   throughput ~ E[A] / L_iter), with the acceptance rule of the speculative
@@ -24,7 +25,8 @@ What it restates, and where it comes from:
   draft token is accepted, draw one more token from the target.
 
 Pins (tests/test_oracle_*.py, run with ``-m "not gpu"``): Philox known-answer
-vectors; attention / RMSNorm / SiLU against PyTorch library routines; RoPE
+vectors; bf16 rounding of the KV cache against hand-worked ties and PyTorch's
+conversion; attention / RMSNorm / SiLU against PyTorch library routines; RoPE
 closed forms; KV-cached decoding equals full recomputation; causality;
 greedy speculative output equals greedy target-only output; a draft equal to
 the target accepts every token; emitted tokens follow the target

@@ -17,13 +17,25 @@ x_1..x_K] against the target's KV cache (Section 2.1, Eq. 1 context; Section
     logits = (RMSNorm(h) * g_final) Wlm^T
 
 Weights arrive as float32 arrays holding bf16 values (exactly representable) and
-are used in float64.  All arithmetic is float64.
+are used in float64.  All arithmetic is float64; the one rounding step is the
+KV cache, which stores K and V as bf16 values (the workload fixes bf16 weights
+and KV cache), so every attention reads bf16 keys and values, the rows just
+appended included.
 """
 from __future__ import annotations
 
 import numpy as np
 
 LAYER_TENSORS = ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate", "w_up", "w_down")
+
+
+def bf16(x: np.ndarray) -> np.ndarray:
+    """Round to the nearest bfloat16 value (8 significant bits, ties to even),
+    float64 in and out: with x = m 2^e, 0.5 <= |m| < 1, the quantum is 2^(e-8)."""
+    x = np.asarray(x, dtype=np.float64)
+    _, e = np.frexp(x)
+    q = np.ldexp(1.0, e - 8)
+    return np.round(x / q) * q          # numpy rounds halves to even
 
 
 def rmsnorm(x: np.ndarray, gain: np.ndarray, eps: float) -> np.ndarray:
@@ -83,7 +95,8 @@ def attention(q: np.ndarray, k_cache: np.ndarray, v_cache: np.ndarray,
 
 
 class KVCache:
-    """Per-layer float64 K and V for positions 0..length-1 (rotated keys)."""
+    """Per-layer K and V for positions 0..length-1 (rotated keys), bf16 values
+    held in float64."""
 
     def __init__(self, n_layers: int, n_kv_heads: int, head_dim: int, capacity: int):
         self.k = np.zeros((n_layers, capacity, n_kv_heads, head_dim))
@@ -138,8 +151,8 @@ class LlamaOracle:
         q = apply_rope(q, positions, s.rope_base)
         k = apply_rope(k, positions, s.rope_base)
         start = int(positions[0])
-        cache.k[li, start:start + M] = k
-        cache.v[li, start:start + M] = v
+        cache.k[li, start:start + M] = bf16(k)
+        cache.v[li, start:start + M] = bf16(v)
         end = start + M
         o = attention(q, cache.k[li, :end], cache.v[li, :end], positions)
         h = h + self._lin(o.reshape(M, s.q_dim), "wo", li)

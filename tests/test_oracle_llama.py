@@ -106,6 +106,9 @@ def _torch_layer(shape, w, li, h, positions):
     rot = lambda x: torch.cat([x[..., :half] * cos - x[..., half:] * sin,
                                x[..., :half] * sin + x[..., half:] * cos], dim=-1)
     q, k = rot(q), rot(k)
+    # the KV cache holds bf16 values: PyTorch's own conversion
+    k = k.to(torch.bfloat16).to(torch.float64)
+    v = v.to(torch.bfloat16).to(torch.float64)
     g = s.n_heads // s.n_kv_heads
     kk = k.repeat_interleave(g, dim=1).permute(1, 0, 2)
     vv = v.repeat_interleave(g, dim=1).permute(1, 0, 2)
@@ -113,6 +116,22 @@ def _torch_layer(shape, w, li, h, positions):
     h = h + F.linear(o.permute(1, 0, 2).reshape(M, -1), W("wo"))
     m = F.rms_norm(h, (s.d_model,), weight=W("ffn_norm"), eps=s.norm_eps)
     return (h + F.linear(F.silu(F.linear(m, W("w_gate"))) * F.linear(m, W("w_up")), W("w_down"))).numpy()
+
+
+def test_bf16_rounding_of_the_kv_cache():
+    from oracle.llama import bf16
+    # values on the bf16 grid are kept; halfway cases go to the even neighbour
+    grid = np.array([0.0, 1.0, -1.0, 1.0 + 2.0 ** -7, 3.0 * 2.0 ** -20, -255.0 * 2.0 ** 10])
+    np.testing.assert_array_equal(bf16(grid), grid)
+    ties = np.array([1.0 + 2.0 ** -8, 1.0 + 3.0 * 2.0 ** -8, -(2.0 + 2.0 ** -7), 0.5 + 2.0 ** -10])
+    np.testing.assert_array_equal(bf16(ties), [1.0, 1.0 + 2.0 ** -6, -2.0, 0.5])
+    np.testing.assert_array_equal(bf16(1.0 + 2.0 ** -8 + 2.0 ** -30), 1.0 + 2.0 ** -7)
+    # PyTorch's conversion agrees on values float32 holds exactly
+    x = np.random.default_rng(2).standard_normal(20000).astype(np.float32).astype(np.float64) * 3.0
+    ref = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(bf16(x), ref)
+    # the rounding error is at most half a quantum: 2^-8 relative (unit roundoff)
+    assert np.all(np.abs(bf16(x) - x) <= np.abs(x) * 2.0 ** -8)
 
 
 @pytest.mark.parametrize("shape", [GQA, SHAPES["tiny_draft"]])
