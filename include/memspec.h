@@ -115,7 +115,8 @@ typedef enum memspec_tensor {
   MEMSPEC_T_LM_HEAD = 9
 } memspec_tensor;
 
-/* Total blob bytes for cfg.  Errors: INVALID_ARG (null / bad cfg). */
+/* Total blob bytes for cfg.  The blob layout is this library's (the paper
+ * prescribes none).  Errors: INVALID_ARG (null / bad cfg). */
 memspec_status memspec_weights_bytes(const memspec_model_cfg* cfg, size_t* bytes);
 
 /* Byte offset and size of one tensor inside the blob.  layer is ignored for
@@ -173,27 +174,33 @@ typedef struct memspec_init_params {
 enum { MEMSPEC_LAUNCH_PER_OP = 0, MEMSPEC_LAUNCH_PASS = 1 };
 enum { MEMSPEC_DRAFT_KERNEL_AUTO = 0, MEMSPEC_DRAFT_KERNEL_PER_OP = 1, MEMSPEC_DRAFT_KERNEL_FUSED = 2 };
 
-/* Device workspace bytes memspec_init needs for these params. */
+/* Device workspace bytes memspec_init needs for these params (all device memory
+ * is the caller's; the paper has no counterpart).  Errors: INVALID_ARG,
+ * UNSUPPORTED. */
 memspec_status memspec_workspace_bytes(const memspec_init_params* p, size_t* bytes);
 
-/* Create a context.  workspace_dev: device memory of memspec_workspace_bytes
+/* Create a context: the target model is loaded once and stays resident
+ * (Section 3.4, Algorithm 3: "load target model" before the runtime loop).
+ * workspace_dev: device memory of memspec_workspace_bytes
  * bytes, 256-byte aligned, caller-owned, untouched by the caller afterwards.
  * Builds TMA descriptors for the target weights.  Errors: INVALID_ARG,
  * UNSUPPORTED (shape), CUDA. */
 memspec_status memspec_init(const memspec_init_params* p, void* workspace_dev,
                             memspec_ctx** out);
 
-/* Release host-side resources (graphs, events).  Does not free caller memory. */
+/* Release host-side resources (graphs, events).  Does not free caller memory.
+ * (Library lifetime; no counterpart in the paper.) */
 void memspec_destroy(memspec_ctx* ctx);
 
-/* Message describing the last error of this context (never NULL). */
+/* Message describing the last error of this context (never NULL; no counterpart
+ * in the paper). */
 const char* memspec_last_error(const memspec_ctx* ctx);
 
 /* ---- drafts (Section 3.3: candidate set D, resident set G under a budget) --*/
 
-/* Register draft draft_id with its weights in pinned host memory (the backing
- * tier) and its own device KV cache (memspec_kv_bytes(cfg, max_batch,
- * max_seq)).  The host blob must stay valid while the draft is registered.
+/* Register draft draft_id of the candidate set D (Section 3.1) with its weights
+ * in pinned host memory - the backing storage tier of Section 3.3 - and its own
+ * device KV cache (memspec_kv_bytes(cfg, max_batch, max_seq)).  The host blob must stay valid while the draft is registered.
  * Errors: INVALID_ARG, UNSUPPORTED, BUSY (id already registered). */
 memspec_status memspec_register_draft(memspec_ctx* ctx, int32_t draft_id,
                                       const memspec_model_cfg* cfg,
@@ -201,22 +208,30 @@ memspec_status memspec_register_draft(memspec_ctx* ctx, int32_t draft_id,
                                       void* kv_dev);
 
 /* Start copying draft_id's weights into the arena on the side stream
- * (non-blocking).  Places the draft first-fit in the arena.  If it does not
+ * (non-blocking): Algorithm 2's "asynchronously prefetch d" (Section 3.3), the
+ * load overlapped with decoding (Section 3.5).  Places the draft first-fit in the arena.  If it does not
  * fit, returns MEMSPEC_ERR_BUDGET and changes nothing: the caller chooses what
  * to evict (the active draft is never evicted implicitly).  Already resident
  * or loading: returns OK.  *slot_offset (optional) receives the arena offset. */
 memspec_status memspec_load_draft_async(memspec_ctx* ctx, int32_t draft_id,
                                         size_t* slot_offset);
 
-/* *state: 0 = not resident, 1 = resident, 2 = loading (copy in flight). */
+/* *state: 0 = not resident, 1 = resident, 2 = loading (copy in flight): the
+ * residency state and prefetch status each draft keeps (Section 3.5).
+ * Errors: INVALID_ARG (unregistered id), CUDA. */
 memspec_status memspec_query_draft(memspec_ctx* ctx, int32_t draft_id, int32_t* state);
 
-/* Drop draft_id from the arena.  Refuses (BUSY) while its copy is in flight
- * or while it is the active draft (the draft of the last draft step that has
+/* Drop draft_id from the arena: Algorithm 2's "evict d_evict" (Section 3.3),
+ * which never evicts the active draft d_i.  Refuses (BUSY) while its copy is in
+ * flight or while it is the active draft (the draft of the last draft step that has
  * not been followed by memspec_set_active_draft to another draft). */
 memspec_status memspec_evict_draft(memspec_ctx* ctx, int32_t draft_id);
 
-/* Make draft_id the active draft.  It must be resident or loading (a loading
+/* Make draft_id the active draft d_i of the next interval (Section 3.4,
+ * Algorithm 3: the best resident draft is selected at each scheduling point).
+ * draft_id = -1 leaves no draft active (then any draft may be evicted and draft
+ * steps return NOT_RESIDENT until a draft is made active again).
+ * It must be resident or loading (a loading
  * draft makes the next draft step wait on the GPU, never on the host).  The
  * new draft's KV cache is brought up to date with the committed tokens by a
  * chunked prefill on the main stream (host-synchronising: it reads the
@@ -225,7 +240,9 @@ memspec_status memspec_set_active_draft(memspec_ctx* ctx, int32_t draft_id);
 
 /* ---- requests ----------------------------------------------------------- */
 
-/* Start request req with prompt tokens_host[0..n) (n >= 1) and Philox seed:
+/* Start request req with prompt tokens_host[0..n) (n >= 1) and Philox seed (the
+ * prompt that precedes the runtime loop of Algorithm 3; its prefill is excluded
+ * from steady-state throughput, Section 4.1):
  * copies the prompt, runs the target and the active draft over all prompt
  * tokens but the last (chunks of up to 128 rows), and resets the request's
  * iteration counter.  Host-synchronising.  Errors: INVALID_ARG, CUDA. */
@@ -233,23 +250,30 @@ memspec_status memspec_prefill(memspec_ctx* ctx, int32_t req, const int32_t* tok
                                int32_t n, uint64_t seed);
 
 /* Number of requests stepped together by the step calls (1..max_batch). All
- * of them must have been prefilled. */
+ * of them must have been prefilled.  (Batching is this library's; the paper
+ * evaluates batch 1.)  Errors: INVALID_ARG. */
 memspec_status memspec_set_batch(memspec_ctx* ctx, int32_t batch);
 
 /* ---- the draft-then-verify step ----------------------------------------- */
 
-/* The active draft proposes x_1..x_K for every request: K forward passes of
+/* Algorithm 3 "run draft d_i" (Section 3.4) - the draft half of the standard
+ * draft-and-verify iteration (Section 2.1, Eq. 1; Section 3.5).
+ * The active draft proposes x_1..x_K for every request: K forward passes of
  * one position each (two for the first pass after a fully accepted step),
  * each followed by sampling x_j ~ softmax(z/T) with Philox uniform slot j-1
  * (T == 0: argmax).  Draft logits are kept for acceptance.  Enqueue only. */
 memspec_status memspec_draft_step(memspec_ctx* ctx, int32_t K, float temperature);
 
-/* One target pass over [t_{L-1}, x_1..x_K] at positions L-1..L-1+K per request,
+/* Algorithm 3 "verify with target model" (Section 3.4; Section 2.1).
+ * One target pass over [t_{L-1}, x_1..x_K] at positions L-1..L-1+K per request,
  * appending their K,V to the target cache and writing fp32 logits for
  * positions L..L+K.  Enqueue only. */
 memspec_status memspec_verify_step(memspec_ctx* ctx, int32_t K);
 
-/* Acceptance, resampling and commit for every request (see the file header):
+/* The accept step of the draft-and-verify iteration (Section 3.5; the
+ * speculative sampling rule the paper cites in Section 1), which yields the
+ * accepted count A of Eq. 1.
+ * Acceptance, resampling and commit for every request (see the file header):
  * n accepted tokens, the correction/bonus token y, L += n + 1, KV rollback by
  * length (target KV valid below L-1; draft KV below L-1, or L-2 when n = K).
  * If results_host_pinned is not NULL, an async copy of int32
@@ -257,7 +281,8 @@ memspec_status memspec_verify_step(memspec_ctx* ctx, int32_t K);
 memspec_status memspec_accept_commit(memspec_ctx* ctx, int32_t K, float temperature,
                                      int32_t* results_host_pinned);
 
-/* Wait for the main stream (timeout_ms < 0: no limit) and return the device
+/* Host synchronisation (no counterpart in the paper).
+ * Wait for the main stream (timeout_ms < 0: no limit) and return the device
  * status word as MEMSPEC_ERR_DEVICE_STATUS if any bit is set (the word is then
  * cleared; *bits, if given, receives it).  Errors: TIMEOUT, CUDA. */
 memspec_status memspec_sync(memspec_ctx* ctx, int32_t timeout_ms, uint32_t* bits);

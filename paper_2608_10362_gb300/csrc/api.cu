@@ -64,6 +64,22 @@ bool encode_map(CUtensorMap* map, const void* base, int rows, int cols, int box_
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D bf16 tensor map, no swizzle (the bytes are copied as stored), zero fill
+// out of bounds: dims {d0, d1, d2} elements, strides of dims 1 and 2 in bytes,
+// box {b0, b1, b2}.
+bool encode_box3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                  uint64_t s1, uint64_t s2, uint32_t b0, uint32_t b1, uint32_t b2) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (fn == nullptr || (reinterpret_cast<uintptr_t>(base) & 15) != 0 || s1 % 16 || s2 % 16) return false;
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {s1, s2};
+  cuuint32_t box[3] = {b0, b1, b2};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 int round_up(int x, int m) { return (x + m - 1) / m * m; }
 int ceil_div(int a, int b) { return (a + b - 1) / b; }
@@ -267,6 +283,9 @@ struct DraftRec {
   cudaEvent_t ev = nullptr;
   ModelRT rt;
   int* d_len = nullptr;  // device [max_batch]
+  // TMA boxes of the fused draft kernel (host copy, and the weights they were built for)
+  std::vector<CUtensorMap> df_maps;
+  const uint8_t* df_maps_for = nullptr;
 };
 
 struct GraphKey {
@@ -346,6 +365,7 @@ struct memspec_ctx {
   float* df_lm = nullptr;
   unsigned int* df_bar = nullptr;
   int* df_cnt = nullptr;
+  CUtensorMap* df_maps = nullptr;   // [kMaxDrafts][kDfMapsPerDraft], 64-byte aligned
   bool df_coop = true;       // cooperative launch attribute (cleared if capture refuses it)
   std::map<std::tuple<const void*, int, int, int>, CUtensorMap> bmaps;
 };
@@ -451,6 +471,7 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   const size_t o_dfl = w.take(static_cast<size_t>(kDfMaxGroups) * nsm * 4 * 4);
   const size_t o_dfb = w.take(64);
   const size_t o_dfc = w.take(static_cast<size_t>(kDfMaxGroups) * (has_draft ? dm.n_heads : 1) * 4);
+  const size_t o_dfm = w.take(has_draft ? static_cast<size_t>(kMaxDrafts) * kDfMapsPerDraft * sizeof(CUtensorMap) : 0);
   const size_t o_ops = w.take(op_bytes);
   const size_t o_done = w.take(done_ints * 4);
   const size_t trace_bytes =
@@ -500,6 +521,7 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
     c->df_lm = reinterpret_cast<float*>(base + o_dfl);
     c->df_bar = reinterpret_cast<unsigned int*>(base + o_dfb);
     c->df_cnt = reinterpret_cast<int*>(base + o_dfc);
+    c->df_maps = has_draft ? reinterpret_cast<CUtensorMap*>(base + o_dfm) : nullptr;
     c->op_area = base + o_ops;
     c->op_area_bytes = op_bytes;
     c->done_area = reinterpret_cast<int*>(base + o_done);
@@ -1217,7 +1239,47 @@ bool fused_draft_plan(memspec_ctx* c, DraftRec& dr, int K, float T, DraftFusedAr
         return false;
       }
   }
+  if (m.n_layers > kDfMaxLayers || c->df_maps == nullptr) {
+    *why = "more than 32 layers";
+    return false;
+  }
+  // TMA boxes over this draft's weights where they are now (rebuilt after a move)
+  const int id = static_cast<int>(&dr - c->drafts);
+  CUtensorMap* dev_maps = c->df_maps + static_cast<size_t>(id) * kDfMapsPerDraft;
+  if (dr.df_maps_for != dr.rt.w) {
+    dr.df_maps.assign(kDfMapsPerDraft, CUtensorMap{});
+    const int d = m.d_model, q = m.n_heads * m.head_dim, kv = m.n_kv_heads * m.head_dim, F = m.d_ffn;
+    auto packed = [&](CUtensorMap* mp, size_t off, long long n, long long k, bool pair, uint32_t rows,
+                      uint32_t tiles) {
+      const uint64_t nt = packed_bytes(n, k, pair) / kPackTileBytes;
+      return encode_box3d(mp, dr.rt.w + off, 64, 128, nt, 128, kPackTileBytes, 64, rows, tiles);
+    };
+    bool ok = true;
+    for (int l = 0; l < m.n_layers && ok; ++l) {
+      CUtensorMap* mp = dr.df_maps.data() + l * 4;
+      ok = packed(mp + 0, lay.wqkv[l], q + 2 * kv, d, false, 4, 8) &&
+           packed(mp + 1, lay.wo[l], d, q, false, 8, 8) && packed(mp + 2, lay.wgate[l], F, d, true, 8, 4) &&
+           packed(mp + 3, lay.wdown[l], d, F, false, 8, 8);
+    }
+    CUtensorMap* lm = dr.df_maps.data() + m.n_layers * 4;
+    if (ok)
+      ok = m.tied_embeddings
+               ? encode_box3d(lm, dr.rt.w + lay.lm_head, static_cast<uint64_t>(d), static_cast<uint64_t>(m.vocab), 1,
+                              static_cast<uint64_t>(d) * 2, static_cast<uint64_t>(d) * 2 * m.vocab, 256, 8, 1)
+               : packed(lm, lay.lm_head, m.vocab, d, false, 8, 8);
+    if (!ok) {
+      *why = "tensor map encoding";
+      return false;
+    }
+    if (cudaMemcpyAsync(dev_maps, dr.df_maps.data(), kDfMapsPerDraft * sizeof(CUtensorMap),
+                        cudaMemcpyHostToDevice, c->main) != cudaSuccess) {
+      *why = "tensor map copy";
+      return false;
+    }
+    dr.df_maps_for = dr.rt.w;
+  }
   DraftFusedArgs& a = *out;
+  a.maps = dev_maps;
   a.w = dr.rt.w;
   a.off_emb = static_cast<long long>(lay.emb);
   a.off_attn_norm = static_cast<long long>(lay.attn_norm[0]);
@@ -1575,6 +1637,10 @@ memspec_status memspec_evict_draft(memspec_ctx* c, int32_t id) {
 
 memspec_status memspec_set_active_draft(memspec_ctx* c, int32_t id) {
   if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (id == -1) {   // no active draft: every draft may be evicted; draft steps are refused
+    c->active = -1;
+    return MEMSPEC_OK;
+  }
   if (id < 0 || id >= c->p.max_drafts || !c->drafts[id].registered)
     return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown draft id");
   DraftRec& d = c->drafts[id];

@@ -16,9 +16,10 @@
 //    pair), assigned round-robin to CTAs; each CTA computes its units' full dot
 //    products (no split-K, no partial sums) on CUDA cores, with fp32 activations
 //    and bf16 weights;
-//  * one copy-issuing warp streams the CTA's weight bytes of every op of every
+//  * one copy-issuing lane streams the CTA's weight bytes of every op of every
 //    pass, in the order the compute warps consume them, into a ring of 8 KB
-//    shared-memory slots with 1-D bulk copies (cp.async.bulk) signalled on
+//    shared-memory slots, each slot one or two multi-dimensional TMA boxes over
+//    the packed tiles (8 rows x 64 columns x up to 8 k tiles), signalled on
 //    mbarriers.  The weights do not depend on activations, so the ring fills
 //    ahead across op and pass boundaries while the compute warps wait at grid
 //    barriers;
@@ -48,9 +49,9 @@ constexpr int kCW = kDfComputeWarps;
 constexpr int kCT = kCW * 32;              // compute threads
 constexpr int kUR = 8;                     // output rows per unit
 constexpr int kKeyBlock = kCT;             // keys per attention block (one per thread)
-// attention scores (2 rows), queries (2 x hd <= 128), key-group partials; the O
-// phase reuses it for the split weights (rows x H x n_splits)
-constexpr int kDfScratchFloats = 2 * kKeyBlock + 2 * 128 + 2 * kCT;
+// attention scores (2 rows), queries (2 x hd <= 128), per-warp o partials
+// [warps][2][hd <= 128]
+constexpr int kDfScratchFloats = 2 * kKeyBlock + 2 * 128 + kCW * 2 * 128;
 
 enum DfOp { OP_QKV = 0, OP_O = 1, OP_GU = 2, OP_DOWN = 3, OP_LM = 4 };
 
@@ -88,6 +89,16 @@ __device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
 }
 __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+// One TMA request per box: a slot is fetched by one or two requests (a request
+// costs about as much as its bytes only from several KB up, measured).
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
+                                            uint64_t* bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_addr(bar)), "l"(pol)
+      : "memory");
 }
 __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
@@ -142,74 +153,62 @@ __device__ __forceinline__ int lm_lo(const Geo& g, int c) {
   return static_cast<int>(static_cast<long long>(c) * g.u_lm / g.G);
 }
 
-// Issue the copies of slot `s` of unit `u` of op `op` (layer `l`) into `dst`,
-// completing on `bar`.  Returns the bytes.
+// Issue the TMA requests of slot `s` of unit `u` of op `op` (layer `l`) into
+// `dst` (one elected lane); returns the bytes they complete.  Shared-memory
+// image of a slot (128-byte rows exactly as packed, swizzle included):
+//   O, DOWN, packed LM: [8 k tiles][8 rows][128 B]            (one request)
+//   QKV:  rows r_lo.. then r_hi..: 2 x [8 k tiles][4 rows][128 B]
+//   GU:   gate rows then up rows:  2 x [4 k tiles][8 rows][128 B]
+//   tied LM (row-major embedding): 2 x [8 rows][256 columns]
 __device__ uint32_t issue_slot(const DraftFusedArgs& a, const Geo& g, int op, int l, int u, int s,
-                               uint8_t* dst, uint64_t* bar, uint64_t pol, bool go) {
-  constexpr uint32_t kTile = kPackTileBytes;
-  uint32_t bytes = 0;
-  auto copy = [&](uint8_t* d, const uint8_t* src, uint32_t n) {
-    if (go) bulk_load(d, src, n, bar, pol);
-    bytes += n;
-  };
+                               uint8_t* dst, uint64_t* bar, uint64_t pol) {
+  const CUtensorMap* maps = a.maps + static_cast<size_t>(l) * 4;
   if (op == OP_QKV) {
-    const uint8_t* base = a.w + a.off_wqkv + static_cast<long long>(l) * a.lstride;
     const int hb = u / (a.hd / kUR), ui = u - hb * (a.hd / kUR);
     const int r_lo = hb * a.hd + 4 * ui, r_hi = r_lo + a.hd / 2;
-    const int kt0 = s * 8, kt1 = min(kt0 + 8, g.kt_d);
-    for (int kt = kt0; kt < kt1; ++kt) {
-      uint8_t* d = dst + (kt - kt0) * 1024;
-      copy(d, base + (static_cast<size_t>(r_lo / 128) * g.kt_d + kt) * kTile + (r_lo % 128) * 128, 512);
-      copy(d + 512, base + (static_cast<size_t>(r_hi / 128) * g.kt_d + kt) * kTile + (r_hi % 128) * 128, 512);
-    }
-  } else if (op == OP_GU) {
-    const uint8_t* base = a.w + a.off_wgate + static_cast<long long>(l) * a.lstride;
-    const int j0 = u * kUR, rt = j0 / 64, rr = j0 % 64;
-    const int kt0 = s * 4, kt1 = min(kt0 + 4, g.kt_d);
-    for (int kt = kt0; kt < kt1; ++kt) {
-      const uint8_t* t = base + (static_cast<size_t>(rt) * g.kt_d + kt) * kTile;
-      uint8_t* d = dst + (kt - kt0) * 2048;
-      copy(d, t + rr * 128, 1024);
-      copy(d + 1024, t + (64 + rr) * 128, 1024);
-    }
-  } else if (op == OP_LM && a.tied) {
-    const uint8_t* base = a.w + a.off_lm;
-    const int c0 = s * 512, nc = min(512, a.d - c0);
-    for (int w = 0; w < kUR; ++w) {
-      const int v = u * kUR + w;
-      if (v >= a.V) break;
-      copy(dst + w * 1024, base + (static_cast<size_t>(v) * a.d + c0) * 2, static_cast<uint32_t>(nc) * 2);
-    }
-  } else {   // O, DOWN, packed LM: 8 contiguous rows of each k tile
-    const uint8_t* base;
-    int kt_n;
-    if (op == OP_O) {
-      base = a.w + a.off_wo + static_cast<long long>(l) * a.lstride;
-      kt_n = g.kt_q;
-    } else if (op == OP_DOWN) {
-      base = a.w + a.off_wdown + static_cast<long long>(l) * a.lstride;
-      kt_n = g.kt_f;
-    } else {
-      base = a.w + a.off_lm;
-      kt_n = g.kt_d;
-    }
-    const int r0 = u * kUR;
-    const int kt0 = s * 8, kt1 = min(kt0 + 8, kt_n);
-    for (int kt = kt0; kt < kt1; ++kt)
-      copy(dst + (kt - kt0) * 1024, base + (static_cast<size_t>(r0 / 128) * kt_n + kt) * kTile + (r0 % 128) * 128,
-           1024);
+    const int kt0 = s * 8;
+    tma_load_3d(dst, maps + 0, 0, r_lo % 128, (r_lo / 128) * g.kt_d + kt0, bar, pol);
+    tma_load_3d(dst + 4096, maps + 0, 0, r_hi % 128, (r_hi / 128) * g.kt_d + kt0, bar, pol);
+    return 8192;
   }
-  return bytes;
+  if (op == OP_GU) {
+    const int j0 = u * kUR, rt = j0 / 64, rr = j0 % 64, kt0 = s * 4;
+    tma_load_3d(dst, maps + 2, 0, rr, rt * g.kt_d + kt0, bar, pol);
+    tma_load_3d(dst + 4096, maps + 2, 0, 64 + rr, rt * g.kt_d + kt0, bar, pol);
+    return 8192;
+  }
+  if (op == OP_LM && a.tied) {
+    const CUtensorMap* m = a.maps + static_cast<size_t>(a.n_layers) * 4;
+    tma_load_3d(dst, m, s * 512, u * kUR, 0, bar, pol);          // map: {d, vocab, 1}, box {256, 8, 1}
+    tma_load_3d(dst + 4096, m, s * 512 + 256, u * kUR, 0, bar, pol);
+    return 8192;
+  }
+  const CUtensorMap* m;
+  int kt_n;
+  if (op == OP_O) {
+    m = maps + 1;
+    kt_n = g.kt_q;
+  } else if (op == OP_DOWN) {
+    m = maps + 3;
+    kt_n = g.kt_f;
+  } else {
+    m = a.maps + static_cast<size_t>(a.n_layers) * 4;
+    kt_n = g.kt_d;
+  }
+  const int r0 = u * kUR;
+  tma_load_3d(dst, m, 0, r0 % 128, (r0 / 128) * kt_n + s * 8, bar, pol);
+  return 8192;
 }
 
-// The copy-issuing lane: every slot of every unit of every op of every pass,
-// in consumption order.
+// The copy-issuing lane: every slot of every unit of every op of every pass, in
+// consumption order.
 __device__ void producer(const DraftFusedArgs& a, DfCtl& ctl, uint8_t* ring) {
   const Geo g = make_geo(a);
   const int S = a.ring_slots;
   const uint64_t pol = l2_policy_evict_first();
   uint32_t n = 0;
   bool ok = true;
+  for (int i = 0; i <= a.n_layers * 4; ++i) tma_prefetch_desc(a.maps + i);
   auto fill = [&](int op, int l, int u, int s) {
     if (!ok) return;
     const int i = static_cast<int>(n % static_cast<uint32_t>(S));
@@ -220,10 +219,8 @@ __device__ void producer(const DraftFusedArgs& a, DfCtl& ctl, uint8_t* ring) {
         return;
       }
     }
-    uint8_t* dst = ring + static_cast<size_t>(i) * kDfSlotBytes;
-    const uint32_t bytes = issue_slot(a, g, op, l, u, s, dst, &ctl.full[i], pol, false);
-    mbar_arrive_expect_tx(&ctl.full[i], bytes);
-    issue_slot(a, g, op, l, u, s, dst, &ctl.full[i], pol, true);
+    mbar_arrive_expect_tx(&ctl.full[i], 8192);
+    issue_slot(a, g, op, l, u, s, ring + static_cast<size_t>(i) * kDfSlotBytes, &ctl.full[i], pol);
     ++n;
   };
   for (int j = 1; j <= a.K && ok; ++j) {
@@ -238,8 +235,17 @@ __device__ void producer(const DraftFusedArgs& a, DfCtl& ctl, uint8_t* ring) {
           for (int s = 0; s < ns[op]; ++s) fill(op, l, u, s);
       }
     }
+    unsigned long long* tr = nullptr;
+    const int phase = j * (5 * a.n_layers + 1) - 1;      // this pass's LM phase
+    if (a.trace != nullptr && phase < a.trace_phases)
+      tr = a.trace + 2 + (static_cast<size_t>(phase) * g.G + g.c) * 16;
+    int lm_fill = 0;
     for (int u = lm_lo(g, g.c); u < lm_lo(g, g.c + 1); ++u)
-      for (int s = 0; s < g.s_lm; ++s) fill(OP_LM, 0, u, s);
+      for (int s = 0; s < g.s_lm; ++s) {
+        if (tr != nullptr && (lm_fill & 7) == 0 && lm_fill < 56) tr[2 + lm_fill / 8] = global_ns();
+        fill(OP_LM, 0, u, s);
+        ++lm_fill;
+      }
   }
   // tear-down: the last fill of every slot must have landed before the CTA exits
   const uint32_t first = n > static_cast<uint32_t>(S) ? n - S : 0;
@@ -279,7 +285,6 @@ __device__ bool grid_sync(const DraftFusedArgs& a, DfCtl& ctl, unsigned& epoch, 
           break;
         }
       }
-      __threadfence();
     }
     t_phase = global_ns();
     if (tr != nullptr && epoch <= static_cast<unsigned>(a.trace_phases)) tr[13] = t_phase;
@@ -389,8 +394,8 @@ __device__ bool unit_dots(const DraftFusedArgs& a, DfCtl& ctl, const uint8_t* ri
         const int ktl = q >> 3, c = q & 7;
         const int kidx = (kt0 + ktl) * 64 + c * 8;
         const int pos = (c ^ ((swz_row_lo + w) & 7)) * 16;
-        const uint4 wg = *reinterpret_cast<const uint4*>(slot + ktl * 2048 + w * 128 + pos);
-        const uint4 wu = *reinterpret_cast<const uint4*>(slot + ktl * 2048 + 1024 + w * 128 + pos);
+        const uint4 wg = *reinterpret_cast<const uint4*>(slot + ktl * 1024 + w * 128 + pos);
+        const uint4 wu = *reinterpret_cast<const uint4*>(slot + 4096 + ktl * 1024 + w * 128 + pos);
 #pragma unroll
         for (int m = 0; m < kDfMaxRows; ++m) {
           if (m >= M) break;
@@ -416,18 +421,23 @@ __device__ bool unit_dots(const DraftFusedArgs& a, DfCtl& ctl, const uint8_t* ri
         const int q = lane + 32 * h;        // chunk of this row in the slot
         bool have;
         int woff, kidx;
-        if (OPK == OP_LM && a.tied) {       // row-major: row w, 512 columns
+        if (OPK == OP_LM && a.tied) {       // row-major: 2 x [8 rows][256 columns]
           const int c0 = s * 512;
           kidx = c0 + q * 8;
           have = kidx < a.d;
-          woff = w * 1024 + q * 16;
+          woff = (q >> 5) * 4096 + w * 512 + (q & 31) * 16;
         } else {
           const int kt0 = s * 8, nkt = min(8, kt_n - kt0);
           const int ktl = q >> 3, c = q & 7;
           have = q < nkt * 8;
           kidx = (kt0 + ktl) * 64 + c * 8;
-          const int trow = (OPK == OP_QKV && w >= 4) ? swz_row_hi + (w - 4) : swz_row_lo + w;
-          woff = ktl * 1024 + w * 128 + ((c ^ (trow & 7)) * 16);
+          if (OPK == OP_QKV) {
+            const int hi = w >> 2, wr = w & 3;
+            const int trow = (hi ? swz_row_hi : swz_row_lo) + wr;
+            woff = hi * 4096 + ktl * 512 + wr * 128 + ((c ^ (trow & 7)) * 16);
+          } else {
+            woff = ktl * 1024 + w * 128 + ((c ^ ((swz_row_lo + w) & 7)) * 16);
+          }
         }
         if (!have) continue;
         const uint4 wv = *reinterpret_cast<const uint4*>(slot + woff);
@@ -491,15 +501,21 @@ __device__ void attention_unit(const DraftFusedArgs& a, DfCtl& ctl, int layer, i
   const bf16* vc = kc + a.layer_kv;
   float* sc = scratch;                    // [2][kKeyBlock] scores, then weights
   float* qs = sc + 2 * kKeyBlock;         // [2][HD]
-  float* op = qs + 2 * HD;                // [kCT][2] o partials (key groups)
+  float* op = qs + 2 * 128;               // [warps][2][HD] o partials
   const float qscale = 1.4426950408889634f / sqrtf(static_cast<float>(HD));
   for (int e = tid; e < nr * HD; e += kCT) {
     const int i = e / HD, dd = e - i * HD;
     qs[e] = ldcg(a.qb + (static_cast<size_t>(g * R + i) * a.H + h) * HD + dd) * qscale;
   }
   float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
-  const int dd = tid % HD, kg = tid / HD;
-  float o_run[2] = {0.f, 0.f};
+  // PV: thread (d8, kg) accumulates dims 8 d8 .. 8 d8 + 7 over keys kg, kg + KG8, ...
+  constexpr int D8 = HD / 8, KG8 = kCT / D8;
+  const int d8 = tid % D8, kg = tid / D8;
+  float o_run[2][8];
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+#pragma unroll
+    for (int e = 0; e < 8; ++e) o_run[i][e] = 0.f;
   csync();
   for (int kb = k0; kb < k1; kb += kKeyBlock) {
     const int t = kb + tid;
@@ -560,31 +576,52 @@ __device__ void attention_unit(const DraftFusedArgs& a, DfCtl& ctl, int layer, i
     for (int i = 0; i < 2; ++i) {
       l_run[i] = l_run[i] * alpha[i] + ctl.red[0][i];
       m_run[i] = mnew[i];
-      o_run[i] *= alpha[i];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) o_run[i][e] *= alpha[i];
     }
     const int nk = min(kKeyBlock, k1 - kb);
-    const bf16* vb = vc + static_cast<size_t>(kb) * HD + dd;
-    for (int t0 = kg; t0 < nk; t0 += 8 * KG) {
-      float v[8];
+    const bf16* vb = vc + static_cast<size_t>(kb) * HD + d8 * 8;
+    constexpr int kPer = (kKeyBlock + KG8 - 1) / KG8;       // keys per thread per block
+    uint4 vv[kPer];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const int tt = t0 + q * KG;
-        v[q] = tt < nk ? __bfloat162float(vb[static_cast<size_t>(tt) * HD]) : 0.f;
-      }
+    for (int q = 0; q < kPer; ++q) {
+      const int tt = kg + q * KG8;
+      vv[q] = tt < nk ? __ldcg(reinterpret_cast<const uint4*>(vb + static_cast<size_t>(tt) * HD))
+                      : make_uint4(0u, 0u, 0u, 0u);
+    }
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const int tt = t0 + q * KG;
-        if (tt < nk) {
-          o_run[0] = fmaf(sc[tt], v[q], o_run[0]);
-          o_run[1] = fmaf(sc[kKeyBlock + tt], v[q], o_run[1]);
+    for (int q = 0; q < kPer; ++q) {
+      const int tt = kg + q * KG8;
+      if (tt < nk) {
+        const float vf[8] = {bf_lo(vv[q].x), bf_hi(vv[q].x), bf_lo(vv[q].y), bf_hi(vv[q].y),
+                             bf_lo(vv[q].z), bf_hi(vv[q].z), bf_lo(vv[q].w), bf_hi(vv[q].w)};
+        const float p0v = sc[tt], p1v = sc[kKeyBlock + tt];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          o_run[0][e] = fmaf(p0v, vf[e], o_run[0][e]);
+          o_run[1][e] = fmaf(p1v, vf[e], o_run[1][e]);
         }
       }
     }
     csync();                                // sc is rewritten by the next block
   }
-  // combine the key groups in order, write (m, l, o)
-  op[tid * 2] = o_run[0];
-  op[tid * 2 + 1] = o_run[1];
+  // key groups: first across the lanes of a warp that share d8 (xor tree), then
+  // the warps in order through shared memory
+  {
+    const int w = tid >> 5, lane = tid & 31;
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+#pragma unroll
+        for (int o = 16; o >= D8; o >>= 1) o_run[i][e] += __shfl_xor_sync(0xffffffffu, o_run[i][e], o);
+    if (lane < D8) {
+#pragma unroll
+      for (int i = 0; i < 2; ++i)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) op[(w * 2 + i) * HD + lane * 8 + e] = o_run[i][e];
+    }
+  }
   csync();
   const int stride = HD + 4;
   float* mine = a.att + (static_cast<size_t>(g * R) * a.H + h) * S * stride;   // row i at + i * H * S * stride
@@ -592,7 +629,7 @@ __device__ void attention_unit(const DraftFusedArgs& a, DfCtl& ctl, int layer, i
     const int i = e / HD, d2 = e - i * HD;
     float o = 0.f;
 #pragma unroll
-    for (int k = 0; k < KG; ++k) o += op[(k * HD + d2) * 2 + i];
+    for (int w = 0; w < kCW; ++w) o += op[(w * 2 + i) * HD + d2];
     mine[(static_cast<size_t>(i) * a.H * S + s) * stride + 4 + d2] = o;
   }
   if (tid < nr) {
@@ -1055,7 +1092,17 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
           load_norm_rows(a, ctl, act, 1, reinterpret_cast<const bf16*>(a.w + a.off_final_norm), true, tid);
         const bool greedy = a.greedy != 0;
         const float it = a.inv_temp;
+        unsigned long long* tr_lm = nullptr;
+        {
+          const int phase = j * (5 * a.n_layers + 1) - 1;
+          if (a.trace != nullptr && phase < a.trace_phases && tid == 0)
+            tr_lm = a.trace + 2 + (static_cast<size_t>(phase) * G + c) * 16;
+        }
         for (int u = ulo; u < uhi && run; ++u) {
+          if (tr_lm != nullptr && ((u - ulo) & 3) == 0 && (u - ulo) < 24) {
+            const int k = (u - ulo) >> 2;               // 0..5 -> slots 9..12, 14, 15
+            tr_lm[k < 4 ? 9 + k : 10 + k] = global_ns();
+          }
           run = csync_and(unit_dots<OP_LM>(a, ctl, ring, act, B, geo.s_lm, geo.kt_d, (u * kUR) % 128, 0,
                                            cons, acc, tid));
           if (!run) break;

@@ -202,8 +202,12 @@ constexpr int kDfSlotBytes = 8192;      // weight ring slot
 constexpr int kDfMaxSlots = 32;
 constexpr int kDfComputeWarps = 8;
 constexpr int kDfThreads = (kDfComputeWarps + 1) * 32;   // + one copy-issuing warp
+constexpr int kDfMaxLayers = 32;
+constexpr int kDfMapsPerDraft = kDfMaxLayers * 4 + 1;
 
 struct DraftFusedArgs {
+  const CUtensorMap* maps;   // device: per layer {QKV, O, gate/up, down} boxes over the packed
+                             // tiles, then the LM head (kDfMaxLayers * 4 + 1 at most)
   const uint8_t* w;          // draft weight blob
   // tensor offsets in the blob; per-layer tensors at off + layer * lstride
   long long off_emb, off_attn_norm, off_wqkv, off_wo, off_ffn_norm, off_wgate, off_wdown,
@@ -244,7 +248,7 @@ struct DraftFusedArgs {
 };
 size_t draft_fused_smem_bytes(int ring_slots, int act_rows, int act_floats);
 size_t draft_fused_static_smem();
-constexpr int kDfScratchFloatsHost = 2 * 256 + 2 * 128 + 2 * 256;   // == kDfScratchFloats
+constexpr int kDfScratchFloatsHost = 2 * 256 + 2 * 128 + 8 * 2 * 128;   // == kDfScratchFloats
 cudaError_t draft_fused_set_max_smem();
 cudaError_t launch_draft_fused(const DraftFusedArgs& a, int grid, cudaStream_t s, bool cooperative);
 

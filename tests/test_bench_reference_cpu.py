@@ -6,6 +6,7 @@ import json
 import os
 import subprocess
 import sys
+import time
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
@@ -14,9 +15,11 @@ def test_reference_arm_line():
     sys.path.insert(0, ROOT)
     import bench
 
+    t0 = time.perf_counter()
     out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
                           "--steps", "2", "--warmup", "3"],
-                         cwd=ROOT, capture_output=True, text=True, timeout=600)
+                         cwd=ROOT, capture_output=True, text=True, timeout=900)
+    wall = time.perf_counter() - t0
     assert out.returncode == 0, out.stderr[-2000:]
     line = json.loads(out.stdout.strip().splitlines()[-1])
     assert line["impl"] == "reference"
@@ -26,8 +29,11 @@ def test_reference_arm_line():
     for k, v in bench.workload_config(bench.K_DRAFT, 1).items():
         assert line["config"][k] == v
     assert line["value"] > 0 and line["ms_per_step"] > 0
+    # the timed steps were executed: they fit inside the run's wall time
+    assert line["ms_per_step"] * line["steps"] / 1000.0 <= wall
     cb = line["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == line["value"] and cb["cores"] >= 1
-    assert "oracle" in cb["sample"]
+    assert "oracle" in cb["sample"] and cb["cpu_model"]
+    assert cb["tokens_per_iteration"] >= 1.0 and cb["full_depth_iteration_s"] > 0
     assert line["e2e"] == {"value": line["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0,
                            "d2h_bytes_per_step": 0}
