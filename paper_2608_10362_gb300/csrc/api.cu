@@ -1214,7 +1214,7 @@ bool fused_draft_plan(memspec_ctx* c, DraftRec& dr, int K, float T, DraftFusedAr
   const size_t fixed = draft_fused_smem_bytes(0, 2 * B, act_floats) + draft_fused_static_smem() + 1024;
   const long long room = 227LL * 1024 - static_cast<long long>(fixed);
   const int slots = static_cast<int>(std::min<long long>(kDfMaxSlots, room / kDfSlotBytes));
-  if (slots < 8) {
+  if (slots < 4) {
     *why = "activation rows leave no room for the weight ring";
     return false;
   }
@@ -1257,16 +1257,16 @@ bool fused_draft_plan(memspec_ctx* c, DraftRec& dr, int K, float T, DraftFusedAr
     bool ok = true;
     for (int l = 0; l < m.n_layers && ok; ++l) {
       CUtensorMap* mp = dr.df_maps.data() + l * 4;
-      ok = packed(mp + 0, lay.wqkv[l], q + 2 * kv, d, false, 4, 8) &&
-           packed(mp + 1, lay.wo[l], d, q, false, 8, 8) && packed(mp + 2, lay.wgate[l], F, d, true, 8, 4) &&
-           packed(mp + 3, lay.wdown[l], d, F, false, 8, 8);
+      ok = packed(mp + 0, lay.wqkv[l], q + 2 * kv, d, false, 8, 8) &&
+           packed(mp + 1, lay.wo[l], d, q, false, 8, 16) && packed(mp + 2, lay.wgate[l], F, d, true, 8, 8) &&
+           packed(mp + 3, lay.wdown[l], d, F, false, 8, 16);
     }
     CUtensorMap* lm = dr.df_maps.data() + m.n_layers * 4;
     if (ok)
       ok = m.tied_embeddings
                ? encode_box3d(lm, dr.rt.w + lay.lm_head, static_cast<uint64_t>(d), static_cast<uint64_t>(m.vocab), 1,
                               static_cast<uint64_t>(d) * 2, static_cast<uint64_t>(d) * 2 * m.vocab, 256, 8, 1)
-               : packed(lm, lay.lm_head, m.vocab, d, false, 8, 8);
+               : packed(lm, lay.lm_head, m.vocab, d, false, 8, 16);
     if (!ok) {
       *why = "tensor map encoding";
       return false;

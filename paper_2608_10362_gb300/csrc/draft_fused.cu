@@ -11,21 +11,20 @@
 //    gate/up + SwiGLU, down + residual; final RMSNorm + LM head; sampling) is a
 //    phase separated from the next by a grid-wide barrier (an arrival counter in
 //    global memory, release / acquire, bounded waits);
-//  * projection weights are split into units of 8 output rows (the rows of a
-//    unit and their RoPE partners for QKV; 8 gate + 8 up rows for the SwiGLU
-//    pair), assigned round-robin to CTAs; each CTA computes its units' full dot
-//    products (no split-K, no partial sums) on CUDA cores, with fp32 activations
-//    and bf16 weights;
+//  * projection weights are split into units of 8 output rows per warp-row (8
+//    rows; 8 RoPE pairs for QKV; 8 gate + 8 up rows for the SwiGLU pair),
+//    assigned round-robin to CTAs; a CTA computes its units' full dot products
+//    (no split-K, no partial sums) on CUDA cores, fp32 activations times bf16
+//    weights, each warp owning one output row (or one row pair);
 //  * one copy-issuing lane streams the CTA's weight bytes of every op of every
-//    pass, in the order the compute warps consume them, into a ring of 8 KB
-//    shared-memory slots, each slot one or two multi-dimensional TMA boxes over
-//    the packed tiles (8 rows x 64 columns x up to 8 k tiles), signalled on
-//    mbarriers.  The weights do not depend on activations, so the ring fills
-//    ahead across op and pass boundaries while the compute warps wait at grid
-//    barriers;
+//    pass, in the order the compute warps consume them, into a ring of 16 KB
+//    shared-memory slots, each slot one to four multi-dimensional TMA boxes over
+//    the packed tiles (8 rows x 64 columns x up to 16 k tiles), signalled on
+//    mbarriers.  Weights do not depend on activations, so the ring fills ahead
+//    across op and pass boundaries while the compute warps wait at barriers;
 //  * attention: one (request, head, key split) unit per CTA; the keys of
 //    positions before the pass are prefetched into L2 while the QKV phase runs;
-//    the O phase combines the splits (m, l, o) itself;
+//    the last split of a head to finish combines the splits (m, l, o);
 //  * LM head: each CTA owns a contiguous vocabulary slice and writes its
 //    logits and (max, first argmax, sum exp) statistics; after the barrier every
 //    CTA redoes the tiny combine and the inverse-CDF search in the owning slice
@@ -47,7 +46,7 @@ namespace {
 
 constexpr int kCW = kDfComputeWarps;
 constexpr int kCT = kCW * 32;              // compute threads
-constexpr int kUR = 8;                     // output rows per unit
+constexpr int kUR = 8;                     // output rows (or row pairs) per unit: one per warp
 constexpr int kKeyBlock = kCT;             // keys per attention block (one per thread)
 // attention scores (2 rows), queries (2 x hd <= 128), per-warp o partials
 // [warps][2][hd <= 128]
@@ -90,8 +89,8 @@ __device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
 __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
-// One TMA request per box: a slot is fetched by one or two requests (a request
-// costs about as much as its bytes only from several KB up, measured).
+// One TMA request per box (a request costs about as much as its bytes only from
+// several KB up, measured).
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
                                             uint64_t* bar, uint64_t pol) {
   asm volatile(
@@ -120,6 +119,18 @@ __device__ __forceinline__ bool csync_and(bool v) {
   return r != 0;
 }
 
+// Position in the weight ring (slot index and the phase parity of its barriers).
+struct Ring {
+  int i = 0, S = 1;
+  uint32_t ph = 0;
+  __device__ void next() {
+    if (++i == S) {
+      i = 0;
+      ph ^= 1u;
+    }
+  }
+};
+
 // ------------------------------------------------------------------ schedule
 // Units of each weight op, and ring slots per unit.
 struct Geo {
@@ -136,52 +147,60 @@ __device__ __forceinline__ Geo make_geo(const DraftFusedArgs& a) {
   g.kt_d = a.d / 64;
   g.kt_q = a.H * a.hd / 64;
   g.kt_f = (a.F + 63) / 64;
-  g.u_qkv = (a.H + 2 * a.Hkv) * a.hd / kUR;
+  g.u_qkv = (a.H + 2 * a.Hkv) * a.hd / (2 * kUR);   // 8 RoPE pairs per unit
   g.u_o = a.d / kUR;
   g.u_gu = a.F / kUR;
   g.u_down = a.d / kUR;
   g.u_lm = (a.V + kUR - 1) / kUR;
   g.s_qkv = (g.kt_d + 7) / 8;
-  g.s_o = (g.kt_q + 7) / 8;
-  g.s_gu = (g.kt_d + 3) / 4;
-  g.s_down = (g.kt_f + 7) / 8;
-  g.s_lm = a.tied ? (a.d + 511) / 512 : (g.kt_d + 7) / 8;
+  g.s_o = (g.kt_q + 15) / 16;
+  g.s_gu = (g.kt_d + 7) / 8;
+  g.s_down = (g.kt_f + 15) / 16;
+  g.s_lm = a.tied ? (a.d + 1023) / 1024 : (g.kt_d + 15) / 16;
   return g;
 }
 __device__ __forceinline__ int first_unit(const Geo& g, int off) { return ((g.c - off) % g.G + g.G) % g.G; }
 __device__ __forceinline__ int lm_lo(const Geo& g, int c) {
   return static_cast<int>(static_cast<long long>(c) * g.u_lm / g.G);
 }
+// The two row blocks of QKV unit u: rows lo..lo+7 and their RoPE partners hi..hi+7.
+__device__ __forceinline__ void qkv_rows(const DraftFusedArgs& a, int u, int* hb, int* ui, int* lo, int* hi) {
+  const int per = a.hd / (2 * kUR);
+  *hb = u / per;
+  *ui = u - *hb * per;
+  *lo = *hb * a.hd + kUR * *ui;
+  *hi = *lo + a.hd / 2;
+}
 
-// Issue the TMA requests of slot `s` of unit `u` of op `op` (layer `l`) into
-// `dst` (one elected lane); returns the bytes they complete.  Shared-memory
-// image of a slot (128-byte rows exactly as packed, swizzle included):
-//   O, DOWN, packed LM: [8 k tiles][8 rows][128 B]            (one request)
-//   QKV:  rows r_lo.. then r_hi..: 2 x [8 k tiles][4 rows][128 B]
-//   GU:   gate rows then up rows:  2 x [4 k tiles][8 rows][128 B]
-//   tied LM (row-major embedding): 2 x [8 rows][256 columns]
-__device__ uint32_t issue_slot(const DraftFusedArgs& a, const Geo& g, int op, int l, int u, int s,
-                               uint8_t* dst, uint64_t* bar, uint64_t pol) {
+// Issue the TMA boxes of slot `s` of unit `u` of op `op` (layer `l`) into `dst`
+// (16 KB, completing on `bar`).  Shared-memory image of a slot (128-byte rows
+// exactly as packed, swizzle included):
+//   O, DOWN, packed LM: [16 k tiles][8 rows][128 B]                 (one box)
+//   QKV: rows lo.. then their partners hi..: 2 x [8 k tiles][8 rows][128 B]
+//   GU:  gate rows then the same up rows:    2 x [8 k tiles][8 rows][128 B]
+//   tied LM (row-major embedding): 4 x [8 rows][256 columns]
+__device__ void issue_slot(const DraftFusedArgs& a, const Geo& g, int op, int l, int u, int s,
+                           uint8_t* dst, uint64_t* bar, uint64_t pol) {
   const CUtensorMap* maps = a.maps + static_cast<size_t>(l) * 4;
   if (op == OP_QKV) {
-    const int hb = u / (a.hd / kUR), ui = u - hb * (a.hd / kUR);
-    const int r_lo = hb * a.hd + 4 * ui, r_hi = r_lo + a.hd / 2;
+    int hb, ui, lo, hi;
+    qkv_rows(a, u, &hb, &ui, &lo, &hi);
     const int kt0 = s * 8;
-    tma_load_3d(dst, maps + 0, 0, r_lo % 128, (r_lo / 128) * g.kt_d + kt0, bar, pol);
-    tma_load_3d(dst + 4096, maps + 0, 0, r_hi % 128, (r_hi / 128) * g.kt_d + kt0, bar, pol);
-    return 8192;
+    tma_load_3d(dst, maps + 0, 0, lo % 128, (lo / 128) * g.kt_d + kt0, bar, pol);
+    tma_load_3d(dst + 8192, maps + 0, 0, hi % 128, (hi / 128) * g.kt_d + kt0, bar, pol);
+    return;
   }
   if (op == OP_GU) {
-    const int j0 = u * kUR, rt = j0 / 64, rr = j0 % 64, kt0 = s * 4;
+    const int j0 = u * kUR, rt = j0 / 64, rr = j0 % 64, kt0 = s * 8;
     tma_load_3d(dst, maps + 2, 0, rr, rt * g.kt_d + kt0, bar, pol);
-    tma_load_3d(dst + 4096, maps + 2, 0, 64 + rr, rt * g.kt_d + kt0, bar, pol);
-    return 8192;
+    tma_load_3d(dst + 8192, maps + 2, 0, 64 + rr, rt * g.kt_d + kt0, bar, pol);
+    return;
   }
-  if (op == OP_LM && a.tied) {
+  if (op == OP_LM && a.tied) {   // map {d, vocab, 1}, box {256, 8, 1}
     const CUtensorMap* m = a.maps + static_cast<size_t>(a.n_layers) * 4;
-    tma_load_3d(dst, m, s * 512, u * kUR, 0, bar, pol);          // map: {d, vocab, 1}, box {256, 8, 1}
-    tma_load_3d(dst + 4096, m, s * 512 + 256, u * kUR, 0, bar, pol);
-    return 8192;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) tma_load_3d(dst + q * 4096, m, s * 1024 + q * 256, u * kUR, 0, bar, pol);
+    return;
   }
   const CUtensorMap* m;
   int kt_n;
@@ -196,31 +215,29 @@ __device__ uint32_t issue_slot(const DraftFusedArgs& a, const Geo& g, int op, in
     kt_n = g.kt_d;
   }
   const int r0 = u * kUR;
-  tma_load_3d(dst, m, 0, r0 % 128, (r0 / 128) * kt_n + s * 8, bar, pol);
-  return 8192;
+  tma_load_3d(dst, m, 0, r0 % 128, (r0 / 128) * kt_n + s * 16, bar, pol);
 }
 
 // The copy-issuing lane: every slot of every unit of every op of every pass, in
 // consumption order.
 __device__ void producer(const DraftFusedArgs& a, DfCtl& ctl, uint8_t* ring) {
   const Geo g = make_geo(a);
-  const int S = a.ring_slots;
   const uint64_t pol = l2_policy_evict_first();
+  Ring rg;
+  rg.S = a.ring_slots;
   uint32_t n = 0;
   bool ok = true;
   for (int i = 0; i <= a.n_layers * 4; ++i) tma_prefetch_desc(a.maps + i);
   auto fill = [&](int op, int l, int u, int s) {
     if (!ok) return;
-    const int i = static_cast<int>(n % static_cast<uint32_t>(S));
-    if (n >= static_cast<uint32_t>(S)) {
-      const uint32_t par = ((n / S) - 1) & 1u;
-      if (!mbar_wait_bounded(&ctl.empty[i], par, &ctl.abort, a.status)) {
-        ok = false;
-        return;
-      }
+    if (n >= static_cast<uint32_t>(rg.S) &&
+        !mbar_wait_bounded(&ctl.empty[rg.i], rg.ph ^ 1u, &ctl.abort, a.status)) {
+      ok = false;
+      return;
     }
-    mbar_arrive_expect_tx(&ctl.full[i], 8192);
-    issue_slot(a, g, op, l, u, s, ring + static_cast<size_t>(i) * kDfSlotBytes, &ctl.full[i], pol);
+    mbar_arrive_expect_tx(&ctl.full[rg.i], kDfSlotBytes);
+    issue_slot(a, g, op, l, u, s, ring + static_cast<size_t>(rg.i) * kDfSlotBytes, &ctl.full[rg.i], pol);
+    rg.next();
     ++n;
   };
   for (int j = 1; j <= a.K && ok; ++j) {
@@ -235,21 +252,12 @@ __device__ void producer(const DraftFusedArgs& a, DfCtl& ctl, uint8_t* ring) {
           for (int s = 0; s < ns[op]; ++s) fill(op, l, u, s);
       }
     }
-    unsigned long long* tr = nullptr;
-    const int phase = j * (5 * a.n_layers + 1) - 1;      // this pass's LM phase
-    if (a.trace != nullptr && phase < a.trace_phases)
-      tr = a.trace + 2 + (static_cast<size_t>(phase) * g.G + g.c) * 16;
-    int lm_fill = 0;
     for (int u = lm_lo(g, g.c); u < lm_lo(g, g.c + 1); ++u)
-      for (int s = 0; s < g.s_lm; ++s) {
-        if (tr != nullptr && (lm_fill & 7) == 0 && lm_fill < 56) tr[2 + lm_fill / 8] = global_ns();
-        fill(OP_LM, 0, u, s);
-        ++lm_fill;
-      }
+      for (int s = 0; s < g.s_lm; ++s) fill(OP_LM, 0, u, s);
   }
   // tear-down: the last fill of every slot must have landed before the CTA exits
-  const uint32_t first = n > static_cast<uint32_t>(S) ? n - S : 0;
-  for (uint32_t m = first; m < n; ++m) mbar_wait_drain(&ctl.full[m % S], (m / S) & 1u);
+  const uint32_t first = n > static_cast<uint32_t>(rg.S) ? n - rg.S : 0;
+  for (uint32_t m = first; m < n; ++m) mbar_wait_drain(&ctl.full[m % rg.S], (m / rg.S) & 1u);
 }
 
 // ------------------------------------------------------------------ helpers (compute warps)
@@ -318,8 +326,9 @@ __device__ void block_row_sums(DfCtl& ctl, float* v, int rows, int tid) {
 }
 
 // act[r][0..d) = RMSNorm(x_r) * gain for the rows of the pass (LM: one row per
-// request, the last valid one).  src: 0 embedding rows of ctl.tok (and CTA 0
-// writes them to the residual stream), 1 residual stream.
+// request, the last valid one), in one round trip for x and the gain.  src: 0
+// embedding rows of ctl.tok (and CTA 0 writes them to the residual stream), 1
+// the residual stream.
 __device__ void load_norm_rows(const DraftFusedArgs& a, DfCtl& ctl, float* act, int src,
                                const bf16* gain, bool lm_rows, int tid) {
   const int d = a.d, AF = a.act_floats;
@@ -328,139 +337,136 @@ __device__ void load_norm_rows(const DraftFusedArgs& a, DfCtl& ctl, float* act, 
 #pragma unroll
   for (int r = 0; r < kDfMaxRows; ++r) ss[r] = 0.f;
   for (int k = tid * 4; k < d; k += kCT * 4) {
+    const uint2 graw = *reinterpret_cast<const uint2*>(gain + k);
+    float4 x[kDfMaxRows];
+#pragma unroll
+    for (int r = 0; r < kDfMaxRows; ++r) {
+      x[r] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (r >= nrow) continue;
+      const int rs = lm_rows ? r * ctl.R + ctl.valid[r] - 1 : r;
+      if (!ctl.ok[rs]) continue;
+      if (src == 0) {
+        const uint2 raw = *reinterpret_cast<const uint2*>(a.w + a.off_emb +
+                                                          (static_cast<size_t>(ctl.tok[rs]) * d + k) * 2);
+        x[r] = make_float4(bf_lo(raw.x), bf_hi(raw.x), bf_lo(raw.y), bf_hi(raw.y));
+        if (blockIdx.x == 0) *reinterpret_cast<float4*>(a.h + static_cast<size_t>(rs) * d + k) = x[r];
+      } else {
+        x[r] = __ldcg(reinterpret_cast<const float4*>(a.h + static_cast<size_t>(rs) * d + k));
+      }
+    }
+    const float g0 = bf_lo(graw.x), g1 = bf_hi(graw.x), g2 = bf_lo(graw.y), g3 = bf_hi(graw.y);
 #pragma unroll
     for (int r = 0; r < kDfMaxRows; ++r) {
       if (r >= nrow) break;
-      const int rs = lm_rows ? r * ctl.R + ctl.valid[r] - 1 : r;
-      float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (ctl.ok[rs]) {
-        if (src == 0) {
-          const uint2 raw = *reinterpret_cast<const uint2*>(a.w + a.off_emb +
-                                                            (static_cast<size_t>(ctl.tok[rs]) * d + k) * 2);
-          x = make_float4(bf_lo(raw.x), bf_hi(raw.x), bf_lo(raw.y), bf_hi(raw.y));
-          if (blockIdx.x == 0) *reinterpret_cast<float4*>(a.h + static_cast<size_t>(rs) * d + k) = x;
-        } else {
-          x = __ldcg(reinterpret_cast<const float4*>(a.h + static_cast<size_t>(rs) * d + k));
-        }
-      }
-      ss[r] += x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w;
-      *reinterpret_cast<float4*>(act + r * AF + k) = x;
+      ss[r] += x[r].x * x[r].x + x[r].y * x[r].y + x[r].z * x[r].z + x[r].w * x[r].w;
+      *reinterpret_cast<float4*>(act + r * AF + k) =
+          make_float4(x[r].x * g0, x[r].y * g1, x[r].z * g2, x[r].w * g3);
     }
   }
   block_row_sums(ctl, ss, nrow, tid);
   if (tid < nrow) ctl.scale[tid] = 1.f / sqrtf(ctl.red[0][tid] / static_cast<float>(d) + a.eps);
   csync();
   for (int k = tid * 4; k < d; k += kCT * 4) {
-    const uint2 graw = *reinterpret_cast<const uint2*>(gain + k);
-    const float g0 = bf_lo(graw.x), g1 = bf_hi(graw.x), g2 = bf_lo(graw.y), g3 = bf_hi(graw.y);
 #pragma unroll
     for (int r = 0; r < kDfMaxRows; ++r) {
       if (r >= nrow) break;
       float4* p = reinterpret_cast<float4*>(act + r * AF + k);
       const float sc = ctl.scale[r];
-      float4 x = *p;
-      x.x = x.x * sc * g0;
-      x.y = x.y * sc * g1;
-      x.z = x.z * sc * g2;
-      x.w = x.w * sc * g3;
-      *p = x;
+      float4 v = *p;
+      v.x *= sc;
+      v.y *= sc;
+      v.z *= sc;
+      v.w *= sc;
+      *p = v;
     }
   }
   csync();
 }
 
-// Dot products of the 8 rows of one unit (NRW = 2: gate and up rows) against
-// the M activation rows, over the unit's ring slots.  Returns false on abort.
+// acc[m] += w(8 bf16 of `wv`) . act row m (8 floats at kidx), for m < M.
+__device__ __forceinline__ void dot8(const uint4 wv, const float* act, int AF, int kidx, int M,
+                                     float (&acc)[kDfMaxRows]) {
+  const float w0 = bf_lo(wv.x), w1 = bf_hi(wv.x), w2 = bf_lo(wv.y), w3 = bf_hi(wv.y);
+  const float w4 = bf_lo(wv.z), w5 = bf_hi(wv.z), w6 = bf_lo(wv.w), w7 = bf_hi(wv.w);
+#pragma unroll
+  for (int m = 0; m < kDfMaxRows; ++m) {
+    if (m >= M) break;
+    const float4 x0 = *reinterpret_cast<const float4*>(act + m * AF + kidx);
+    const float4 x1 = *reinterpret_cast<const float4*>(act + m * AF + kidx + 4);
+    float t = acc[m];
+    t = fmaf(w0, x0.x, t);
+    t = fmaf(w1, x0.y, t);
+    t = fmaf(w2, x0.z, t);
+    t = fmaf(w3, x0.w, t);
+    t = fmaf(w4, x1.x, t);
+    t = fmaf(w5, x1.y, t);
+    t = fmaf(w6, x1.z, t);
+    t = fmaf(w7, x1.w, t);
+    acc[m] = t;
+  }
+}
+
+// This warp's dot products for one unit: its output row (PAIR: its two rows,
+// lo / hi for QKV, gate / up for GU) against the M activation rows, over the
+// unit's ring slots.  Each lane handles 4 16-byte weight chunks per slot.  The
+// warp releases each slot on its own; no CTA-wide step.  Every lane ends with
+// the row totals.  false: a wait gave up.
 template <int OPK>
 __device__ bool unit_dots(const DraftFusedArgs& a, DfCtl& ctl, const uint8_t* ring, const float* act,
-                          int M, int n_slots, int kt_n, int swz_row_lo, int swz_row_hi,
-                          uint32_t& cons, float (&acc)[2][kDfMaxRows], int tid) {
-  const int w = tid >> 5, lane = tid & 31;
-  const int S = a.ring_slots, AF = a.act_floats;
+                          int M, int n_slots, int kt_n, int trow_lo, int trow_hi, Ring& rg,
+                          float (&acc)[2][kDfMaxRows], int w, int lane) {
+  constexpr bool PAIR = OPK == OP_QKV || OPK == OP_GU;
+  const int AF = a.act_floats;
 #pragma unroll
   for (int q = 0; q < 2; ++q)
 #pragma unroll
     for (int m = 0; m < kDfMaxRows; ++m) acc[q][m] = 0.f;
-  for (int s = 0; s < n_slots; ++s, ++cons) {
-    const int i = static_cast<int>(cons % static_cast<uint32_t>(S));
-    if (!mbar_wait_bounded(const_cast<uint64_t*>(&ctl.full[i]), (cons / S) & 1u, &ctl.abort, a.status))
-      return false;
-    const uint8_t* slot = ring + static_cast<size_t>(i) * kDfSlotBytes;
-    if constexpr (OPK == OP_GU) {
-      // 4 k tiles x (8 gate rows | 8 up rows) of 128-byte swizzled rows
-      const int kt0 = s * 4, nkt = min(4, kt_n - kt0);
-      const int q = lane;                   // chunk: k tile q / 8, column chunk q % 8
-      if (q < nkt * 8) {
-        const int ktl = q >> 3, c = q & 7;
-        const int kidx = (kt0 + ktl) * 64 + c * 8;
-        const int pos = (c ^ ((swz_row_lo + w) & 7)) * 16;
-        const uint4 wg = *reinterpret_cast<const uint4*>(slot + ktl * 1024 + w * 128 + pos);
-        const uint4 wu = *reinterpret_cast<const uint4*>(slot + 4096 + ktl * 1024 + w * 128 + pos);
+  const int sw_lo = (trow_lo + w) & 7, sw_hi = (trow_hi + w) & 7;
+  for (int s = 0; s < n_slots; ++s) {
+    if (!mbar_wait_bounded(&ctl.full[rg.i], rg.ph, &ctl.abort, a.status)) return false;
+    const uint8_t* slot = ring + static_cast<size_t>(rg.i) * kDfSlotBytes;
+    if constexpr (PAIR) {
+      const int kt0 = s * 8, nkt = min(8, kt_n - kt0);
 #pragma unroll
-        for (int m = 0; m < kDfMaxRows; ++m) {
-          if (m >= M) break;
-          const float4 x0 = *reinterpret_cast<const float4*>(act + m * AF + kidx);
-          const float4 x1 = *reinterpret_cast<const float4*>(act + m * AF + kidx + 4);
-          float t = acc[0][m];
-          t = fmaf(bf_lo(wg.x), x0.x, t); t = fmaf(bf_hi(wg.x), x0.y, t);
-          t = fmaf(bf_lo(wg.y), x0.z, t); t = fmaf(bf_hi(wg.y), x0.w, t);
-          t = fmaf(bf_lo(wg.z), x1.x, t); t = fmaf(bf_hi(wg.z), x1.y, t);
-          t = fmaf(bf_lo(wg.w), x1.z, t); t = fmaf(bf_hi(wg.w), x1.w, t);
-          acc[0][m] = t;
-          float v = acc[1][m];
-          v = fmaf(bf_lo(wu.x), x0.x, v); v = fmaf(bf_hi(wu.x), x0.y, v);
-          v = fmaf(bf_lo(wu.y), x0.z, v); v = fmaf(bf_hi(wu.y), x0.w, v);
-          v = fmaf(bf_lo(wu.z), x1.x, v); v = fmaf(bf_hi(wu.z), x1.y, v);
-          v = fmaf(bf_lo(wu.w), x1.z, v); v = fmaf(bf_hi(wu.w), x1.w, v);
-          acc[1][m] = v;
+      for (int h = 0; h < 2; ++h) {
+        const int q = lane + 32 * h, ktl = q >> 3, c = q & 7;
+        if (ktl < nkt) {
+          const int kidx = (kt0 + ktl) * 64 + c * 8;
+          const uint4 wa = *reinterpret_cast<const uint4*>(slot + ktl * 1024 + w * 128 + ((c ^ sw_lo) << 4));
+          const uint4 wb =
+              *reinterpret_cast<const uint4*>(slot + 8192 + ktl * 1024 + w * 128 + ((c ^ sw_hi) << 4));
+          dot8(wa, act, AF, kidx, M, acc[0]);
+          dot8(wb, act, AF, kidx, M, acc[1]);
+        }
+      }
+    } else if (OPK == OP_LM && a.tied) {
+      const int c0 = s * 1024;
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        const int q = lane + 32 * h, kidx = c0 + q * 8;
+        if (kidx < a.d) {
+          const uint4 wv = *reinterpret_cast<const uint4*>(slot + h * 4096 + w * 512 + (lane << 4));
+          dot8(wv, act, AF, kidx, M, acc[0]);
         }
       }
     } else {
+      const int kt0 = s * 16, nkt = min(16, kt_n - kt0);
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int q = lane + 32 * h;        // chunk of this row in the slot
-        bool have;
-        int woff, kidx;
-        if (OPK == OP_LM && a.tied) {       // row-major: 2 x [8 rows][256 columns]
-          const int c0 = s * 512;
-          kidx = c0 + q * 8;
-          have = kidx < a.d;
-          woff = (q >> 5) * 4096 + w * 512 + (q & 31) * 16;
-        } else {
-          const int kt0 = s * 8, nkt = min(8, kt_n - kt0);
-          const int ktl = q >> 3, c = q & 7;
-          have = q < nkt * 8;
-          kidx = (kt0 + ktl) * 64 + c * 8;
-          if (OPK == OP_QKV) {
-            const int hi = w >> 2, wr = w & 3;
-            const int trow = (hi ? swz_row_hi : swz_row_lo) + wr;
-            woff = hi * 4096 + ktl * 512 + wr * 128 + ((c ^ (trow & 7)) * 16);
-          } else {
-            woff = ktl * 1024 + w * 128 + ((c ^ ((swz_row_lo + w) & 7)) * 16);
-          }
-        }
-        if (!have) continue;
-        const uint4 wv = *reinterpret_cast<const uint4*>(slot + woff);
-#pragma unroll
-        for (int m = 0; m < kDfMaxRows; ++m) {
-          if (m >= M) break;
-          const float4 x0 = *reinterpret_cast<const float4*>(act + m * AF + kidx);
-          const float4 x1 = *reinterpret_cast<const float4*>(act + m * AF + kidx + 4);
-          float t = acc[0][m];
-          t = fmaf(bf_lo(wv.x), x0.x, t); t = fmaf(bf_hi(wv.x), x0.y, t);
-          t = fmaf(bf_lo(wv.y), x0.z, t); t = fmaf(bf_hi(wv.y), x0.w, t);
-          t = fmaf(bf_lo(wv.z), x1.x, t); t = fmaf(bf_hi(wv.z), x1.y, t);
-          t = fmaf(bf_lo(wv.w), x1.z, t); t = fmaf(bf_hi(wv.w), x1.w, t);
-          acc[0][m] = t;
+      for (int h = 0; h < 4; ++h) {
+        const int q = lane + 32 * h, ktl = q >> 3, c = q & 7;
+        if (ktl < nkt) {
+          const uint4 wv = *reinterpret_cast<const uint4*>(slot + ktl * 1024 + w * 128 + ((c ^ sw_lo) << 4));
+          dot8(wv, act, AF, (kt0 + ktl) * 64 + c * 8, M, acc[0]);
         }
       }
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(const_cast<uint64_t*>(&ctl.empty[i]));
+    if (lane == 0) mbar_arrive(&ctl.empty[rg.i]);
+    rg.next();
   }
   // fixed xor tree: every lane ends with the row totals
 #pragma unroll
-  for (int q = 0; q < 2; ++q)
+  for (int q = 0; q < (PAIR ? 2 : 1); ++q)
 #pragma unroll
     for (int m = 0; m < kDfMaxRows; ++m) {
       if (m >= M) break;
@@ -851,53 +857,54 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
   } else {
     const Geo geo = make_geo(a);
     const int G = geo.G, c = geo.c;
-    uint32_t cons = 0;
+    Ring rg;
+    rg.S = a.ring_slots;
     unsigned epoch = 0;
     unsigned long long t_phase = global_ns();
     bool run = true;
     float acc[2][kDfMaxRows];
     for (int j = 1; j <= a.K && run; ++j) {
-      // ---------------- the rows of this pass
-      if (tid == 0) {
-        const int R = j == 1 ? 2 : 1;
-        ctl.R = R;
-        ctl.rows = a.B * R;
-        for (int g = 0; g < a.B; ++g) {
-          const int L = a.seq_state[g * kStateInts + 0];
-          int valid, pos0;
-          if (j == 1) {
-            int nv = L - a.draft_len[g];
-            if (nv < 1 || nv > 2) {
-              atomicOr(a.status, 0x4u);     // draft cache not caught up
-              nv = nv < 1 ? 1 : 2;
-            }
-            valid = nv;
-            pos0 = L - nv;
-          } else {
-            valid = 1;
-            pos0 = L + j - 2;
+      // ---------------- the rows of this pass (one thread per request)
+      if (tid < a.B) {
+        const int g = tid, R = j == 1 ? 2 : 1;
+        const int L = a.seq_state[g * kStateInts + 0];
+        int valid, pos0;
+        if (j == 1) {
+          int nv = L - a.draft_len[g];
+          if (nv < 1 || nv > 2) {
+            atomicOr(a.status, 0x4u);     // draft cache not caught up
+            nv = nv < 1 ? 1 : 2;
           }
-          ctl.valid[g] = valid;
-          ctl.pos0[g] = pos0;
-          for (int i = 0; i < R; ++i) {
-            const int r = g * R + i, pos = pos0 + i;
-            bool ok = i < valid;
-            int tok = 0;
-            if (ok && (pos < 0 || pos >= a.max_seq)) {
-              atomicOr(a.status, 0x4u);
-              ok = false;
-            }
-            if (ok) {
-              tok = j == 1 ? a.tokens[static_cast<size_t>(g) * a.max_seq + pos] : ctl.next_tok[g];
-              if (tok < 0 || tok >= a.V) {
-                atomicOr(a.status, 0x2u);
-                tok = 0;
-              }
-            }
-            ctl.ok[r] = ok ? 1 : 0;
-            ctl.tok[r] = tok;
-          }
+          valid = nv;
+          pos0 = L - nv;
+        } else {
+          valid = 1;
+          pos0 = L + j - 2;
         }
+        ctl.valid[g] = valid;
+        ctl.pos0[g] = pos0;
+        for (int i = 0; i < R; ++i) {
+          const int r = g * R + i, pos = pos0 + i;
+          bool ok = i < valid;
+          int tok = 0;
+          if (ok && (pos < 0 || pos >= a.max_seq)) {
+            atomicOr(a.status, 0x4u);
+            ok = false;
+          }
+          if (ok) {
+            tok = j == 1 ? a.tokens[static_cast<size_t>(g) * a.max_seq + pos] : ctl.next_tok[g];
+            if (tok < 0 || tok >= a.V) {
+              atomicOr(a.status, 0x2u);
+              tok = 0;
+            }
+          }
+          ctl.ok[r] = ok ? 1 : 0;
+          ctl.tok[r] = tok;
+        }
+      }
+      if (tid == 0) {
+        ctl.R = j == 1 ? 2 : 1;
+        ctl.rows = a.B * ctl.R;
       }
       csync();
       const int R = ctl.R, rows = ctl.rows;
@@ -914,7 +921,7 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
               const int ctx = ctl.pos0[g] + ctl.valid[g];
               const int chunk = (ctx + a.n_splits - 1) / a.n_splits;
               const int k0 = s * chunk, k1 = min(min(k0 + chunk, ctx), ctl.pos0[g]);
-              if (k1 > k0 && ctl.pos0[g] + ctl.valid[g] <= a.max_seq) {
+              if (k1 > k0 && ctx <= a.max_seq) {
                 const int kvh = h / (a.H / a.Hkv);
                 const bf16* kc = a.kv + static_cast<size_t>(l) * 2 * a.layer_kv +
                                  (static_cast<size_t>(g) * a.Hkv + kvh) * a.max_seq * a.hd;
@@ -927,20 +934,19 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
                          reinterpret_cast<const bf16*>(a.w + a.off_attn_norm + loff), false, tid);
           const int off = cum % G;
           cum += geo.u_qkv;
-          const int upb = a.hd / kUR;               // units per head block
-          for (int u = first_unit(geo, off); u < geo.u_qkv && run; u += G) {
-            const int hb = u / upb, ui = u - hb * upb;
-            const int r_lo = hb * a.hd + 4 * ui, r_hi = r_lo + a.hd / 2;
-            run = csync_and(unit_dots<OP_QKV>(a, ctl, ring, act, rows, geo.s_qkv, geo.kt_d, r_lo % 128,
-                                              r_hi % 128, cons, acc, tid));
-            if (!run) break;
-            if (lane < rows) ctl.xch[warp][lane] = pick(acc[0], lane);
-            csync();
-            if (warp < 4 && lane < rows && ctl.ok[lane]) {
+          bool ok = true;
+          const int half = a.hd / 2;
+          for (int u = first_unit(geo, off); u < geo.u_qkv && ok; u += G) {
+            int hb, ui, lo, hi;
+            qkv_rows(a, u, &hb, &ui, &lo, &hi);
+            ok = unit_dots<OP_QKV>(a, ctl, ring, act, rows, geo.s_qkv, geo.kt_d, lo % 128, hi % 128, rg, acc,
+                                   warp, lane);
+            if (!ok) break;
+            // this warp's pair (fi, fi + hd/2) of head block hb; lane m: row m
+            const int fi = kUR * ui + warp;
+            if (lane < rows && ctl.ok[lane]) {
               const int m = lane, g = m / R, pos = ctl.pos0[g] + (m - g * R);
-              const float x1 = ctl.xch[warp][m], x2 = ctl.xch[warp + 4][m];
-              const int fi = 4 * ui + warp;         // pair (fi, fi + hd/2) of the head
-              const int half = a.hd / 2;
+              const float x1 = pick(acc[0], m), x2 = pick(acc[1], m);
               if (hb < a.H + a.Hkv) {
                 const float cs = a.rope_cos[static_cast<size_t>(pos) * half + fi];
                 const float sn = a.rope_sin[static_cast<size_t>(pos) * half + fi];
@@ -962,8 +968,8 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
                 vd[fi + half] = __float2bfloat16_rn(x2);
               }
             }
-            csync();
           }
+          run = csync_and(ok);
           if (run) run = grid_sync(a, ctl, epoch, tid, t_phase);
         }
         // ---------------- attention
@@ -983,7 +989,7 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
           }
           run = grid_sync(a, ctl, epoch, tid, t_phase);
         }
-        // ---------------- O projection + residual (combines the key splits)
+        // ---------------- O projection + residual
         if (run) {
           const int off = cum % G;
           cum += geo.u_o;
@@ -1011,15 +1017,17 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
             }
             csync();
           }
-          for (int u = fu; u < geo.u_o && run; u += G) {
-            run = csync_and(unit_dots<OP_O>(a, ctl, ring, act, rows, geo.s_o, geo.kt_q, (u * kUR) % 128, 0,
-                                            cons, acc, tid));
-            if (!run) break;
-            if (lane < rows && ctl.ok[lane]) {
-              float* hp = a.h + static_cast<size_t>(lane) * a.d + u * kUR + warp;
-              *hp = ldcg(hp) + pick(acc[0], lane);
-            }
+          bool ok = true;
+          for (int u = fu; u < geo.u_o && ok; u += G) {
+            const int row = u * kUR + warp;
+            float hold = 0.f;
+            if (lane < rows && ctl.ok[lane]) hold = ldcg(a.h + static_cast<size_t>(lane) * a.d + row);
+            ok = unit_dots<OP_O>(a, ctl, ring, act, rows, geo.s_o, geo.kt_q, (u * kUR) % 128, 0, rg, acc, warp,
+                                 lane);
+            if (ok && lane < rows && ctl.ok[lane])
+              a.h[static_cast<size_t>(lane) * a.d + row] = hold + pick(acc[0], lane);
           }
+          run = csync_and(ok);
           if (run) run = grid_sync(a, ctl, epoch, tid, t_phase);
         }
         // ---------------- gate/up + SwiGLU
@@ -1030,16 +1038,17 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
           if (fu < geo.u_gu)
             load_norm_rows(a, ctl, act, 1, reinterpret_cast<const bf16*>(a.w + a.off_ffn_norm + loff), false,
                            tid);
-          for (int u = fu; u < geo.u_gu && run; u += G) {
-            run = csync_and(unit_dots<OP_GU>(a, ctl, ring, act, rows, geo.s_gu, geo.kt_d, (u * kUR) % 64, 0,
-                                             cons, acc, tid));
-            if (!run) break;
-            if (lane < rows && ctl.ok[lane]) {
+          bool ok = true;
+          for (int u = fu; u < geo.u_gu && ok; u += G) {
+            ok = unit_dots<OP_GU>(a, ctl, ring, act, rows, geo.s_gu, geo.kt_d, (u * kUR) % 64, (u * kUR) % 64, rg,
+                                  acc, warp, lane);
+            if (ok && lane < rows && ctl.ok[lane]) {
               const float gt = pick(acc[0], lane), up = pick(acc[1], lane);
               const float sg = gt / (1.f + expf(-gt));
               a.act[static_cast<size_t>(lane) * a.F + u * kUR + warp] = sg * up;
             }
           }
+          run = csync_and(ok);
           if (run) run = grid_sync(a, ctl, epoch, tid, t_phase);
         }
         // ---------------- down + residual
@@ -1070,15 +1079,17 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
             }
             csync();
           }
-          for (int u = fu; u < geo.u_down && run; u += G) {
-            run = csync_and(unit_dots<OP_DOWN>(a, ctl, ring, act, rows, geo.s_down, geo.kt_f, (u * kUR) % 128,
-                                               0, cons, acc, tid));
-            if (!run) break;
-            if (lane < rows && ctl.ok[lane]) {
-              float* hp = a.h + static_cast<size_t>(lane) * a.d + u * kUR + warp;
-              *hp = ldcg(hp) + pick(acc[0], lane);
-            }
+          bool ok = true;
+          for (int u = fu; u < geo.u_down && ok; u += G) {
+            const int row = u * kUR + warp;
+            float hold = 0.f;
+            if (lane < rows && ctl.ok[lane]) hold = ldcg(a.h + static_cast<size_t>(lane) * a.d + row);
+            ok = unit_dots<OP_DOWN>(a, ctl, ring, act, rows, geo.s_down, geo.kt_f, (u * kUR) % 128, 0, rg, acc,
+                                    warp, lane);
+            if (ok && lane < rows && ctl.ok[lane])
+              a.h[static_cast<size_t>(lane) * a.d + row] = hold + pick(acc[0], lane);
           }
+          run = csync_and(ok);
           if (run) run = grid_sync(a, ctl, epoch, tid, t_phase);
         }
       }
@@ -1092,24 +1103,15 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
           load_norm_rows(a, ctl, act, 1, reinterpret_cast<const bf16*>(a.w + a.off_final_norm), true, tid);
         const bool greedy = a.greedy != 0;
         const float it = a.inv_temp;
-        unsigned long long* tr_lm = nullptr;
-        {
-          const int phase = j * (5 * a.n_layers + 1) - 1;
-          if (a.trace != nullptr && phase < a.trace_phases && tid == 0)
-            tr_lm = a.trace + 2 + (static_cast<size_t>(phase) * G + c) * 16;
-        }
-        for (int u = ulo; u < uhi && run; ++u) {
-          if (tr_lm != nullptr && ((u - ulo) & 3) == 0 && (u - ulo) < 24) {
-            const int k = (u - ulo) >> 2;               // 0..5 -> slots 9..12, 14, 15
-            tr_lm[k < 4 ? 9 + k : 10 + k] = global_ns();
-          }
-          run = csync_and(unit_dots<OP_LM>(a, ctl, ring, act, B, geo.s_lm, geo.kt_d, (u * kUR) % 128, 0,
-                                           cons, acc, tid));
-          if (!run) break;
+        float* zrow = a.zd + (static_cast<size_t>(lane) * a.K + (j - 1)) * a.V;
+        bool ok = true;
+        for (int u = ulo; u < uhi && ok; ++u) {
+          ok = unit_dots<OP_LM>(a, ctl, ring, act, B, geo.s_lm, geo.kt_d, (u * kUR) % 128, 0, rg, acc, warp,
+                                lane);
           const int v = u * kUR + warp;
-          if (lane < B && v < a.V) {
+          if (ok && lane < B && v < a.V) {
             const float z = pick(acc[0], lane);
-            a.zd[(static_cast<size_t>(lane) * a.K + (j - 1)) * a.V + v] = z;
+            zrow[v] = z;
             if (z > sm_m) {
               if (!greedy) sm_s = (sm_m == -INFINITY) ? 0.f : sm_s * __expf((sm_m - z) * it);
               sm_m = z;
@@ -1118,6 +1120,7 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
             if (!greedy) sm_s += __expf((z - sm_m) * it);
           }
         }
+        run = csync_and(ok);
         if (run) {
           // this CTA's statistics per request: warps combined in order
           if (lane < B) {
@@ -1186,11 +1189,16 @@ size_t draft_fused_smem_bytes(int ring_slots, int act_rows, int act_floats) {
          static_cast<size_t>(kDfScratchFloats) * 4;
 }
 
-size_t draft_fused_static_smem() { return sizeof(DfCtl); }
+// Static shared memory of the kernel as compiled (the control block, padded).
+size_t draft_fused_static_smem() {
+  cudaFuncAttributes fa{};
+  if (cudaFuncGetAttributes(&fa, draft_fused_kernel) != cudaSuccess) return 4096;
+  return fa.sharedSizeBytes;
+}
 
 cudaError_t draft_fused_set_max_smem() {
   return cudaFuncSetAttribute(draft_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(227 * 1024 - sizeof(DfCtl) - 64));
+                              static_cast<int>(227 * 1024 - draft_fused_static_smem()));
 }
 
 cudaError_t launch_draft_fused(const DraftFusedArgs& a, int grid, cudaStream_t s, bool cooperative) {

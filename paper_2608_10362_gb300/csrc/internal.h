@@ -198,8 +198,8 @@ struct AcceptArgs {
 // kDfMaxGroups requests.
 constexpr int kDfMaxGroups = 4;
 constexpr int kDfMaxRows = 2 * kDfMaxGroups;
-constexpr int kDfSlotBytes = 8192;      // weight ring slot
-constexpr int kDfMaxSlots = 32;
+constexpr int kDfSlotBytes = 16384;     // weight ring slot
+constexpr int kDfMaxSlots = 16;
 constexpr int kDfComputeWarps = 8;
 constexpr int kDfThreads = (kDfComputeWarps + 1) * 32;   // + one copy-issuing warp
 constexpr int kDfMaxLayers = 32;
