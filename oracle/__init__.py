@@ -16,6 +16,10 @@ What it restates, and where it comes from:
   RMSNorm, rotary position embedding, causal grouped-query attention over a
   KV cache that holds bf16 values (the workload's KV precision), SwiGLU
   feed-forward, LM head.
+* ``int4`` - the group-wise INT4 weight-only linear layer of the paper's GPTQ
+  INT4 targets (Section 4.1): w = (q - z) s per group of inputs, y = x W^T.
+* ``scheduler`` - MemSpec's draft cache update and runtime loop (Sections
+  3.3-3.4, Algorithms 2-3) and the MAB-Async baseline (Sections 2.3, 4.1).
 * ``speculative`` - the draft-and-verify iteration that MemSpec runs unchanged
   (Section 3.5: "the standard draft-and-verify process"; Section 2.1, Eq. 1:
   throughput ~ E[A] / L_iter), with the acceptance rule of the speculative

@@ -25,7 +25,7 @@ import numpy as np
 __all__ = [
     "ModelShape", "SHAPES", "tensor_names", "tensor_shape", "gen_tensor",
     "iter_weights", "gen_weights", "gen_prompt", "gen_logits", "gen_kv",
-    "bf16_round", "gen_score_stream",
+    "bf16_round", "gen_score_stream", "gen_int4_weights",
 ]
 
 
@@ -194,3 +194,15 @@ def gen_score_stream(seed: int, points: int, n_drafts: int, phase: int = 4,
         row[best] = 1.0
         out[i] = (row + rng.standard_normal(n_drafts) * noise).astype(np.float32)
     return out
+
+
+def gen_int4_weights(seed: int, n: int, k: int, group: int = 128, scale: float = 0.004):
+    """Random group-wise INT4 weights: packed codes uint8 [n][k/2] (two 4-bit codes
+    per byte, low nibble first), scales [n][k/group] as bf16-valued float32 (about
+    `scale` in size), zero points uint8 [n][k/group] in 0..15."""
+    rng = np.random.default_rng([seed, 0x696E7434, n, k])
+    codes = rng.integers(0, 16, size=(n, k), dtype=np.int64)
+    packed = (codes[:, 0::2] | (codes[:, 1::2] << 4)).astype(np.uint8)
+    scales = bf16_round((rng.random((n, k // group)) * 1.5 + 0.5).astype(np.float32) * np.float32(scale))
+    zeros = rng.integers(0, 16, size=(n, k // group), dtype=np.int64).astype(np.uint8)
+    return packed, scales, zeros
