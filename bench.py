@@ -612,6 +612,77 @@ def run_switching_case(args):
             "prefix": prefix, "K": K, "T": T, "policies": results, "device_status": bits}
 
 
+def run_int4_case(args):
+    """The 7B target's projections as group-wise INT4 weights (the paper's GPTQ
+    INT4 targets): 32 layers x (qkv 12288x4096, o 4096x4096, gate_up 22016x4096,
+    down 4096x11008) with distinct random codes (3.6 GB packed, far above L2),
+    one launch per projection at `rows` activation rows (K + 1 = 5 for one
+    verify pass), replayed from a CUDA graph.  Reports each shape's mean launch time over the 32 layers and
+    the whole stack's algorithmic bytes / time against the measured HBM peak."""
+    import torch
+
+    from paper_2608_10362_gb300 import int4_pack, op_linear_int4
+    from seeded_inputs import SHAPES
+    t = SHAPES[TARGET]
+    shapes = {"qkv": (t.q_dim + 2 * t.kv_dim, t.d_model), "o": (t.d_model, t.q_dim),
+              "gate_up": (2 * t.d_ffn, t.d_model), "down": (t.d_model, t.d_ffn)}
+    rows = args.rows
+    gen = torch.Generator(device="cuda").manual_seed(0)
+    layers = []
+    for _ in range(t.n_layers):
+        ent = {}
+        for name, (n, k) in shapes.items():
+            qw = torch.randint(0, 256, (n, k // 2), dtype=torch.uint8, device="cuda", generator=gen)
+            sc = (torch.rand(n, k // 128, device="cuda", generator=gen) * 0.006 + 0.002).to(torch.bfloat16)
+            zs = torch.randint(0, 16, (n, k // 128), dtype=torch.uint8, device="cuda", generator=gen)
+            ent[name] = int4_pack(qw, sc, zs)
+            del qw, sc, zs
+        layers.append(ent)
+    xs = {k: (torch.randn(rows, k, device="cuda", generator=gen)).to(torch.bfloat16)
+          for k in {t.d_model, t.q_dim, t.d_ffn}}
+    ys = {name: torch.empty(rows, n, device="cuda") for name, (n, k) in shapes.items()}
+
+    def nbytes(name):
+        n, k = shapes[name]
+        return ((n + 15) // 16) * (k // 128) * 1072 + rows * k * 2 + rows * n * 4
+
+    def run(names):
+        for ent in layers:
+            for name in names:
+                n, k = shapes[name]
+                op_linear_int4(xs[k], ent[name], n, y=ys[name])
+
+    out = {"case": "int4", "target": TARGET, "rows": rows, "layers": t.n_layers, "group": 128, "shapes": {}}
+    peak, peak_src = measured_peaks()
+    out["peak"] = {"hbm_GBps": peak, "source": peak_src}
+    for names in [[nm] for nm in shapes] + [list(shapes)]:
+        for _ in range(args.warmup):
+            run(names)
+        torch.cuda.synchronize()
+        # the pass's launches replayed from a CUDA graph: the timing is the
+        # kernels', not the Python loop's
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            run(names)
+        graph.replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(1, args.steps)
+        a.record()
+        for _ in range(reps):
+            graph.replay()
+        b.record()
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / reps
+        byt = sum(nbytes(nm) for nm in names) * t.n_layers
+        gbs = byt / ms / 1e6
+        key = names[0] if len(names) == 1 else "all"
+        out["shapes"][key] = {"us_per_launch": ms * 1e3 / (t.n_layers * len(names)),
+                              "ms_per_pass": ms, "bytes_per_pass": byt, "GB/s": gbs,
+                              "frac_of_hbm_peak": gbs / peak}
+    return out
+
+
 def run_case(args):
     """Diagnostic cases (not the headline metric)."""
     import numpy as np
@@ -638,6 +709,8 @@ def run_case(args):
         nbytes = args.n * args.kdim * 2 + args.rows * (args.kdim * 2 + args.n * 4)
         return {"case": "gemm", "n_out": args.n, "k": args.kdim, "rows": args.rows,
                 "us_per_launch": ms * 1e3, "GB/s": nbytes / ms / 1e6}
+    if args.case == "int4":
+        return run_int4_case(args)
     from paper_2608_10362_gb300 import Engine
     if args.case == "edge":
         return {"case": "edge", **run_pair_case(args, "target_1b1", "draft_68m", [512], 5, args.temp)}
@@ -782,7 +855,7 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--case", default="step", choices=["step", "gemm", "small", "verify", "prefill", "edge", "batched",
-                                                          "switching"],
+                                                          "switching", "int4"],
                     help="step: the workload above; gemm / small: diagnostic cases sized for "
                          "profiler captures (one projection GEMM; a 160M target with a 68M draft)")
     ap.add_argument("--temp", type=float, default=0.8, help="(--case edge) temperature")

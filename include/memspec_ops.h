@@ -58,6 +58,38 @@ memspec_status memspec_op_linear_noalloc(const void* x_dev, const void* w_dev, f
                                          int32_t rows, int32_t n_out, int32_t k,
                                          uint32_t* status_dev, void* stream);
 
+/* Group-wise INT4 weight-only linear layer (the paper's targets are GPTQ INT4
+ * models, Section 4.1).  The weights W[n_out][k] are given GPTQ-style,
+ *   W[r][c] = (q[r][c] - zeros[r][c/128]) * scales[r][c/128],
+ *   qweight: uint8 [n_out][k/2], byte j of row r = q[r][2j] | q[r][2j+1] << 4
+ *   scales:  bf16  [n_out][k/128];   zeros: uint8 [n_out][k/128], values 0..15
+ * and are repacked once, by memspec_int4_pack, into the kernel's layout (one
+ * 1072-byte record per 16-row tile and 128-column group; rows past n_out are
+ * zero-filled).  The layout is private to this library: only
+ * memspec_op_linear_int4 reads it.
+ *
+ * memspec_int4_packed_bytes: bytes of the packed copy, or -1 for bad sizes
+ * (n_out >= 1, k a positive multiple of 128). */
+int64_t memspec_int4_packed_bytes(int32_t n_out, int32_t k);
+
+/* Repack on `stream` (device pointers; qweight 4-byte, scales 2-byte, packed
+ * 16-byte aligned; packed holds memspec_int4_packed_bytes).  The caller owns
+ * every buffer; nothing is allocated.  Errors: INVALID_ARG (n_out outside
+ * 1..1048576, k not a positive multiple of 128, NULL, misalignment), CUDA. */
+memspec_status memspec_int4_pack(const void* qweight_dev, const void* scales_dev, const void* zeros_dev,
+                                 int32_t n_out, int32_t k, void* packed_dev, void* stream);
+
+/* y[rows][n_out] (fp32) = x[rows][k] (bf16, row-major) . W^T, enqueued on
+ * `stream`.  rows in 1..16; x and packed 16-byte aligned, y 4-byte aligned;
+ * rows <= 8 needs 16 (k + 32) + k/16 + 16384 bytes of shared memory, rows
+ * 9..16 twice that, at most 220 KB (else UNSUPPORTED).  Results are
+ * deterministic.  Allocates nothing: the cross-CTA partial sums and tile
+ * counters live in static device arrays, so calls on one device must not run
+ * concurrently (stream-ordered calls are fine).  Errors: INVALID_ARG,
+ * UNSUPPORTED, CUDA. */
+memspec_status memspec_op_linear_int4(const void* x_dev, const void* packed_dev, float* y_dev, int32_t rows,
+                                      int32_t n_out, int32_t k, void* stream);
+
 /* Categorical sampling of each row of logits[rows][vocab] (fp32): with T > 0,
  * out[r] = smallest j with sum_{i<=j} exp(z_i/T - m) > u[r] * sum_i exp(z_i/T - m);
  * with T == 0, out[r] = argmax (lowest id on ties).  u_dev: fp32 [rows] in

@@ -7,5 +7,5 @@ built (python -m paper_2608_10362_gb300.build).
 """
 from ._lib import MemSpecError, load  # noqa: F401
 from .engine import (Engine, fill_blob, kv_bytes, model_cfg, op_linear, pack_matrix,  # noqa: F401
-                     op_linear_noalloc, op_sample, weights_bytes)
+                     int4_pack, op_linear_int4, op_linear_noalloc, op_sample, weights_bytes)
 from .sched import DraftScheduler  # noqa: F401

@@ -117,6 +117,11 @@ EXPORTS = {
                                     C.c_int32, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
     "memspec_op_linear_noalloc": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
                                             C.c_int32, C.c_int32, C.c_void_p, C.c_void_p]),
+    "memspec_int4_packed_bytes": (C.c_int64, [C.c_int32, C.c_int32]),
+    "memspec_int4_pack": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p,
+                                    C.c_void_p]),
+    "memspec_op_linear_int4": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
+                                         C.c_void_p]),
     "memspec_op_sample": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_float, C.c_void_p,
                                     C.c_void_p, C.c_void_p]),
     "memspec_op_last_error": (C.c_char_p, []),

@@ -120,6 +120,11 @@ bool ensure_func_attrs() {
     g_attr_error = std::string("fused draft kernel smem attribute: ") + cudaGetErrorString(e);
     return false;
   }
+  e = int4_set_max_smem();
+  if (e != cudaSuccess) {
+    g_attr_error = std::string("int4 kernel smem attribute: ") + cudaGetErrorString(e);
+    return false;
+  }
   done = true;
   return true;
 }
@@ -2074,6 +2079,76 @@ memspec_status memspec_op_linear(const void* x, const void* w, float* y, int32_t
                               static_cast<cudaStream_t>(stream), false);
   if (e != cudaSuccess) {
     g_op_error = std::string("gemm launch: ") + cudaGetErrorString(e);
+    return MEMSPEC_ERR_CUDA;
+  }
+  return MEMSPEC_OK;
+}
+
+int64_t memspec_int4_packed_bytes(int32_t n_out, int32_t k) {
+  if (n_out < 1 || k < 128 || k % 128 != 0) return -1;
+  return static_cast<int64_t>(int4_packed_bytes(n_out, k));
+}
+
+memspec_status memspec_int4_pack(const void* qweight, const void* scales, const void* zeros, int32_t n_out,
+                                 int32_t k, void* packed, void* stream) {
+  if (qweight == nullptr || scales == nullptr || zeros == nullptr || packed == nullptr) {
+    g_op_error = "null pointer";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (n_out < 1 || k < 128 || k % 128 != 0 || n_out > int4_max_rows()) {
+    g_op_error = "n_out in 1..1048576 and k a positive multiple of 128 required";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if ((reinterpret_cast<uintptr_t>(qweight) & 3) || (reinterpret_cast<uintptr_t>(scales) & 1) ||
+      (reinterpret_cast<uintptr_t>(packed) & 15)) {
+    g_op_error = "qweight must be 4-byte, scales 2-byte and packed 16-byte aligned";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  cudaError_t e = launch_int4_pack(static_cast<const uint8_t*>(qweight), static_cast<const bf16*>(scales),
+                                   static_cast<const uint8_t*>(zeros), static_cast<uint8_t*>(packed), n_out, k,
+                                   static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) {
+    g_op_error = std::string("int4 pack launch: ") + cudaGetErrorString(e);
+    return MEMSPEC_ERR_CUDA;
+  }
+  return MEMSPEC_OK;
+}
+
+memspec_status memspec_op_linear_int4(const void* x, const void* packed, float* y, int32_t rows,
+                                      int32_t n_out, int32_t k, void* stream) {
+  if (x == nullptr || packed == nullptr || y == nullptr) {
+    g_op_error = "null pointer";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (rows < 1 || rows > kInt4MaxRows || n_out < 1 || k < 128 || k % 128 != 0 || n_out > int4_max_rows()) {
+    g_op_error = "rows in 1..16, n_out in 1..1048576 and k a positive multiple of 128 required";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if ((reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(packed) & 15) ||
+      (reinterpret_cast<uintptr_t>(y) & 3)) {
+    g_op_error = "x and packed must be 16-byte aligned, y 4-byte aligned";
+    return MEMSPEC_ERR_INVALID_ARG;
+  }
+  if (int4_smem_bytes(rows, k) > static_cast<size_t>(kInt4MaxSmem)) {
+    g_op_error = "rows x k too large for the activations in shared memory";
+    return MEMSPEC_ERR_UNSUPPORTED;
+  }
+  if (!ensure_func_attrs()) {
+    g_op_error = g_attr_error;
+    return MEMSPEC_ERR_CUDA;
+  }
+  Int4Args a{};
+  a.x = static_cast<const bf16*>(x);
+  a.packed = static_cast<const uint8_t*>(packed);
+  a.y = y;
+  a.rows = rows;
+  a.n = n_out;
+  a.k = k;
+  const long long units = static_cast<long long>((n_out + 15) / 16) * (k / 128);
+  const int grid = static_cast<int>(std::max(1LL, std::min<long long>(std::min(sm_count(), int4_max_ctas()), units)));
+  cudaError_t e = launch_int4_linear(a, grid, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) {
+    g_op_error = std::string("int4 launch: ") + cudaGetErrorString(e);
     return MEMSPEC_ERR_CUDA;
   }
   return MEMSPEC_OK;

@@ -252,6 +252,26 @@ constexpr int kDfScratchFloatsHost = 2 * 256 + 2 * 128 + 8 * 2 * 128;   // == kD
 cudaError_t draft_fused_set_max_smem();
 cudaError_t launch_draft_fused(const DraftFusedArgs& a, int grid, cudaStream_t s, bool cooperative);
 
+// Group-wise INT4 weight-only linear layer (int4.cu): y = x (q - z) s^T over a
+// repacked weight copy of one 1072-byte record per (16-row tile, 128-column group).
+constexpr int kInt4MaxRows = 16;
+constexpr int kInt4RecordBytes = 1072;
+constexpr int kInt4MaxSmem = 220 * 1024;
+struct Int4Args {
+  const bf16* x;            // [rows][k] bf16
+  const uint8_t* packed;    // records, tile-major
+  float* y;                 // [rows][n]
+  int rows, n, k;
+};
+size_t int4_packed_bytes(long long n, int k);
+size_t int4_smem_bytes(int rows, int k);
+int int4_max_ctas();
+long long int4_max_rows();
+cudaError_t int4_set_max_smem();
+cudaError_t launch_int4_linear(const Int4Args& a, int grid, cudaStream_t s);
+cudaError_t launch_int4_pack(const uint8_t* qweight, const bf16* scales, const uint8_t* zeros, uint8_t* out,
+                             int n, int k, cudaStream_t s);
+
 // launchers (each returns the launch's cudaError_t)
 cudaError_t launch_embed(const EmbedArgs& a, int rows, cudaStream_t s, bool pdl);
 cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s, bool pdl);

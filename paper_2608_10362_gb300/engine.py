@@ -370,6 +370,38 @@ def op_linear_noalloc(x: torch.Tensor, w: torch.Tensor, y: torch.Tensor | None =
     return y
 
 
+def int4_pack(qweight: torch.Tensor, scales: torch.Tensor, zeros: torch.Tensor,
+              stream: torch.cuda.Stream | None = None) -> torch.Tensor:
+    """Repack GPTQ-style INT4 weights (qweight uint8 [n][k/2], scales bf16
+    [n][k/128], zeros uint8 [n][k/128], all on cuda) into the layout
+    op_linear_int4 reads; returns the packed uint8 buffer."""
+    lib = _lib.load()
+    n_out, half_k = qweight.shape
+    k = 2 * half_k
+    nbytes = lib.memspec_int4_packed_bytes(n_out, k)
+    if nbytes < 0:
+        raise MemSpecError(_lib.ERR_INVALID_ARG, f"bad INT4 shape n={n_out} k={k}")
+    packed = torch.empty(nbytes, dtype=torch.uint8, device=qweight.device)
+    s = stream or torch.cuda.current_stream(qweight.device)
+    _check(lib, lib.memspec_int4_pack(qweight.data_ptr(), scales.data_ptr(), zeros.data_ptr(), n_out, k,
+                                      packed.data_ptr(), s.cuda_stream))
+    return packed
+
+
+def op_linear_int4(x: torch.Tensor, packed: torch.Tensor, n_out: int, y: torch.Tensor | None = None,
+                   stream: torch.cuda.Stream | None = None) -> torch.Tensor:
+    """y = x . W^T (fp32 [rows][n_out]) for x bf16 [rows][k] and W packed by
+    int4_pack."""
+    lib = _lib.load()
+    rows, k = x.shape
+    if y is None:
+        y = torch.empty(rows, n_out, dtype=torch.float32, device=x.device)
+    s = stream or torch.cuda.current_stream(x.device)
+    _check(lib, lib.memspec_op_linear_int4(x.data_ptr(), packed.data_ptr(), y.data_ptr(), rows, n_out, k,
+                                           s.cuda_stream))
+    return y
+
+
 def op_sample(logits: torch.Tensor, temperature: float, u: torch.Tensor | None = None):
     lib = _lib.load()
     rows, vocab = logits.shape
