@@ -628,8 +628,9 @@ def run_int4_case(args):
               "gate_up": (2 * t.d_ffn, t.d_model), "down": (t.d_model, t.d_ffn)}
     rows = args.rows
     gen = torch.Generator(device="cuda").manual_seed(0)
+    n_layers = args.int4_layers or t.n_layers
     layers = []
-    for _ in range(t.n_layers):
+    for _ in range(n_layers):
         ent = {}
         for name, (n, k) in shapes.items():
             qw = torch.randint(0, 256, (n, k // 2), dtype=torch.uint8, device="cuda", generator=gen)
@@ -652,7 +653,7 @@ def run_int4_case(args):
                 n, k = shapes[name]
                 op_linear_int4(xs[k], ent[name], n, y=ys[name])
 
-    out = {"case": "int4", "target": TARGET, "rows": rows, "layers": t.n_layers, "group": 128, "shapes": {}}
+    out = {"case": "int4", "target": TARGET, "rows": rows, "layers": n_layers, "group": 128, "shapes": {}}
     peak, peak_src = measured_peaks()
     out["peak"] = {"hbm_GBps": peak, "source": peak_src}
     for names in [[nm] for nm in shapes] + [list(shapes)]:
@@ -674,10 +675,10 @@ def run_int4_case(args):
         b.record()
         torch.cuda.synchronize()
         ms = a.elapsed_time(b) / reps
-        byt = sum(nbytes(nm) for nm in names) * t.n_layers
+        byt = sum(nbytes(nm) for nm in names) * n_layers
         gbs = byt / ms / 1e6
         key = names[0] if len(names) == 1 else "all"
-        out["shapes"][key] = {"us_per_launch": ms * 1e3 / (t.n_layers * len(names)),
+        out["shapes"][key] = {"us_per_launch": ms * 1e3 / (n_layers * len(names)),
                               "ms_per_pass": ms, "bytes_per_pass": byt, "GB/s": gbs,
                               "frac_of_hbm_peak": gbs / peak}
     return out
@@ -871,6 +872,8 @@ def main():
     ap.add_argument("--n", type=int, default=22016)
     ap.add_argument("--kdim", type=int, default=4096)
     ap.add_argument("--rows", type=int, default=5)
+    ap.add_argument("--int4-layers", type=int, default=0,
+                    help="(--case int4) layers of INT4 weights (default: all of the 7B target's)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.case != "step":

@@ -81,12 +81,11 @@ memspec_status memspec_int4_pack(const void* qweight_dev, const void* scales_dev
 
 /* y[rows][n_out] (fp32) = x[rows][k] (bf16, row-major) . W^T, enqueued on
  * `stream`.  rows in 1..16; x and packed 16-byte aligned, y 4-byte aligned;
- * rows <= 8 needs 16 (k + 32) + k/16 + 16384 bytes of shared memory, rows
- * 9..16 twice that, at most 220 KB (else UNSUPPORTED).  Results are
- * deterministic.  Allocates nothing: the cross-CTA partial sums and tile
- * counters live in static device arrays, so calls on one device must not run
- * concurrently (stream-ordered calls are fine).  Errors: INVALID_ARG,
- * UNSUPPORTED, CUDA. */
+ * the activations (rows (2k + 64) bytes) plus a ring of at least two
+ * 1072-byte records per warp (16 warps) must fit in 220 KB of shared memory
+ * (else UNSUPPORTED: e.g. rows 9..16 at k = 11008).  Results are
+ * deterministic.  Allocates nothing and keeps no state between calls.
+ * Errors: INVALID_ARG (sizes, NULL, misalignment), UNSUPPORTED, CUDA. */
 memspec_status memspec_op_linear_int4(const void* x_dev, const void* packed_dev, float* y_dev, int32_t rows,
                                       int32_t n_out, int32_t k, void* stream);
 

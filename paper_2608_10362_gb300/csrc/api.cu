@@ -2095,7 +2095,7 @@ memspec_status memspec_int4_pack(const void* qweight, const void* scales, const 
     g_op_error = "null pointer";
     return MEMSPEC_ERR_INVALID_ARG;
   }
-  if (n_out < 1 || k < 128 || k % 128 != 0 || n_out > int4_max_rows()) {
+  if (n_out < 1 || k < 128 || k % 128 != 0 || n_out > (1 << 20)) {
     g_op_error = "n_out in 1..1048576 and k a positive multiple of 128 required";
     return MEMSPEC_ERR_INVALID_ARG;
   }
@@ -2120,7 +2120,7 @@ memspec_status memspec_op_linear_int4(const void* x, const void* packed, float* 
     g_op_error = "null pointer";
     return MEMSPEC_ERR_INVALID_ARG;
   }
-  if (rows < 1 || rows > kInt4MaxRows || n_out < 1 || k < 128 || k % 128 != 0 || n_out > int4_max_rows()) {
+  if (rows < 1 || rows > kInt4MaxRows || n_out < 1 || k < 128 || k % 128 != 0 || n_out > (1 << 20)) {
     g_op_error = "rows in 1..16, n_out in 1..1048576 and k a positive multiple of 128 required";
     return MEMSPEC_ERR_INVALID_ARG;
   }
@@ -2129,14 +2129,18 @@ memspec_status memspec_op_linear_int4(const void* x, const void* packed, float* 
     g_op_error = "x and packed must be 16-byte aligned, y 4-byte aligned";
     return MEMSPEC_ERR_INVALID_ARG;
   }
-  if (int4_smem_bytes(rows, k) > static_cast<size_t>(kInt4MaxSmem)) {
-    g_op_error = "rows x k too large for the activations in shared memory";
+  if (int4_pick_depth(rows, k) == 0) {
+    g_op_error = "rows x k too large for the activations and a 2-slot ring per warp in shared memory";
     return MEMSPEC_ERR_UNSUPPORTED;
   }
   if (!ensure_func_attrs()) {
     g_op_error = g_attr_error;
     return MEMSPEC_ERR_CUDA;
   }
+  // whole 16-row tiles, the same number per CTA, at most one CTA per SM
+  const int tiles = (n_out + 15) / 16;
+  const int per_cta = (tiles + sm_count() - 1) / sm_count();
+  const int grid = (tiles + per_cta - 1) / per_cta;
   Int4Args a{};
   a.x = static_cast<const bf16*>(x);
   a.packed = static_cast<const uint8_t*>(packed);
@@ -2144,8 +2148,7 @@ memspec_status memspec_op_linear_int4(const void* x, const void* packed, float* 
   a.rows = rows;
   a.n = n_out;
   a.k = k;
-  const long long units = static_cast<long long>((n_out + 15) / 16) * (k / 128);
-  const int grid = static_cast<int>(std::max(1LL, std::min<long long>(std::min(sm_count(), int4_max_ctas()), units)));
+  a.tiles_per_cta = per_cta;
   cudaError_t e = launch_int4_linear(a, grid, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) {
     g_op_error = std::string("int4 launch: ") + cudaGetErrorString(e);

@@ -262,11 +262,11 @@ struct Int4Args {
   const uint8_t* packed;    // records, tile-major
   float* y;                 // [rows][n]
   int rows, n, k;
+  int tiles_per_cta;        // whole 16-row tiles per CTA
 };
 size_t int4_packed_bytes(long long n, int k);
+int int4_pick_depth(int rows, int k);   // cp.async ring slots per warp; 0: does not fit
 size_t int4_smem_bytes(int rows, int k);
-int int4_max_ctas();
-long long int4_max_rows();
 cudaError_t int4_set_max_smem();
 cudaError_t launch_int4_linear(const Int4Args& a, int grid, cudaStream_t s);
 cudaError_t launch_int4_pack(const uint8_t* qweight, const bf16* scales, const uint8_t* zeros, uint8_t* out,
