@@ -64,8 +64,8 @@ memspec_status memspec_op_linear_noalloc(const void* x_dev, const void* w_dev, f
  *   qweight: uint8 [n_out][k/2], byte j of row r = q[r][2j] | q[r][2j+1] << 4
  *   scales:  bf16  [n_out][k/128];   zeros: uint8 [n_out][k/128], values 0..15
  * and are repacked once, by memspec_int4_pack, into the kernel's layout (one
- * 1072-byte record per 16-row tile and 128-column group; rows past n_out are
- * zero-filled).  The layout is private to this library: only
+ * 1072-byte record per 16-row tile and 128-column group, codes regrouped
+ * within each 32-bit word; rows past n_out are zero-filled).  The layout is private to this library: only
  * memspec_op_linear_int4 reads it.
  *
  * memspec_int4_packed_bytes: bytes of the packed copy, or -1 for bad sizes
@@ -84,10 +84,12 @@ memspec_status memspec_int4_pack(const void* qweight_dev, const void* scales_dev
  * the activations (rows (2k + 64) bytes) plus a ring of at least two
  * 1072-byte records per warp (16 warps) must fit in 220 KB of shared memory
  * (else UNSUPPORTED: e.g. rows 9..16 at k = 11008).  Results are
- * deterministic.  Allocates nothing and keeps no state between calls.
+ * deterministic.  status_dev: optional uint32 device word; bit 0 is set if a
+ * wait for a bulk copy ran out (about a second; y is then incomplete).
+ * Allocates nothing and keeps no state between calls.
  * Errors: INVALID_ARG (sizes, NULL, misalignment), UNSUPPORTED, CUDA. */
 memspec_status memspec_op_linear_int4(const void* x_dev, const void* packed_dev, float* y_dev, int32_t rows,
-                                      int32_t n_out, int32_t k, void* stream);
+                                      int32_t n_out, int32_t k, uint32_t* status_dev, void* stream);
 
 /* Categorical sampling of each row of logits[rows][vocab] (fp32): with T > 0,
  * out[r] = smallest j with sum_{i<=j} exp(z_i/T - m) > u[r] * sum_i exp(z_i/T - m);

@@ -121,7 +121,7 @@ EXPORTS = {
     "memspec_int4_pack": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_void_p,
                                     C.c_void_p]),
     "memspec_op_linear_int4": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_int32, C.c_int32,
-                                         C.c_void_p]),
+                                         C.c_void_p, C.c_void_p]),
     "memspec_op_sample": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_float, C.c_void_p,
                                     C.c_void_p, C.c_void_p]),
     "memspec_op_last_error": (C.c_char_p, []),

@@ -2115,7 +2115,7 @@ memspec_status memspec_int4_pack(const void* qweight, const void* scales, const 
 }
 
 memspec_status memspec_op_linear_int4(const void* x, const void* packed, float* y, int32_t rows,
-                                      int32_t n_out, int32_t k, void* stream) {
+                                      int32_t n_out, int32_t k, uint32_t* status, void* stream) {
   if (x == nullptr || packed == nullptr || y == nullptr) {
     g_op_error = "null pointer";
     return MEMSPEC_ERR_INVALID_ARG;
@@ -2130,7 +2130,7 @@ memspec_status memspec_op_linear_int4(const void* x, const void* packed, float* 
     return MEMSPEC_ERR_INVALID_ARG;
   }
   if (int4_pick_depth(rows, k) == 0) {
-    g_op_error = "rows x k too large for the activations and a 2-slot ring per warp in shared memory";
+    g_op_error = "rows x k too large for the activations and a 2-record ring per warp in shared memory";
     return MEMSPEC_ERR_UNSUPPORTED;
   }
   if (!ensure_func_attrs()) {
@@ -2138,9 +2138,7 @@ memspec_status memspec_op_linear_int4(const void* x, const void* packed, float* 
     return MEMSPEC_ERR_CUDA;
   }
   // whole 16-row tiles, the same number per CTA, at most one CTA per SM
-  const int tiles = (n_out + 15) / 16;
-  const int per_cta = (tiles + sm_count() - 1) / sm_count();
-  const int grid = (tiles + per_cta - 1) / per_cta;
+  const Int4Plan plan = int4_plan(rows, n_out, k, sm_count());
   Int4Args a{};
   a.x = static_cast<const bf16*>(x);
   a.packed = static_cast<const uint8_t*>(packed);
@@ -2148,8 +2146,9 @@ memspec_status memspec_op_linear_int4(const void* x, const void* packed, float* 
   a.rows = rows;
   a.n = n_out;
   a.k = k;
-  a.tiles_per_cta = per_cta;
-  cudaError_t e = launch_int4_linear(a, grid, static_cast<cudaStream_t>(stream));
+  a.tiles_per_cta = plan.tiles_per_cta;
+  a.status = status;
+  cudaError_t e = launch_int4_linear(a, plan, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) {
     g_op_error = std::string("int4 launch: ") + cudaGetErrorString(e);
     return MEMSPEC_ERR_CUDA;

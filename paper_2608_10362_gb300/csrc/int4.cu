@@ -19,9 +19,11 @@
 // (exponent of 128, q in the mantissa's low bits: one LOP3 per two codes), the
 // zero point is folded out per group:
 //   sum_c x (q - z) = sum_c x (128 + q) - (128 + z) sum_c x,
-// with sum_c x over the group (sx) formed once per CTA.  Products are exact;
-// the MMA's fp32 accumulation of the biased terms is the only rounding beyond
-// the epilogue's.
+// with the group sum of x formed by the tensor pipe too: one more MMA per step
+// with an all-ones A operand meets the same B fragments and leaves sum_c x in
+// exactly the accumulator layout of the products (no separate pass over x, no
+// extra ALU work).  Products are exact; the MMAs' fp32 accumulation is the
+// only rounding beyond the epilogue's.
 //
 // Layout (memspec_int4_pack).  The kernel reads a repacked copy: one record per
 // (16-row tile, group) unit, in tile-major order:
@@ -30,20 +32,23 @@
 //                                   column offsets g*128 + 32 j + 8 t + (0..7)
 //   bytes [1024, 1056) eight bf16 pairs (s[r], s[r + 8])
 //   bytes [1056, 1072) eight byte pairs (z[r], z[r + 8])
-// so a warp copies a record with three 16-byte-per-lane copies and lane L reads
-// exactly its MMA fragment.  Word j's 8 nibbles e = 0..7 become the k slots
-// {2t, 2t+1, 2t+8, 2t+9} of two k16 steps as pairs (e, e+4); the activations
-// are staged in shared memory with each 16-byte vector permuted the same way,
-// so one 16-byte load gives both steps' B fragments and each step contracts
-// matching columns.
+// and within each word the codes of columns e = 0..7 sit at nibble positions
+// 0 4 1 5 2 6 3 7 (e = 0..7), so that masking nibbles p and p + 4 of
+// (word >> 4 p) yields the bf16 pair of columns (2p, 2p + 1): exactly the
+// A-fragment pair that meets the activation pair (x[2p], x[2p + 1]) in the
+// natural bf16 layout.  Lane L's record bytes are its A fragments and one
+// 16-byte load of x gives the B fragments of two k16 steps.
 //
 // Work split.  Whole 16-row tiles are dealt to CTAs, the same number to each
 // (ceil(tiles / SMs); the grid shrinks to fit), so no output is shared between
 // CTAs.  A CTA's units (its tiles x groups, contiguous in memory) are cut into
 // 16 equal contiguous ranges, one per warp.  Each warp streams its range
-// through its own ring of D record slots with cp.async (D = 8, 4 or 2, the most
-// that fits beside the activations), so D records per warp are in flight while
-// it computes.  A tile a warp covers whole is stored directly; the partial sums
+// through its own ring of D record slots (D = 8, 4 or 2, the most that fits
+// beside the activations) with cp.async, one commit group per record (small
+// copies: per-request cost decides, and 1 KB bulk copies were slower).  The
+// activations arrive as one 1-D bulk copy (TMA) per row, outside the
+// load/store unit's queue.  That wait is bounded: on expiry the kernel sets
+// bit 0 of the optional status word and finishes without computing.  A tile a warp covers whole is stored directly; the partial sums
 // of a tile shared by several warps are added in warp order at the end.  Every
 // sum has a fixed order: results are bit-reproducible.  Launched with
 // programmatic stream serialisation: a CTA starts its weight copies, then
@@ -51,6 +56,7 @@
 #include <cuda_bf16.h>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace memspec {
 namespace {
@@ -79,11 +85,8 @@ __device__ __forceinline__ void mma_bf16(float (&c)[4], uint32_t a0, uint32_t a1
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-__device__ __forceinline__ uint32_t saddr(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
 __device__ __forceinline__ void cp16(void* dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(saddr(dst)), "l"(src) : "memory");
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
 }
 __device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
@@ -105,81 +108,79 @@ __device__ __forceinline__ int part_of(int v, int total, int parts) {
   return ((v + 1) * parts + total - 1) / total - 1;
 }
 
+// Bounded mbarrier wait with a warp-uniform outcome (the MMAs after it need
+// every lane): true once every lane has seen the phase complete; false if the
+// budget ran out or another warp gave up (then lane 0 raises the flag and the
+// status bit).
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          uint32_t* status) {
+  const long long t0 = clock64();
+  for (;;) {
+    const bool ok = mbar_try_wait(bar, parity);
+    if (__all_sync(0xffffffffu, ok)) return true;
+    const bool bad = *abort_flag != 0 || clock64() - t0 > kWaitBudgetCycles;
+    if (__any_sync(0xffffffffu, bad)) {
+      if ((threadIdx.x & 31) == 0) {
+        *abort_flag = 1;
+        if (status != nullptr) atomicOr(status, 0x1u);
+      }
+      return false;
+    }
+  }
+}
+
 template <int NT, int D>
 __global__ void __launch_bounds__(kI4Threads, 1) int4_linear_kernel(const __grid_constant__ Int4Args a) {
   constexpr int Mp = 8 * NT;
   extern __shared__ __align__(128) uint8_t dsm[];
+  __shared__ uint64_t xbar;
+  __shared__ int abort_flag;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rq = lane >> 2, t = lane & 3;
   const int M = a.rows, k = a.k, G = k >> 7, n = a.n;
   const int P = 2 * k + 64;   // bytes per staged activation row (the pad makes the fragment loads conflict-free)
   uint8_t* xs = dsm;                                                        // [M][P]
-  float* sx = reinterpret_cast<float*>(dsm + ((static_cast<size_t>(M) * P + 15) & ~static_cast<size_t>(15)));
-  uint8_t* ring = reinterpret_cast<uint8_t*>(sx) + ((static_cast<size_t>(G) * Mp * 4 + 127) & ~static_cast<size_t>(127));
+  uint8_t* ring = dsm + ((static_cast<size_t>(M) * P + 127) & ~static_cast<size_t>(127));
   uint8_t* my_ring = ring + static_cast<size_t>(warp) * D * kInt4RecordBytes;
+  volatile int* abort_v = &abort_flag;
 
   // this CTA's tiles [T0, T1) and this warp's units [lo, hi) of them
   const int tiles = (n + 15) >> 4;
-  const int T0 = blockIdx.x * a.tiles_per_cta;
+  const int T0 = min(tiles, static_cast<int>(blockIdx.x) * a.tiles_per_cta);   // CTAs past the end: no tiles
   const int T1 = min(tiles, T0 + a.tiles_per_cta);
   const int L = (T1 - T0) * G;
   const int lo = L * warp / kI4Warps, hi = L * (warp + 1) / kI4Warps;
   const int cnt = hi - lo;
   const uint8_t* src = a.packed + (static_cast<size_t>(T0) * G + lo) * kInt4RecordBytes;
 
-  // ---- start this warp's weight stream first (it does not depend on the
-  // previous kernel); one commit group per unit, empty ones included
+  if (tid == 0) {
+    mbar_init(&xbar, 1);
+    abort_flag = 0;
+  }
+  fence_mbar_init();
+  __syncthreads();
+
+  // ---- this warp's weight stream first (it does not depend on the previous
+  // kernel); one commit group per record, empty ones included
 #pragma unroll
   for (int i = 0; i < D; ++i) {
     if (i < cnt) copy_record(my_ring + i * kInt4RecordBytes, src + static_cast<size_t>(i) * kInt4RecordBytes, lane);
     cp_commit();
   }
 
-  // the activations are the previous kernel's output
-  asm volatile("griddepcontrol.wait;" ::: "memory");
-
-  // ---- activations into shared memory, each 16-byte vector (8 columns e) in
-  // the order (e0,e4)(e1,e5)(e2,e6)(e3,e7) of the B fragments; and their
-  // per-group sums sx[g][m]: half a warp covers one group of one row (16
-  // vectors), summed by a fixed xor tree
-  {
-    const int per_row = k >> 3;
-    const int total = M * per_row;
-    constexpr int kBatch = 4;
-    for (int base = warp * 32; base < total; base += kBatch * kI4Threads) {
-      uint4 xv[kBatch];
-#pragma unroll
-      for (int b = 0; b < kBatch; ++b) {
-        const int idx = base + b * kI4Threads + lane;
-        xv[b] = idx < total ? __ldg(reinterpret_cast<const uint4*>(a.x) + idx) : make_uint4(0u, 0u, 0u, 0u);
-      }
-#pragma unroll
-      for (int b = 0; b < kBatch; ++b) {
-        const int idx = base + b * kI4Threads + lane;
-        const uint4 X = xv[b];
-        float sum = 0.f;
-        const uint32_t w4[4] = {X.x, X.y, X.z, X.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) sum += __uint_as_float(w4[e] << 16) + __uint_as_float(w4[e] & 0xffff0000u);
-#pragma unroll
-        for (int o = 8; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-        if (idx < total) {
-          const int m = idx / per_row, v = idx - m * per_row;
-          *reinterpret_cast<uint4*>(xs + static_cast<size_t>(m) * P + v * 16) =
-              make_uint4(prmt(X.x, X.z, 0x5410), prmt(X.x, X.z, 0x7632), prmt(X.y, X.w, 0x5410),
-                         prmt(X.y, X.w, 0x7632));
-          if ((lane & 15) == 0) sx[(v >> 4) * Mp + m] = sum;
-        }
-      }
-    }
-    for (int i = tid; i < (Mp - M) * G; i += kI4Threads) {   // padding rows: zero sums
-      const int g = i / (Mp - M), m = M + i % (Mp - M);
-      sx[g * Mp + m] = 0.f;
-    }
+  // ---- the activations (the previous kernel's output): one bulk copy per row
+  pdl_wait();
+  if (tid == 0) {
+    const uint64_t pol = l2_policy_evict_last();
+    mbar_arrive_expect_tx(&xbar, static_cast<uint32_t>(M) * 2 * k);
+    for (int m = 0; m < M; ++m)
+      bulk_load(xs + static_cast<size_t>(m) * P, a.x + static_cast<size_t>(m) * k, 2 * k, &xbar, pol);
   }
+  bool ok = warp_wait(&xbar, 0, abort_v, a.status);
   __syncthreads();
+  ok = ok && *abort_v == 0;
 
-  // ---- main loop: unit j of the warp sits in ring slot j % D
+  // ---- main loop: unit u of the warp sits in ring slot u % D
   float o[NT][4], of[NT][4];
 #pragma unroll
   for (int j = 0; j < NT; ++j)
@@ -195,101 +196,106 @@ __global__ void __launch_bounds__(kI4Threads, 1) int4_linear_kernel(const __grid
     xrow[j] = xs + static_cast<size_t>(8 * j + rq) * P + 16 * t;
     xok[j] = 8 * j + rq < M;
   }
-
-  for (int base = 0; base < cnt; base += D) {
+  for (int base = 0; base < cnt && ok; base += D) {
 #pragma unroll
     for (int i = 0; i < D; ++i) {
       const int u = base + i;
       if (u < cnt) {
-        cp_wait<D - 1>();
-        __syncwarp();
-        const uint8_t* slot = my_ring + i * kInt4RecordBytes;
-        const uint4 qa = *reinterpret_cast<const uint4*>(slot + lane * 16);
-        const uint4 qb = *reinterpret_cast<const uint4*>(slot + 512 + lane * 16);
-        const uint32_t sp = *reinterpret_cast<const uint32_t*>(slot + 1024 + rq * 4);
-        const uint32_t zp = *reinterpret_cast<const uint16_t*>(slot + 1056 + rq * 2);
-        float acc0[NT][4], acc1[NT][4];
+        {
+          cp_wait<D - 1>();   // this lane's copies of unit u have landed
+          __syncwarp();       // ... and every other lane's
+          const uint8_t* slot = my_ring + i * kInt4RecordBytes;
+          const uint4 qa = *reinterpret_cast<const uint4*>(slot + lane * 16);
+          const uint4 qb = *reinterpret_cast<const uint4*>(slot + 512 + lane * 16);
+          const uint32_t sp = *reinterpret_cast<const uint32_t*>(slot + 1024 + rq * 4);
+          const uint32_t zp = *reinterpret_cast<const uint16_t*>(slot + 1056 + rq * 2);
+          __syncwarp();   // every lane has read the slot: refill it
+          if (u + D < cnt)
+            copy_record(my_ring + i * kInt4RecordBytes, src + static_cast<size_t>(u + D) * kInt4RecordBytes, lane);
+          cp_commit();
+          float acc0[NT][4], acc1[NT][4], sum0[NT][4], sum1[NT][4];
 #pragma unroll
-        for (int j = 0; j < NT; ++j)
+          for (int j = 0; j < NT; ++j)
 #pragma unroll
-          for (int e = 0; e < 4; ++e) acc0[j][e] = acc1[j][e] = 0.f;
-        const uint32_t wa[4] = {qa.x, qa.y, qa.z, qa.w};
-        const uint32_t wb[4] = {qb.x, qb.y, qb.z, qb.w};
+            for (int e = 0; e < 4; ++e) acc0[j][e] = acc1[j][e] = sum0[j][e] = sum1[j][e] = 0.f;
+          constexpr uint32_t kOnes = 0x3F803F80u;   // bf16 pair (1, 1)
+          const uint32_t wa[4] = {qa.x, qa.y, qa.z, qa.w};
+          const uint32_t wb[4] = {qb.x, qb.y, qb.z, qb.w};
 #pragma unroll
-        for (int w = 0; w < 4; ++w) {
-          const uint32_t a0 = nib2(wa[w]), a1 = nib2(wb[w]);
-          const uint32_t a2 = nib2(wa[w] >> 4), a3 = nib2(wb[w] >> 4);
-          const uint32_t a4 = nib2(wa[w] >> 8), a5 = nib2(wb[w] >> 8);
-          const uint32_t a6 = nib2(wa[w] >> 12), a7 = nib2(wb[w] >> 12);
-#pragma unroll
-          for (int j = 0; j < NT; ++j) {
-            uint4 X = make_uint4(0u, 0u, 0u, 0u);
-            if (xok[j]) X = *reinterpret_cast<const uint4*>(xrow[j] + g * 256 + w * 64);
-            // k slots (2t, 2t+1) <- columns (e, e + 4); (2t+8, 2t+9) <- (e+1, e+5)
-            mma_bf16(acc0[j], a0, a1, a2, a3, X.x, X.y);
-            mma_bf16(acc1[j], a4, a5, a6, a7, X.z, X.w);
-          }
-        }
-        __syncwarp();   // every lane has read the slot: refill it
-        if (u + D < cnt)
-          copy_record(my_ring + i * kInt4RecordBytes, src + static_cast<size_t>(u + D) * kInt4RecordBytes, lane);
-        cp_commit();
-        // fold the scale and zero point of this group
-        const float s0 = __uint_as_float(sp << 16), s1 = __uint_as_float(sp & 0xffff0000u);
-        const float z0 = 128.f + static_cast<float>(zp & 0xffu), z1 = 128.f + static_cast<float>(zp >> 8);
-#pragma unroll
-        for (int j = 0; j < NT; ++j) {
-          const float2 sv = *reinterpret_cast<const float2*>(sx + g * Mp + 8 * j + 2 * t);
-          o[j][0] = fmaf(s0, fmaf(-z0, sv.x, acc0[j][0] + acc1[j][0]), o[j][0]);
-          o[j][1] = fmaf(s0, fmaf(-z0, sv.y, acc0[j][1] + acc1[j][1]), o[j][1]);
-          o[j][2] = fmaf(s1, fmaf(-z1, sv.x, acc0[j][2] + acc1[j][2]), o[j][2]);
-          o[j][3] = fmaf(s1, fmaf(-z1, sv.y, acc0[j][3] + acc1[j][3]), o[j][3]);
-        }
-        // end of a tile, or of the warp's range
-        ++g;
-        const bool last = u + 1 == cnt;
-        if (g == G || last) {
-          const bool whole = g == G && (T != T_first || lo == (T - T0) * G);
-          if (whole) {
-            const int r0 = T * 16 + rq, r1 = r0 + 8;
+          for (int w = 0; w < 4; ++w) {
+            const uint32_t a0 = nib2(wa[w]), a1 = nib2(wb[w]);
+            const uint32_t a2 = nib2(wa[w] >> 4), a3 = nib2(wb[w] >> 4);
+            const uint32_t a4 = nib2(wa[w] >> 8), a5 = nib2(wb[w] >> 8);
+            const uint32_t a6 = nib2(wa[w] >> 12), a7 = nib2(wb[w] >> 12);
 #pragma unroll
             for (int j = 0; j < NT; ++j) {
-              const int m = 8 * j + 2 * t;
-              if (m < M) {
-                if (r0 < n) a.y[static_cast<size_t>(m) * n + r0] = o[j][0];
-                if (r1 < n) a.y[static_cast<size_t>(m) * n + r1] = o[j][2];
-              }
-              if (m + 1 < M) {
-                if (r0 < n) a.y[static_cast<size_t>(m + 1) * n + r0] = o[j][1];
-                if (r1 < n) a.y[static_cast<size_t>(m + 1) * n + r1] = o[j][3];
-              }
+              uint4 X = make_uint4(0u, 0u, 0u, 0u);
+              if (xok[j]) X = *reinterpret_cast<const uint4*>(xrow[j] + g * 256 + w * 64);
+              // k slots (2t, 2t+1) <- columns (0, 1) of the 8; (2t+8, 2t+9) <- (2, 3); then (4, 5), (6, 7)
+              mma_bf16(acc0[j], a0, a1, a2, a3, X.x, X.y);
+              mma_bf16(acc1[j], a4, a5, a6, a7, X.z, X.w);
+              mma_bf16(sum0[j], kOnes, kOnes, kOnes, kOnes, X.x, X.y);   // the group sums of x
+              mma_bf16(sum1[j], kOnes, kOnes, kOnes, kOnes, X.z, X.w);
             }
-          } else if (T == T_first) {
-            first_partial = true;
-#pragma unroll
-            for (int j = 0; j < NT; ++j)
-#pragma unroll
-              for (int e = 0; e < 4; ++e) of[j][e] = o[j][e];
-          } else {
-            last_partial = true;   // the range ends inside this tile: keep o
           }
-          if (!last || whole || T == T_first) {
+          // fold the scale and zero point of this group
+          const float s0 = __uint_as_float(sp << 16), s1 = __uint_as_float(sp & 0xffff0000u);
+          const float z0 = 128.f + static_cast<float>(zp & 0xffu), z1 = 128.f + static_cast<float>(zp >> 8);
 #pragma unroll
-            for (int j = 0; j < NT; ++j)
-#pragma unroll
-              for (int e = 0; e < 4; ++e) o[j][e] = 0.f;
+          for (int j = 0; j < NT; ++j) {
+            o[j][0] = fmaf(s0, fmaf(-z0, sum0[j][0] + sum1[j][0], acc0[j][0] + acc1[j][0]), o[j][0]);
+            o[j][1] = fmaf(s0, fmaf(-z0, sum0[j][1] + sum1[j][1], acc0[j][1] + acc1[j][1]), o[j][1]);
+            o[j][2] = fmaf(s1, fmaf(-z1, sum0[j][2] + sum1[j][2], acc0[j][2] + acc1[j][2]), o[j][2]);
+            o[j][3] = fmaf(s1, fmaf(-z1, sum0[j][3] + sum1[j][3], acc0[j][3] + acc1[j][3]), o[j][3]);
           }
-          if (g == G) {
-            g = 0;
-            ++T;
+          // end of a tile, or of the warp's range
+          ++g;
+          const bool last = u + 1 == cnt;
+          if (g == G || last) {
+            const bool whole = g == G && (T != T_first || lo == (T - T0) * G);
+            if (whole) {
+              const int r0 = T * 16 + rq, r1 = r0 + 8;
+#pragma unroll
+              for (int j = 0; j < NT; ++j) {
+                const int m = 8 * j + 2 * t;
+                if (m < M) {
+                  if (r0 < n) a.y[static_cast<size_t>(m) * n + r0] = o[j][0];
+                  if (r1 < n) a.y[static_cast<size_t>(m) * n + r1] = o[j][2];
+                }
+                if (m + 1 < M) {
+                  if (r0 < n) a.y[static_cast<size_t>(m + 1) * n + r0] = o[j][1];
+                  if (r1 < n) a.y[static_cast<size_t>(m + 1) * n + r1] = o[j][3];
+                }
+              }
+            } else if (T == T_first) {
+              first_partial = true;
+#pragma unroll
+              for (int j = 0; j < NT; ++j)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) of[j][e] = o[j][e];
+            } else {
+              last_partial = true;   // the range ends inside this tile: keep o
+            }
+            if (!last || whole || T == T_first) {
+#pragma unroll
+              for (int j = 0; j < NT; ++j)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) o[j][e] = 0.f;
+            }
+            if (g == G) {
+              g = 0;
+              ++T;
+            }
           }
         }
       }
     }
   }
-  asm volatile("griddepcontrol.launch_dependents;");
+  pdl_launch_dependents();
   cp_wait<0>();
+  if (tid == 0 && *abort_v) mbar_wait_drain(&xbar, 0);   // after a timeout: let the copies land before exit
   __syncthreads();   // the rings are free: they hold the partial sums from here on
+  if (*abort_v) return;
 
   // ---- partial tiles: slot 0 = the warp's first tile, slot 1 = its last
   float* part = reinterpret_cast<float*>(ring);   // [warp][2][16][Mp]
@@ -329,6 +335,14 @@ __global__ void __launch_bounds__(kI4Threads, 1) int4_linear_kernel(const __grid
   }
 }
 
+// code of column e (nibble e of the GPTQ word) -> nibble position (e >> 1) + 4 (e & 1)
+__device__ __forceinline__ uint32_t interleave_nibbles(uint32_t w) {
+  uint32_t r = 0;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) r |= ((w >> (4 * e)) & 0xFu) << (4 * ((e >> 1) + 4 * (e & 1)));
+  return r;
+}
+
 // One thread per 16-byte code block (64 per unit) plus one per unit tail.
 __global__ void int4_pack_kernel(const uint8_t* __restrict__ qweight, const bf16* __restrict__ scales,
                                  const uint8_t* __restrict__ zeros, uint8_t* __restrict__ out, int n, int k,
@@ -348,7 +362,7 @@ __global__ void int4_pack_kernel(const uint8_t* __restrict__ qweight, const bf16
     if (row < n) {
       const uint8_t* src = qweight + row * (k / 2) + g * 64 + 4 * t;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) w4[j] = *reinterpret_cast<const uint32_t*>(src + 16 * j);
+      for (int j = 0; j < 4; ++j) w4[j] = interleave_nibbles(*reinterpret_cast<const uint32_t*>(src + 16 * j));
     }
     *reinterpret_cast<uint4*>(rec + half * 512 + lane * 16) = make_uint4(w4[0], w4[1], w4[2], w4[3]);
   } else {
@@ -384,12 +398,11 @@ size_t int4_packed_bytes(long long n, int k) {
 
 static size_t int4_smem_for(int rows, int k, int depth) {
   const int Mp = rows <= 8 ? 8 : 16;
-  const size_t xs = (static_cast<size_t>(rows) * (2 * k + 64) + 15) & ~static_cast<size_t>(15);
-  const size_t sxb = (static_cast<size_t>(k / 128) * Mp * 4 + 127) & ~static_cast<size_t>(127);
+  const size_t xs = (static_cast<size_t>(rows) * (2 * k + 64) + 127) & ~static_cast<size_t>(127);
   size_t ring = static_cast<size_t>(kI4Warps) * depth * kInt4RecordBytes;
   const size_t part = static_cast<size_t>(kI4Warps) * 2 * 16 * Mp * 4;
   if (ring < part) ring = part;
-  return xs + sxb + ring;
+  return xs + ring;
 }
 
 int int4_pick_depth(int rows, int k) {
@@ -417,13 +430,22 @@ cudaError_t int4_set_max_smem() {
   return cudaSuccess;
 }
 
-cudaError_t launch_int4_linear(const Int4Args& a, int grid, cudaStream_t s) {
-  const int d = int4_pick_depth(a.rows, a.k);
-  if (d == 0) return cudaErrorInvalidValue;
+Int4Plan int4_plan(int rows, int n, int k, int sms) {
+  Int4Plan p{};
+  p.depth = int4_pick_depth(rows, k);
+  if (p.depth == 0) return p;
+  const int tiles = (n + 15) / 16;
+  p.tiles_per_cta = (tiles + sms - 1) / sms;
+  p.grid = (tiles + p.tiles_per_cta - 1) / p.tiles_per_cta;
+  return p;
+}
+
+cudaError_t launch_int4_linear(const Int4Args& a, const Int4Plan& p, cudaStream_t s) {
+  if (p.depth == 0) return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
+  cfg.gridDim = dim3(p.grid);
   cfg.blockDim = dim3(kI4Threads);
-  cfg.dynamicSmemBytes = int4_smem_for(a.rows, a.k, d);
+  cfg.dynamicSmemBytes = int4_smem_for(a.rows, a.k, p.depth);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -431,10 +453,10 @@ cudaError_t launch_int4_linear(const Int4Args& a, int grid, cudaStream_t s) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   const bool wide = a.rows > 8;
-  if (d == 8) return wide ? cudaLaunchKernelEx(&cfg, int4_linear_kernel<2, 8>, a)
-                          : cudaLaunchKernelEx(&cfg, int4_linear_kernel<1, 8>, a);
-  if (d == 4) return wide ? cudaLaunchKernelEx(&cfg, int4_linear_kernel<2, 4>, a)
-                          : cudaLaunchKernelEx(&cfg, int4_linear_kernel<1, 4>, a);
+  if (p.depth == 8) return wide ? cudaLaunchKernelEx(&cfg, int4_linear_kernel<2, 8>, a)
+                                : cudaLaunchKernelEx(&cfg, int4_linear_kernel<1, 8>, a);
+  if (p.depth == 4) return wide ? cudaLaunchKernelEx(&cfg, int4_linear_kernel<2, 4>, a)
+                                : cudaLaunchKernelEx(&cfg, int4_linear_kernel<1, 4>, a);
   return wide ? cudaLaunchKernelEx(&cfg, int4_linear_kernel<2, 2>, a)
               : cudaLaunchKernelEx(&cfg, int4_linear_kernel<1, 2>, a);
 }

@@ -263,12 +263,19 @@ struct Int4Args {
   float* y;                 // [rows][n]
   int rows, n, k;
   int tiles_per_cta;        // whole 16-row tiles per CTA
+  uint32_t* status;         // optional device word: bit 0 = a copy wait ran out
 };
 size_t int4_packed_bytes(long long n, int k);
 int int4_pick_depth(int rows, int k);   // cp.async ring slots per warp; 0: does not fit
 size_t int4_smem_bytes(int rows, int k);
 cudaError_t int4_set_max_smem();
-cudaError_t launch_int4_linear(const Int4Args& a, int grid, cudaStream_t s);
+struct Int4Plan {
+  int depth;           // record slots per warp (0: does not fit)
+  int tiles_per_cta;
+  int grid;
+};
+Int4Plan int4_plan(int rows, int n, int k, int sms);
+cudaError_t launch_int4_linear(const Int4Args& a, const Int4Plan& p, cudaStream_t s);
 cudaError_t launch_int4_pack(const uint8_t* qweight, const bf16* scales, const uint8_t* zeros, uint8_t* out,
                              int n, int k, cudaStream_t s);
 

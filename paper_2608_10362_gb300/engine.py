@@ -389,16 +389,18 @@ def int4_pack(qweight: torch.Tensor, scales: torch.Tensor, zeros: torch.Tensor,
 
 
 def op_linear_int4(x: torch.Tensor, packed: torch.Tensor, n_out: int, y: torch.Tensor | None = None,
+                   status: torch.Tensor | None = None,
                    stream: torch.cuda.Stream | None = None) -> torch.Tensor:
     """y = x . W^T (fp32 [rows][n_out]) for x bf16 [rows][k] and W packed by
-    int4_pack."""
+    int4_pack; `status` (int32 [1] on cuda, optional) receives the kernel's
+    error bits."""
     lib = _lib.load()
     rows, k = x.shape
     if y is None:
         y = torch.empty(rows, n_out, dtype=torch.float32, device=x.device)
     s = stream or torch.cuda.current_stream(x.device)
     _check(lib, lib.memspec_op_linear_int4(x.data_ptr(), packed.data_ptr(), y.data_ptr(), rows, n_out, k,
-                                           s.cuda_stream))
+                                           None if status is None else status.data_ptr(), s.cuda_stream))
     return y
 
 

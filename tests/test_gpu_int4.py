@@ -47,8 +47,9 @@ def _x(seed, rows, k):
 def _pack_reference(qweight, scales, zeros):
     """The record layout written out from its definition (16-row tiles x
     128-column groups, tile-major; lane L = 4 r + t holds the words at column
-    offsets 32 j + 8 t of rows r and r + 8; then the (s[r], s[r+8]) bf16 pairs
-    and the (z[r], z[r+8]) byte pairs)."""
+    offsets 32 j + 8 t of rows r and r + 8, each word's codes of columns
+    e = 0..7 moved to nibble positions 0 4 1 5 2 6 3 7; then the (s[r], s[r+8])
+    bf16 pairs and the (z[r], z[r+8]) byte pairs)."""
     n, half = qweight.shape
     k = 2 * half
     G, tiles = k // 128, (n + 15) // 16
@@ -68,7 +69,12 @@ def _pack_reference(qweight, scales, zeros):
                     row = T * 16 + 8 * h + r
                     for j in range(4):
                         o = g * 64 + 16 * j + 4 * t
-                        rec[h * 512 + lane * 16 + 4 * j: h * 512 + lane * 16 + 4 * j + 4] = qw[row, o:o + 4]
+                        word = int.from_bytes(qw[row, o:o + 4].tobytes(), "little")
+                        moved = 0
+                        for e in range(8):
+                            moved |= ((word >> (4 * e)) & 15) << (4 * [0, 4, 1, 5, 2, 6, 3, 7][e])
+                        rec[h * 512 + lane * 16 + 4 * j: h * 512 + lane * 16 + 4 * j + 4] = \
+                            np.frombuffer(moved.to_bytes(4, "little"), np.uint8)
             pairs = np.stack([sb[T * 16:T * 16 + 8, g], sb[T * 16 + 8:T * 16 + 16, g]], axis=1)
             rec[1024:1056] = np.frombuffer(pairs.astype("<u2").tobytes(), np.uint8)
             zp = np.stack([zb[T * 16:T * 16 + 8, g], zb[T * 16 + 8:T * 16 + 16, g]], axis=1)
@@ -96,7 +102,9 @@ def test_int4_linear_matches_oracle(rows, n, k):
     packed = int4_pack(*_device(qw, sc, zs))
     xt = torch.from_numpy(x).to(torch.bfloat16).cuda()
     y = torch.full((rows, n), float("nan"), device="cuda")
-    op_linear_int4(xt, packed, n, y=y)
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    op_linear_int4(xt, packed, n, y=y, status=status)
+    assert int(status.item()) == 0
     got = y.cpu().numpy().astype(np.float64)
     ref = linear_int4(x, qw, sc, zs, 128)
     bound = _bound(x, qw, sc, zs)
@@ -153,8 +161,8 @@ def test_int4_entry_points_refuse_bad_arguments():
     bad = [(p, p, p, 0, 128, 128), (p, p, p, 17, 128, 128), (p, p, p, 1, 128, 100), (p, p, p, 1, 0, 128),
            (C.c_void_p(base + 8), p, p, 1, 128, 128), (None, p, p, 1, 128, 128)]
     for x, w, y, rows, n, k in bad:
-        assert lib.memspec_op_linear_int4(x, w, y, rows, n, k, None) == _lib.ERR_INVALID_ARG
+        assert lib.memspec_op_linear_int4(x, w, y, rows, n, k, None, None) == _lib.ERR_INVALID_ARG
     # 16 rows of k = 8192 need more shared memory than the kernel may use
-    assert lib.memspec_op_linear_int4(p, p, p, 16, 128, 8192, None) == _lib.ERR_UNSUPPORTED
+    assert lib.memspec_op_linear_int4(p, p, p, 16, 128, 8192, None, None) == _lib.ERR_UNSUPPORTED
     assert lib.memspec_int4_pack(p, p, p, 16, 100, p, None) == _lib.ERR_INVALID_ARG
     assert lib.memspec_int4_pack(p, p, p, 16, 128, C.c_void_p(base + 4), None) == _lib.ERR_INVALID_ARG
