@@ -750,8 +750,13 @@ def run_case(args):
                 "tokens_per_s": PREFIX / ms * 1e3, "device_status": bits}
     if args.case == "verify":
         # the 7B verify pass alone, one launch per op and no graph, inside an NVTX
-        # range "verify" (for profilers: ncu --nvtx --nvtx-include "verify/")
+        # range "verify" (for profilers: ncu --nvtx --nvtx-include "verify/");
+        # --layers N keeps only N of the 7B target's layers (every per-layer
+        # kernel and the LM head keep their full size: a profiler-sized case)
+        import dataclasses
         t = SHAPES[TARGET]
+        if args.layers:
+            t = dataclasses.replace(t, n_layers=args.layers)
         K = args.k
         max_seq = PREFIX + (args.steps + args.warmup + 2) * (K + 1) + 16
         eng = Engine(t, iter_weights(t, 0), max_batch=1, max_seq=max_seq, max_k=K, max_drafts=0,
@@ -776,8 +781,8 @@ def run_case(args):
         bits = eng.sync()
         ms = a.elapsed_time(b) / args.steps
         eng.close()
-        return {"case": "verify", "target": TARGET, "K": K, "prefix": PREFIX, "graphs": False,
-                "ms_per_verify": ms, "device_status": bits}
+        return {"case": "verify", "target": TARGET, "layers": t.n_layers, "K": K, "prefix": PREFIX,
+                "graphs": False, "ms_per_verify": ms, "device_status": bits}
     t, d = SHAPES["draft_160m"], SHAPES["draft_68m"]
     K = args.k
     max_seq = 512 + (args.steps + args.warmup + 4) * (K + 1) + 16
@@ -811,27 +816,28 @@ def run_case(args):
             "device_status": bits}
 
 
-TRAFFIC_PROFILE = os.path.join(ROOT, "profiles", "verify_7b_k4_ctx2048_dram.md")
+TRAFFIC_PROFILE = os.path.join(ROOT, "profiles", "verify_7b_2layers_k4_ctx2048_dram.md")
+# the sources of the kernels a verify pass launches (and of their launch set-up)
+VERIFY_SOURCES = ("api.cu", "attention.cu", "attn_body.cuh", "embed.cu", "embed_body.cuh", "gemm.cu",
+                  "gemm_epi.cuh", "internal.h", "pack.cu", "ptx.cuh")
 
 
-def kernel_sources_hash() -> str:
-    """sha256 over the CUDA sources (name + content, sorted by name)."""
-    import glob
+def kernel_sources_hash(names=VERIFY_SOURCES) -> str:
+    """sha256 over the named CUDA sources (name + content, in name order)."""
     import hashlib
     csrc = os.path.join(ROOT, "paper_2608_10362_gb300", "csrc")
-    files = sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh")) +
-                   glob.glob(os.path.join(csrc, "*.h")))
     h = hashlib.sha256()
-    for f in files:
-        h.update(os.path.basename(f).encode())
-        with open(f, "rb") as fh:
+    for name in sorted(names):
+        h.update(name.encode())
+        with open(os.path.join(csrc, name), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()
 
 
 def recorded_traffic():
-    """DRAM bytes of one verify pass from the committed ncu summary, if it was
-    taken on the kernel sources as they are now (else None)."""
+    """DRAM bytes of one full verify pass, scaled from the committed ncu summary
+    of a 2-layer pass (per-layer kernels x 32 + LM head + embedding), if it was
+    taken on the verify kernels' sources as they are now (else None)."""
     try:
         with open(TRAFFIC_PROFILE) as fh:
             text = fh.read()
@@ -872,6 +878,8 @@ def main():
     ap.add_argument("--n", type=int, default=22016)
     ap.add_argument("--kdim", type=int, default=4096)
     ap.add_argument("--rows", type=int, default=5)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="(--case verify) layers of the 7B target to keep (default: all)")
     ap.add_argument("--int4-layers", type=int, default=0,
                     help="(--case int4) layers of INT4 weights (default: all of the 7B target's)")
     args = ap.parse_args()
@@ -931,9 +939,9 @@ def main():
                      "bound": "hbm", "achieved": achieved, "peak": peak,
                      "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                      "traffic": recorded_traffic(),
-                     "traffic_source": "ncu dram__bytes_read+write of one verify pass "
-                                       "(profiles/verify_7b_k4_ctx2048_dram.md); null when the "
-                                       "kernels changed since",
+                     "traffic_source": "ncu dram__bytes_read+write per kernel of a 2-layer 7B verify "
+                                       "pass, scaled to 32 layers (profiles/verify_7b_2layers_k4_"
+                                       "ctx2048_dram.md); null when the verify kernels changed since",
                      "verify_ms": r["verify_ms"],
                      "algorithmic_bytes": r["verify_bytes"],
                      "frac_of_8000": achieved / 8000.0},

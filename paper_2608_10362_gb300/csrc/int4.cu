@@ -43,9 +43,11 @@
 // (ceil(tiles / SMs); the grid shrinks to fit), so no output is shared between
 // CTAs.  A CTA's units (its tiles x groups, contiguous in memory) are cut into
 // 16 equal contiguous ranges, one per warp.  Each warp streams its range
-// through its own ring of D record slots (D = 8, 4 or 2, the most that fits
-// beside the activations) with cp.async, one commit group per record (small
-// copies: per-request cost decides, and 1 KB bulk copies were slower).  The
+// through its own ring of D = 2 record slots with cp.async, one commit group
+// per record (small copies: per-request cost decides, and 1 KB bulk copies
+// were slower).  Measured on GB300, rings of 4 and 8 slots were no faster
+// (the load/store pipe's throughput, not the bytes in flight, is the limit)
+// and took longer to issue.  The
 // activations arrive as one 1-D bulk copy (TMA) per row, outside the
 // load/store unit's queue.  That wait is bounded: on expiry the kernel sets
 // bit 0 of the optional status word and finishes without computing.  A tile a warp covers whole is stored directly; the partial sums
@@ -63,6 +65,7 @@ namespace {
 
 constexpr int kI4Warps = 16;
 constexpr int kI4Threads = kI4Warps * 32;
+constexpr int kI4Depth = 2;   // record slots per warp
 
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
   uint32_t d;
@@ -406,23 +409,12 @@ static size_t int4_smem_for(int rows, int k, int depth) {
 }
 
 int int4_pick_depth(int rows, int k) {
-  for (int d : {8, 4, 2})
-    if (int4_smem_for(rows, k, d) <= static_cast<size_t>(kInt4MaxSmem)) return d;
-  return 0;
-}
-
-size_t int4_smem_bytes(int rows, int k) {
-  const int d = int4_pick_depth(rows, k);
-  return int4_smem_for(rows, k, d == 0 ? 2 : d);
+  return int4_smem_for(rows, k, kI4Depth) <= static_cast<size_t>(kInt4MaxSmem) ? kI4Depth : 0;
 }
 
 cudaError_t int4_set_max_smem() {
-  const void* fns[] = {reinterpret_cast<const void*>(int4_linear_kernel<1, 8>),
-                       reinterpret_cast<const void*>(int4_linear_kernel<1, 4>),
-                       reinterpret_cast<const void*>(int4_linear_kernel<1, 2>),
-                       reinterpret_cast<const void*>(int4_linear_kernel<2, 8>),
-                       reinterpret_cast<const void*>(int4_linear_kernel<2, 4>),
-                       reinterpret_cast<const void*>(int4_linear_kernel<2, 2>)};
+  const void* fns[] = {reinterpret_cast<const void*>(int4_linear_kernel<1, kI4Depth>),
+                       reinterpret_cast<const void*>(int4_linear_kernel<2, kI4Depth>)};
   for (const void* f : fns) {
     cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, kInt4MaxSmem);
     if (e != cudaSuccess) return e;
@@ -452,13 +444,8 @@ cudaError_t launch_int4_linear(const Int4Args& a, const Int4Plan& p, cudaStream_
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  const bool wide = a.rows > 8;
-  if (p.depth == 8) return wide ? cudaLaunchKernelEx(&cfg, int4_linear_kernel<2, 8>, a)
-                                : cudaLaunchKernelEx(&cfg, int4_linear_kernel<1, 8>, a);
-  if (p.depth == 4) return wide ? cudaLaunchKernelEx(&cfg, int4_linear_kernel<2, 4>, a)
-                                : cudaLaunchKernelEx(&cfg, int4_linear_kernel<1, 4>, a);
-  return wide ? cudaLaunchKernelEx(&cfg, int4_linear_kernel<2, 2>, a)
-              : cudaLaunchKernelEx(&cfg, int4_linear_kernel<1, 2>, a);
+  return a.rows > 8 ? cudaLaunchKernelEx(&cfg, int4_linear_kernel<2, kI4Depth>, a)
+                    : cudaLaunchKernelEx(&cfg, int4_linear_kernel<1, kI4Depth>, a);
 }
 
 cudaError_t launch_int4_pack(const uint8_t* qweight, const bf16* scales, const uint8_t* zeros, uint8_t* out,

@@ -267,7 +267,6 @@ struct Int4Args {
 };
 size_t int4_packed_bytes(long long n, int k);
 int int4_pick_depth(int rows, int k);   // cp.async ring slots per warp; 0: does not fit
-size_t int4_smem_bytes(int rows, int k);
 cudaError_t int4_set_max_smem();
 struct Int4Plan {
   int depth;           // record slots per warp (0: does not fit)
