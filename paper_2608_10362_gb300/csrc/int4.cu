@@ -19,11 +19,11 @@
 // (exponent of 128, q in the mantissa's low bits: one LOP3 per two codes), the
 // zero point is folded out per group:
 //   sum_c x (q - z) = sum_c x (128 + q) - (128 + z) sum_c x,
-// with the group sum of x formed by the tensor pipe too: one more MMA per step
-// with an all-ones A operand meets the same B fragments and leaves sum_c x in
-// exactly the accumulator layout of the products (no separate pass over x, no
-// extra ALU work).  Products are exact; the MMAs' fp32 accumulation is the
-// only rounding beyond the epilogue's.
+// with the group sums of x formed once per CTA by the tensor pipe too: MMAs with
+// an all-ones A operand on the same B fragments leave sum_c x in exactly the
+// accumulator layout of the products (no shuffles, no extra ALU work), kept in
+// shared memory for the fold.  Products are exact; the MMAs' fp32
+// accumulation is the only rounding beyond the epilogue's.
 //
 // Layout (memspec_int4_pack).  The kernel reads a repacked copy: one record per
 // (16-row tile, group) unit, in tile-major order:
@@ -143,7 +143,8 @@ __global__ void __launch_bounds__(kI4Threads, 1) int4_linear_kernel(const __grid
   const int M = a.rows, k = a.k, G = k >> 7, n = a.n;
   const int P = 2 * k + 64;   // bytes per staged activation row (the pad makes the fragment loads conflict-free)
   uint8_t* xs = dsm;                                                        // [M][P]
-  uint8_t* ring = dsm + ((static_cast<size_t>(M) * P + 127) & ~static_cast<size_t>(127));
+  float* sx = reinterpret_cast<float*>(dsm + ((static_cast<size_t>(M) * P + 127) & ~static_cast<size_t>(127)));
+  uint8_t* ring = reinterpret_cast<uint8_t*>(sx) + ((static_cast<size_t>(G) * Mp * 4 + 127) & ~static_cast<size_t>(127));
   uint8_t* my_ring = ring + static_cast<size_t>(warp) * D * kInt4RecordBytes;
   volatile int* abort_v = &abort_flag;
 
@@ -180,6 +181,32 @@ __global__ void __launch_bounds__(kI4Threads, 1) int4_linear_kernel(const __grid
       bulk_load(xs + static_cast<size_t>(m) * P, a.x + static_cast<size_t>(m) * k, 2 * k, &xbar, pol);
   }
   bool ok = warp_wait(&xbar, 0, abort_v, a.status);
+  const uint8_t* xrow[NT];
+  bool xok[NT];
+#pragma unroll
+  for (int j = 0; j < NT; ++j) {
+    xrow[j] = xs + static_cast<size_t>(8 * j + rq) * P + 16 * t;
+    xok[j] = 8 * j + rq < M;
+  }
+  constexpr uint32_t kOnes = 0x3F803F80u;   // bf16 pair (1, 1)
+  // group sums sx[g][m] = sum of x[m][128 g .. 128 g + 127]: MMAs with an
+  // all-ones A operand, one group per warp at a time (rows past M read as 0)
+  if (ok) {
+    for (int gg = warp; gg < G; gg += kI4Warps) {
+#pragma unroll
+      for (int j = 0; j < NT; ++j) {
+        float c[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          uint4 X = make_uint4(0u, 0u, 0u, 0u);
+          if (xok[j]) X = *reinterpret_cast<const uint4*>(xrow[j] + gg * 256 + w * 64);
+          mma_bf16(c, kOnes, kOnes, kOnes, kOnes, X.x, X.y);
+          mma_bf16(c, kOnes, kOnes, kOnes, kOnes, X.z, X.w);
+        }
+        if (rq == 0) *reinterpret_cast<float2*>(sx + gg * Mp + 8 * j + 2 * t) = make_float2(c[0], c[1]);
+      }
+    }
+  }
   __syncthreads();
   ok = ok && *abort_v == 0;
 
@@ -192,13 +219,6 @@ __global__ void __launch_bounds__(kI4Threads, 1) int4_linear_kernel(const __grid
   int T = T0 + lo / G, g = lo - (lo / G) * G;
   const int T_first = T;
   bool first_partial = false, last_partial = false;
-  const uint8_t* xrow[NT];
-  bool xok[NT];
-#pragma unroll
-  for (int j = 0; j < NT; ++j) {
-    xrow[j] = xs + static_cast<size_t>(8 * j + rq) * P + 16 * t;
-    xok[j] = 8 * j + rq < M;
-  }
   for (int base = 0; base < cnt && ok; base += D) {
 #pragma unroll
     for (int i = 0; i < D; ++i) {
@@ -216,12 +236,11 @@ __global__ void __launch_bounds__(kI4Threads, 1) int4_linear_kernel(const __grid
           if (u + D < cnt)
             copy_record(my_ring + i * kInt4RecordBytes, src + static_cast<size_t>(u + D) * kInt4RecordBytes, lane);
           cp_commit();
-          float acc0[NT][4], acc1[NT][4], sum0[NT][4], sum1[NT][4];
+          float acc0[NT][4], acc1[NT][4];
 #pragma unroll
           for (int j = 0; j < NT; ++j)
 #pragma unroll
-            for (int e = 0; e < 4; ++e) acc0[j][e] = acc1[j][e] = sum0[j][e] = sum1[j][e] = 0.f;
-          constexpr uint32_t kOnes = 0x3F803F80u;   // bf16 pair (1, 1)
+            for (int e = 0; e < 4; ++e) acc0[j][e] = acc1[j][e] = 0.f;
           const uint32_t wa[4] = {qa.x, qa.y, qa.z, qa.w};
           const uint32_t wb[4] = {qb.x, qb.y, qb.z, qb.w};
 #pragma unroll
@@ -237,8 +256,6 @@ __global__ void __launch_bounds__(kI4Threads, 1) int4_linear_kernel(const __grid
               // k slots (2t, 2t+1) <- columns (0, 1) of the 8; (2t+8, 2t+9) <- (2, 3); then (4, 5), (6, 7)
               mma_bf16(acc0[j], a0, a1, a2, a3, X.x, X.y);
               mma_bf16(acc1[j], a4, a5, a6, a7, X.z, X.w);
-              mma_bf16(sum0[j], kOnes, kOnes, kOnes, kOnes, X.x, X.y);   // the group sums of x
-              mma_bf16(sum1[j], kOnes, kOnes, kOnes, kOnes, X.z, X.w);
             }
           }
           // fold the scale and zero point of this group
@@ -246,10 +263,11 @@ __global__ void __launch_bounds__(kI4Threads, 1) int4_linear_kernel(const __grid
           const float z0 = 128.f + static_cast<float>(zp & 0xffu), z1 = 128.f + static_cast<float>(zp >> 8);
 #pragma unroll
           for (int j = 0; j < NT; ++j) {
-            o[j][0] = fmaf(s0, fmaf(-z0, sum0[j][0] + sum1[j][0], acc0[j][0] + acc1[j][0]), o[j][0]);
-            o[j][1] = fmaf(s0, fmaf(-z0, sum0[j][1] + sum1[j][1], acc0[j][1] + acc1[j][1]), o[j][1]);
-            o[j][2] = fmaf(s1, fmaf(-z1, sum0[j][2] + sum1[j][2], acc0[j][2] + acc1[j][2]), o[j][2]);
-            o[j][3] = fmaf(s1, fmaf(-z1, sum0[j][3] + sum1[j][3], acc0[j][3] + acc1[j][3]), o[j][3]);
+            const float2 sv = *reinterpret_cast<const float2*>(sx + g * Mp + 8 * j + 2 * t);
+            o[j][0] = fmaf(s0, fmaf(-z0, sv.x, acc0[j][0] + acc1[j][0]), o[j][0]);
+            o[j][1] = fmaf(s0, fmaf(-z0, sv.y, acc0[j][1] + acc1[j][1]), o[j][1]);
+            o[j][2] = fmaf(s1, fmaf(-z1, sv.x, acc0[j][2] + acc1[j][2]), o[j][2]);
+            o[j][3] = fmaf(s1, fmaf(-z1, sv.y, acc0[j][3] + acc1[j][3]), o[j][3]);
           }
           // end of a tile, or of the warp's range
           ++g;
@@ -402,10 +420,11 @@ size_t int4_packed_bytes(long long n, int k) {
 static size_t int4_smem_for(int rows, int k, int depth) {
   const int Mp = rows <= 8 ? 8 : 16;
   const size_t xs = (static_cast<size_t>(rows) * (2 * k + 64) + 127) & ~static_cast<size_t>(127);
+  const size_t sxb = (static_cast<size_t>(k / 128) * Mp * 4 + 127) & ~static_cast<size_t>(127);
   size_t ring = static_cast<size_t>(kI4Warps) * depth * kInt4RecordBytes;
   const size_t part = static_cast<size_t>(kI4Warps) * 2 * 16 * Mp * 4;
   if (ring < part) ring = part;
-  return xs + ring;
+  return xs + sxb + ring;
 }
 
 int int4_pick_depth(int rows, int k) {
