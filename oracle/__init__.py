@@ -20,6 +20,11 @@ What it restates, and where it comes from:
   INT4 targets (Section 4.1): w = (q - z) s per group of inputs, y = x W^T.
 * ``scheduler`` - MemSpec's draft cache update and runtime loop (Sections
   3.3-3.4, Algorithms 2-3) and the MAB-Async baseline (Sections 2.3, 4.1).
+* ``tree`` - verification of a draft tree in one target pass and the walk that
+  accepts a path of it, as in the engine MemSpec is built on (Section 3.5,
+  "System Implementation"); pinned against a tree-masked attention pass
+  (torch SDPA), chi-square draws from the target and E[accepted] in closed
+  form (tests/test_oracle_tree.py).
 * ``speculative`` - the draft-and-verify iteration that MemSpec runs unchanged
   (Section 3.5: "the standard draft-and-verify process"; Section 2.1, Eq. 1:
   throughput ~ E[A] / L_iter), with the acceptance rule of the speculative
