@@ -8,6 +8,9 @@
  *   memspec_draft_step    the draft model's K autoregressive M=1 proposals
  *   memspec_verify_step   one target pass over the K+1 positions
  *                         [last committed token, x_1..x_K] against its KV cache
+ *   memspec_tree_step     (alternative to the three calls above) one target
+ *                         pass over a caller-built draft tree, the
+ *                         root-down acceptance walk and the commit
  *   memspec_accept_commit speculative-sampling acceptance (accept x_i with
  *                         probability min(1, p_i(x_i)/q_i(x_i)), else resample
  *                         from norm(max(0, p - q)); bonus token when all K are
@@ -281,6 +284,31 @@ memspec_status memspec_verify_step(memspec_ctx* ctx, int32_t K);
 memspec_status memspec_accept_commit(memspec_ctx* ctx, int32_t K, float temperature,
                                      int32_t* results_host_pinned);
 
+/* Tree verification step, as in the speculative-decoding engine MemSpec is
+ * built on (Section 3.5, "System Implementation"; that engine verifies draft
+ * trees, the paper's own runs use a chain).  Request 0, batch 1.
+ * The caller's tree: node i has token tokens_host[i] and parent
+ * parents_host[i] (-1: a child of the root, the last committed token t_{L-1};
+ * else a smaller node index); 1 <= n_nodes <= 31.  One target pass scores the
+ * root and every node: the root at position L-1, node i at L + depth(i) (depth
+ * 0 below the root), each row attending to the committed prefix, its
+ * ancestors and itself; the nodes' K,V go to the scratch slots L..L-1+n_nodes.
+ * Then a token is drawn from each row's softmax(z/T) (Philox slot 64 + e for
+ * the step's e-th emitted token; T == 0: argmax), and the walk descends from
+ * the root while the drawn token is a child's token (lowest index among equal
+ * siblings); the first drawn token that is no child is the step's final
+ * token.  Commit: the accepted tokens and the final token (L += accepted + 1),
+ * the accepted nodes' K,V moved to consecutive positions after the root.
+ * The drafts' caches are not advanced (a following memspec_draft_step catches
+ * up at most two tokens; more is reported as device status 0x4).
+ * If results_host is not NULL, an async copy of int32 [66] =
+ * {n_emit, L_before, emitted[32], accepted_rows[32]} (rows: node index + 1;
+ * n_emit = accepted + 1, or 0 if the sequence would pass max_seq) is enqueued.
+ * Needs batch 1.  Errors: INVALID_ARG (tree, tokens, T), UNSUPPORTED (batch),
+ * CUDA.  Enqueue only. */
+memspec_status memspec_tree_step(memspec_ctx* ctx, int32_t n_nodes, const int32_t* tokens_host,
+                                 const int32_t* parents_host, float temperature, int32_t* results_host);
+
 /* Host synchronisation (no counterpart in the paper).
  * Wait for the main stream (timeout_ms < 0: no limit) and return the device
  * status word as MEMSPEC_ERR_DEVICE_STATUS if any bit is set (the word is then
@@ -302,7 +330,8 @@ typedef enum memspec_buffer {
                                     first MMA issued, partials stored, arrival counted,
                                     reduction inputs loaded, reduction done, then
                                     epilogue-internal points}; 2048 ops at most */
-  MEMSPEC_BUF_SEEDS = 8          /* u64 [max_batch] Philox keys of the requests (set by prefill) */
+  MEMSPEC_BUF_SEEDS = 8,         /* u64 [max_batch] Philox keys of the requests (set by prefill) */
+  MEMSPEC_BUF_TREE_LOGITS = 9    /* fp32 [32][vocab] rows of the last tree step (row 0 = the root) */
 } memspec_buffer;
 
 /* Facts about the last step calls (host-side, no wait).  what:

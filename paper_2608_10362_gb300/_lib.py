@@ -22,7 +22,7 @@ T_TOK_EMB, T_ATTN_NORM, T_WQKV, T_WO, T_FFN_NORM, T_WGATE, T_WUP, T_WDOWN, T_FIN
 
 # buffer ids (memspec_buffer)
 BUF_TARGET_LOGITS, BUF_DRAFT_LOGITS, BUF_DRAFT_TOKENS, BUF_TOKENS, BUF_SEQ_STATE, \
-    BUF_ACCEPT_DEBUG, BUF_RESIDUAL, BUF_PASS_TRACE, BUF_SEEDS = range(9)
+    BUF_ACCEPT_DEBUG, BUF_RESIDUAL, BUF_PASS_TRACE, BUF_SEEDS, BUF_TREE_LOGITS = range(10)
 
 # launch modes (memspec_init_params.launch_mode)
 LAUNCH_PER_OP, LAUNCH_PASS = 0, 1
@@ -106,6 +106,7 @@ EXPORTS = {
     "memspec_set_batch": (C.c_int, [C.c_void_p, C.c_int32]),
     "memspec_draft_step": (C.c_int, [C.c_void_p, C.c_int32, C.c_float]),
     "memspec_verify_step": (C.c_int, [C.c_void_p, C.c_int32]),
+    "memspec_tree_step": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_float, C.c_void_p]),
     "memspec_accept_commit": (C.c_int, [C.c_void_p, C.c_int32, C.c_float, C.c_void_p]),
     "memspec_sync": (C.c_int, [C.c_void_p, C.c_int32, C.POINTER(C.c_uint32)]),
     "memspec_read_buffer": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_size_t]),

@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libmemspec.so")
-SOURCES = ["gemm.cu", "attention.cu", "embed.cu", "sampling.cu", "api.cu", "noalloc.cu", "pass.cu", "pack.cu",
+SOURCES = ["gemm.cu", "attention.cu", "embed.cu", "sampling.cu", "api.cu", "noalloc.cu", "pass.cu", "pack.cu", "tree.cu",
            "draft_fused.cu", "sched.cpp", "int4.cu"]
 HEADERS = ["ptx.cuh", "internal.h", "gemm_epi.cuh", "attn_body.cuh", "sample_body.cuh", "embed_body.cuh", "pass.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

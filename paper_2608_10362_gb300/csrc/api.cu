@@ -341,6 +341,10 @@ struct memspec_ctx {
   float* acc_dbg = nullptr;
   int* acc_cnt = nullptr;
   int* smp_cnt = nullptr;
+  TreeDesc* tree_desc = nullptr;            // tree steps: the tree, its rows' draws,
+  int* tree_samples = nullptr;              // the walk's outcome and the rows' logits
+  TreeResult* tree_result = nullptr;
+  float* tree_z = nullptr;
   float* rope_cos[2] = {nullptr, nullptr};  // hd 64, hd 128
   float* rope_sin[2] = {nullptr, nullptr};
   size_t ws_bytes = 0;
@@ -459,6 +463,10 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   const size_t o_ad = w.take(static_cast<size_t>(B) * (2 * K + 2) * 4);
   const size_t o_ac = w.take(static_cast<size_t>(B) * 4);
   const size_t o_sc = w.take(static_cast<size_t>(B) * 4);
+  const size_t o_td = w.take(sizeof(TreeDesc));
+  const size_t o_ts = w.take(static_cast<size_t>(kTreeRows) * 4);
+  const size_t o_tr = w.take(sizeof(TreeResult));
+  const size_t o_tz = w.take(static_cast<size_t>(kTreeRows) * V * 4);
   const size_t o_rc64 = w.take(static_cast<size_t>(p->max_seq) * 32 * 4);
   const size_t o_rs64 = w.take(static_cast<size_t>(p->max_seq) * 32 * 4);
   const size_t o_rc128 = w.take(static_cast<size_t>(p->max_seq) * 64 * 4);
@@ -517,6 +525,10 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
     c->acc_dbg = reinterpret_cast<float*>(base + o_ad);
     c->acc_cnt = reinterpret_cast<int*>(base + o_ac);
     c->smp_cnt = reinterpret_cast<int*>(base + o_sc);
+    c->tree_desc = reinterpret_cast<TreeDesc*>(base + o_td);
+    c->tree_samples = reinterpret_cast<int*>(base + o_ts);
+    c->tree_result = reinterpret_cast<TreeResult*>(base + o_tr);
+    c->tree_z = reinterpret_cast<float*>(base + o_tz);
     c->rope_cos[0] = reinterpret_cast<float*>(base + o_rc64);
     c->rope_sin[0] = reinterpret_cast<float*>(base + o_rs64);
     c->rope_cos[1] = reinterpret_cast<float*>(base + o_rc128);
@@ -981,6 +993,8 @@ memspec_status run_ops_separately(memspec_ctx* c, const std::vector<PassOp>& ops
       case OP_ATTN: e = launch_attention(op.u.at, op.grid, c->main, c->pdl && !op.full_dep); break;
       case OP_SAMPLE: e = launch_sample(op.u.s, c->main, c->pdl); break;
       case OP_ACCEPT: e = launch_accept(op.u.acc, c->main, false); break;
+      case OP_TREE_WALK: e = launch_tree_walk(op.u.tw, c->main); break;
+      case OP_TREE_COMPACT: e = launch_tree_compact(op.u.tc, op.n_units, c->main); break;
       default: return fail(c, MEMSPEC_ERR_INVALID_ARG, "unknown op");
     }
     if (e != cudaSuccess) return cuda_fail(c, e, "op launch");
@@ -1080,7 +1094,7 @@ memspec_status launch_table(memspec_ctx* c, const OpTable& t) {
 template <class Emit>
 memspec_status run_pass(memspec_ctx* c, const GraphKey& key, bool use_pass, Emit&& emit) {
   const bool pass = use_pass && c->pass_kernel;
-  const int slot = key.kind == 1 ? 1 : (key.kind == 2 ? 2 : 0);
+  const int slot = (key.kind == 1 || key.kind == 4) ? 1 : (key.kind == 2 ? 2 : 0);
   if (c->p.use_graphs) {
     auto it = c->graphs.find(key);
     if (it != c->graphs.end()) {
@@ -1847,6 +1861,90 @@ memspec_status memspec_accept_commit(memspec_ctx* c, int32_t K, float T, int32_t
   return MEMSPEC_OK;
 }
 
+memspec_status memspec_tree_step(memspec_ctx* c, int32_t n_nodes, const int32_t* tokens_host,
+                                 const int32_t* parents_host, float T, int32_t* results_host) {
+  if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
+  if (tokens_host == nullptr || parents_host == nullptr)
+    return fail(c, MEMSPEC_ERR_INVALID_ARG, "tree tokens and parents required");
+  if (n_nodes < 1 || n_nodes > kTreeRows - 1) return fail(c, MEMSPEC_ERR_INVALID_ARG, "tree of 1..31 nodes");
+  if (!(T >= 0.f)) return fail(c, MEMSPEC_ERR_INVALID_ARG, "temperature must be >= 0");
+  if (c->batch != 1) return fail(c, MEMSPEC_ERR_UNSUPPORTED, "tree steps run one request (batch 1)");
+  // the tree as rows: row 0 = the root, row i + 1 = node i
+  TreeDesc t{};
+  t.n_rows = n_nodes + 1;
+  t.parent_row[0] = -1;
+  t.rope_off[0] = 0;
+  t.anc[0] = 1u;
+  for (int i = 0; i < n_nodes; ++i) {
+    const int p = parents_host[i];
+    if (p < -1 || p >= i) return fail(c, MEMSPEC_ERR_INVALID_ARG, "tree parent must be -1 or a smaller node");
+    if (tokens_host[i] < 0 || tokens_host[i] >= c->vocab)
+      return fail(c, MEMSPEC_ERR_INVALID_ARG, "tree token out of the vocabulary");
+    const int r = i + 1, pr = p + 1;
+    t.tokens[r] = tokens_host[i];
+    t.parent_row[r] = pr;
+    t.rope_off[r] = t.rope_off[pr] + 1;
+    t.anc[r] = t.anc[pr] | (1u << r);
+  }
+  // outside any captured graph: the graph reads only the device copy
+  cudaError_t e = cudaMemcpyAsync(c->tree_desc, &t, sizeof(TreeDesc), cudaMemcpyHostToDevice, c->main);
+  if (e != cudaSuccess) return cuda_fail(c, e, "tree copy");
+  const int R = t.n_rows;
+  const ModelRT& tm = c->target;
+  GraphKey key{4, -1, R, fbits(T), 1};
+  memspec_status s = run_pass(c, key, false, [&](std::vector<PassOp>& ops) -> memspec_status {
+    FwdSpec f{};
+    f.mode = PLAN_TREE;
+    f.n_groups = 1;
+    f.R = R;
+    f.logits = c->tree_z;
+    f.last_only = 0;
+    memspec_status st = emit_forward(c, c->target, f, ops);
+    if (st != MEMSPEC_OK) return st;
+    if (!ops.empty() && ops.front().type == OP_EMBED) ops.front().u.e.tree = c->tree_desc;
+    SampleArgs sa{};
+    sa.logits = c->tree_z;
+    sa.row_stride = c->vocab;
+    sa.vocab = c->vocab;
+    sa.n_groups = R;
+    sa.greedy = T == 0.f;
+    sa.inv_temp = T == 0.f ? 0.f : 1.f / T;
+    sa.slot = kTreeSlot0;
+    sa.row_slots = c->tree_desc->rope_off;
+    sa.seq_state = c->state;
+    sa.seeds = c->seeds;
+    sa.out_tok = c->tree_samples;
+    sa.out_stride = 1;
+    sa.counters = c->smp_cnt;
+    sa.status = c->status;
+    PassOp op{};
+    op.type = OP_SAMPLE;
+    op.n_units = R;
+    op.u.s = sa;
+    ops.push_back(op);
+    PassOp w{};
+    w.type = OP_TREE_WALK;
+    w.n_units = 1;
+    w.u.tw = TreeWalkArgs{c->tree_desc, c->tree_samples, c->state, c->tokens, c->p.max_seq, c->tree_result,
+                          c->status};
+    ops.push_back(w);
+    PassOp k{};
+    k.type = OP_TREE_COMPACT;
+    k.n_units = tm.cfg.n_layers;
+    k.u.tc = TreeCompactArgs{tm.kv,
+                             static_cast<size_t>(c->p.max_batch) * tm.cfg.n_kv_heads * c->p.max_seq * tm.cfg.head_dim,
+                             tm.cfg.n_kv_heads, tm.cfg.head_dim, c->p.max_seq, c->tree_result};
+    ops.push_back(k);
+    return MEMSPEC_OK;
+  });
+  if (s != MEMSPEC_OK) return s;
+  if (results_host != nullptr) {
+    e = cudaMemcpyAsync(results_host, c->tree_result, sizeof(TreeResult), cudaMemcpyDeviceToHost, c->main);
+    if (e != cudaSuccess) return cuda_fail(c, e, "tree results copy");
+  }
+  return MEMSPEC_OK;
+}
+
 memspec_status memspec_sync(memspec_ctx* c, int32_t timeout_ms, uint32_t* bits) {
   if (c == nullptr) return MEMSPEC_ERR_INVALID_ARG;
   cudaError_t e;
@@ -1912,6 +2010,7 @@ static memspec_status buffer_span(memspec_ctx* c, int32_t buf, void** ptr, size_
     case MEMSPEC_BUF_ACCEPT_DEBUG: *ptr = c->acc_dbg; *cap = static_cast<size_t>(B) * (2 * K + 2) * 4; break;
     case MEMSPEC_BUF_RESIDUAL: *ptr = c->h; *cap = static_cast<size_t>(kMaxRows) * c->p.target.d_model * 4; break;
     case MEMSPEC_BUF_SEEDS: *ptr = c->seeds; *cap = static_cast<size_t>(B) * 8; break;
+    case MEMSPEC_BUF_TREE_LOGITS: *ptr = c->tree_z; *cap = static_cast<size_t>(kTreeRows) * V * 4; break;
     case MEMSPEC_BUF_PASS_TRACE:
       if (c->trace == nullptr) return fail(c, MEMSPEC_ERR_INVALID_ARG, "tracing is off (init param trace)");
       *ptr = c->trace;

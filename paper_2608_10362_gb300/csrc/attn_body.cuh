@@ -90,13 +90,14 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   if (!early) wait();
   const RowPlan* plan = a.plan;
   // every plan field in one round trip (g < kMaxGroups: in bounds before the check)
-  int n_groups = 1, R = a.rows_per_block, req = 0, valid = a.rows_per_block, pos0 = 0;
+  int n_groups = 1, R = a.rows_per_block, req = 0, valid = a.rows_per_block, pos0 = 0, tree = 0;
   if (!dry) {
     n_groups = plan->n_groups;
     R = plan->rows_per_group;
     req = plan->req[g];
     valid = plan->valid[g];
     pos0 = plan->pos0[g];
+    tree = plan->tree;
   }
   if (g >= n_groups) return;
   const int r_lo = rb * a.rows_per_block;
@@ -194,11 +195,14 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     }
   }
   // positions of this thread's two rows (v = mt*16 + lane/4 and +8); -1: padding row
+  // tree passes: beyond pos0 a row sees only the rows in its ancestor mask
   int prow[2];
+  uint32_t amask[2] = {0u, 0u};
 #pragma unroll
   for (int h2 = 0; h2 < 2; ++h2) {
     const int v = mt * 16 + (lane >> 2) + 8 * h2;
     prow[h2] = (active && v < nq) ? pos0 + r_lo + (v % nr) : -1;
+    if (tree && prow[h2] >= 0 && r_lo + (v % nr) < kTreeRows) amask[h2] = plan->anc[r_lo + (v % nr)];
   }
   float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
   float o[kNT][4];
@@ -237,12 +241,21 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
       for (int h2 = 0; h2 < 2; ++h2) {
         const int p = prow[h2];
         const int lim = min(p, k1 - 1);
+        const uint32_t am = amask[h2];
+        // key visible: causal (and in this split) and, in a tree pass, below
+        // pos0 or an ancestor row (rows past 31 never appear in a tree pass)
+        auto vis = [&](int key) {
+          if (key > lim) return false;
+          if (!tree) return true;
+          const int rel = key - pos0;
+          return rel < 0 || (rel < kTreeRows && ((am >> rel) & 1u) != 0u);
+        };
         float* a0 = s0 + 2 * h2;
         float* a1 = s1 + 2 * h2;
-        a0[0] = (key_c <= lim) ? a0[0] : -INFINITY;
-        a0[1] = (key_c + 1 <= lim) ? a0[1] : -INFINITY;
-        a1[0] = (key_c + 8 <= lim) ? a1[0] : -INFINITY;
-        a1[1] = (key_c + 9 <= lim) ? a1[1] : -INFINITY;
+        a0[0] = vis(key_c) ? a0[0] : -INFINITY;
+        a0[1] = vis(key_c + 1) ? a0[1] : -INFINITY;
+        a1[0] = vis(key_c + 8) ? a1[0] : -INFINITY;
+        a1[1] = vis(key_c + 9) ? a1[1] : -INFINITY;
         mx[h2] = fmaxf(fmaxf(a0[0], a0[1]), fmaxf(a1[0], a1[1]));
         mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 1));
         mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 2));

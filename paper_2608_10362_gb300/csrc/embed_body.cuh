@@ -16,7 +16,7 @@ static __device__ void compute_group(const EmbedArgs& a, int g, int* req, int* v
   }
   *req = g;
   const int L = a.seq_state[g * kStateInts + 0];
-  if (a.mode == PLAN_VERIFY) {
+  if (a.mode == PLAN_VERIFY || a.mode == PLAN_TREE) {
     *valid = a.R;
     *pos0 = L - 1;
   } else if (a.mode == PLAN_DRAFT_FIRST) {
@@ -40,6 +40,7 @@ static __device__ int row_token(const EmbedArgs& a, int req, int pos, int i) {
     return i == 0 ? a.tokens[static_cast<size_t>(req) * a.max_seq + L - 1]
                   : a.draft_tokens[req * a.max_k + i - 1];
   }
+  if (a.mode == PLAN_TREE) return i == 0 ? a.tokens[static_cast<size_t>(req) * a.max_seq + L - 1] : a.tree->tokens[i];
   if (a.mode == PLAN_DRAFT_NEXT) return a.draft_tokens[req * a.max_k + a.j - 2];
   return a.tokens[static_cast<size_t>(req) * a.max_seq + pos];
 }
@@ -59,7 +60,13 @@ __device__ void embed_row(const EmbedArgs& a, int r, float* red, int tid, Sync s
     a.plan->valid[tid] = vl;
     a.plan->pos0[tid] = p0;
   }
+  if (r == 0 && tid < kTreeRows) {   // tree passes: per-row RoPE offsets and visibility
+    const bool tr = a.mode == PLAN_TREE;
+    a.plan->rope_off[tid] = tr ? a.tree->rope_off[tid] : tid;
+    a.plan->anc[tid] = tr ? a.tree->anc[tid] : 0u;
+  }
   if (r == 0 && tid == 0) {
+    a.plan->tree = a.mode == PLAN_TREE ? 1 : 0;
     a.plan->n_groups = a.n_groups;
     a.plan->rows_per_group = a.R;
     a.plan->rows_total = a.n_groups * a.R;

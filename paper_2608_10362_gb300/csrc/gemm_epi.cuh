@@ -48,7 +48,8 @@ __device__ __forceinline__ bool row_valid(const GemmArgs& a, int r) {
 // global memory: each such read would be a dependent L2 round trip there.
 constexpr int kCtxRopeRows = 16;   // rows whose RoPE cos/sin are staged (the first chunk)
 struct EpiCtx {
-  int pos[kMaxRows];               // position of each row (plan rows)
+  int pos[kMaxRows];               // KV slot of each row (plan rows)
+  int rpos[kTreeRows];             // RoPE position of rows < 32 (differs in tree passes)
   int req[kMaxRows];               // its request
   int grp[kMaxRows];               // its group
   uint32_t valid[kMaxRows / 32];   // bit r: row r is valid
@@ -68,7 +69,7 @@ __device__ __forceinline__ void epi_prologue(const GemmArgs& a, EpiCtx* ctx, int
   for (int base = 0; base < n_pad; base += 128) {   // uniform trip count: ballots below
     const int r = base + et;
     bool valid = false, last = false;
-    int g = 0, pos = 0, req = 0;
+    int g = 0, pos = 0, rpos = 0, req = 0;
     if (r < rows_total) {
       if (plan == nullptr) {
         valid = true;
@@ -79,11 +80,13 @@ __device__ __forceinline__ void epi_prologue(const GemmArgs& a, EpiCtx* ctx, int
         valid = i < nv;
         last = i == nv - 1;
         pos = plan->pos0[g] + i;
+        rpos = (plan->tree && i < kTreeRows) ? plan->pos0[g] + plan->rope_off[i] : pos;
         req = plan->req[g];
       }
     }
     if (r < n_pad) {
       ctx->pos[r] = pos;
+      if (r < kTreeRows) ctx->rpos[r] = rpos;
       ctx->req[r] = req;
       ctx->grp[r] = g;
     }
@@ -102,7 +105,7 @@ __device__ __forceinline__ void epi_prologue(const GemmArgs& a, EpiCtx* ctx, int
       const int j = idx / half, ip = idx - j * half;
       const int pos = ctx->pos[j];
       const bool ok = ctx_bit(ctx->valid, j) && pos >= 0 && pos < a.max_seq;
-      const size_t ri = ok ? static_cast<size_t>(pos) * half + ip : 0;
+      const size_t ri = ok ? static_cast<size_t>(j < kTreeRows ? ctx->rpos[j] : pos) * half + ip : 0;
       ctx->rc[j][ip] = a.rope_cos[ri];
       ctx->rs[j][ip] = a.rope_sin[ri];
     }
@@ -296,7 +299,7 @@ static __device__ __noinline__ void apply_epilogue(const GemmArgs& a, const EpiC
           if (ok) ok_mask |= 1u << j;
           y[j] = stage[et * kStagePitch + j];
           if (seg < 2) {
-            const size_t ri = ok ? static_cast<size_t>(pos) * half_hd + ip : 0;
+            const size_t ri = ok ? static_cast<size_t>(r < kTreeRows ? ctx->rpos[r] : pos) * half_hd + ip : 0;
             const float c = rope_cos[ri], sn = rope_sin[ri];
             const float x1 = stage[e1 * kStagePitch + j];
             const float x2 = stage[(e1 + half_hd) * kStagePitch + j];
@@ -384,6 +387,7 @@ __device__ __forceinline__ void reduce_partials(const GemmArgs& a, int rt, int c
 __device__ __forceinline__ void epi_ctx_dry(EpiCtx* ctx, int n_pad, int et) {
   for (int r = et; r < n_pad; r += 128) {
     ctx->pos[r] = 0;
+    if (r < kTreeRows) ctx->rpos[r] = 0;
     ctx->req[r] = 0;
     ctx->grp[r] = 0;
   }

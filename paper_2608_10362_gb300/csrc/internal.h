@@ -23,6 +23,8 @@ constexpr int kStateInts = 4;       // per request: L, Lt, step, unused
 // (a request), index i = r % R; it is valid iff i < valid[g]; its position is
 // pos0[g] + i.  Written by the embedding kernel, read by every later kernel of
 // the same forward pass.
+constexpr int kTreeRows = 32;       // a tree pass: the root and up to 31 draft-tree nodes
+
 struct RowPlan {
   int n_groups;
   int rows_per_group;  // R
@@ -31,7 +33,51 @@ struct RowPlan {
   int req[kMaxGroups];
   int valid[kMaxGroups];
   int pos0[kMaxGroups];
+  // tree passes (one group): row r holds KV slot pos0 + r but sits at RoPE
+  // position pos0 + rope_off[r] and sees, beyond pos0, only the rows of anc[r]
+  int tree;
+  int rope_off[kTreeRows];
+  uint32_t anc[kTreeRows];   // bit j: row r sees row j (its ancestors and itself)
 };
+
+// A draft tree, written by the host before a tree step (row 0 = the root, the
+// last committed token; row i + 1 = node i).
+struct TreeDesc {
+  int n_rows;
+  int tokens[kTreeRows];       // rows >= 1: the node's token
+  int parent_row[kTreeRows];   // row of the parent (0 = the root); -1 for row 0
+  int rope_off[kTreeRows];     // 0 for the root, 1 + depth for a node
+  uint32_t anc[kTreeRows];
+};
+
+// The walk's outcome (device), also copied back to the host.
+struct TreeResult {
+  int n_emit;                  // accepted nodes + the final token (0: nothing committed)
+  int L_before;                // committed length before the step
+  int emitted[kTreeRows];      // accepted tokens, then the final token
+  int rows[kTreeRows];         // rows of the accepted nodes, in path order
+};
+
+constexpr int kTreeSlot0 = 64;   // Philox slot of the step's emitted token e: kTreeSlot0 + e
+
+struct TreeWalkArgs {            // tree.cu: the root-down walk and the commit (request 0)
+  const TreeDesc* tree;
+  const int* samples;            // [n_rows]: the token drawn from each row
+  int* seq_state;                // request 0: L, Lt, step
+  int* tokens;                   // request 0's committed tokens [max_seq]
+  int max_seq;
+  TreeResult* result;
+  uint32_t* status;
+};
+
+struct TreeCompactArgs {         // tree.cu: the accepted nodes' K / V moved to consecutive slots
+  bf16* kv;                      // layer l: K at kv + l * 2 * layer_kv, V layer_kv further
+  size_t layer_kv;               // elements of one layer's K (request-major [B][Hkv][max_seq][hd])
+  int Hkv, hd, max_seq;
+  const TreeResult* result;
+};
+cudaError_t launch_tree_walk(const TreeWalkArgs& a, cudaStream_t s);
+cudaError_t launch_tree_compact(const TreeCompactArgs& a, int n_layers, cudaStream_t s);
 
 __host__ __device__ inline bool plan_row_valid(const RowPlan* p, int r) {
   if (r >= p->rows_total) return false;
@@ -39,7 +85,7 @@ __host__ __device__ inline bool plan_row_valid(const RowPlan* p, int r) {
   return (r - g * p->rows_per_group) < p->valid[g];
 }
 
-enum PlanMode : int { PLAN_VERIFY = 0, PLAN_DRAFT_FIRST = 1, PLAN_DRAFT_NEXT = 2, PLAN_PREFILL = 3 };
+enum PlanMode : int { PLAN_VERIFY = 0, PLAN_DRAFT_FIRST = 1, PLAN_DRAFT_NEXT = 2, PLAN_PREFILL = 3, PLAN_TREE = 4 };
 
 struct EmbedArgs {
   int mode;
@@ -62,6 +108,7 @@ struct EmbedArgs {
   float* ss;                // [ss_tiles][ss_stride]: row sums of squares (partial)
   int ss_stride;
   RowPlan* plan;
+  const TreeDesc* tree;     // PLAN_TREE: the tree of this pass
   uint32_t* status;
 };
 
@@ -163,6 +210,7 @@ struct SampleArgs {         // draft sampling of pass j
   const int* seq_state;     // for Philox step; nullptr for explicit uniforms
   const unsigned long long* seeds;
   const float* u_explicit;  // [groups] (op-level entry)
+  const int* row_slots;     // tree steps: group g is row g of request 0, Philox slot row_slots[g]
   int* out_tok;             // [groups] at stride out_stride
   int out_stride;
   float* part;              // [groups][chunks][4] scratch

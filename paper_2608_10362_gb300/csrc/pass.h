@@ -6,7 +6,9 @@
 
 namespace memspec {
 
-enum OpType : int { OP_EMBED = 0, OP_GEMM = 1, OP_ATTN = 2, OP_SAMPLE = 3, OP_ACCEPT = 4 };
+// OP_TREE_WALK / OP_TREE_COMPACT run only as their own launches (tree steps)
+enum OpType : int { OP_EMBED = 0, OP_GEMM = 1, OP_ATTN = 2, OP_SAMPLE = 3, OP_ACCEPT = 4, OP_TREE_WALK = 5,
+                    OP_TREE_COMPACT = 6 };
 
 struct alignas(64) PassOp {
   int type;
@@ -22,6 +24,8 @@ struct alignas(64) PassOp {
     EmbedArgs e;
     SampleArgs s;
     AcceptArgs acc;
+    TreeWalkArgs tw;
+    TreeCompactArgs tc;
   } u;
 };
 

@@ -275,6 +275,8 @@ __device__ void sample_group(const SampleArgs& a, int g, SampleSmem& sm, int tid
     float u;
     if (a.u_explicit != nullptr) {
       u = a.u_explicit[g];
+    } else if (a.row_slots != nullptr) {   // tree step: rows of request 0
+      u = philox_uniform(a.seeds[0], 0, a.seq_state[2], a.slot + a.row_slots[g]);
     } else {
       const int step = a.seq_state[g * kStateInts + 2];
       u = philox_uniform(a.seeds[g], g, step, a.slot);

@@ -254,6 +254,18 @@ class Engine:
         ptr = None if results is None else results.data_ptr()
         self._call(self.lib.memspec_accept_commit, K, C.c_float(temperature), ptr)
 
+    def tree_step(self, tokens, parents, temperature: float, results: torch.Tensor | None = None):
+        """One tree verification step (request 0, batch 1): node i carries
+        tokens[i] and parents[i] (-1: child of the root).  With `results` (int32
+        [66], pinned) the outcome {n_emit, L_before, emitted[32], rows[32]} is
+        copied there; read it after sync()."""
+        t = np.ascontiguousarray(np.asarray(tokens, dtype=np.int32))
+        p = np.ascontiguousarray(np.asarray(parents, dtype=np.int32))
+        if t.shape != p.shape or t.ndim != 1:
+            raise ValueError("tokens and parents must be 1-D of equal length")
+        ptr = None if results is None else results.data_ptr()
+        self._call(self.lib.memspec_tree_step, len(t), t.ctypes.data, p.ctypes.data, C.c_float(temperature), ptr)
+
     def sync(self, timeout_ms: int = -1) -> int:
         bits = C.c_uint32()
         st = self.lib.memspec_sync(self.ctx, timeout_ms, C.byref(bits))

@@ -1,0 +1,155 @@
+"""Tree verification on the GPU (memspec_tree_step) against the oracle
+(oracle/tree.py), on the tiny target, with and without CUDA graphs:
+
+* every row of the tree pass (root and nodes) against the oracle's per-path
+  rows, within the lock-step logit tolerance;
+* the walk: the emitted tokens and accepted nodes equal the oracle's walk over
+  the oracle's rows with the same Philox uniforms, unless a decision is
+  exempt (|u - CDF| < 1e-3, or a greedy top-2 gap below 0.03 max|z|);
+* the commit: committed tokens, lengths and step counter, and the K/V of the
+  root and the accepted nodes at consecutive positions equal to the oracle's
+  chain forward over those tokens (bf16 storage).
+
+Trees: a "spine" built from the oracle's own top tokens (deep acceptance,
+accepted nodes spread over the rows, so the K/V really move) and seeded random
+trees (general shapes, mostly rejected at the root).
+"""
+import numpy as np
+import pytest
+import torch
+
+from lockstep import LOGIT_TOL, RECORDS, U_TOL
+from oracle.llama import LlamaOracle
+from oracle.speculative import argmax_first, softmax_t
+from oracle.tree import accept_tree, tree_logits, tree_uniforms
+from seeded_inputs import SHAPES, gen_prompt, gen_weights
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def tiny_target():
+    from paper_2608_10362_gb300 import Engine
+    t = SHAPES["tiny_target"]
+    wt = gen_weights(t, 0)
+    engines = {g: Engine(t, wt, max_batch=1, max_seq=256, max_k=8, max_drafts=0, use_graphs=g)
+               for g in (False, True)}
+    yield engines, LlamaOracle(t, wt, keep_f64=True), t
+    for e in engines.values():
+        e.close()
+
+
+def _spine_tree(model, cache, root, widths):
+    """Level by level below the current spine node: its `w` most likely tokens
+    (oracle rows); the spine continues through the most likely one."""
+    tokens, parents, cur, path = [], [], -1, [root]
+    L0 = cache.length
+    for w in widths:
+        z = model.forward(cache, path)[-1]
+        cache.truncate(L0)
+        top = np.argsort(-z, kind="stable")[:w]
+        first = len(tokens)
+        for tok in top:
+            tokens.append(int(tok))
+            parents.append(cur)
+        cur = first
+        path = path + [int(top[0])]
+    return tokens, parents
+
+
+def _random_tree(seed, n, vocab):
+    rng = np.random.default_rng(seed)
+    parents = [-1] + [int(rng.integers(-1, i)) for i in range(1, n)]
+    tokens = [int(x) for x in rng.integers(0, vocab, n)]
+    return tokens, parents
+
+
+def _exempt(z_rows, tokens, parents, T, u, res):
+    """A decision of the oracle's walk that the tolerance exempts."""
+    from oracle.tree import children
+    v = 0
+    for e, x in enumerate(res.emitted):
+        z = z_rows[v]
+        if T == 0.0:
+            s = np.sort(z)
+            if s[-1] - s[-2] < LOGIT_TOL * np.abs(z).max():
+                return True
+        else:
+            p = softmax_t(z, T)
+            cdf = np.cumsum(p)
+            if min(abs(u[e] - cdf[x]), abs(u[e] - (cdf[x - 1] if x > 0 else 0.0))) < U_TOL:
+                return True
+        if e < len(res.accepted):
+            v = res.accepted[e] + 1
+    return False
+
+
+def _kv(eng, shape):
+    return eng.kv.view(torch.bfloat16).view(shape.n_layers, 2, eng.max_batch, shape.n_kv_heads,
+                                            eng.max_seq, shape.head_dim)
+
+
+@pytest.mark.parametrize("graphs", [False, True])
+@pytest.mark.parametrize("T", [0.0, 1.0])
+@pytest.mark.parametrize("kind", ["spine", "random"])
+def test_tree_step_matches_oracle(tiny_target, graphs, T, kind):
+    from paper_2608_10362_gb300 import _lib
+    engines, model, t = tiny_target
+    eng = engines[graphs]
+    seed = 101 + (kind == "random") * 7 + int(T)
+    prompt = [int(x) for x in gen_prompt(seed, 40, t.vocab)]
+    eng.prefill(0, prompt, seed=seed)
+    cache = model.new_cache(256)
+    model.forward(cache, prompt[:-1], want_logits=False)
+    root, L = prompt[-1], len(prompt)
+    if kind == "spine":
+        tokens, parents = _spine_tree(model, cache, root, (3, 2, 3, 2, 2))
+    else:
+        tokens, parents = _random_tree(seed, 13, t.vocab)
+    res_host = torch.zeros(66, dtype=torch.int32).pin_memory()
+    eng.tree_step(tokens, parents, T, res_host)
+    assert eng.sync() == 0
+    res = res_host.numpy().copy()
+    n = len(tokens)
+    zg = eng.read_buffer(_lib.BUF_TREE_LOGITS, np.float32, 32 * t.vocab).reshape(32, t.vocab)[:n + 1]
+    zo = tree_logits(model, cache, root, tokens, parents)
+    err = max(float(np.abs(zg[r] - zo[r]).max() / np.abs(zo[r]).max()) for r in range(n + 1))
+    assert err <= LOGIT_TOL, err
+    u = tree_uniforms(seed, 0, 0, n + 1)
+    ro = accept_tree(zo, tokens, parents, T, u)
+    n_emit, L_before = int(res[0]), int(res[1])
+    emitted = [int(x) for x in res[2:2 + n_emit]]
+    rows = [int(x) - 1 for x in res[34:34 + n_emit - 1]]
+    assert L_before == L
+    # a mismatch is allowed only where the tolerance exempts a decision
+    match = (emitted, rows) == (ro.emitted, ro.accepted)
+    if not match:
+        assert _exempt(zo, tokens, parents, T, u, ro), (emitted, rows, ro.emitted, ro.accepted)
+    RECORDS.append(f"tree {kind} T={T} graphs={graphs}: {n} nodes, accepted {n_emit - 1}, "
+                   f"max logit err {err:.2e} of max, tolerance-flags {int(not match)}")
+    # commit: tokens, lengths, step counter
+    st = eng.seq_state()[0]
+    assert tuple(int(x) for x in st[:3]) == (L + n_emit, L + n_emit - 1, 1)
+    toks = eng.read_buffer(_lib.BUF_TOKENS, np.int32, eng.max_batch * eng.max_seq)[:eng.max_seq]
+    assert list(toks[L:L + n_emit]) == emitted
+    # K/V of the root and the accepted nodes at positions L-1 .. L-1+accepted
+    acc_tokens = emitted[:-1]
+    model.forward(cache, [root] + acc_tokens, want_logits=False)
+    a = len(acc_tokens)
+    got = _kv(eng, t)[:, :, 0, :, L - 1:L + a, :].float().cpu().numpy()
+    for kvi, ref in ((0, cache.k), (1, cache.v)):
+        r = ref[:, L - 1:L + a].transpose(0, 2, 1, 3)
+        scale = np.abs(r).max(axis=(1, 2, 3), keepdims=True)
+        assert np.all(np.abs(got[:, kvi] - r) <= 0.03 * scale)
+    if kind == "spine" and T == 0.0 and match:
+        assert n_emit - 1 == 5      # the whole spine of the oracle's own top tokens
+
+
+def test_tree_step_rejects_bad_trees(tiny_target):
+    from paper_2608_10362_gb300 import MemSpecError
+    engines, _, t = tiny_target
+    eng = engines[False]
+    eng.prefill(0, [1, 2, 3, 4], seed=1)
+    for tokens, parents in (([1, 2], [-1, 1]), ([1], [-2]), ([t.vocab], [-1]), ([1] * 32, [-1] * 32), ([], [])):
+        with pytest.raises(MemSpecError):
+            eng.tree_step(tokens, parents, 1.0)
