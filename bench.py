@@ -684,6 +684,80 @@ def run_int4_case(args):
     return out
 
 
+def run_tree_case(args):
+    """Tree verification on the 7B target at prefix 2048 (the engine MemSpec
+    builds on verifies draft trees): one step = the tree pass (root + nodes,
+    ancestor-masked attention), a draw from every row, the walk, the commit and
+    the K/V compaction, replayed from a CUDA graph.  Trees of 4, 8, 15 and 31
+    nodes (widths per depth below), random tokens; the chain verify pass at
+    K = 4 (5 rows) is timed alongside.  With random weights almost nothing is
+    accepted: the line reports cost per step and bytes per second, not
+    tokens per step."""
+    import numpy as np
+    import torch
+
+    from paper_2608_10362_gb300 import Engine, _lib
+    from seeded_inputs import SHAPES, gen_prompt, iter_weights
+    t = SHAPES[TARGET]
+    reps = max(1, args.steps)
+    max_seq = PREFIX + (reps + args.warmup + 4) * 33 + 64
+    eng = Engine(t, iter_weights(t, 0), max_batch=1, max_seq=max_seq, max_k=args.k, max_drafts=0,
+                 use_graphs=True)
+    prompt = gen_prompt(3, PREFIX, t.vocab)
+    rng = np.random.default_rng(9)
+    shapes = {4: (2, 1, 1), 8: (2, 2, 1, 1, 1, 1), 15: (4, 3, 3, 2, 2, 1), 31: (6, 5, 5, 4, 4, 3, 2, 2)}
+    out = {"case": "tree", "target": TARGET, "prefix": PREFIX, "graphs": True, "trees": {}}
+    s = eng.stream
+    for n_nodes, widths in shapes.items():
+        # a spine with `w` children per level, continued through the first child
+        tokens, parents, cur = [], [], -1
+        for w in widths:
+            first = len(tokens)
+            for _ in range(w):
+                tokens.append(int(rng.integers(0, t.vocab)))
+                parents.append(cur)
+            cur = first
+        assert len(tokens) == n_nodes, (n_nodes, len(tokens))
+        eng.prefill(0, prompt, seed=1)
+        for _ in range(args.warmup):
+            eng.tree_step(tokens, parents, TEMP)
+        eng.sync()
+        L0 = int(eng.seq_state()[0, 0])
+        pass_bytes = verify_bytes(t, L0 - 1, n_nodes)   # the pass over n_nodes + 1 rows
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(s)
+        for _ in range(reps):
+            eng.tree_step(tokens, parents, TEMP)
+        b.record(s)
+        torch.cuda.synchronize()
+        bits = eng.sync()
+        ms = a.elapsed_time(b) / reps
+        L1 = int(eng.seq_state()[0, 0])
+        out["trees"][n_nodes] = {"rows": n_nodes + 1, "depth": len(widths), "ms_per_step": ms,
+                                 "tokens_per_step": (L1 - L0) / reps, "pass_GBps": pass_bytes / ms / 1e6,
+                                 "device_status": bits}
+    # the chain verify pass over K + 1 rows, same prefix, for comparison
+    eng.prefill(0, prompt, seed=1)
+    dt = np.zeros((1, eng.max_k), dtype=np.int32)
+    dt[0, :args.k] = gen_prompt(4, args.k, t.vocab)
+    eng.write_buffer(_lib.BUF_DRAFT_TOKENS, dt)
+    for _ in range(args.warmup):
+        eng.verify_step(args.k)
+    eng.sync()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(s)
+    for _ in range(reps):
+        eng.verify_step(args.k)
+    b.record(s)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / reps
+    out["chain_verify"] = {"K": args.k, "rows": args.k + 1, "ms": ms,
+                           "pass_GBps": verify_bytes(t, PREFIX - 1, args.k) / ms / 1e6,
+                           "device_status": eng.sync()}
+    eng.close()
+    return out
+
+
 def run_case(args):
     """Diagnostic cases (not the headline metric)."""
     import numpy as np
@@ -712,6 +786,8 @@ def run_case(args):
                 "us_per_launch": ms * 1e3, "GB/s": nbytes / ms / 1e6}
     if args.case == "int4":
         return run_int4_case(args)
+    if args.case == "tree":
+        return run_tree_case(args)
     from paper_2608_10362_gb300 import Engine
     if args.case == "edge":
         return {"case": "edge", **run_pair_case(args, "target_1b1", "draft_68m", [512], 5, args.temp)}
@@ -862,7 +938,7 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--case", default="step", choices=["step", "gemm", "small", "verify", "prefill", "edge", "batched",
-                                                          "switching", "int4"],
+                                                          "switching", "int4", "tree"],
                     help="step: the workload above; gemm / small: diagnostic cases sized for "
                          "profiler captures (one projection GEMM; a 160M target with a 68M draft)")
     ap.add_argument("--temp", type=float, default=0.8, help="(--case edge) temperature")

@@ -90,13 +90,13 @@ def _kv(eng, shape):
 
 
 @pytest.mark.parametrize("graphs", [False, True])
-@pytest.mark.parametrize("T", [0.0, 1.0])
+@pytest.mark.parametrize("T", [0.0, 0.3, 1.0])
 @pytest.mark.parametrize("kind", ["spine", "random"])
 def test_tree_step_matches_oracle(tiny_target, graphs, T, kind):
     from paper_2608_10362_gb300 import _lib
     engines, model, t = tiny_target
     eng = engines[graphs]
-    seed = 101 + (kind == "random") * 7 + int(T)
+    seed = 101 + (kind == "random") * 7 + int(10 * T)
     prompt = [int(x) for x in gen_prompt(seed, 40, t.vocab)]
     eng.prefill(0, prompt, seed=seed)
     cache = model.new_cache(256)
