@@ -373,7 +373,6 @@ struct memspec_ctx {
   size_t df_att_floats = 0;
   float* df_lm = nullptr;
   unsigned int* df_bar = nullptr;
-  int* df_cnt = nullptr;
   CUtensorMap* df_maps = nullptr;   // [kMaxDrafts][kDfMapsPerDraft], 64-byte aligned
   bool df_coop = true;       // cooperative launch attribute (cleared if capture refuses it)
   std::map<std::tuple<const void*, int, int, int>, CUtensorMap> bmaps;
@@ -483,7 +482,6 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
   const size_t o_dfa = w.take(df_att_floats * 4);
   const size_t o_dfl = w.take(static_cast<size_t>(kDfMaxGroups) * nsm * 4 * 4);
   const size_t o_dfb = w.take(64);
-  const size_t o_dfc = w.take(static_cast<size_t>(kDfMaxGroups) * (has_draft ? dm.n_heads : 1) * 4);
   const size_t o_dfm = w.take(has_draft ? static_cast<size_t>(kMaxDrafts) * kDfMapsPerDraft * sizeof(CUtensorMap) : 0);
   const size_t o_ops = w.take(op_bytes);
   const size_t o_done = w.take(done_ints * 4);
@@ -537,7 +535,6 @@ size_t layout_workspace(const memspec_init_params* p, memspec_ctx* c, uint8_t* b
     c->df_att_floats = df_att_floats;
     c->df_lm = reinterpret_cast<float*>(base + o_dfl);
     c->df_bar = reinterpret_cast<unsigned int*>(base + o_dfb);
-    c->df_cnt = reinterpret_cast<int*>(base + o_dfc);
     c->df_maps = has_draft ? reinterpret_cast<CUtensorMap*>(base + o_dfm) : nullptr;
     c->op_area = base + o_ops;
     c->op_area_bytes = op_bytes;
@@ -1238,7 +1235,7 @@ bool fused_draft_plan(memspec_ctx* c, DraftRec& dr, int K, float T, DraftFusedAr
     return false;
   }
   int S = std::max(1, G / (B * m.n_heads));
-  S = std::min({S, 32, std::max(1, ceil_div(c->p.max_seq, 64))});
+  S = std::min({S, kDfMaxSplits, std::max(1, ceil_div(c->p.max_seq, 64))});
   if (static_cast<size_t>(2 * B) * m.n_heads * S * (m.head_dim + 4) > c->df_att_floats) {
     *why = "too many attention units for the scratch";
     return false;
@@ -1338,8 +1335,6 @@ bool fused_draft_plan(memspec_ctx* c, DraftRec& dr, int K, float T, DraftFusedAr
   a.h = c->h;
   a.qb = c->q;
   a.att = c->df_att;
-  a.att_cnt = c->df_cnt;
-  a.ao = reinterpret_cast<float*>(c->o);
   a.act = reinterpret_cast<float*>(c->act);
   a.lm_part = c->df_lm;
   a.bar = c->df_bar;

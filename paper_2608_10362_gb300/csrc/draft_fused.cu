@@ -487,9 +487,9 @@ __device__ __forceinline__ float pick(const float (&v)[kDfMaxRows], int m) {
 }
 
 // One (request, head, key split) of attention for the rows of request g: writes
-// (m, l, o) in log2 units to the partial buffer; the last split of (g, h) to
-// finish (arrival counter) combines all splits in split order and writes the
-// attention output of the head to a.ao.  scratch: kDfScratchFloats floats.
+// (m, l, o) in log2 units to the partial buffer; the O phase combines the
+// splits (in split order) as it loads its input.  scratch: kDfScratchFloats
+// floats.
 template <int HD>
 __device__ void attention_unit(const DraftFusedArgs& a, DfCtl& ctl, int layer, int g, int h, int s,
                                float* scratch, int tid) {
@@ -509,6 +509,18 @@ __device__ void attention_unit(const DraftFusedArgs& a, DfCtl& ctl, int layer, i
   float* qs = sc + 2 * kKeyBlock;         // [2][HD]
   float* op = qs + 2 * 128;               // [warps][2][HD] o partials
   const float qscale = 1.4426950408889634f / sqrtf(static_cast<float>(HD));
+  // HD 64: the first key block's K row (one per thread) does not depend on q and
+  // is requested before q is read, so q and K share one round trip (an HD 128
+  // row held across the q loads would not fit the registers)
+  constexpr bool kEarlyK = HD <= 64;
+  uint4 kr0[kEarlyK ? HD / 8 : 1];
+  if constexpr (kEarlyK) {
+    if (k0 + tid < k1) {
+      const uint4* src = reinterpret_cast<const uint4*>(kc + static_cast<size_t>(k0 + tid) * HD);
+#pragma unroll
+      for (int c = 0; c < HD / 8; ++c) kr0[c] = __ldcg(src + c);
+    }
+  }
   for (int e = tid; e < nr * HD; e += kCT) {
     const int i = e / HD, dd = e - i * HD;
     qs[e] = ldcg(a.qb + (static_cast<size_t>(g * R + i) * a.H + h) * HD + dd) * qscale;
@@ -530,8 +542,13 @@ __device__ void attention_unit(const DraftFusedArgs& a, DfCtl& ctl, int layer, i
       // the whole key row in one round trip
       uint4 kr[HD / 8];
       const uint4* src = reinterpret_cast<const uint4*>(kc + static_cast<size_t>(t) * HD);
+      if (kEarlyK && kb == k0) {
 #pragma unroll
-      for (int c = 0; c < HD / 8; ++c) kr[c] = __ldcg(src + c);
+        for (int c = 0; c < HD / 8; ++c) kr[c] = kr0[kEarlyK ? c : 0];
+      } else {
+#pragma unroll
+        for (int c = 0; c < HD / 8; ++c) kr[c] = __ldcg(src + c);
+      }
       float dot[2] = {0.f, 0.f};
 #pragma unroll
       for (int c = 0; c < HD / 8; ++c) {
@@ -643,58 +660,7 @@ __device__ void attention_unit(const DraftFusedArgs& a, DfCtl& ctl, int layer, i
     hdr[0] = tid == 0 ? m_run[0] : m_run[1];
     hdr[1] = tid == 0 ? l_run[0] : l_run[1];
   }
-  // the last split of (g, h) to arrive combines them all
-  csync();
-  if (tid == 0) {
-    __threadfence();
-    const int old = atomicAdd(&a.att_cnt[g * a.H + h], 1);
-    ctl.samp_i[0] = old == S - 1 ? 1 : 0;
-    if (old == S - 1) {
-      a.att_cnt[g * a.H + h] = 0;             // ready for the next layer
-      __threadfence();
-    }
-  }
-  csync();
-  if (!ctl.samp_i[0]) return;
-  float* w = scratch;                          // [2][32] split weights (scores are done)
-  if (tid < nr) {
-    const float* base = mine + static_cast<size_t>(tid) * a.H * S * stride;
-    float mv[32], lv[32];
-#pragma unroll
-    for (int q = 0; q < 32; ++q) {
-      float2 ml = make_float2(-INFINITY, 0.f);
-      if (q < S) ml = __ldcg(reinterpret_cast<const float2*>(base + q * stride));
-      mv[q] = ml.x;
-      lv[q] = ml.y;
-    }
-    float M = -INFINITY;
-#pragma unroll
-    for (int q = 0; q < 32; ++q)
-      if (lv[q] > 0.f) M = fmaxf(M, mv[q]);
-    float Lsum = 0.f;
-#pragma unroll
-    for (int q = 0; q < 32; ++q) {
-      const float wv = lv[q] > 0.f ? exp2f(mv[q] - M) : 0.f;
-      mv[q] = wv;
-      Lsum += wv * lv[q];
-    }
-    const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-#pragma unroll
-    for (int q = 0; q < 32; ++q) w[tid * 32 + q] = mv[q] * inv;
-  }
-  csync();
-  for (int e = tid; e < nr * HD; e += kCT) {
-    const int i = e / HD, d2 = e - i * HD;
-    const float* base = mine + static_cast<size_t>(i) * a.H * S * stride + 4 + d2;
-    float v[32];
-#pragma unroll
-    for (int q = 0; q < 32; ++q) v[q] = q < S ? ldcg(base + q * stride) : 0.f;
-    float o = 0.f;
-#pragma unroll
-    for (int q = 0; q < 32; ++q)
-      if (q < S) o = fmaf(w[i * 32 + q], v[q], o);
-    a.ao[static_cast<size_t>(g * R + i) * a.H * HD + h * HD + d2] = o;
-  }
+  // the splits are combined by every CTA of the O phase as it loads its input
 }
 
 // Sample request g's token of pass j from the LM-head statistics (warp 0);
@@ -995,25 +961,50 @@ __global__ void __launch_bounds__(kDfThreads, 1) draft_fused_kernel(const __grid
           cum += geo.u_o;
           const int fu = first_unit(geo, off);
           if (fu < geo.u_o) {
-            // the heads' attention outputs (combined by the last split of each)
-            const int qd = a.H * a.hd, n4 = rows * qd / 4;
-            for (int e0 = tid; e0 < n4; e0 += 4 * kCT) {
-              float4 v[4];
+            // the heads' attention outputs: every split's (m, l, o) of this
+            // element in one round trip, combined here in split order
+            //   o = sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s,  M = max_s m_s
+            // (every CTA redoes it: cheaper than one more barrier)
+            // hd / 4 lanes per (row, head), four features each, so that every
+            // split's loads of a pair are in flight together
+            const int S = a.n_splits, stride = a.hd + 4;
+            const int lpp = a.hd / 4, pairs = rows * a.H, per_pass = kCT / lpp;
+            for (int p0 = 0; p0 < pairs; p0 += per_pass) {
+              const int p = p0 + tid / lpp, d = (tid % lpp) * 4;
+              if (tid >= per_pass * lpp || p >= pairs) continue;
+              const int m = p / a.H, hh = p - m * a.H;
+              float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+              if (ctl.ok[m]) {
+                const float* base = a.att + (static_cast<size_t>(m) * a.H + hh) * S * stride;
+                float2 ml[kDfMaxSplits];
+                float4 ov[kDfMaxSplits];
 #pragma unroll
-              for (int q = 0; q < 4; ++q) {
-                const int e = e0 + q * kCT;
-                const int m = e < n4 ? (4 * e) / qd : 0;
-                v[q] = (e < n4 && ctl.ok[m]) ? __ldcg(reinterpret_cast<const float4*>(a.ao) + e)
-                                              : make_float4(0.f, 0.f, 0.f, 0.f);
-              }
-#pragma unroll
-              for (int q = 0; q < 4; ++q) {
-                const int e = e0 + q * kCT;
-                if (e < n4) {
-                  const int m = (4 * e) / qd, k = 4 * e - m * qd;
-                  *reinterpret_cast<float4*>(act + m * a.act_floats + k) = v[q];
+                for (int q = 0; q < kDfMaxSplits; ++q) {
+                  ml[q] = make_float2(-INFINITY, 0.f);
+                  ov[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+                  if (q < S) {
+                    ml[q] = __ldcg(reinterpret_cast<const float2*>(base + q * stride));
+                    ov[q] = __ldcg(reinterpret_cast<const float4*>(base + q * stride + 4 + d));
+                  }
                 }
+                float M = -INFINITY;
+#pragma unroll
+                for (int q = 0; q < kDfMaxSplits; ++q)
+                  if (ml[q].y > 0.f) M = fmaxf(M, ml[q].x);
+                float L = 0.f;
+#pragma unroll
+                for (int q = 0; q < kDfMaxSplits; ++q) {
+                  const float w = ml[q].y > 0.f ? exp2f(ml[q].x - M) : 0.f;
+                  L = fmaf(w, ml[q].y, L);
+                  o.x = fmaf(w, ov[q].x, o.x);
+                  o.y = fmaf(w, ov[q].y, o.y);
+                  o.z = fmaf(w, ov[q].z, o.z);
+                  o.w = fmaf(w, ov[q].w, o.w);
+                }
+                const float inv = L > 0.f ? 1.f / L : 0.f;
+                o = make_float4(o.x * inv, o.y * inv, o.z * inv, o.w * inv);
               }
+              *reinterpret_cast<float4*>(act + m * a.act_floats + hh * a.hd + d) = o;
             }
             csync();
           }

@@ -245,6 +245,7 @@ struct AcceptArgs {
 // between the ops of a pass.  Rows: at most 2 per request (catch-up) and at most
 // kDfMaxGroups requests.
 constexpr int kDfMaxGroups = 4;
+constexpr int kDfMaxSplits = 12;   // key splits per head of the fused draft attention
 constexpr int kDfMaxRows = 2 * kDfMaxGroups;
 constexpr int kDfSlotBytes = 16384;     // weight ring slot
 constexpr int kDfMaxSlots = 16;
@@ -281,8 +282,6 @@ struct DraftFusedArgs {
   float* h;                  // residual stream [kDfMaxRows][d]
   float* qb;                 // rotated queries [kDfMaxRows][H * hd]
   float* att;                // attention partials [kDfMaxRows][H][n_splits][hd + 4]
-  int* att_cnt;              // split arrivals [kDfMaxGroups][H], zero between phases
-  float* ao;                 // combined attention output [kDfMaxRows][H * hd]
   float* act;                // SwiGLU output [kDfMaxRows][F]
   float* lm_part;            // per-CTA LM-head statistics [B][grid][4]
   unsigned int* bar;         // [0] barrier arrivals, [1] exits, [2] abort flag
