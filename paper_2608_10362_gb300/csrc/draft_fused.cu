@@ -278,11 +278,14 @@ __device__ bool grid_sync(const DraftFusedArgs& a, DfCtl& ctl, unsigned& epoch, 
     }
     int ok = *reinterpret_cast<volatile int*>(&ctl.abort) ? 0 : 1;
     if (ok) {
-      __threadfence();
+      // the block barrier above orders every thread's writes before this
+      // thread's release, which publishes them at GPU scope (cumulativity); the
+      // acquire below and the block barrier after it order the other CTAs'
+      // writes before this block's next reads
       red_release_add(&a.bar[0], 1u);
       const long long t0 = clock64();
-      while (ld_acquire_u32(&a.bar[0]) < target) {
-        if (ld_relaxed_u32(&a.bar[2]) != 0u) {
+      for (unsigned it = 0; ld_acquire_u32(&a.bar[0]) < target; ++it) {
+        if ((it & 31u) == 31u && ld_relaxed_u32(&a.bar[2]) != 0u) {   // the abort word, now and then
           ok = 0;
           break;
         }
