@@ -857,6 +857,14 @@ memspec_status emit_forward(memspec_ctx* c, ModelRT& m, const FwdSpec& f,
       at.out_lo = c->o_lo;
       at.plan = c->plan;
       at.status = c->status;
+      // per-op launches stream K/V tiles by TMA (the persistent pass kernel keeps cp.async)
+      if (!c->pass_kernel) {
+        const int kv_rows = c->p.max_batch * cf.n_kv_heads * c->p.max_seq;
+        if (!encode_map(&at.kmap, kl, kv_rows, cf.head_dim, 64) ||
+            !encode_map(&at.vmap, vl, kv_rows, cf.head_dim, 64))
+          return fail(c, MEMSPEC_ERR_CUDA, "KV tensor map");
+        at.tma = 1;
+      }
       PassOp op{};
       op.type = OP_ATTN;
       op.n_units = at.n_splits * at.Hkv * at.row_blocks * f.n_groups;

@@ -30,6 +30,14 @@ using namespace attn;
 template <int HD>
 __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant__ AttnArgs a) {
   extern __shared__ __align__(128) uint8_t smem_raw[];
+  __shared__ uint64_t bars[kStages];   // TMA stages
+  if (a.tma && threadIdx.x == 0) {
+    for (int i = 0; i < kStages; ++i) mbar_init(&bars[i], 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&a.kmap);
+    tma_prefetch_desc(&a.vmap);
+  }
+  __syncthreads();
   pdl_launch_dependents();
   const int lin = (blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
   unsigned long long* trace =
@@ -46,7 +54,7 @@ __global__ void __launch_bounds__(kAttThreads) attn_kernel(const __grid_constant
   };
   const int kvh = blockIdx.y / a.row_blocks, rb = blockIdx.y - kvh * a.row_blocks;
   attention_cta<HD>(a, blockIdx.z, kvh, rb, blockIdx.x, smem_raw, threadIdx.x, sync, wait,
-                    a.ctx_early != 0, trace);
+                    a.ctx_early != 0, trace, false, a.tma ? bars : nullptr);
   trace_at(trace, 1);
 }
 

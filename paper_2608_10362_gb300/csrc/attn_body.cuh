@@ -50,20 +50,28 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&t);
 }
 
-// byte offset of 16-byte chunk `ch` of row `row` in a swizzled [rows][HD] bf16 tile
+// Byte offset of 16-byte chunk `ch` of row `row` in a [64 rows][HD] bf16 tile:
+// 64-column halves one after the other, each [64 rows][128 bytes] with chunk c
+// of row r at c ^ (r % 8) - the layout a TMA box {64, 64} with the 128-byte
+// swizzle writes (and the cp.async path mirrors).
 template <int HD>
 __device__ __forceinline__ uint32_t swz(int row, int ch) {
-  return static_cast<uint32_t>(row * (HD * 2) + ((ch ^ (row & 7)) << 4));
+  return static_cast<uint32_t>((ch >> 3) * (kKeyTile * 128) + row * 128 + (((ch & 7) ^ (row & 7)) << 4));
 }
 
 template <int HD>
-__host__ __device__ constexpr size_t attention_smem_bytes_hd() {
-  // kStages x (K tile + V tile); the merge buffers (o, (m, l), weights, (M, L))
-  // reuse it; the last 16 bytes hold a flag
+__host__ __device__ constexpr size_t attention_body_bytes() {
+  // kStages x (K tile + V tile); the merge buffers (o, (m, l), weights, (M, L)) reuse it
   return static_cast<size_t>(kStages) * 2 * kKeyTile * HD * 2 >
-                 static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + kMaxQ * 6 * 4 + 16
+                 static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + kMaxQ * 6 * 4
              ? static_cast<size_t>(kStages) * 2 * kKeyTile * HD * 2
-             : static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + kMaxQ * 6 * 4 + 16;
+             : static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + kMaxQ * 6 * 4;
+}
+// + up to 1008 bytes to align the stages to 1024 (the swizzle's period), + a
+// 16-byte flag at the end
+template <int HD>
+__host__ __device__ constexpr size_t attention_smem_bytes_hd() {
+  return 1008 + attention_body_bytes<HD>() + 16;
 }
 
 // One CTA of split-KV attention for unit (g, kvh, rb, split), run by 128 threads
@@ -79,11 +87,12 @@ __host__ __device__ constexpr size_t attention_smem_bytes_hd() {
 // and the cached keys / values before the group's first new position are final
 // before wait() (see AttnArgs::ctx_early): the plan is read, and the first tiles
 // that hold only such keys are requested, before it.
+// bars: kStages mbarriers (count 1) for the TMA path (a.tma, not dry), else nullptr.
 template <int HD, class Sync, class Wait>
 __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh, int rb, int split,
                                               uint8_t* smem_raw, int tid, Sync sync, Wait wait,
                                               bool early, unsigned long long* ts = nullptr,
-                                              bool dry = false) {
+                                              bool dry = false, uint64_t* bars = nullptr) {
   constexpr int kChunks = HD / 8;                        // 16-byte chunks per row
   constexpr int kTileBytes = kKeyTile * HD * 2;          // one K (or V) tile
   constexpr int kNT = HD / 8;                            // n8 tiles of the output
@@ -123,7 +132,10 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   const int mt = warp / kg, kgi = warp - mt * kg;
   const bool active = mt < n_mt;
 
-  uint8_t* kv = smem_raw;                                 // kStages x (K tile, V tile)
+  // kStages x (K tile, V tile), 1024-byte aligned
+  uint8_t* kv = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
+  const bool tma = bars != nullptr && !dry;
+  int* flag = reinterpret_cast<int*>(smem_raw + attention_smem_bytes_hd<HD>() - 16);
   // Q (hi and lo planes, [64][HD] bf16 each, swizzled) is staged in the last
   // pipeline stage, which the prologue leaves empty; the fragments move to
   // registers before that stage is first filled.
@@ -132,10 +144,24 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   const bf16* kc = a.kcache + kv_base * HD;
   const bf16* vc = a.vcache + kv_base * HD;
 
+  const int kv_row0 = (req * a.Hkv + kvh) * a.max_seq;   // first row of this head in the maps
   auto load_tile = [&](int t) {
     uint8_t* ks = kv + (t % kStages) * 2 * kTileBytes;
     uint8_t* vs = ks + kTileBytes;
     const int kt0 = k0 + t * kKeyTile;
+    if (tma) {   // one thread: the K and V boxes of the tile (rows past k1 are masked / zeroed later)
+      if (tid == 0) {
+        uint64_t* bar = &bars[t % kStages];
+        const uint64_t pol = l2_policy_evict_first();
+        mbar_arrive_expect_tx(bar, 2u * kTileBytes);
+#pragma unroll
+        for (int hf = 0; hf < HD / 64; ++hf) {
+          tma_load_2d(ks + hf * kKeyTile * 128, &a.kmap, hf * 64, kv_row0 + kt0, bar, pol);
+          tma_load_2d(vs + hf * kKeyTile * 128, &a.vmap, hf * 64, kv_row0 + kt0, bar, pol);
+        }
+      }
+      return;
+    }
     for (int c = tid; c < kKeyTile * kChunks; c += kAttThreads) {
       const int row = c / kChunks, ch = c - row * kChunks;
       const bool ok = kt0 + row < k1 && !dry;   // dry: zero-fill, no global read
@@ -210,9 +236,32 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   for (int i = 0; i < kNT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
 
   const int sub_per_warp = (kKeyTile / 16) / kg;          // 16-key sub-blocks per warp per tile
+  int waited = 0;   // TMA: tiles whose stage completion was observed
   for (int t = 0; t < n_tiles; ++t) {
-    cp_async_wait<kStages - 2>();
-    sync();
+    if (tma) {
+      // one thread waits (bounded); all follow its outcome
+      if (tid == 0)
+        *flag = mbar_wait_bounded(&bars[t % kStages], static_cast<uint32_t>(t / kStages) & 1u, nullptr, a.status)
+                    ? 1
+                    : 0;
+      sync();
+      if (!*flag) break;
+      waited = t + 1;
+      const int nk = min(kKeyTile, k1 - (k0 + t * kKeyTile));
+      if (nk < kKeyTile) {   // V rows past the split's end hold other positions (or garbage): zero them
+        uint8_t* vs = kv + (t % kStages) * 2 * kTileBytes + kTileBytes;
+        for (int c = tid; c < (kKeyTile - nk) * kChunks; c += kAttThreads) {
+          const int row = nk + c / kChunks, ch = c % kChunks;
+          *reinterpret_cast<uint4*>(vs + swz<HD>(row, ch)) = make_uint4(0u, 0u, 0u, 0u);
+        }
+        sync();
+      }
+      // the stage refilled next was last read (ldmatrix, generic proxy) before the barrier above
+      if (tid == 0) fence_proxy_async_smem();
+    } else {
+      cp_async_wait<kStages - 2>();
+      sync();
+    }
     if (t == 0) trace_at(ts, 10);
     if (t + kStages - 1 < n_tiles) load_tile(t + kStages - 1);
     cp_async_commit();
@@ -316,6 +365,13 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     }
   }
   cp_async_wait<0>();
+  if (tma && waited < n_tiles) {   // a wait ran out: let the copies still in flight land, then stop
+    if (tid == 0)
+      for (int t = waited; t < min(n_tiles, waited + kStages); ++t)
+        mbar_wait_drain(&bars[t % kStages], static_cast<uint32_t>(t / kStages) & 1u);
+    sync();
+    return;
+  }
   sync();
   trace_at(ts, 9);
   if (ts != nullptr) trace_after(ts, 12, o[0][0] + o[kNT - 1][3]);   // last MMAs retired
@@ -387,7 +443,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   // partial stores before thread 0's acq_rel arrival; the last split's acquire
   // and the next barrier order every split's partials before its loads
   sync();
-  int* last = reinterpret_cast<int*>(kv + attention_smem_bytes_hd<HD>() - 16);
+  int* last = flag;
   if (tid == 0)
     *last = dry ? 1 : ((atom_add_acq_rel_gpu(&a.counters[unit], 1) == n_active - 1) ? 1 : 0);
   sync();

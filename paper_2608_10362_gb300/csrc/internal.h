@@ -175,6 +175,9 @@ struct GemmArgs {
 };
 
 struct AttnArgs {
+  CUtensorMap kmap;         // tma: this layer's K cache as [max_batch * Hkv * max_seq][hd] bf16,
+  CUtensorMap vmap;         //   box {64, 64}, 128-byte swizzle; V likewise
+  int tma;                  // 1: K/V tiles by cp.async.bulk.tensor into mbarrier stages
   const float* q;           // [rows][H][hd] fp32, rotated
   const bf16* kcache;       // [req][Hkv][max_seq][hd]
   const bf16* vcache;
