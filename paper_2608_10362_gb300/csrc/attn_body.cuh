@@ -45,6 +45,13 @@ __device__ __forceinline__ void mma16816(float* c, const uint32_t* a, uint32_t b
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
+// 8x8 b16 matrix held as the ldmatrix fragment (lane: row lane/4, columns
+// 2(lane%4), +1) -> the same fragment of its transpose
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
+  uint32_t y;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
+}
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 t = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&t);
@@ -88,7 +95,10 @@ __host__ __device__ constexpr size_t attention_smem_bytes_hd() {
 // before wait() (see AttnArgs::ctx_early): the plan is read, and the first tiles
 // that hold only such keys are requested, before it.
 // bars: kStages mbarriers (count 1) for the TMA path (a.tma, not dry), else nullptr.
-template <int HD, class Sync, class Wait>
+// kTQ: at most 8 query vectors (the launch's qmax <= 8; checked): the keys are the
+// MMA's M side, S^T = K Q^T and O^T = V^T P^T with the queries as N = 8, half the
+// MMAs, accumulator registers and rescaling work of the 16-row form.
+template <int HD, bool kTQ = false, class Sync, class Wait>
 __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh, int rb, int split,
                                               uint8_t* smem_raw, int tid, Sync sync, Wait wait,
                                               bool early, unsigned long long* ts = nullptr,
@@ -116,7 +126,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   const int gs = a.H / a.Hkv;
   const int nq = gs * nr;
   const int kmax = pos0 + r_hi - 1;
-  if (pos0 < 0 || kmax >= a.max_seq || nq > kMaxQ || a.n_splits > 16) {   // reported, never read
+  if (pos0 < 0 || kmax >= a.max_seq || nq > (kTQ ? 8 : kMaxQ) || a.n_splits > 16) {   // reported, never read
     if (threadIdx.x == 0 && split == 0) atomicOr(a.status, 0x4u);
     return;
   }
@@ -136,10 +146,6 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   uint8_t* kv = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
   const bool tma = bars != nullptr && !dry;
   int* flag = reinterpret_cast<int*>(smem_raw + attention_smem_bytes_hd<HD>() - 16);
-  // Q (hi and lo planes, [64][HD] bf16 each, swizzled) is staged in the last
-  // pipeline stage, which the prologue leaves empty; the fragments move to
-  // registers before that stage is first filled.
-  uint8_t* qs = kv + (kStages - 1) * 2 * kTileBytes;
   const size_t kv_base = (static_cast<size_t>(req) * a.Hkv + kvh) * a.max_seq;
   const bf16* kc = a.kcache + kv_base * HD;
   const bf16* vc = a.vcache + kv_base * HD;
@@ -171,69 +177,97 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     }
   };
 
-  // prologue: start the first kStages-1 tiles (early: those below pos0 before the
-  // wait), then stage Q (fp32 -> bf16, scaled)
+  // prologue: the TMA path requests every stage (Q goes straight to registers),
+  // the cp.async path the first kStages-1 tiles (one commit group per stage);
+  // early: the tiles that hold only keys below pos0 go before the wait
+  const int depth = tma ? kStages : kStages - 1;
   int s_pre = 0;
   if (early) {
-    for (; s_pre < kStages - 1 && s_pre < n_tiles && k0 + (s_pre + 1) * kKeyTile <= pos0; ++s_pre) {
+    for (; s_pre < depth && s_pre < n_tiles && k0 + (s_pre + 1) * kKeyTile <= pos0; ++s_pre) {
       load_tile(s_pre);
       cp_async_commit();
     }
     wait();
   }
-  for (int s = s_pre; s < kStages - 1; ++s) {
+  for (int s = s_pre; s < depth; ++s) {
     if (s < n_tiles) load_tile(s);
     cp_async_commit();
   }
-  for (int c = tid; c < kMaxQ * kChunks; c += kAttThreads) {
-    const int v = c / kChunks, ch = c - v * kChunks;
-    __nv_bfloat16 e[8], el[8];
-    if (v < nq && !dry) {
-      const int hl = v / nr, rr = v - hl * nr;
-      const int row = g * R + r_lo + rr;
-      const int h = kvh * gs + hl;
-      const float* src = a.q + (static_cast<size_t>(row) * a.H + h) * HD + ch * 8;
-      const float4 x0 = *reinterpret_cast<const float4*>(src);
-      const float4 x1 = *reinterpret_cast<const float4*>(src + 4);
-      const float f[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-#pragma unroll
-      for (int i = 0; i < 8; ++i) split_bf16(f[i] * a.scale_log2, e[i], el[i]);
-    } else {
-#pragma unroll
-      for (int i = 0; i < 8; ++i) e[i] = el[i] = __float2bfloat16_rn(0.f);
-    }
-    *reinterpret_cast<uint4*>(qs + swz<HD>(v, ch)) = *reinterpret_cast<const uint4*>(e);
-    *reinterpret_cast<uint4*>(qs + kTileBytes + swz<HD>(v, ch)) = *reinterpret_cast<const uint4*>(el);
-  }
-  sync();
-  trace_at(ts, 8);
+  int next = min(depth, n_tiles);   // tiles requested so far
 
-  // Q fragments (hi and lo) of this warp's m-tile stay in registers
-  uint32_t qa[HD / 16][4], ql[HD / 16][4];
-  if (active) {
+  // Q fragments (hi and lo planes, pre-scaled), loaded from the fp32 rows
+  // straight into registers.  16-row form: A operand of m16n8k16 for this
+  // warp's m-tile, register j of k-step ks holds row lane/4 (+8 if j is odd) and
+  // columns 2(lane%4), +1 (+8 if j >= 2).  kTQ: B operand, query lane/4, register
+  // j of k-step ks holds columns 2(lane%4), +1 (+8 if j == 1).
+  // Query vector v of the block is head v / nr of the group, row v % nr.
+  auto q_row = [&](int v) {
+    const int hl = v / nr, rr = v - hl * nr;
+    return a.q + (static_cast<size_t>(g * R + r_lo + rr) * a.H + kvh * gs + hl) * HD + 2 * (lane & 3);
+  };
+  auto split2 = [&](float2 x, uint32_t& hi, uint32_t& lo) {
+    __nv_bfloat16 h0, l0, h1, l1;
+    split_bf16(x.x * a.scale_log2, h0, l0);
+    split_bf16(x.y * a.scale_log2, h1, l1);
+    hi = pack_bf16x2(__bfloat162float(h0), __bfloat162float(h1));
+    lo = pack_bf16x2(__bfloat162float(l0), __bfloat162float(l1));
+  };
+  uint32_t qa[kTQ ? 1 : HD / 16][4], ql[kTQ ? 1 : HD / 16][4];
+  uint32_t qb[kTQ ? HD / 16 : 1][2], qbl[kTQ ? HD / 16 : 1][2];
+  if constexpr (kTQ) {
+    const int v = lane >> 2;
+    const float* src = (v < nq && !dry) ? q_row(v) : nullptr;
+    float2 x[HD / 16][2];
 #pragma unroll
-    for (int ks = 0; ks < HD / 16; ++ks) {
-      const int row = mt * 16 + (lane & 15);
-      const int ch = ks * 2 + (lane >> 4);
-      ldsm_x4(smem_addr(qs) + swz<HD>(row, ch), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
-      ldsm_x4(smem_addr(qs + kTileBytes) + swz<HD>(row, ch), ql[ks][0], ql[ks][1], ql[ks][2],
-              ql[ks][3]);
+    for (int ks = 0; ks < HD / 16; ++ks)
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+        x[ks][j] = src != nullptr ? *reinterpret_cast<const float2*>(src + ks * 16 + j * 8) : make_float2(0.f, 0.f);
+#pragma unroll
+    for (int ks = 0; ks < HD / 16; ++ks)
+#pragma unroll
+      for (int j = 0; j < 2; ++j) split2(x[ks][j], qb[ks][j], qbl[ks][j]);
+    if (ts != nullptr) trace_after(ts, 8, __uint_as_float(qb[0][0] ^ qbl[HD / 16 - 1][1]));
+  } else {
+    const float* qsrc[2] = {nullptr, nullptr};
+#pragma unroll
+    for (int h2 = 0; h2 < 2; ++h2) {
+      const int v = mt * 16 + (lane >> 2) + 8 * h2;
+      if (active && v < nq && !dry) qsrc[h2] = q_row(v);
     }
+    float2 x[HD / 16][4];
+#pragma unroll
+    for (int ks = 0; ks < HD / 16; ++ks)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float* src = qsrc[j & 1];
+        x[ks][j] = src != nullptr ? *reinterpret_cast<const float2*>(src + ks * 16 + (j >> 1) * 8)
+                                  : make_float2(0.f, 0.f);
+      }
+#pragma unroll
+    for (int ks = 0; ks < HD / 16; ++ks)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) split2(x[ks][j], qa[ks][j], ql[ks][j]);
+    if (ts != nullptr) trace_after(ts, 8, __uint_as_float(qa[0][0] ^ ql[HD / 16 - 1][3]));
   }
-  // positions of this thread's two rows (v = mt*16 + lane/4 and +8); -1: padding row
-  // tree passes: beyond pos0 a row sees only the rows in its ancestor mask
+  // positions of this thread's two query vectors (16-row form: v = mt*16 +
+  // lane/4 and +8; kTQ: v = 2(lane%4) and +1); -1: padding.  Tree passes:
+  // beyond pos0 a vector sees only the rows in its ancestor mask
   int prow[2];
   uint32_t amask[2] = {0u, 0u};
 #pragma unroll
   for (int h2 = 0; h2 < 2; ++h2) {
-    const int v = mt * 16 + (lane >> 2) + 8 * h2;
+    const int v = kTQ ? 2 * (lane & 3) + h2 : mt * 16 + (lane >> 2) + 8 * h2;
     prow[h2] = (active && v < nq) ? pos0 + r_lo + (v % nr) : -1;
     if (tree && prow[h2] >= 0 && r_lo + (v % nr) < kTreeRows) amask[h2] = plan->anc[r_lo + (v % nr)];
   }
   float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
-  float o[kNT][4];
+  // output accumulators: 16-row form [n8 tile of features][4]; kTQ: [16-feature
+  // block][4] of O^T (features lane/4 and +8, queries 2(lane%4) and +1)
+  constexpr int kNO = kTQ ? HD / 16 : kNT;
+  float o[kNO][4];
 #pragma unroll
-  for (int i = 0; i < kNT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  for (int i = 0; i < kNO; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
 
   const int sub_per_warp = (kKeyTile / 16) / kg;          // 16-key sub-blocks per warp per tile
   int waited = 0;   // TMA: tiles whose stage completion was observed
@@ -256,125 +290,257 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
         }
         sync();
       }
-      // the stage refilled next was last read (ldmatrix, generic proxy) before the barrier above
-      if (tid == 0) fence_proxy_async_smem();
+      // the stage refilled next (tile t-1's) was last read (ldmatrix, generic
+      // proxy) before the barrier above
+      if (next < n_tiles && next < t + kStages) {
+        if (tid == 0) fence_proxy_async_smem();
+        load_tile(next);
+        ++next;
+      }
     } else {
       cp_async_wait<kStages - 2>();
       sync();
+      if (t + kStages - 1 < n_tiles) load_tile(t + kStages - 1);
+      cp_async_commit();
     }
     if (t == 0) trace_at(ts, 10);
-    if (t + kStages - 1 < n_tiles) load_tile(t + kStages - 1);
-    cp_async_commit();
     if (!active) continue;
     const uint32_t ks_addr = smem_addr(kv + (t % kStages) * 2 * kTileBytes);
     const uint32_t vs_addr = ks_addr + kTileBytes;
     const int kt0 = k0 + t * kKeyTile;
-    for (int sb = 0; sb < sub_per_warp; ++sb) {
-      const int kb = (kgi * sub_per_warp + sb) * 16;      // key offset within the tile
-      float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+    if constexpr (kTQ) {
+      for (int sb = 0; sb < sub_per_warp; ++sb) {
+        const int kb = (kgi * sub_per_warp + sb) * 16;    // key offset within the tile
+        // S^T (16 keys x 8 queries): A = K rows from the stage, B = Q; chains
+        // per Q plane and (hd 128) k-step parity, summed at the end
+        constexpr int kPar = HD >= 128 ? 2 : 1;
+        float sp[2][kPar][4];
 #pragma unroll
-      for (int ks = 0; ks < HD / 16; ++ks) {
-        uint32_t b0, b1, b2, b3;
-        const int row = kb + (lane & 7) + ((lane >> 4) << 3);
-        const int ch = ks * 2 + ((lane >> 3) & 1);
-        ldsm_x4(ks_addr + swz<HD>(row, ch), b0, b1, b2, b3);
-        mma16816(s0, qa[ks], b0, b1);
-        mma16816(s0, ql[ks], b0, b1);
-        mma16816(s1, qa[ks], b2, b3);
-        mma16816(s1, ql[ks], b2, b3);
-      }
-      // causal / range mask, then online softmax (base 2)
-      const int key_c = kt0 + kb + ((lane & 3) << 1);
-      float mx[2];
+        for (int pl = 0; pl < 2; ++pl)
 #pragma unroll
-      for (int h2 = 0; h2 < 2; ++h2) {
-        const int p = prow[h2];
-        const int lim = min(p, k1 - 1);
-        const uint32_t am = amask[h2];
-        // key visible: causal (and in this split) and, in a tree pass, below
-        // pos0 or an ancestor row (rows past 31 never appear in a tree pass)
-        auto vis = [&](int key) {
-          if (key > lim) return false;
-          if (!tree) return true;
-          const int rel = key - pos0;
-          return rel < 0 || (rel < kTreeRows && ((am >> rel) & 1u) != 0u);
-        };
-        float* a0 = s0 + 2 * h2;
-        float* a1 = s1 + 2 * h2;
-        a0[0] = vis(key_c) ? a0[0] : -INFINITY;
-        a0[1] = vis(key_c + 1) ? a0[1] : -INFINITY;
-        a1[0] = vis(key_c + 8) ? a1[0] : -INFINITY;
-        a1[1] = vis(key_c + 9) ? a1[1] : -INFINITY;
-        mx[h2] = fmaxf(fmaxf(a0[0], a0[1]), fmaxf(a1[0], a1[1]));
-        mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 1));
-        mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 2));
-      }
-      float scale[2];
+          for (int par = 0; par < kPar; ++par)
 #pragma unroll
-      for (int h2 = 0; h2 < 2; ++h2) {
-        const float m_new = fmaxf(m_run[h2], mx[h2]);
-        float* a0 = s0 + 2 * h2;
-        float* a1 = s1 + 2 * h2;
-        if (m_new == -INFINITY) {
-          scale[h2] = 1.f;
-          a0[0] = a0[1] = a1[0] = a1[1] = 0.f;
-        } else {
-          scale[h2] = exp2f(m_run[h2] - m_new);
-          a0[0] = exp2f(a0[0] - m_new);
-          a0[1] = exp2f(a0[1] - m_new);
-          a1[0] = exp2f(a1[0] - m_new);
-          a1[1] = exp2f(a1[1] - m_new);
+            for (int i = 0; i < 4; ++i) sp[pl][par][i] = 0.f;
+#pragma unroll
+        for (int ks = 0; ks < HD / 16; ++ks) {
+          uint32_t ka[4];
+          const int row = kb + (lane & 7) + (((lane >> 3) & 1) << 3);
+          const int ch = ks * 2 + (lane >> 4);
+          ldsm_x4(ks_addr + swz<HD>(row, ch), ka[0], ka[1], ka[2], ka[3]);
+          const int par = ks % kPar;
+          mma16816(sp[0][par], ka, qb[ks][0], qb[ks][1]);
+          mma16816(sp[1][par], ka, qbl[ks][0], qbl[ks][1]);
         }
-        float rs = (a0[0] + a0[1]) + (a1[0] + a1[1]);
-        rs += __shfl_xor_sync(0xffffffffu, rs, 1);
-        rs += __shfl_xor_sync(0xffffffffu, rs, 2);
-        l_run[h2] = l_run[h2] * scale[h2] + rs;
-        m_run[h2] = m_new;
-      }
-#pragma unroll
-      for (int i = 0; i < kNT; ++i) {
-        o[i][0] *= scale[0];
-        o[i][1] *= scale[0];
-        o[i][2] *= scale[1];
-        o[i][3] *= scale[1];
-      }
-      // P as hi + lo bf16 fragments
-      uint32_t pa[4], pl[4];
-      {
-        const float pv[8] = {s0[0], s0[1], s0[2], s0[3], s1[0], s1[1], s1[2], s1[3]};
-        float lo[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) lo[i] = pv[i] - __bfloat162float(__float2bfloat16_rn(pv[i]));
+        // sc[0], sc[1]: key kb + lane/4, queries 2(lane%4) and +1; sc[2], sc[3]: key + 8
+        float sc[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-          pa[i] = pack_bf16x2(pv[2 * i], pv[2 * i + 1]);
-          pl[i] = pack_bf16x2(lo[2 * i], lo[2 * i + 1]);
+          if constexpr (kPar == 2)
+            sc[i] = (sp[0][0][i] + sp[0][1][i]) + (sp[1][0][i] + sp[1][1][i]);
+          else
+            sc[i] = sp[0][0][i] + sp[1][0][i];
+        }
+        const int key_c = kt0 + kb + (lane >> 2);
+        float mx[2];
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          const int p = prow[h2];
+          const int lim = min(p, k1 - 1);
+          const uint32_t am = amask[h2];
+          auto vis = [&](int key) {
+            if (key > lim) return false;
+            if (!tree) return true;
+            const int rel = key - pos0;
+            return rel < 0 || (rel < kTreeRows && ((am >> rel) & 1u) != 0u);
+          };
+          sc[h2] = vis(key_c) ? sc[h2] : -INFINITY;
+          sc[2 + h2] = vis(key_c + 8) ? sc[2 + h2] : -INFINITY;
+          mx[h2] = fmaxf(sc[h2], sc[2 + h2]);
+          mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 4));
+          mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 8));
+          mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 16));
+        }
+        float scale[2];
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          const float m_new = fmaxf(m_run[h2], mx[h2]);
+          if (m_new == -INFINITY) {
+            scale[h2] = 1.f;
+            sc[h2] = sc[2 + h2] = 0.f;
+          } else {
+            scale[h2] = exp2f(m_run[h2] - m_new);
+            sc[h2] = exp2f(sc[h2] - m_new);
+            sc[2 + h2] = exp2f(sc[2 + h2] - m_new);
+          }
+          float rs = sc[h2] + sc[2 + h2];
+          rs += __shfl_xor_sync(0xffffffffu, rs, 4);
+          rs += __shfl_xor_sync(0xffffffffu, rs, 8);
+          rs += __shfl_xor_sync(0xffffffffu, rs, 16);
+          l_run[h2] = l_run[h2] * scale[h2] + rs;
+          m_run[h2] = m_new;
+        }
+#pragma unroll
+        for (int i = 0; i < kNO; ++i) {
+          o[i][0] *= scale[0];
+          o[i][1] *= scale[1];
+          o[i][2] *= scale[0];
+          o[i][3] *= scale[1];
+        }
+        // P^T as the B operand (keys x queries), hi + lo planes: the 8x8 blocks
+        // [key][query] this lane holds (rows lane/4, columns 2(lane%4), +1) are
+        // transposed across the warp, giving query lane/4, keys 2(lane%4), +1
+        uint32_t pb[2], pbl[2];
+#pragma unroll
+        for (int hk = 0; hk < 2; ++hk) {
+          const float x0 = sc[2 * hk], x1 = sc[2 * hk + 1];
+          const float h0 = __bfloat162float(__float2bfloat16_rn(x0));
+          const float h1 = __bfloat162float(__float2bfloat16_rn(x1));
+          pb[hk] = movmatrix_trans(pack_bf16x2(x0, x1));
+          pbl[hk] = movmatrix_trans(pack_bf16x2(x0 - h0, x1 - h1));
+        }
+        // O^T += V^T P^T: A = V^T (16 features x 16 keys) by transposing loads
+#pragma unroll
+        for (int i = 0; i < kNO; ++i) {
+          uint32_t va[4];
+          const int row = kb + (lane & 7) + ((lane >> 4) << 3);
+          const int ch = i * 2 + ((lane >> 3) & 1);
+          ldsm_x4_t(vs_addr + swz<HD>(row, ch), va[0], va[1], va[2], va[3]);
+          mma16816(o[i], va, pb[0], pb[1]);
+          mma16816(o[i], va, pbl[0], pbl[1]);
         }
       }
-#pragma unroll
-      for (int n2 = 0; n2 < HD / 16; ++n2) {
-        uint32_t b0, b1, b2, b3;
-        const int row = kb + (lane & 7) + (((lane >> 3) & 1) << 3);
-        const int ch = n2 * 2 + (lane >> 4);
-        ldsm_x4_t(vs_addr + swz<HD>(row, ch), b0, b1, b2, b3);
-        mma16816(o[2 * n2], pa, b0, b1);
-        mma16816(o[2 * n2], pl, b0, b1);
-        mma16816(o[2 * n2 + 1], pa, b2, b3);
-        mma16816(o[2 * n2 + 1], pl, b2, b3);
+    } else {
+      for (int sb = 0; sb < sub_per_warp; ++sb) {
+        const int kb = (kgi * sub_per_warp + sb) * 16;      // key offset within the tile
+        // independent accumulator chains (n8 tile x Q plane x, at hd 128, k-step
+        // parity), summed at the end: one chain per n8 tile would serialise
+        // 2 hd / 16 dependent MMAs per sub-block
+        constexpr int kPar = HD >= 128 ? 2 : 1;
+        float sp[2][2][kPar][4];
+  #pragma unroll
+        for (int n = 0; n < 2; ++n)
+  #pragma unroll
+          for (int pl = 0; pl < 2; ++pl)
+  #pragma unroll
+            for (int par = 0; par < kPar; ++par)
+  #pragma unroll
+              for (int i = 0; i < 4; ++i) sp[n][pl][par][i] = 0.f;
+  #pragma unroll
+        for (int ks = 0; ks < HD / 16; ++ks) {
+          uint32_t b0, b1, b2, b3;
+          const int row = kb + (lane & 7) + ((lane >> 4) << 3);
+          const int ch = ks * 2 + ((lane >> 3) & 1);
+          ldsm_x4(ks_addr + swz<HD>(row, ch), b0, b1, b2, b3);
+          const int par = ks % kPar;
+          mma16816(sp[0][0][par], qa[ks], b0, b1);
+          mma16816(sp[0][1][par], ql[ks], b0, b1);
+          mma16816(sp[1][0][par], qa[ks], b2, b3);
+          mma16816(sp[1][1][par], ql[ks], b2, b3);
+        }
+        float s0[4], s1[4];
+  #pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          if constexpr (kPar == 2) {
+            s0[i] = (sp[0][0][0][i] + sp[0][0][1][i]) + (sp[0][1][0][i] + sp[0][1][1][i]);
+            s1[i] = (sp[1][0][0][i] + sp[1][0][1][i]) + (sp[1][1][0][i] + sp[1][1][1][i]);
+          } else {
+            s0[i] = sp[0][0][0][i] + sp[0][1][0][i];
+            s1[i] = sp[1][0][0][i] + sp[1][1][0][i];
+          }
+        }
+        // causal / range mask, then online softmax (base 2)
+        const int key_c = kt0 + kb + ((lane & 3) << 1);
+        float mx[2];
+  #pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          const int p = prow[h2];
+          const int lim = min(p, k1 - 1);
+          const uint32_t am = amask[h2];
+          // key visible: causal (and in this split) and, in a tree pass, below
+          // pos0 or an ancestor row (rows past 31 never appear in a tree pass)
+          auto vis = [&](int key) {
+            if (key > lim) return false;
+            if (!tree) return true;
+            const int rel = key - pos0;
+            return rel < 0 || (rel < kTreeRows && ((am >> rel) & 1u) != 0u);
+          };
+          float* a0 = s0 + 2 * h2;
+          float* a1 = s1 + 2 * h2;
+          a0[0] = vis(key_c) ? a0[0] : -INFINITY;
+          a0[1] = vis(key_c + 1) ? a0[1] : -INFINITY;
+          a1[0] = vis(key_c + 8) ? a1[0] : -INFINITY;
+          a1[1] = vis(key_c + 9) ? a1[1] : -INFINITY;
+          mx[h2] = fmaxf(fmaxf(a0[0], a0[1]), fmaxf(a1[0], a1[1]));
+          mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 1));
+          mx[h2] = fmaxf(mx[h2], __shfl_xor_sync(0xffffffffu, mx[h2], 2));
+        }
+        float scale[2];
+  #pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          const float m_new = fmaxf(m_run[h2], mx[h2]);
+          float* a0 = s0 + 2 * h2;
+          float* a1 = s1 + 2 * h2;
+          if (m_new == -INFINITY) {
+            scale[h2] = 1.f;
+            a0[0] = a0[1] = a1[0] = a1[1] = 0.f;
+          } else {
+            scale[h2] = exp2f(m_run[h2] - m_new);
+            a0[0] = exp2f(a0[0] - m_new);
+            a0[1] = exp2f(a0[1] - m_new);
+            a1[0] = exp2f(a1[0] - m_new);
+            a1[1] = exp2f(a1[1] - m_new);
+          }
+          float rs = (a0[0] + a0[1]) + (a1[0] + a1[1]);
+          rs += __shfl_xor_sync(0xffffffffu, rs, 1);
+          rs += __shfl_xor_sync(0xffffffffu, rs, 2);
+          l_run[h2] = l_run[h2] * scale[h2] + rs;
+          m_run[h2] = m_new;
+        }
+  #pragma unroll
+        for (int i = 0; i < kNT; ++i) {
+          o[i][0] *= scale[0];
+          o[i][1] *= scale[0];
+          o[i][2] *= scale[1];
+          o[i][3] *= scale[1];
+        }
+        // P as hi + lo bf16 fragments
+        uint32_t pa[4], pl[4];
+        {
+          const float pv[8] = {s0[0], s0[1], s0[2], s0[3], s1[0], s1[1], s1[2], s1[3]};
+          float lo[8];
+  #pragma unroll
+          for (int i = 0; i < 8; ++i) lo[i] = pv[i] - __bfloat162float(__float2bfloat16_rn(pv[i]));
+  #pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            pa[i] = pack_bf16x2(pv[2 * i], pv[2 * i + 1]);
+            pl[i] = pack_bf16x2(lo[2 * i], lo[2 * i + 1]);
+          }
+        }
+  #pragma unroll
+        for (int n2 = 0; n2 < HD / 16; ++n2) {
+          uint32_t b0, b1, b2, b3;
+          const int row = kb + (lane & 7) + (((lane >> 3) & 1) << 3);
+          const int ch = n2 * 2 + (lane >> 4);
+          ldsm_x4_t(vs_addr + swz<HD>(row, ch), b0, b1, b2, b3);
+          mma16816(o[2 * n2], pa, b0, b1);
+          mma16816(o[2 * n2], pl, b0, b1);
+          mma16816(o[2 * n2 + 1], pa, b2, b3);
+          mma16816(o[2 * n2 + 1], pl, b2, b3);
+        }
       }
     }
   }
   cp_async_wait<0>();
   if (tma && waited < n_tiles) {   // a wait ran out: let the copies still in flight land, then stop
     if (tid == 0)
-      for (int t = waited; t < min(n_tiles, waited + kStages); ++t)
+      for (int t = waited; t < next; ++t)
         mbar_wait_drain(&bars[t % kStages], static_cast<uint32_t>(t / kStages) & 1u);
     sync();
     return;
   }
   sync();
   trace_at(ts, 9);
-  if (ts != nullptr) trace_after(ts, 12, o[0][0] + o[kNT - 1][3]);   // last MMAs retired
+  if (ts != nullptr) trace_after(ts, 12, o[0][0] + o[kNO - 1][3]);   // last MMAs retired
 
   // merge the key groups of each m-tile (shared memory reuses the K/V stages):
   // the query vectors' rows of o go to shared memory (padding rows are not
@@ -385,11 +551,28 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   float* ml = mo + 4 * 16 * HD;                             // [4 warps][16][2]
   float* mf = ml + 4 * 16 * 2;                              // [kMaxQ][4] weights
   float* mml = mf + kMaxQ * 4;                              // [kMaxQ][2] M, L
-  if (active) {
+  if (kTQ) {   // O^T fragments: features 16i + lane/4 (+8), queries 2(lane%4), +1
+    const int f0 = lane >> 2;
+#pragma unroll
+    for (int h2 = 0; h2 < 2; ++h2) {
+      const int v = 2 * (lane & 3) + h2;
+      if (v >= nq) continue;
+      float* dst = mo + (warp * 16 + v) * HD + f0;
+#pragma unroll
+      for (int i = 0; i < kNO; ++i) {
+        dst[i * 16] = o[i][h2];
+        dst[i * 16 + 8] = o[i][2 + h2];
+      }
+      if (f0 == 0) {
+        ml[(warp * 16 + v) * 2] = m_run[h2];
+        ml[(warp * 16 + v) * 2 + 1] = l_run[h2];
+      }
+    }
+  } else if (active) {
     const int r0 = lane >> 2, cc = (lane & 3) << 1;
     const bool lo_ok = mt * 16 + r0 < nq, hi_ok = mt * 16 + r0 + 8 < nq;
 #pragma unroll
-    for (int i = 0; i < kNT; ++i) {
+    for (int i = 0; i < kNO; ++i) {
       float* dst = mo + (warp * 16) * HD + i * 8 + cc;
       if (lo_ok) *reinterpret_cast<float2*>(dst + r0 * HD) = make_float2(o[i][0], o[i][1]);
       if (hi_ok) *reinterpret_cast<float2*>(dst + (r0 + 8) * HD) = make_float2(o[i][2], o[i][3]);
@@ -453,57 +636,99 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   const int qmax = a.qmax;
   const float* part_ml = a.part_ml;
   const float* part_o = a.part_o;
-  // One round trip: each thread fetches, for its query vector v and its four
-  // features, every split's (m_s, l_s) (the 32 threads of a vector read the same
-  // words: one transaction) together with its o_s (n_active <= 16: the geometry
-  // caps the splits), then M = max m_s, weights 2^(m_s - M), L and the weighted
-  // sum, all in ascending split order.
   constexpr int kV4 = HD / 4;
   bf16* out = a.out;
   bf16* out_lo = a.out_lo;
   const int H = a.H;
-  for (int idx = tid; idx < nq * kV4; idx += kAttThreads) {
-    const int v = idx / kV4, d = (idx - v * kV4) * 4;
-    float2 mlv[16];
-    float4 ov[16];
-#pragma unroll
-    for (int q = 0; q < 16; ++q) {
-      if (q < n_active) {
-        const size_t pv = ubase + static_cast<size_t>(q) * qmax + v;
-        mlv[q] = ld_cg_f2(part_ml + pv * 2);
-        ov[q] = ld_cg_f4(part_o + pv * HD + d);
-      }
-    }
-    if (idx == tid) trace_after(ts, 6, mlv[0].x + ov[0].x);
-    float M = -INFINITY;
-#pragma unroll
-    for (int q = 0; q < 16; ++q)
-      if (q < n_active) M = fmaxf(M, mlv[q].x);
-    float L = 0.f;
-    float O[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-    for (int q = 0; q < 16; ++q) {
-      if (q < n_active) {
-        const float w = mlv[q].x == -INFINITY ? 0.f : exp2f(mlv[q].x - M);
-        L += w * mlv[q].y;
-        O[0] += w * ov[q].x;
-        O[1] += w * ov[q].y;
-        O[2] += w * ov[q].z;
-        O[3] += w * ov[q].w;
-      }
-    }
+  // o = O / L of query vector v, features d..d+3: hi and lo planes, one 8-byte
+  // store each (the index is a multiple of 4)
+  auto emit = [&](int v, int d, float O0, float O1, float O2, float O3, float L) {
+    const float O[4] = {O0, O1, O2, O3};
     const float li = 1.f / L;
     const int hl = v / nr, rr = v - hl * nr;
     const int row = g * R + r_lo + rr;
     const int h = kvh * gs + hl;
     const size_t oi = (static_cast<size_t>(row) * H + h) * HD + d;
-    if (dry) continue;
-    // four features: one 8-byte store per plane (oi is a multiple of 4)
+    if (dry) return;
     __nv_bfloat16 hv[4], lv[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) split_bf16(O[e] * li, hv[e], lv[e]);
     *reinterpret_cast<uint2*>(out + oi) = *reinterpret_cast<const uint2*>(hv);
     if (out_lo != nullptr) *reinterpret_cast<uint2*>(out_lo + oi) = *reinterpret_cast<const uint2*>(lv);
+  };
+  // Both ways below compute M = max m_s, weights 2^(m_s - M), L and the weighted
+  // sum of the o_s in ascending split order (identical results).
+  const size_t land_o = static_cast<size_t>(n_active) * qmax * HD;   // floats
+  if ((land_o + static_cast<size_t>(n_active) * qmax * 2) * 4 <= attention_body_bytes<HD>()) {
+    // every active split's o (contiguous, [split][qmax][HD]) by 16-byte cp.async
+    // (L2) and its (m, l) by ld.cg land in the stages - free now: this CTA's own
+    // partial went out above - in one round trip; the sums read shared memory
+    float* so = reinterpret_cast<float*>(kv);
+    float* sml = so + land_o;
+    const float* src = part_o + ubase * HD;
+    for (size_t i = tid; i < land_o / 4; i += kAttThreads) cp_async16_zfill(so + 4 * i, src + 4 * i, true);
+    cp_async_commit();
+    for (int i = tid; i < n_active * qmax; i += kAttThreads)
+      *reinterpret_cast<float2*>(sml + 2 * i) = ld_cg_f2(part_ml + (ubase + i) * 2);
+    cp_async_wait<0>();
+    sync();
+    trace_at(ts, 6);
+    for (int idx = tid; idx < nq * kV4; idx += kAttThreads) {
+      const int v = idx / kV4, d = (idx - v * kV4) * 4;
+      float M = -INFINITY;
+      for (int q = 0; q < n_active; ++q) M = fmaxf(M, sml[(q * qmax + v) * 2]);
+      float L = 0.f;
+      float O[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+      for (int q = 0; q < n_active; ++q) {
+        const float2 ml = *reinterpret_cast<const float2*>(sml + (q * qmax + v) * 2);
+        const float4 ov = *reinterpret_cast<const float4*>(so + (static_cast<size_t>(q) * qmax + v) * HD + d);
+        const float w = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);
+        L += w * ml.y;
+        O[0] += w * ov.x;
+        O[1] += w * ov.y;
+        O[2] += w * ov.z;
+        O[3] += w * ov.w;
+      }
+      emit(v, d, O[0], O[1], O[2], O[3], L);
+    }
+  } else {
+    // too many splits or vectors to land: each thread fetches, for its query
+    // vector v and its four features, every split's (m_s, l_s) (the 32 threads
+    // of a vector read the same words: one transaction) together with its o_s
+    // (n_active <= 16: the geometry caps the splits), one round trip per pass
+    for (int idx = tid; idx < nq * kV4; idx += kAttThreads) {
+      const int v = idx / kV4, d = (idx - v * kV4) * 4;
+      float2 mlv[16];
+      float4 ov[16];
+#pragma unroll
+      for (int q = 0; q < 16; ++q) {
+        if (q < n_active) {
+          const size_t pv = ubase + static_cast<size_t>(q) * qmax + v;
+          mlv[q] = ld_cg_f2(part_ml + pv * 2);
+          ov[q] = ld_cg_f4(part_o + pv * HD + d);
+        }
+      }
+      if (idx == tid) trace_after(ts, 6, mlv[0].x + ov[0].x);
+      float M = -INFINITY;
+#pragma unroll
+      for (int q = 0; q < 16; ++q)
+        if (q < n_active) M = fmaxf(M, mlv[q].x);
+      float L = 0.f;
+      float O[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int q = 0; q < 16; ++q) {
+        if (q < n_active) {
+          const float w = mlv[q].x == -INFINITY ? 0.f : exp2f(mlv[q].x - M);
+          L += w * mlv[q].y;
+          O[0] += w * ov[q].x;
+          O[1] += w * ov[q].y;
+          O[2] += w * ov[q].z;
+          O[3] += w * ov[q].w;
+        }
+      }
+      emit(v, d, O[0], O[1], O[2], O[3], L);
+    }
   }
   trace_at(ts, 7);
   if (tid == 0 && !dry) a.counters[unit] = 0;
