@@ -227,15 +227,19 @@ AttnGeo attn_geometry(const memspec_model_cfg& c, int groups, int R, int max_seq
   g.qmax = gs * rpb;
   const int units = groups * c.n_kv_heads * g.row_blocks;
   const int max_splits = ceil_div(max_seq, 64);
-  // at most two CTAs per SM in one wave (an extra partial wave would double the time)
-  // (and at most 16 splits: the combine fetches 16 splits' outputs per round trip)
-  int want = std::max(1, std::min(16, (2 * sm_count()) / units));
+  // one wave of CTAs: the transposed form (at most 8 query vectors per CTA, 2
+  // stages) fits three per SM, the 16-row form (3 stages) two (an extra partial
+  // wave would double the time); at most 16 splits (the combine fetches 16
+  // splits' outputs per round trip)
+  const bool tq = g.qmax <= 8;
+  const int per_sm = tq ? 3 : 2;
+  int want = std::max(1, std::min(16, (per_sm * sm_count()) / units));
   want = std::min(want, max_splits);
   g.chunk = round_up(ceil_div(max_seq, want), 64);
   g.n_splits = ceil_div(max_seq, g.chunk);
   // the combine keeps (2 n_splits + 1) x qmax floats of split statistics in the
-  // CTA's shared memory (3 stages x 64 keys x hd x 2 x 2 bytes, last 16 bytes reserved)
-  const size_t smem = static_cast<size_t>(3) * 2 * 64 * c.head_dim * 2 - 16;
+  // CTA's shared memory (stages x 64 keys x hd x 2 x 2 bytes, last 16 bytes reserved)
+  const size_t smem = static_cast<size_t>(tq ? 2 : 3) * 2 * 64 * c.head_dim * 2 - 16;
   while (static_cast<size_t>(2 * g.n_splits + 1) * g.qmax * 4 > smem) {
     g.chunk *= 2;
     g.n_splits = ceil_div(max_seq, g.chunk);

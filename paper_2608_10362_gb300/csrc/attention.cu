@@ -32,7 +32,7 @@ namespace {
 using namespace attn;
 
 template <int HD, bool TQ>
-__global__ void __launch_bounds__(kAttThreads, 2) attn_kernel(const __grid_constant__ AttnArgs a) {
+__global__ void __launch_bounds__(kAttThreads, TQ ? 3 : 2) attn_kernel(const __grid_constant__ AttnArgs a) {
   extern __shared__ __align__(128) uint8_t smem_raw[];
   __shared__ uint64_t bars[kStages];   // TMA stages
   if (a.tma && threadIdx.x == 0) {
@@ -52,6 +52,9 @@ __global__ void __launch_bounds__(kAttThreads, 2) attn_kernel(const __grid_const
   // global memory (see attention_cta)
   attention_cta<HD, TQ>(a, 0, 0, 0, 0, smem_raw, threadIdx.x, sync, [] {}, false, nullptr, true);
   __syncthreads();
+  // the dry run wrote the stages through the generic proxy; the copies into them
+  // come through the async proxy
+  if (a.tma && threadIdx.x == 0) fence_proxy_async_smem();
   auto wait = [&] {
     pdl_wait();
     trace_at(trace, 13);
@@ -65,7 +68,9 @@ __global__ void __launch_bounds__(kAttThreads, 2) attn_kernel(const __grid_const
 }  // namespace
 
 size_t attention_smem_bytes(const AttnArgs& a) {
-  return a.hd == 64 ? attention_smem_bytes_hd<64>() : attention_smem_bytes_hd<128>();
+  const bool tq = a.qmax <= 8;
+  if (a.hd == 64) return tq ? attention_smem_bytes_hd<64, true>() : attention_smem_bytes_hd<64, false>();
+  return tq ? attention_smem_bytes_hd<128, true>() : attention_smem_bytes_hd<128, false>();
 }
 cudaError_t attention_set_max_smem() {
   for (const void* f : {reinterpret_cast<const void*>(attn_kernel<64, false>),

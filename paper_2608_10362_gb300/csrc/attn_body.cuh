@@ -66,19 +66,26 @@ __device__ __forceinline__ uint32_t swz(int row, int ch) {
   return static_cast<uint32_t>((ch >> 3) * (kKeyTile * 128) + row * 128 + (((ch & 7) ^ (row & 7)) << 4));
 }
 
-template <int HD>
+// Pipeline stages: 3; the transposed form (at most 8 query vectors, three CTAs
+// per SM) runs 2.
+template <bool kTQ>
+__host__ __device__ constexpr int attention_stages() {
+  return kTQ ? 2 : kStages;
+}
+
+template <int HD, bool kTQ = false>
 __host__ __device__ constexpr size_t attention_body_bytes() {
-  // kStages x (K tile + V tile); the merge buffers (o, (m, l), weights, (M, L)) reuse it
-  return static_cast<size_t>(kStages) * 2 * kKeyTile * HD * 2 >
+  // stages x (K tile + V tile); the merge buffers (o, (m, l), weights, (M, L)) reuse it
+  return static_cast<size_t>(attention_stages<kTQ>()) * 2 * kKeyTile * HD * 2 >
                  static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + kMaxQ * 6 * 4
-             ? static_cast<size_t>(kStages) * 2 * kKeyTile * HD * 2
+             ? static_cast<size_t>(attention_stages<kTQ>()) * 2 * kKeyTile * HD * 2
              : static_cast<size_t>(4) * 16 * HD * 4 + 4 * 16 * 2 * 4 + kMaxQ * 6 * 4;
 }
 // + up to 1008 bytes to align the stages to 1024 (the swizzle's period), + a
 // 16-byte flag at the end
-template <int HD>
+template <int HD, bool kTQ = false>
 __host__ __device__ constexpr size_t attention_smem_bytes_hd() {
-  return 1008 + attention_body_bytes<HD>() + 16;
+  return 1008 + attention_body_bytes<HD, kTQ>() + 16;
 }
 
 // One CTA of split-KV attention for unit (g, kvh, rb, split), run by 128 threads
@@ -94,7 +101,8 @@ __host__ __device__ constexpr size_t attention_smem_bytes_hd() {
 // and the cached keys / values before the group's first new position are final
 // before wait() (see AttnArgs::ctx_early): the plan is read, and the first tiles
 // that hold only such keys are requested, before it.
-// bars: kStages mbarriers (count 1) for the TMA path (a.tma, not dry), else nullptr.
+// bars: attention_stages<kTQ>() mbarriers (count 1) for the TMA path (a.tma, not
+// dry), else nullptr.
 // kTQ: at most 8 query vectors (the launch's qmax <= 8; checked): the keys are the
 // MMA's M side, S^T = K Q^T and O^T = V^T P^T with the queries as N = 8, half the
 // MMAs, accumulator registers and rescaling work of the 16-row form.
@@ -104,6 +112,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
                                               bool early, unsigned long long* ts = nullptr,
                                               bool dry = false, uint64_t* bars = nullptr) {
   constexpr int kChunks = HD / 8;                        // 16-byte chunks per row
+  constexpr int kSt = attention_stages<kTQ>();           // pipeline stages
   constexpr int kTileBytes = kKeyTile * HD * 2;          // one K (or V) tile
   constexpr int kNT = HD / 8;                            // n8 tiles of the output
   if (!early) wait();
@@ -142,22 +151,22 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   const int mt = warp / kg, kgi = warp - mt * kg;
   const bool active = mt < n_mt;
 
-  // kStages x (K tile, V tile), 1024-byte aligned
+  // kSt x (K tile, V tile), 1024-byte aligned
   uint8_t* kv = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
   const bool tma = bars != nullptr && !dry;
-  int* flag = reinterpret_cast<int*>(smem_raw + attention_smem_bytes_hd<HD>() - 16);
+  int* flag = reinterpret_cast<int*>(smem_raw + attention_smem_bytes_hd<HD, kTQ>() - 16);
   const size_t kv_base = (static_cast<size_t>(req) * a.Hkv + kvh) * a.max_seq;
   const bf16* kc = a.kcache + kv_base * HD;
   const bf16* vc = a.vcache + kv_base * HD;
 
   const int kv_row0 = (req * a.Hkv + kvh) * a.max_seq;   // first row of this head in the maps
   auto load_tile = [&](int t) {
-    uint8_t* ks = kv + (t % kStages) * 2 * kTileBytes;
+    uint8_t* ks = kv + (t % kSt) * 2 * kTileBytes;
     uint8_t* vs = ks + kTileBytes;
     const int kt0 = k0 + t * kKeyTile;
     if (tma) {   // one thread: the K and V boxes of the tile (rows past k1 are masked / zeroed later)
       if (tid == 0) {
-        uint64_t* bar = &bars[t % kStages];
+        uint64_t* bar = &bars[t % kSt];
         const uint64_t pol = l2_policy_evict_first();
         mbar_arrive_expect_tx(bar, 2u * kTileBytes);
 #pragma unroll
@@ -178,9 +187,9 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   };
 
   // prologue: the TMA path requests every stage (Q goes straight to registers),
-  // the cp.async path the first kStages-1 tiles (one commit group per stage);
+  // the cp.async path the first kSt-1 tiles (one commit group per stage);
   // early: the tiles that hold only keys below pos0 go before the wait
-  const int depth = tma ? kStages : kStages - 1;
+  const int depth = tma ? kSt : kSt - 1;
   int s_pre = 0;
   if (early) {
     for (; s_pre < depth && s_pre < n_tiles && k0 + (s_pre + 1) * kKeyTile <= pos0; ++s_pre) {
@@ -275,7 +284,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     if (tma) {
       // one thread waits (bounded); all follow its outcome
       if (tid == 0)
-        *flag = mbar_wait_bounded(&bars[t % kStages], static_cast<uint32_t>(t / kStages) & 1u, nullptr, a.status)
+        *flag = mbar_wait_bounded(&bars[t % kSt], static_cast<uint32_t>(t / kSt) & 1u, nullptr, a.status)
                     ? 1
                     : 0;
       sync();
@@ -283,7 +292,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
       waited = t + 1;
       const int nk = min(kKeyTile, k1 - (k0 + t * kKeyTile));
       if (nk < kKeyTile) {   // V rows past the split's end hold other positions (or garbage): zero them
-        uint8_t* vs = kv + (t % kStages) * 2 * kTileBytes + kTileBytes;
+        uint8_t* vs = kv + (t % kSt) * 2 * kTileBytes + kTileBytes;
         for (int c = tid; c < (kKeyTile - nk) * kChunks; c += kAttThreads) {
           const int row = nk + c / kChunks, ch = c % kChunks;
           *reinterpret_cast<uint4*>(vs + swz<HD>(row, ch)) = make_uint4(0u, 0u, 0u, 0u);
@@ -292,20 +301,20 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
       }
       // the stage refilled next (tile t-1's) was last read (ldmatrix, generic
       // proxy) before the barrier above
-      if (next < n_tiles && next < t + kStages) {
+      if (next < n_tiles && next < t + kSt) {
         if (tid == 0) fence_proxy_async_smem();
         load_tile(next);
         ++next;
       }
     } else {
-      cp_async_wait<kStages - 2>();
+      cp_async_wait<kSt - 2>();
       sync();
-      if (t + kStages - 1 < n_tiles) load_tile(t + kStages - 1);
+      if (t + kSt - 1 < n_tiles) load_tile(t + kSt - 1);
       cp_async_commit();
     }
     if (t == 0) trace_at(ts, 10);
     if (!active) continue;
-    const uint32_t ks_addr = smem_addr(kv + (t % kStages) * 2 * kTileBytes);
+    const uint32_t ks_addr = smem_addr(kv + (t % kSt) * 2 * kTileBytes);
     const uint32_t vs_addr = ks_addr + kTileBytes;
     const int kt0 = k0 + t * kKeyTile;
     if constexpr (kTQ) {
@@ -534,7 +543,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   if (tma && waited < n_tiles) {   // a wait ran out: let the copies still in flight land, then stop
     if (tid == 0)
       for (int t = waited; t < next; ++t)
-        mbar_wait_drain(&bars[t % kStages], static_cast<uint32_t>(t / kStages) & 1u);
+        mbar_wait_drain(&bars[t % kSt], static_cast<uint32_t>(t / kSt) & 1u);
     sync();
     return;
   }
@@ -659,7 +668,7 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
   // Both ways below compute M = max m_s, weights 2^(m_s - M), L and the weighted
   // sum of the o_s in ascending split order (identical results).
   const size_t land_o = static_cast<size_t>(n_active) * qmax * HD;   // floats
-  if ((land_o + static_cast<size_t>(n_active) * qmax * 2) * 4 <= attention_body_bytes<HD>()) {
+  if ((land_o + static_cast<size_t>(n_active) * qmax * 2) * 4 <= attention_body_bytes<HD, kTQ>()) {
     // every active split's o (contiguous, [split][qmax][HD]) by 16-byte cp.async
     // (L2) and its (m, l) by ld.cg land in the stages - free now: this CTA's own
     // partial went out above - in one round trip; the sums read shared memory
