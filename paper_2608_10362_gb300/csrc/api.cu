@@ -732,12 +732,28 @@ void emit_gemm(memspec_ctx* c, GemmArgs& a, std::vector<PassOp>& ops) {
   a.partials = c->gemm_part;
   a.counters = c->gemm_cnt;
   a.status = c->status;
+  // Many rows (batched verify, prefill): split row tiles get their own epilogue
+  // launch, one CTA per (row tile, 16-row chunk), instead of one contributor
+  // folding every chunk in turn.  MEMSPEC_SPLIT_EPI_ROWS sets the threshold
+  // (0: never; measurement).
+  static const int split_rows = env_int("MEMSPEC_SPLIT_EPI_ROWS", 64);
+  a.split_epi = (!c->pass_kernel && a.csk == 0 && split_rows > 0 && a.n_pad >= split_rows &&
+                 !sk_split_free(a.row_tiles * a.k_tiles, a.k_tiles, grid))
+                    ? 1
+                    : 0;
   PassOp op{};
   op.type = OP_GEMM;
   op.grid = grid;
   op.smem = static_cast<int>(gemm_smem_bytes(a.n_pad, a.stages, planes, a.csk));
   op.u.g = a;
   ops.push_back(op);
+  if (a.split_epi) {
+    PassOp ep{};
+    ep.type = OP_GEMM_EPI;
+    ep.grid = grid;
+    ep.u.g = a;
+    ops.push_back(ep);
+  }
 }
 
 // Launches as separate kernels: the op after the embedding kernel (which writes
@@ -999,6 +1015,7 @@ memspec_status run_ops_separately(memspec_ctx* c, const std::vector<PassOp>& ops
     switch (op.type) {
       case OP_EMBED: e = launch_embed(op.u.e, op.n_units, c->main, c->pdl); break;
       case OP_GEMM: e = launch_gemm(op.u.g, op.grid, op.smem, c->main, c->pdl && !op.full_dep); break;
+      case OP_GEMM_EPI: e = launch_gemm_split_epi(op.u.g, op.grid, c->main, c->pdl); break;
       case OP_ATTN: e = launch_attention(op.u.at, op.grid, c->main, c->pdl && !op.full_dep); break;
       case OP_SAMPLE: e = launch_sample(op.u.s, c->main, c->pdl); break;
       case OP_ACCEPT: e = launch_accept(op.u.acc, c->main, false); break;

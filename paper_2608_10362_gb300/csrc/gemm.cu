@@ -344,6 +344,33 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_stream_kernel(const __grid_c
   if (threadIdx.x == 64) trace_at(trace, 1);
 }
 
+// The epilogue of the split row tiles of a GEMM launched with split_epi (at
+// least 64 rows: one CTA folding every 16-row chunk of a tile in turn would
+// hold the launch for tens of microseconds).  CTA (rt, chunk), 128 threads
+// (thread = feature within the tile): if row tile rt had several contributors,
+// sum their partials in ascending CTA order (the order of the in-kernel
+// reduction) and run the epilogue for the chunk's 16 rows; row tiles owned by
+// one CTA were finished by it.  gemm_grid: the GEMM's grid (its stream-K split).
+template <int EPI>
+__global__ void __launch_bounds__(128) gemm_split_epi_kernel(const __grid_constant__ GemmArgs a,
+                                                             int gemm_grid) {
+  __shared__ EpiCtx ectx;
+  __shared__ float stage[kStageFloats];
+  __shared__ float rms[kMaxRows];
+  __shared__ float red[4][16];
+  const int rt = blockIdx.x, chunk = blockIdx.y, et = threadIdx.x;
+  const int KT = a.k_tiles, T = a.row_tiles * KT, G = gemm_grid;
+  const int c_first = sk_cta_of(rt * KT, T, G), c_last = sk_cta_of((rt + 1) * KT - 1, T, G);
+  pdl_launch_dependents();
+  if (c_first == c_last) return;
+  pdl_wait();
+  float v[16];
+  reduce_partials(a, rt, c_first, c_last, chunk, et, T, G, v);
+  if (a.rms) rms_chunk(a, rms, chunk, et);
+  epi_prologue<EPI>(a, &ectx, et);
+  apply_epilogue<EPI>(a, &ectx, red, stage, rms, rt, chunk, et, v, nullptr, false);
+}
+
 }  // namespace
 
 // Shared-memory budget of the stage ring.  A deep ring keeps more weight bytes
@@ -467,6 +494,26 @@ cudaError_t launch_gemm(const GemmArgs& a, int grid, size_t smem, cudaStream_t s
     case EPI_RESIDUAL: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_RESIDUAL, false>, a);
     case EPI_SWIGLU: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_SWIGLU, false>, a);
     case EPI_QKV: return cudaLaunchKernelEx(&cfg, gemm_stream_kernel<EPI_QKV, false>, a);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_gemm_split_epi(const GemmArgs& a, int gemm_grid, cudaStream_t s, bool pdl) {
+  if (a.n_pad % 16 != 0 || a.n_pad > kMaxRows) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.row_tiles, a.n_pad / 16);
+  cfg.blockDim = dim3(128);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  switch (a.epi) {
+    case EPI_F32: return cudaLaunchKernelEx(&cfg, gemm_split_epi_kernel<EPI_F32>, a, gemm_grid);
+    case EPI_RESIDUAL: return cudaLaunchKernelEx(&cfg, gemm_split_epi_kernel<EPI_RESIDUAL>, a, gemm_grid);
+    case EPI_SWIGLU: return cudaLaunchKernelEx(&cfg, gemm_split_epi_kernel<EPI_SWIGLU>, a, gemm_grid);
+    case EPI_QKV: return cudaLaunchKernelEx(&cfg, gemm_split_epi_kernel<EPI_QKV>, a, gemm_grid);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -347,6 +347,30 @@ __device__ __forceinline__ void rms_prologue(const GemmArgs& a, float* rms, int 
   named_bar_sync(1, 128);
 }
 
+// rms_prologue for the 16 rows of one chunk only (threads et < 16, the same
+// summation order, every partial sum of a row in flight at once); ends with a
+// barrier over the 128 threads.
+__device__ __forceinline__ void rms_chunk(const GemmArgs& a, float* rms, int chunk, int et) {
+  const int r = chunk * 16 + et;
+  if (et < 16 && r < a.n_pad) {
+    float val = 0.f;
+    if (r < a.rows_total) {
+      float sum = 0.f;
+      for (int i0 = 0; i0 < a.ss_count; i0 += 32) {
+        float t[32];
+#pragma unroll
+        for (int q = 0; q < 32; ++q)
+          t[q] = (i0 + q < a.ss_count) ? a.ss[static_cast<size_t>(i0 + q) * a.ss_stride + r] : 0.f;
+#pragma unroll
+        for (int q = 0; q < 32; ++q) sum += t[q];
+      }
+      val = rsqrtf(sum / static_cast<float>(a.k_in) + a.eps);
+    }
+    rms[r] = val;
+  }
+  named_bar_sync(1, 128);
+}
+
 // Sum of the split-K partials of row tile rt, chunk `chunk`, for feature et:
 // contributors in ascending CTA order, four fetched at once.
 __device__ __forceinline__ void reduce_partials(const GemmArgs& a, int rt, int c_first, int c_last,
@@ -533,6 +557,7 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, const EpiCtx
   if (lane == 0) mbar_arrive(&acc_empty[buf]);
   if (full) return;
   trace_at(ts, 4);
+  if (a.split_epi) return;   // the split epilogue kernel finishes this row tile
   if (CSK && dsm) {
     if (c != c_first) return;
     // one thread waits; the epilogue threads follow (or stop) together, then each

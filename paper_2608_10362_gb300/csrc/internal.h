@@ -139,6 +139,9 @@ struct GemmArgs {
   // split-K scratch
   float* partials;          // [2 * grid][n_pad * 128]
   int* counters;            // [row_tiles], zero on entry, left zero
+  int split_epi;            // 1: contributors to a split row tile only store their partials;
+                            // gemm_split_epi_kernel (the next launch) sums them and runs the
+                            // epilogue, one CTA per (row tile, 16-row chunk)
   int csk;                  // > 1: launched in clusters of csk CTAs (n_pad == 16 only); a
                             // row tile whose contributors share a cluster is summed by
                             // its first contributor from partials the others push into
@@ -337,6 +340,7 @@ int gemm_pick_stages(int n_pad, int planes = 1, int csk = 0);
 // `smem` bytes of dynamic shared memory that can be resident at once (0: none).
 int gemm_max_active_clusters(int epi, int csk, size_t smem);
 cudaError_t gemm_set_max_smem();
+cudaError_t launch_gemm_split_epi(const GemmArgs& a, int gemm_grid, cudaStream_t s, bool pdl);
 cudaError_t launch_attention(const AttnArgs& a, int n_groups, cudaStream_t s, bool pdl);
 size_t attention_smem_bytes(const AttnArgs& a);
 cudaError_t attention_set_max_smem();

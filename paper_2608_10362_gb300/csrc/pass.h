@@ -8,7 +8,7 @@ namespace memspec {
 
 // OP_TREE_WALK / OP_TREE_COMPACT run only as their own launches (tree steps)
 enum OpType : int { OP_EMBED = 0, OP_GEMM = 1, OP_ATTN = 2, OP_SAMPLE = 3, OP_ACCEPT = 4, OP_TREE_WALK = 5,
-                    OP_TREE_COMPACT = 6 };
+                    OP_TREE_COMPACT = 6, OP_GEMM_EPI = 7 };   // OP_GEMM_EPI: u.g, grid = the GEMM's
 
 struct alignas(64) PassOp {
   int type;
