@@ -1096,6 +1096,10 @@ memspec_status attach_trace(memspec_ctx* c, std::vector<PassOp>& ops) {
   for (size_t n = 0; n < ops.size() && n < static_cast<size_t>(kPassTraceOps); ++n) {
     unsigned long long* row = c->trace + 2 + n * nsm * kPassTraceSlots;
     if (ops[n].type == OP_GEMM) ops[n].u.g.trace = row;
+    if (ops[n].type == OP_GEMM_EPI) {
+      ops[n].u.g.trace = row;
+      ops[n].u.g.trace_ctas = nsm;
+    }
     if (ops[n].type == OP_ATTN) {
       ops[n].u.at.trace = row;
       ops[n].u.at.trace_ctas = nsm;

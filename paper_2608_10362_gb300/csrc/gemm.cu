@@ -361,14 +361,24 @@ __global__ void __launch_bounds__(128) gemm_split_epi_kernel(const __grid_consta
   const int rt = blockIdx.x, chunk = blockIdx.y, et = threadIdx.x;
   const int KT = a.k_tiles, T = a.row_tiles * KT, G = gemm_grid;
   const int c_first = sk_cta_of(rt * KT, T, G), c_last = sk_cta_of((rt + 1) * KT - 1, T, G);
+  // optional trace (a.trace: 16 slots per CTA, CTAs in launch order up to the
+  // row's width): 0 entry, 13 dependency released, 2 partials summed, 3 context
+  // built, 1 done
+  const int lin = blockIdx.y * gridDim.x + blockIdx.x;
+  unsigned long long* ts = (a.trace != nullptr && et == 0 && lin < a.trace_ctas) ? a.trace + lin * 16 : nullptr;
+  trace_at(ts, 0);
   pdl_launch_dependents();
   if (c_first == c_last) return;
   pdl_wait();
+  trace_at(ts, 13);
   float v[16];
   reduce_partials(a, rt, c_first, c_last, chunk, et, T, G, v);
+  if (ts != nullptr) trace_after(ts, 2, v[0] + v[15]);
   if (a.rms) rms_chunk(a, rms, chunk, et);
   epi_prologue<EPI>(a, &ectx, et);
+  trace_at(ts, 3);
   apply_epilogue<EPI>(a, &ectx, red, stage, rms, rt, chunk, et, v, nullptr, false);
+  trace_at(ts, 1);
 }
 
 }  // namespace

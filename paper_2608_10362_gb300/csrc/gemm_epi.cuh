@@ -386,7 +386,7 @@ __device__ __forceinline__ void reduce_partials(const GemmArgs& a, int rt, int c
       if (cc <= c_last) {
         const int sl = (sk_begin(cc, T, G) >= rt * KT) ? 0 : 1;
         const float* pp = a.partials + static_cast<size_t>(2 * cc + sl) * a.n_pad * kTileM +
-                          static_cast<size_t>(et) * a.n_pad + chunk * 16;
+                          (static_cast<size_t>(chunk) * kTileM + et) * 16;
 #pragma unroll
         for (int e = 0; e < 4; ++e) tmp[q][e] = ld_cg_f4(pp + 4 * e);
       }
@@ -541,13 +541,15 @@ __device__ __forceinline__ void epilogue_segment(const GemmArgs& a, const EpiCtx
         st_async_f4(raddr + 16 * q, v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3], rbar);
     }
   } else {
-    // partial sums, feature-major: thread et owns n_pad consecutive floats
+    // partial sums, chunk-major: the 16 rows of chunk k for feature et at
+    // ((k * 128) + et) * 16 (a warp's stores, and a reader's loads, of one chunk
+    // are one contiguous 2 KB run)
     const int slot = (seg == 0) ? 0 : 1;
     float* pb = a.partials + static_cast<size_t>(2 * c + slot) * a.n_pad * kTileM +
-                static_cast<size_t>(et) * a.n_pad;
+                static_cast<size_t>(et) * 16;
     for (int chunk = 0; chunk < a.n_pad / 16; ++chunk) {
       load_chunk(chunk);
-      float4* dst = reinterpret_cast<float4*>(pb + chunk * 16);
+      float4* dst = reinterpret_cast<float4*>(pb + static_cast<size_t>(chunk) * kTileM * 16);
 #pragma unroll
       for (int q = 0; q < 4; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
     }

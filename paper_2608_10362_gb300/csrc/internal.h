@@ -170,6 +170,7 @@ struct GemmArgs {
   const RowPlan* plan;      // nullptr: rows < rows_total are valid, no positions
   uint32_t* status;
   unsigned long long* trace;  // nullptr, or this op's trace row (16 slots per CTA)
+  int trace_ctas;           // split epilogue kernel: CTAs (linear index) that record
   int warm;                 // 1: dry run of the tail before griddepcontrol.wait
   int ctx_early;            // 1: every kernel before the previous one has completed when
                             // this one starts (an earlier launch of the pass had a full
