@@ -139,10 +139,13 @@ __device__ __forceinline__ void attention_cta(const AttnArgs& a, int g, int kvh,
     if (threadIdx.x == 0 && split == 0) atomicOr(a.status, 0x4u);
     return;
   }
-  const int n_active = (kmax + a.chunk) / a.chunk;   // ceil((kmax + 1) / chunk)
+  // the keys 0..kmax spread evenly over the launch's splits, whole 64-key tiles
+  // each (a.chunk sizes the splits for max_seq; the context may be far shorter)
+  const int chunk = ((kmax + a.n_splits) / a.n_splits + kKeyTile - 1) / kKeyTile * kKeyTile;
+  const int n_active = (kmax + chunk) / chunk;   // ceil((kmax + 1) / chunk)
   if (split >= n_active) return;
-  const int k0 = split * a.chunk;
-  const int k1 = min(k0 + a.chunk, kmax + 1);
+  const int k0 = split * chunk;
+  const int k1 = min(k0 + chunk, kmax + 1);
   const int n_tiles = (k1 - k0 + kKeyTile - 1) / kKeyTile;
 
   const int n_mt = (nq + 15) >> 4;

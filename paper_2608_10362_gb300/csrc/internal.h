@@ -188,7 +188,8 @@ struct AttnArgs {
   int H, Hkv, hd, max_seq;
   int rows_per_block;       // query rows (positions) per CTA
   int row_blocks;           // blocks per group
-  int chunk;                // keys per split
+  int chunk;                // keys per split at max_seq (the kernel spreads the actual
+                            // context over n_splits, in whole 64-key tiles)
   int n_splits;             // gridDim.x
   float scale_log2;         // log2(e) / sqrt(hd)
   float* part_o;            // [groups][Hkv][row_blocks][n_splits][qmax][hd]
