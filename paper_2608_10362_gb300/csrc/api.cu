@@ -2207,8 +2207,13 @@ memspec_status memspec_op_linear(const void* x, const void* w, float* y, int32_t
                                                              align256(static_cast<size_t>(a.row_tiles) * 4));
   a.plan = nullptr;
   const int grid = gemm_grid(a.row_tiles, a.k_tiles);
+  // at least 64 rows: split row tiles finished by the split epilogue kernel (as in
+  // the passes)
+  a.split_epi = (n_pad >= 64 && !sk_split_free(a.row_tiles * a.k_tiles, a.k_tiles, grid)) ? 1 : 0;
   cudaError_t e = launch_gemm(a, grid, gemm_smem_bytes(n_pad, a.stages),
                               static_cast<cudaStream_t>(stream), false);
+  if (e == cudaSuccess && a.split_epi)
+    e = launch_gemm_split_epi(a, grid, static_cast<cudaStream_t>(stream), false);
   if (e != cudaSuccess) {
     g_op_error = std::string("gemm launch: ") + cudaGetErrorString(e);
     return MEMSPEC_ERR_CUDA;
