@@ -24,8 +24,8 @@ memspec_status memspec_op_linear_scratch_bytes(int32_t rows, int32_t n_out, int3
  * This is the weight-streaming GEMM every projection of the verify and draft
  * passes runs (Q/K/V, O, gate/up, down, LM head): TMA-staged weight tiles,
  * tcgen05 MMA into TMEM, stream-K over all SMs, deterministic split-K
- * reduction (at 64 rows or more, split row tiles are finished by a second
- * launch on the same stream, one CTA per row tile and 16-row chunk).
+ * reduction (above 16 rows, split row tiles are finished by a second launch
+ * on the same stream, one CTA per row tile and 16-row chunk).
  * rows in 1..256, k a multiple of 8, n_out >= 1, and
  * ceil(n_out/128) * ceil(k/64) * (SMs + 1) below 2^32.
  * scratch_dev: memspec_op_linear_scratch_bytes bytes, 256-byte aligned; its

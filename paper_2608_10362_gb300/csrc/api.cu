@@ -737,11 +737,12 @@ void emit_gemm(memspec_ctx* c, GemmArgs& a, std::vector<PassOp>& ops) {
   a.partials = c->gemm_part;
   a.counters = c->gemm_cnt;
   a.status = c->status;
-  // Many rows (batched verify, prefill): split row tiles get their own epilogue
-  // launch, one CTA per (row tile, 16-row chunk), instead of one contributor
-  // folding every chunk in turn.  MEMSPEC_SPLIT_EPI_ROWS sets the threshold
-  // (0: never; measurement).
-  static const int split_rows = env_int("MEMSPEC_SPLIT_EPI_ROWS", 64);
+  // Two or more 16-row chunks (trees, batched verify, prefill): split row tiles
+  // get their own epilogue launch, one CTA per (row tile, 16-row chunk), instead
+  // of one contributor folding every chunk in turn (a 31-node tree step 5.02 ->
+  // 4.81 ms, batched 8B verify 17.6 -> 12.0 ms).  MEMSPEC_SPLIT_EPI_ROWS sets the
+  // threshold (0: never; measurement).
+  static const int split_rows = env_int("MEMSPEC_SPLIT_EPI_ROWS", 32);
   a.split_epi = (!c->pass_kernel && a.csk == 0 && split_rows > 0 && a.n_pad >= split_rows &&
                  !sk_split_free(a.row_tiles * a.k_tiles, a.k_tiles, grid))
                     ? 1
@@ -2207,9 +2208,9 @@ memspec_status memspec_op_linear(const void* x, const void* w, float* y, int32_t
                                                              align256(static_cast<size_t>(a.row_tiles) * 4));
   a.plan = nullptr;
   const int grid = gemm_grid(a.row_tiles, a.k_tiles);
-  // at least 64 rows: split row tiles finished by the split epilogue kernel (as in
-  // the passes)
-  a.split_epi = (n_pad >= 64 && !sk_split_free(a.row_tiles * a.k_tiles, a.k_tiles, grid)) ? 1 : 0;
+  // more than 16 rows: split row tiles finished by the split epilogue kernel (as
+  // in the passes)
+  a.split_epi = (n_pad >= 32 && !sk_split_free(a.row_tiles * a.k_tiles, a.k_tiles, grid)) ? 1 : 0;
   cudaError_t e = launch_gemm(a, grid, gemm_smem_bytes(n_pad, a.stages),
                               static_cast<cudaStream_t>(stream), false);
   if (e == cudaSuccess && a.split_epi)
