@@ -422,7 +422,9 @@ def run_pair_case(args, tname: str, dname: str, prefixes, K: int, T: float, seed
     for i in range(steps):
         eng.draft_step(K, T)
         ev[i][0].record(s)
+        torch.cuda.nvtx.range_push("verify")   # for profilers: --nvtx --nvtx-include "verify/"
         eng.verify_step(K)
+        torch.cuda.nvtx.range_pop()
         ev[i][1].record(s)
         eng.accept_commit(K, T)
     b_.record(s)
