@@ -4,11 +4,12 @@
 //
 // Grid: (key split, kv_head x row_block, request group).  A CTA takes the query
 // vectors of one KV head's group of query heads for a block of rows (at most 64
-// vectors, 16 per m-tile), streams its chunk of keys/values once through a
-// 3-stage ring of TMA boxes (128-byte swizzle, mbarrier per stage; the tiles
-// below the pass's first new position are requested before the launch waits for
-// its predecessor) and computes on tensor cores (mma.sync m16n8k16, bf16 in,
-// fp32 accumulate):
+// vectors, 16 per m-tile), streams its share of the keys/values (the context
+// spread evenly over the splits, whole 64-key tiles) once through a ring of TMA
+// boxes (128-byte swizzle, mbarrier per stage, 3 stages; 2 in the transposed
+// form; the tiles below the pass's first new position are requested before the
+// launch waits for its predecessor) and computes on tensor cores (mma.sync
+// m16n8k16, bf16 in, fp32 accumulate):
 //   S = Q K^T (Q pre-scaled by log2(e)/sqrt(hd), loaded straight into the
 //   A-operand registers), online softmax in registers (running max m, sum l),
 //   O += P V with P re-packed from the S fragments.
